@@ -1,0 +1,407 @@
+/*
+ * tfg_oracle.c -- plain, slow, fp64 CPU oracle for graph message aggregation.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the test-suite, the smoke check and the
+ * benchmark's CPU-baseline leg may load this file's library.  It shares no
+ * code, header or constant with the CUDA library and includes nothing of it.
+ *
+ * What it follows (tf_geometric, arXiv:2101.11552):
+ *   - Graph data structure, Section 2.1.1: edge_index is [2, E] int64, row 0
+ *     the source and row 1 the target of each edge; A_ij > 0 is an edge i -> j.
+ *   - Graph map-reduce framework, Section 2.1.2 / Fig. 5: a reducer groups
+ *     elements by a key (here the target node index) and reduces each group;
+ *     the GAT workflow is map (edge -> unnormalised score), reduce (segment
+ *     sum -> softmax denominator), map (divide).
+ *   - BatchGraph / graph pooling, Section 2.1.1 and Fig. 2a: nodes are reduced
+ *     per graph by node_graph_index.
+ *   - GCN normalisation D^-1/2 (A+I) D^-1/2 and GAT additive attention come
+ *     from the works the paper cites for those models (Section 2.2).
+ *
+ * Every function loops over edges (or nodes) in their original order and
+ * accumulates in double precision.  Empty groups reduce to 0 for every
+ * reducer (the paper does not fix this; it is the convention of this library).
+ *
+ * Planted-mistake switches (ORACLE_PLANT_*) exist only so that the pin tests
+ * can demonstrate that a plausible bug is caught; the normal build defines
+ * none of them.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define OK 0
+#define E_ARG (-1)
+#define E_RANGE (-5)
+#define E_UNSORTED (-6)
+
+#define R_SUM 0
+#define R_MEAN 1
+#define R_MAX 2
+
+/* ---------------------------------------------------------------------------
+ * CSR grouped by target: a stable counting sort of the edges by edge_index[1].
+ * The "reduce key" of Section 2.1.2 is the target node; grouping by it makes
+ * each group a contiguous row.  Within a row, edges keep their original order,
+ * which fixes a single canonical CSR.
+ *   rowptr[N+1], col[E] (source of each edge), perm[E] (original edge id),
+ *   in_degree[N].
+ * ------------------------------------------------------------------------- */
+int oracle_build_csr(int64_t n, int64_t e, const int64_t *edge_index,
+                     int32_t *rowptr, int32_t *col, int32_t *perm, int32_t *in_degree)
+{
+    if (n < 0 || e < 0) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+    for (int64_t i = 0; i < e; ++i)
+        if (src[i] < 0 || src[i] >= n || dst[i] < 0 || dst[i] >= n) return E_RANGE;
+    for (int64_t t = 0; t < n; ++t) in_degree[t] = 0;
+    for (int64_t i = 0; i < e; ++i) in_degree[dst[i]] += 1;
+    rowptr[0] = 0;
+    for (int64_t t = 0; t < n; ++t) rowptr[t + 1] = rowptr[t] + in_degree[t];
+    int32_t *cursor = (int32_t *)malloc(sizeof(int32_t) * (size_t)(n > 0 ? n : 1));
+    if (!cursor) return E_ARG;
+    for (int64_t t = 0; t < n; ++t) cursor[t] = rowptr[t];
+#ifdef ORACLE_PLANT_UNSTABLE_CSR
+    /* planted mistake: place edges in reverse order inside each row */
+    for (int64_t t = 0; t < n; ++t) cursor[t] = rowptr[t + 1];
+    for (int64_t i = 0; i < e; ++i) {
+        int32_t p = --cursor[dst[i]];
+        col[p] = (int32_t)src[i];
+        perm[p] = (int32_t)i;
+    }
+#else
+    for (int64_t i = 0; i < e; ++i) {
+        int32_t p = cursor[dst[i]]++;
+        col[p] = (int32_t)src[i];
+        perm[p] = (int32_t)i;
+    }
+#endif
+    free(cursor);
+    return OK;
+}
+
+/* ---------------------------------------------------------------------------
+ * GCN symmetric normalisation of (A + I) (Kipf & Welling, cited in Sec. 2.2).
+ *   deg[t]  = sum of the weights of the edges whose target is t
+ *             (+ fill when an implicit self-loop is added to every node)
+ *   dinv[t] = deg[t]^-1/2, or 0 when deg[t] == 0
+ *   w_norm[e] = w_e * dinv[src_e] * dinv[dst_e]         (COO order)
+ *   self_w[t] = fill * dinv[t]^2  when add_self_loops, else 0
+ * edge_weight == NULL means every weight is 1.
+ * ------------------------------------------------------------------------- */
+int oracle_gcn_norm(int64_t n, int64_t e, const int64_t *edge_index,
+                    const double *edge_weight, int add_self_loops, double fill,
+                    double *deg, double *dinv, double *w_norm, double *self_w)
+{
+    if (n < 0 || e < 0) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+    for (int64_t i = 0; i < e; ++i)
+        if (src[i] < 0 || src[i] >= n || dst[i] < 0 || dst[i] >= n) return E_RANGE;
+    for (int64_t t = 0; t < n; ++t) deg[t] = add_self_loops ? fill : 0.0;
+#ifdef ORACLE_PLANT_DROP_SELF_LOOP_DEGREE
+    for (int64_t t = 0; t < n; ++t) deg[t] = 0.0;
+#endif
+    for (int64_t i = 0; i < e; ++i) {
+#ifdef ORACLE_PLANT_OUT_DEGREE
+        deg[src[i]] += edge_weight ? edge_weight[i] : 1.0;   /* planted: by source */
+#else
+        deg[dst[i]] += edge_weight ? edge_weight[i] : 1.0;
+#endif
+    }
+    for (int64_t t = 0; t < n; ++t) dinv[t] = deg[t] > 0.0 ? 1.0 / sqrt(deg[t]) : 0.0;
+    for (int64_t i = 0; i < e; ++i) {
+        double w = edge_weight ? edge_weight[i] : 1.0;
+        w_norm[i] = w * dinv[src[i]] * dinv[dst[i]];
+    }
+    if (self_w)
+        for (int64_t t = 0; t < n; ++t) self_w[t] = add_self_loops ? fill * dinv[t] * dinv[t] : 0.0;
+    return OK;
+}
+
+/* ---------------------------------------------------------------------------
+ * Message aggregation (Fig. 1; reducer of Fig. 5b keyed by the target node):
+ *   out[t, :] = REDUCE over edges e with dst_e == t of  w_e * x[src_e, :]
+ * SUM, MEAN (= SUM / number of incoming edges) or MAX.  Empty rows give 0.
+ * self_w (optional, SUM only) adds self_w[t] * x[t, :], the implicit
+ * self-loop of GCN.  absout[t, f] = sum of |w_e * x[src_e, f]| (+ |self term|),
+ * the scale that a floating-point tolerance is measured against.
+ * ------------------------------------------------------------------------- */
+int oracle_aggregate(int reduce, int64_t n, int64_t e, const int64_t *edge_index,
+                     const double *w, const double *x, int64_t f,
+                     const double *self_w, double *out, double *absout)
+{
+    if (n < 0 || e < 0 || f < 0) return E_ARG;
+    if (reduce != R_SUM && reduce != R_MEAN && reduce != R_MAX) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+#ifdef ORACLE_PLANT_SWAP_DIRECTION
+    src = edge_index + e; dst = edge_index;          /* planted: aggregate into sources */
+#endif
+    for (int64_t i = 0; i < e; ++i)
+        if (src[i] < 0 || src[i] >= n || dst[i] < 0 || dst[i] >= n) return E_RANGE;
+    int64_t *count = (int64_t *)calloc((size_t)(n > 0 ? n : 1), sizeof(int64_t));
+    if (!count) return E_ARG;
+    for (int64_t k = 0; k < n * f; ++k) { out[k] = 0.0; absout[k] = 0.0; }
+    for (int64_t i = 0; i < e; ++i) {
+        int64_t s = src[i], t = dst[i];
+        double we = w ? w[i] : 1.0;
+        for (int64_t c = 0; c < f; ++c) {
+            double m = we * x[s * f + c];
+            if (reduce == R_MAX) {
+#ifdef ORACLE_PLANT_MAX_FROM_ZERO
+                if (m > out[t * f + c]) out[t * f + c] = m;      /* planted: max starts at 0 */
+#else
+                if (count[t] == 0 || m > out[t * f + c]) out[t * f + c] = m;
+#endif
+            } else {
+                out[t * f + c] += m;
+            }
+            absout[t * f + c] += fabs(m);
+        }
+        count[t] += 1;
+    }
+    if (reduce == R_MEAN) {
+        for (int64_t t = 0; t < n; ++t) {
+            if (count[t] == 0) continue;
+#ifdef ORACLE_PLANT_MEAN_PLUS_ONE
+            double cnt = (double)(count[t] + 1);              /* planted: off-by-one count */
+#else
+            double cnt = (double)count[t];
+#endif
+            for (int64_t c = 0; c < f; ++c) { out[t * f + c] /= cnt; absout[t * f + c] /= cnt; }
+        }
+    }
+    if (self_w && reduce == R_SUM) {
+        for (int64_t t = 0; t < n; ++t)
+            for (int64_t c = 0; c < f; ++c) {
+                double m = self_w[t] * x[t * f + c];
+                out[t * f + c] += m;
+                absout[t * f + c] += fabs(m);
+            }
+    }
+    free(count);
+    return OK;
+}
+
+/* Same definition, evaluated only for the listed target rows, walking the
+ * oracle's own stable CSR (rowptr/col/perm from oracle_build_csr).  A row's
+ * edges in that CSR are exactly the edges with that target, in original
+ * order, so each value equals the one oracle_aggregate computes.  w (COO
+ * order, NULL = 1) is indexed through perm.  out/absout are [nrows, f]. */
+int oracle_aggregate_rows(int reduce, int64_t n, const int32_t *rowptr, const int32_t *col,
+                          const int32_t *perm, const double *w, const double *x, int64_t f,
+                          const double *self_w, const int64_t *rows, int64_t nrows,
+                          double *out, double *absout)
+{
+    if (reduce != R_SUM && reduce != R_MEAN && reduce != R_MAX) return E_ARG;
+    for (int64_t r = 0; r < nrows; ++r) {
+        int64_t t = rows[r];
+        if (t < 0 || t >= n) return E_RANGE;
+        double *o = out + r * f, *a = absout + r * f;
+        for (int64_t c = 0; c < f; ++c) { o[c] = 0.0; a[c] = 0.0; }
+        int64_t cnt = 0;
+        for (int64_t k = rowptr[t]; k < rowptr[t + 1]; ++k) {
+            int64_t s = col[k];
+            double we = w ? w[perm[k]] : 1.0;
+            for (int64_t c = 0; c < f; ++c) {
+                double m = we * x[s * f + c];
+                if (reduce == R_MAX) {
+                    if (cnt == 0 || m > o[c]) o[c] = m;
+                } else {
+                    o[c] += m;
+                }
+                a[c] += fabs(m);
+            }
+            cnt += 1;
+        }
+        if (reduce == R_MEAN && cnt > 0)
+            for (int64_t c = 0; c < f; ++c) { o[c] /= (double)cnt; a[c] /= (double)cnt; }
+        if (self_w && reduce == R_SUM)
+            for (int64_t c = 0; c < f; ++c) {
+                double m = self_w[t] * x[t * f + c];
+                o[c] += m;
+                a[c] += fabs(m);
+            }
+    }
+    return OK;
+}
+
+/* ---------------------------------------------------------------------------
+ * GAT edge-softmax aggregation, following the map-reduce workflow of Fig. 5a:
+ *   node scores  s_src[n,h] = sum_c x[n,h,c] a_src[h,c];  s_dst likewise
+ *   map          l[e,h] = LeakyReLU(s_src[src_e,h] + s_dst[dst_e,h])
+ *   reduce       m[t,h] = max over edges into t of l[e,h]          (stability)
+ *                den[t,h] = sum over edges into t of exp(l[e,h] - m[t,h])
+ *   map          alpha[e,h] = exp(l[e,h] - m[dst_e,h]) / den[dst_e,h]
+ *   aggregate    out[t,h,:] = sum over edges into t of alpha[e,h] x[src_e,h,:]
+ * Subtracting the per-target max does not change alpha mathematically.
+ * x is [n, H*C] with the channels of head h at columns h*C .. h*C+C-1.
+ * alpha is [e, H] in COO order.  Targets without incoming edges give 0.
+ * absout[t, h*C+c] = sum of alpha[e,h] |x[src_e,h,c]|.
+ * ------------------------------------------------------------------------- */
+static double leaky(double v, double slope)
+{
+#ifdef ORACLE_PLANT_NO_LEAKY
+    (void)slope;
+    return v;                                             /* planted: no LeakyReLU */
+#else
+    return v > 0.0 ? v : slope * v;
+#endif
+}
+
+int oracle_edge_softmax(int64_t n, int64_t e, const int64_t *edge_index, const double *x,
+                        int h, int c, const double *a_src, const double *a_dst, double slope,
+                        double *out, double *alpha, double *absout)
+{
+    if (n < 0 || e < 0 || h <= 0 || c <= 0) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+    for (int64_t i = 0; i < e; ++i)
+        if (src[i] < 0 || src[i] >= n || dst[i] < 0 || dst[i] >= n) return E_RANGE;
+    int64_t f = (int64_t)h * c;
+    size_t nh = (size_t)(n > 0 ? n : 1) * (size_t)h;
+    double *s_src = (double *)calloc(nh, sizeof(double));
+    double *s_dst = (double *)calloc(nh, sizeof(double));
+    double *mx = (double *)calloc(nh, sizeof(double));
+    double *den = (double *)calloc(nh, sizeof(double));
+    char *seen = (char *)calloc(nh, 1);
+    double *logit = (double *)calloc((size_t)(e > 0 ? e : 1) * (size_t)h, sizeof(double));
+    if (!s_src || !s_dst || !mx || !den || !seen || !logit) {
+        free(s_src); free(s_dst); free(mx); free(den); free(seen); free(logit);
+        return E_ARG;
+    }
+    for (int64_t v = 0; v < n; ++v)
+        for (int hh = 0; hh < h; ++hh) {
+            double a = 0.0, b = 0.0;
+            for (int cc = 0; cc < c; ++cc) {
+                a += x[v * f + hh * c + cc] * a_src[hh * c + cc];
+                b += x[v * f + hh * c + cc] * a_dst[hh * c + cc];
+            }
+            s_src[v * h + hh] = a;
+            s_dst[v * h + hh] = b;
+        }
+    /* map: unnormalised scores; reduce: per-target max */
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            double l = leaky(s_src[src[i] * h + hh] + s_dst[dst[i] * h + hh], slope);
+            logit[i * h + hh] = l;
+            size_t k = (size_t)dst[i] * h + hh;
+            if (!seen[k] || l > mx[k]) mx[k] = l;
+            seen[k] = 1;
+        }
+    /* reduce: segment sum of exp -> softmax denominator */
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh)
+            den[(size_t)dst[i] * h + hh] += exp(logit[i * h + hh] - mx[(size_t)dst[i] * h + hh]);
+    /* map: divide; then the attention-weighted sum */
+    for (int64_t k = 0; k < n * f; ++k) { out[k] = 0.0; absout[k] = 0.0; }
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            size_t k = (size_t)dst[i] * h + hh;
+            double al = exp(logit[i * h + hh] - mx[k]) / den[k];
+            if (alpha) alpha[i * h + hh] = al;
+            for (int cc = 0; cc < c; ++cc) {
+                double m = al * x[src[i] * f + hh * c + cc];
+                out[dst[i] * f + hh * c + cc] += m;
+                absout[dst[i] * f + hh * c + cc] += fabs(m);
+            }
+        }
+    free(s_src); free(s_dst); free(mx); free(den); free(seen); free(logit);
+    return OK;
+}
+
+/* The same three passes, restricted to the in-edges of the listed target rows
+ * (walked through the oracle's stable CSR).  alpha_rows, when given, receives
+ * for each listed row its alpha values [deg, H] in CSR order, rows packed one
+ * after another (the caller sizes it from rowptr). */
+int oracle_edge_softmax_rows(int64_t n, const int32_t *rowptr, const int32_t *col,
+                             const double *x, int h, int c, const double *a_src,
+                             const double *a_dst, double slope, const int64_t *rows,
+                             int64_t nrows, double *out, double *alpha_rows, double *absout)
+{
+    if (h <= 0 || c <= 0) return E_ARG;
+    int64_t f = (int64_t)h * c;
+    int64_t apos = 0;
+    for (int64_t r = 0; r < nrows; ++r) {
+        int64_t t = rows[r];
+        if (t < 0 || t >= n) return E_RANGE;
+        int64_t k0 = rowptr[t], k1 = rowptr[t + 1], deg = k1 - k0;
+        double *o = out + r * f, *ab = absout + r * f;
+        for (int64_t q = 0; q < f; ++q) { o[q] = 0.0; ab[q] = 0.0; }
+        if (deg == 0) continue;
+        double *lg = (double *)malloc(sizeof(double) * (size_t)deg * (size_t)h);
+        if (!lg) return E_ARG;
+        for (int hh = 0; hh < h; ++hh) {
+            double sd = 0.0;
+            for (int cc = 0; cc < c; ++cc) sd += x[t * f + hh * c + cc] * a_dst[hh * c + cc];
+            double mx = 0.0, den = 0.0;
+            for (int64_t k = k0; k < k1; ++k) {
+                int64_t s = col[k];
+                double ss = 0.0;
+                for (int cc = 0; cc < c; ++cc) ss += x[s * f + hh * c + cc] * a_src[hh * c + cc];
+                double l = leaky(ss + sd, slope);
+                lg[(k - k0) * h + hh] = l;
+                if (k == k0 || l > mx) mx = l;
+            }
+            for (int64_t k = k0; k < k1; ++k) den += exp(lg[(k - k0) * h + hh] - mx);
+            for (int64_t k = k0; k < k1; ++k) {
+                int64_t s = col[k];
+                double al = exp(lg[(k - k0) * h + hh] - mx) / den;
+                if (alpha_rows) alpha_rows[(apos + (k - k0)) * h + hh] = al;
+                for (int cc = 0; cc < c; ++cc) {
+                    double m = al * x[s * f + hh * c + cc];
+                    o[hh * c + cc] += m;
+                    ab[hh * c + cc] += fabs(m);
+                }
+            }
+        }
+        apos += deg;
+        free(lg);
+    }
+    return OK;
+}
+
+/* ---------------------------------------------------------------------------
+ * Graph pooling keyed by node_graph_index (Fig. 2a; Section 2.1.1):
+ *   out[g, :] = REDUCE over nodes v with batch[v] == g of x[v, :]
+ * SUM, MEAN (divide by the node count) or MAX; empty graphs give 0.
+ * batch must be non-decreasing (a BatchGraph stacks graphs in order) and
+ * inside [0, G).
+ * ------------------------------------------------------------------------- */
+int oracle_segment_pool(int reduce, int64_t n, int64_t f, int64_t g, const int64_t *batch,
+                        const double *x, double *out, double *absout)
+{
+    if (n < 0 || f < 0 || g < 0) return E_ARG;
+    if (reduce != R_SUM && reduce != R_MEAN && reduce != R_MAX) return E_ARG;
+    for (int64_t v = 0; v < n; ++v) {
+        if (batch[v] < 0 || batch[v] >= g) return E_RANGE;
+        if (v > 0 && batch[v] < batch[v - 1]) return E_UNSORTED;
+    }
+    int64_t *count = (int64_t *)calloc((size_t)(g > 0 ? g : 1), sizeof(int64_t));
+    if (!count) return E_ARG;
+    for (int64_t k = 0; k < g * f; ++k) { out[k] = 0.0; absout[k] = 0.0; }
+#ifdef ORACLE_PLANT_POOL_SKIP_LAST
+    n = n > 0 ? n - 1 : 0;                                /* planted: drops the last node */
+#endif
+    for (int64_t v = 0; v < n; ++v) {
+        int64_t b = batch[v];
+        for (int64_t c = 0; c < f; ++c) {
+            double m = x[v * f + c];
+            if (reduce == R_MAX) {
+                if (count[b] == 0 || m > out[b * f + c]) out[b * f + c] = m;
+            } else {
+                out[b * f + c] += m;
+            }
+            absout[b * f + c] += fabs(m);
+        }
+        count[b] += 1;
+    }
+    if (reduce == R_MEAN)
+        for (int64_t b = 0; b < g; ++b) {
+            if (count[b] == 0) continue;
+            for (int64_t c = 0; c < f; ++c) {
+                out[b * f + c] /= (double)count[b];
+                absout[b * f + c] /= (double)count[b];
+            }
+        }
+    free(count);
+    return OK;
+}

@@ -1,0 +1,391 @@
+"""Pins of the fp64 oracle against facts fixed outside the oracle itself.
+
+Each pin is a function of an oracle object so that the same check can be run
+against a build with a planted mistake (``test_planted_mistakes_are_caught``):
+every plausible slip planted in ``oracle/tfg_oracle.c`` must make at least
+one pin fail.  No GPU is used here.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2101_11552_gb300 import graphgen as gg
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _golden(name):
+    with open(os.path.join(GOLDEN, name)) as fh:
+        return json.load(fh)
+
+
+def _undirected_random(n, m, seed, self_loops=False):
+    rng = np.random.default_rng(seed)
+    ei = gg.symmetrise(gg.er_pairs(n, m, rng))
+    return gg.with_self_loops(ei, n) if self_loops else ei
+
+
+# ---------------------------------------------------------------------------
+# CSR by target: brute force with Python's (stable) sort
+# ---------------------------------------------------------------------------
+def pin_csr_is_stable_grouping(o):
+    for seed, (n, e) in enumerate([(7, 40), (50, 300), (1, 5), (30, 0), (200, 2000)]):
+        w = gg.random_edge_case_graph(n, e, 1, seed, hub=0 if n > 1 else -1, isolated=min(3, n - 1))
+        ei = w.edge_index
+        rowptr, col, perm, deg = o.build_csr(ei, n)
+        order = sorted(range(e), key=lambda k: int(ei[1, k]))       # stable
+        assert list(perm) == order
+        assert list(col) == [int(ei[0, k]) for k in order]
+        counts = [0] * n
+        for k in range(e):
+            counts[int(ei[1, k])] += 1
+        assert list(deg) == counts
+        acc = [0]
+        for c in counts:
+            acc.append(acc[-1] + c)
+        assert list(rowptr) == acc
+
+
+def test_csr_is_stable_grouping():
+    pin_csr_is_stable_grouping(oracle.default)
+
+
+def test_csr_rejects_out_of_range():
+    ei = np.array([[0, 3], [1, 0]], dtype=np.int64)
+    with pytest.raises(oracle.OracleError) as exc:
+        oracle.build_csr(ei, 3)
+    assert exc.value.code == -5
+
+
+# ---------------------------------------------------------------------------
+# GCN normalisation and sum: hand examples, eigenvector identity, dense form
+# ---------------------------------------------------------------------------
+def pin_gcn_p4(o):
+    g = _golden("gcn_p4.json")
+    ei = gg.symmetrise(np.array(g["edges_undirected"], dtype=np.int64))
+    x = np.array(g["x"], dtype=np.float32)[:, None]
+    out, _ = o.gcn_aggregate(ei, 4, x, add_self_loops=g["add_self_loops"])
+    np.testing.assert_allclose(out[:, 0], g["out"], rtol=0, atol=g["abs_tol"])
+    closed = [1 / 2 + 2 / math.sqrt(6), 1 / math.sqrt(6) + 2 / 3 + 1, 2 / 3 + 1 + 4 / math.sqrt(6),
+              3 / math.sqrt(6) + 2]
+    np.testing.assert_allclose(out[:, 0], closed, rtol=1e-14)
+    nrm = o.gcn_norm(ei, 4, add_self_loops=1)
+    np.testing.assert_allclose(nrm["deg"], g["degree"], rtol=0, atol=0)
+
+
+def test_gcn_p4():
+    pin_gcn_p4(oracle.default)
+
+
+def pin_gcn_directed(o):
+    g = _golden("gcn_directed3.json")
+    ei = np.array(g["edge_index"], dtype=np.int64)
+    x = np.array(g["x"], dtype=np.float32)[:, None]
+    out, _ = o.gcn_aggregate(ei, 3, x, add_self_loops=1)
+    np.testing.assert_allclose(out[:, 0], g["out"], rtol=0, atol=g["abs_tol"])
+    nrm = o.gcn_norm(ei, 3, add_self_loops=1)
+    np.testing.assert_array_equal(nrm["deg"], g["in_degree_with_self_loop"])
+
+
+def test_gcn_directed_hand_example():
+    pin_gcn_directed(oracle.default)
+
+
+def pin_gcn_sqrt_degree_eigenvector(o):
+    """For a symmetric graph, D^-1/2 A' D^-1/2 sqrt(d) = sqrt(d) exactly (math).
+
+    (A' = A + fill I with weighted degrees d = row sums of A'.)  Holds with
+    and without implicit self-loops and with symmetric edge weights.
+    """
+    for seed, (n, m, selfl, weighted) in enumerate(
+            [(40, 90, 1, False), (300, 1200, 0, False), (120, 400, 1, True), (64, 64, 0, True)]):
+        rng = np.random.default_rng(50 + seed)
+        pairs = gg.er_pairs(n, m, rng)
+        ei = gg.symmetrise(pairs)
+        w = None
+        if weighted:
+            wp = rng.uniform(0.5, 2.0, size=m)
+            w = np.concatenate([wp, wp])
+        nrm = o.gcn_norm(ei, n, w, add_self_loops=selfl, fill=1.0)
+        x = np.sqrt(nrm["deg"])[:, None]
+        out, _ = o.aggregate(ei, n, x, "sum", w=nrm["w_norm"], self_w=nrm["self_w"])
+        np.testing.assert_allclose(out[:, 0], x[:, 0], rtol=1e-12, atol=1e-14)
+
+
+def test_gcn_sqrt_degree_eigenvector():
+    pin_gcn_sqrt_degree_eigenvector(oracle.default)
+
+
+def pin_dense_equivalence(o):
+    """Per-edge loops == numpy dense matrices for tiny random multigraphs."""
+    for seed in range(6):
+        n = [1, 5, 17, 33, 64, 64][seed]
+        e = [3, 12, 80, 200, 500, 0][seed]
+        wl = gg.random_edge_case_graph(n, e, 7, seed, hub=0 if n > 2 else -1, isolated=min(2, n - 1))
+        ei, x = wl.edge_index, wl.x
+        rng = np.random.default_rng(seed)
+        ew = rng.uniform(0.1, 3.0, size=e)
+        xd = x.astype(np.float64)
+        for selfl in (0, 1):
+            out, _ = o.gcn_aggregate(ei, n, x, ew, add_self_loops=selfl, fill=1.5)
+            ref = oracle.dense_gcn_matrix(ei, n, ew, selfl, 1.5) @ xd
+            np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-12)
+        m = oracle.dense_adjacency(ei, n, ew)
+        cnt = oracle.dense_adjacency(ei, n, None).sum(axis=1)
+        out, _ = o.aggregate(ei, n, x, "sum", w=ew)
+        np.testing.assert_allclose(out, m @ xd, rtol=1e-12, atol=1e-12)
+        out, _ = o.aggregate(ei, n, x, "mean", w=ew)
+        ref = np.where(cnt[:, None] > 0, (m @ xd) / np.maximum(cnt, 1)[:, None], 0.0)
+        np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_dense_equivalence():
+    pin_dense_equivalence(oracle.default)
+
+
+def pin_ones_give_in_degree(o):
+    for seed in range(3):
+        wl = gg.random_edge_case_graph(90, 700, 3, 10 + seed, hub=4, isolated=5)
+        ones = np.ones((90, 3), np.float32)
+        out, _ = o.aggregate(wl.edge_index, 90, ones, "sum")
+        deg = np.bincount(wl.edge_index[1], minlength=90)
+        np.testing.assert_array_equal(out, np.repeat(deg[:, None], 3, axis=1).astype(float))
+        out, _ = o.aggregate(wl.edge_index, 90, ones * 2.5, "mean")
+        np.testing.assert_array_equal(out, np.where(deg[:, None] > 0, 2.5, 0.0) * np.ones((1, 3)))
+
+
+def test_ones_give_in_degree_and_mean_of_constant():
+    pin_ones_give_in_degree(oracle.default)
+
+
+def pin_max_brute_force(o):
+    for seed in range(4):
+        n, e = 40, 300
+        wl = gg.random_edge_case_graph(n, e, 5, 20 + seed, hub=1, isolated=4)
+        ei, x = wl.edge_index, wl.x
+        rng = np.random.default_rng(seed)
+        w = rng.uniform(-2, 2, size=e).astype(np.float32)
+        for weights in (None, w):
+            out, _ = o.aggregate(ei, n, x, "max", w=weights)
+            for t in range(n):
+                ks = [k for k in range(e) if ei[1, k] == t]
+                for c in range(5):
+                    if not ks:
+                        assert out[t, c] == 0.0
+                        continue
+                    vals = [(1.0 if weights is None else float(weights[k])) * float(x[ei[0, k], c])
+                            for k in ks]
+                    assert out[t, c] == max(vals)
+
+
+def test_max_brute_force():
+    pin_max_brute_force(oracle.default)
+
+
+def test_permutation_invariance():
+    wl = gg.random_edge_case_graph(300, 4000, 9, 77, hub=3, isolated=10)
+    ei, x = wl.edge_index, wl.x
+    p = np.random.default_rng(1).permutation(ei.shape[1])
+    a, _ = oracle.aggregate(ei, 300, x, "max")
+    b, _ = oracle.aggregate(ei[:, p], 300, x, "max")
+    np.testing.assert_array_equal(a, b)
+    a, _ = oracle.gcn_aggregate(ei, 300, x, add_self_loops=1)
+    b, _ = oracle.gcn_aggregate(ei[:, p], 300, x, add_self_loops=1)
+    np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-13)
+    rp, col, perm, _ = oracle.build_csr(ei[:, p], 300)
+    # the permuted CSR holds the same multiset of sources per row
+    r0, c0, _, _ = oracle.build_csr(ei, 300)
+    np.testing.assert_array_equal(rp, r0)
+    for t in range(300):
+        assert sorted(col[rp[t]:rp[t + 1]]) == sorted(c0[r0[t]:r0[t + 1]])
+
+
+# ---------------------------------------------------------------------------
+# Edge softmax (GAT): hand values, normalisation, reduction to mean
+# ---------------------------------------------------------------------------
+def pin_star_softmax(o):
+    g = _golden("gat_star.json")
+    ei = np.array(g["edge_index"], dtype=np.int64)
+    for case in g["cases"]:
+        x = np.array([[case["x0"]], [1.0], [2.0], [3.0]], dtype=np.float32)
+        out, alpha, _ = o.edge_softmax(ei, 4, x, 1, 1, g["a_src"], g["a_dst"], g["negative_slope"])
+        np.testing.assert_allclose(alpha[:, 0], case["alpha"], rtol=0, atol=g["abs_tol"])
+        np.testing.assert_allclose(out[0, 0], case["out0"], rtol=0, atol=g["abs_tol"])
+        np.testing.assert_array_equal(out[1:, 0], 0.0)
+        ex = np.exp(np.array(case["logits"]))
+        np.testing.assert_allclose(alpha[:, 0], ex / ex.sum(), rtol=1e-13)
+
+
+def test_star_softmax():
+    pin_star_softmax(oracle.default)
+
+
+def pin_softmax_normalised_and_mean_limit(o):
+    for seed in range(3):
+        n, e, h, c = 60, 500, 3, 4
+        wl = gg.random_edge_case_graph(n, e, h * c, 30 + seed, hub=2, isolated=5)
+        ei, x = wl.edge_index, wl.x
+        rng = np.random.default_rng(seed)
+        a_s = rng.standard_normal(h * c)
+        a_d = rng.standard_normal(h * c)
+        _, alpha, _ = o.edge_softmax(ei, n, x, h, c, a_s, a_d, 0.2)
+        sums = np.zeros((n, h))
+        np.add.at(sums, ei[1], alpha)
+        deg = np.bincount(ei[1], minlength=n)
+        np.testing.assert_allclose(sums[deg > 0], 1.0, rtol=1e-12)
+        np.testing.assert_array_equal(sums[deg == 0], 0.0)
+        # zero attention vectors: every logit is 0, alpha = 1/in-degree -> mean
+        out, alpha, _ = o.edge_softmax(ei, n, x, h, c, np.zeros(h * c), np.zeros(h * c), 0.2)
+        mean, _ = o.aggregate(ei, n, x, "mean")
+        np.testing.assert_allclose(out, mean, rtol=1e-12, atol=1e-13)
+        np.testing.assert_allclose(alpha[:, 0], 1.0 / deg[ei[1]], rtol=1e-13)
+
+
+def test_softmax_normalised_and_mean_limit():
+    pin_softmax_normalised_and_mean_limit(oracle.default)
+
+
+def test_softmax_heads_are_independent():
+    n, e, c = 50, 400, 5
+    wl = gg.random_edge_case_graph(n, e, 2 * c, 41, hub=1)
+    ei, x = wl.edge_index, wl.x
+    rng = np.random.default_rng(3)
+    a_s0, a_d0 = rng.standard_normal(c), rng.standard_normal(c)
+    a_s = np.concatenate([a_s0, np.zeros(c)])
+    a_d = np.concatenate([a_d0, np.zeros(c)])
+    out, alpha, _ = oracle.edge_softmax(ei, n, x, 2, c, a_s, a_d, 0.2)
+    one, alpha1, _ = oracle.edge_softmax(ei, n, x[:, :c].copy(), 1, c, a_s0, a_d0, 0.2)
+    np.testing.assert_allclose(out[:, :c], one, rtol=1e-13, atol=1e-14)
+    np.testing.assert_allclose(alpha[:, 0], alpha1[:, 0], rtol=1e-13)
+    mean, _ = oracle.aggregate(ei, n, x[:, c:].copy(), "mean")
+    np.testing.assert_allclose(out[:, c:], mean, rtol=1e-12, atol=1e-13)
+
+
+def test_row_variants_match_full():
+    wl = gg.random_edge_case_graph(120, 1500, 8, 5, hub=7, isolated=6)
+    ei, x, n = wl.edge_index, wl.x, 120
+    csr = oracle.build_csr(ei, n)
+    rows = np.array([0, 7, 119, 118, 50, 3], dtype=np.int64)
+    rng = np.random.default_rng(0)
+    w = rng.uniform(-1, 1, ei.shape[1])
+    for red in ("sum", "mean", "max"):
+        full, fab = oracle.aggregate(ei, n, x, red, w=w)
+        part, pab = oracle.aggregate_rows(csr, n, x, red, rows, w=w)
+        np.testing.assert_array_equal(part, full[rows])
+        np.testing.assert_allclose(pab, fab[rows], rtol=1e-15)
+    a_s, a_d = rng.standard_normal(8), rng.standard_normal(8)
+    full, alpha, _ = oracle.edge_softmax(ei, n, x, 2, 4, a_s, a_d, 0.2)
+    part, alpha_r, _ = oracle.edge_softmax_rows(csr, n, x, 2, 4, a_s, a_d, 0.2, rows)
+    np.testing.assert_allclose(part, full[rows], rtol=1e-13, atol=1e-14)
+    rowptr, _, perm, _ = csr
+    want = np.concatenate([alpha[perm[rowptr[r]:rowptr[r + 1]]] for r in rows])
+    np.testing.assert_allclose(alpha_r, want, rtol=1e-13)
+
+
+# ---------------------------------------------------------------------------
+# BatchGraph: the paper's reindexing example and batched == per-graph
+# ---------------------------------------------------------------------------
+def test_batch_reindex_example():
+    g = _golden("batch_reindex.json")
+    sizes = g["graph_sizes"]
+    parts = [np.zeros((2, 0), np.int64) for _ in sizes]
+    _, batch, offsets = gg.batch_graphs(parts, sizes)
+    assert list(offsets) == g["offsets"]
+    for item in g["one_based"]:          # the paper counts from 1
+        assert item["node"] + offsets[item["graph"] - 1] == item["index"]
+    for item in g["zero_based"]:
+        assert item["node"] + offsets[item["graph"]] == item["index"]
+    assert list(batch) == [0, 0, 0, 0, 1, 1, 2, 2, 2]
+
+
+def pin_batched_equals_per_graph(o):
+    """Applying the aggregation to a BatchGraph equals applying it per graph
+    and concatenating (Section 2.1.1); pooling equals per-graph full reductions."""
+    rng = np.random.default_rng(9)
+    sizes = [int(s) for s in rng.integers(5, 30, size=12)] + [1]
+    graphs = [gg.with_self_loops(gg.symmetrise(gg.er_pairs(s, min(2 * s, s * (s - 1) // 2), rng)), s)
+              for s in sizes]
+    ei, batch, offsets = gg.batch_graphs(graphs, sizes)
+    n = sum(sizes)
+    x = rng.standard_normal((n, 6)).astype(np.float32)
+    full_gcn, _ = o.gcn_aggregate(ei, n, x)
+    full_max, _ = o.aggregate(ei, n, x, "max")
+    for g, (s, off) in enumerate(zip(sizes, offsets)):
+        xs = x[off:off + s]
+        part, _ = o.gcn_aggregate(graphs[g], s, xs)
+        np.testing.assert_array_equal(part, full_gcn[off:off + s])
+        part, _ = o.aggregate(graphs[g], s, xs, "max")
+        np.testing.assert_array_equal(part, full_max[off:off + s])
+    g_n = len(sizes)
+    for red, fn in (("sum", np.sum), ("mean", np.mean), ("max", np.max)):
+        pooled, _ = o.segment_pool(full_gcn, batch, g_n, red)
+        for g, (s, off) in enumerate(zip(sizes, offsets)):
+            np.testing.assert_allclose(pooled[g], fn(full_gcn[off:off + s], axis=0),
+                                       rtol=1e-13, atol=1e-14)
+
+
+def test_batched_equals_per_graph():
+    pin_batched_equals_per_graph(oracle.default)
+
+
+def pin_pool_counts(o):
+    batch = np.array([0, 0, 0, 2, 2, 4, 4, 4, 4], dtype=np.int64)
+    ones = np.ones((9, 2), np.float32)
+    out, _ = o.segment_pool(ones, batch, 6, "sum")
+    np.testing.assert_array_equal(out[:, 0], [3, 0, 2, 0, 4, 0])
+    # x[v] = [2v - 10, 2v - 9]
+    x = np.arange(18, dtype=np.float32).reshape(9, 2) - 10
+    out, _ = o.segment_pool(x, batch, 6, "max")
+    np.testing.assert_array_equal(out[:, 1], [-5, 0, -1, 0, 7, 0])
+    out, _ = o.segment_pool(x, batch, 6, "mean")
+    np.testing.assert_array_equal(out[:, 0], [-8, 0, -3, 0, 3, 0])
+
+
+def test_pool_counts_and_empty_graphs():
+    pin_pool_counts(oracle.default)
+
+
+def test_pool_rejects_unsorted_and_out_of_range():
+    x = np.ones((3, 1), np.float32)
+    with pytest.raises(oracle.OracleError) as exc:
+        oracle.segment_pool(x, np.array([0, 1, 0]), 2, "sum")
+    assert exc.value.code == -6
+    with pytest.raises(oracle.OracleError) as exc:
+        oracle.segment_pool(x, np.array([0, 1, 2]), 2, "sum")
+    assert exc.value.code == -5
+
+
+def test_bf16_widening_is_exact():
+    x = np.random.default_rng(0).standard_normal((10, 8)).astype(np.float32)
+    bits = gg.bf16_bits_rne(x)
+    wide = oracle.widen(bits)
+    np.testing.assert_array_equal(wide, gg.bf16_bits_to_f32(bits).astype(np.float64))
+    # RNE: at most half an ulp of bf16 (2^-8 relative) from the fp32 value
+    assert np.all(np.abs(wide - x) <= np.abs(x) * 2.0 ** -8)
+
+
+# ---------------------------------------------------------------------------
+# Planted mistakes: each one must trip at least one pin
+# ---------------------------------------------------------------------------
+PLANTS = {
+    "UNSTABLE_CSR": [pin_csr_is_stable_grouping],
+    "DROP_SELF_LOOP_DEGREE": [pin_gcn_p4, pin_gcn_sqrt_degree_eigenvector],
+    "OUT_DEGREE": [pin_gcn_directed],
+    "SWAP_DIRECTION": [pin_gcn_directed, pin_ones_give_in_degree],
+    "MAX_FROM_ZERO": [pin_max_brute_force],
+    "MEAN_PLUS_ONE": [pin_ones_give_in_degree, pin_softmax_normalised_and_mean_limit],
+    "NO_LEAKY": [pin_star_softmax],
+    "POOL_SKIP_LAST": [pin_pool_counts],
+}
+
+
+@pytest.mark.parametrize("plant", sorted(PLANTS))
+def test_planted_mistakes_are_caught(plant):
+    bad = oracle.planted(plant)
+    for pin in PLANTS[plant]:
+        with pytest.raises((AssertionError, oracle.OracleError)):
+            pin(bad)
