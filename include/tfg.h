@@ -1,0 +1,212 @@
+/*
+ * tfg.h -- C ABI of the GB300 (sm_103a) graph message-aggregation library.
+ *
+ * The library implements the data-parallel core of the graph map-reduce
+ * framework of tf_geometric (arXiv:2101.11552): gathering source-node
+ * features along the edges of a COO edge list, weighting them, and reducing
+ * them per target node; plus the per-graph segment reduction used for graph
+ * pooling over a BatchGraph.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - edge_index is the COO adjacency of Section 2.1.1 ("Graph Data
+ *    Structure"): int64 [2, E] row-major, row 0 = source node of each edge,
+ *    row 1 = target node.  An entry A_ij > 0 is an edge i -> j; messages flow
+ *    from source to target and are reduced at the target (Fig. 1).
+ *  - The "reduce key" of the map-reduce framework (Section 2.1.2, Fig. 5b) is
+ *    the target node.  tfg_build_csr groups the edges by that key once; every
+ *    aggregation then reads the grouped form (rowptr, col).
+ *  - Node features are dense row-major [N, F]; fp32, or bf16 storage where a
+ *    dtype argument allows it.  Every reduction accumulates in fp32.
+ *  - Pointers marked (device) are device memory owned by the caller; the
+ *    library never allocates, frees or keeps them.  Workspace buffers are
+ *    caller-provided device memory of at least the queried size.
+ *  - Every call is stateless (the functional style of Section 2.1.5): all
+ *    parameters, including attention vectors, are passed per call.  The
+ *    graph-level cache of Section 3 is the caller keeping the outputs of
+ *    tfg_build_csr / tfg_gcn_norm and passing them back.
+ *  - Calls enqueue work on `stream` (NULL = the legacy default stream) and
+ *    return immediately; results are ready once the stream reaches them.
+ *  - Return value: TFG_OK (0) or a negative tfg_status.  Host-side checks
+ *    (null pointers, sizes, workspace) fail before anything is enqueued;
+ *    tfg_last_error() then describes the failure (thread-local).
+ *  - Checks that need the data (edge ids outside [0, N), an unsorted batch
+ *    vector) run on the device: the call first sets *status to 0 and a kernel
+ *    that finds a bad value writes the error code there.  Out-of-range
+ *    values are clamped, so no kernel reads or writes out of bounds, but the
+ *    outputs of a call whose status is non-zero are unspecified.
+ *  - Empty reductions (a node without incoming edges, a graph without
+ *    nodes) give 0 for every reducer.
+ *  - Results are deterministic: the same inputs give bit-identical outputs.
+ */
+#ifndef TFG_H
+#define TFG_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* cudaStream_t without pulling in the CUDA headers. */
+typedef struct CUstream_st *tfg_stream_t;
+
+typedef enum {
+    TFG_OK = 0,
+    TFG_ERR_INVALID_ARG = -1, /* null pointer, negative/zero size, bad enum    */
+    TFG_ERR_TOO_LARGE = -2,   /* N or E >= 2^31 (CSR indices are int32)       */
+    TFG_ERR_WORKSPACE = -3,   /* workspace missing or smaller than required   */
+    TFG_ERR_CUDA = -4,        /* a CUDA runtime call or launch failed         */
+    TFG_ERR_INDEX_RANGE = -5, /* (status word) an index outside its range     */
+    TFG_ERR_UNSORTED = -6,    /* (status word) batch vector not non-decreasing */
+    TFG_ERR_TIMEOUT = -7      /* reserved: a bounded device wait gave up      */
+} tfg_status;
+
+typedef enum { TFG_F32 = 0, TFG_BF16 = 1 } tfg_dtype;
+typedef enum { TFG_SUM = 0, TFG_MEAN = 1, TFG_MAX = 2 } tfg_reduce;
+
+/* Library version (major * 10000 + minor * 100 + patch). */
+int tfg_version(void);
+
+/* Description of the last host-side failure on this thread ("" if none). */
+const char *tfg_last_error(void);
+
+/* ------------------------------------------------------------------------
+ * Grouping by the reduce key: COO -> CSR by target.
+ * Section 2.1.2 / Fig. 5b: a reducer gathers the elements that share a key
+ * (here the target node) into one group.
+ *
+ *   edge_index (device) int64 [2, num_edges]: sources then targets.
+ *   rowptr     (device) int32 [num_nodes + 1]: edges into node t are
+ *                       positions rowptr[t] .. rowptr[t+1]-1.
+ *   col        (device) int32 [num_edges]: source node of each position.
+ *   perm       (device) int32 [num_edges]: original edge id of each position.
+ *   in_degree  (device) int32 [num_nodes]: number of edges into each node.
+ *   workspace  (device) >= tfg_build_csr_workspace_size() bytes, 256-byte
+ *                       aligned; contents are scratch.
+ *   status     (device) int32 [1]: 0, or TFG_ERR_INDEX_RANGE when an edge id
+ *                       lies outside [0, num_nodes).
+ * The grouping is stable: inside a row, edges keep their original order, so
+ * (rowptr, col, perm) is unique.  num_edges may be 0; num_nodes >= 1 when
+ * num_edges > 0.
+ * ---------------------------------------------------------------------- */
+int tfg_build_csr_workspace_size(int64_t num_nodes, int64_t num_edges, size_t *bytes);
+int tfg_build_csr(const int64_t *edge_index, int64_t num_edges, int64_t num_nodes,
+                  int32_t *rowptr, int32_t *col, int32_t *perm, int32_t *in_degree,
+                  void *workspace, size_t workspace_bytes, int32_t *status,
+                  tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * GCN symmetric normalisation of A + I (the propagation rule of the GCN
+ * model that Section 2.2 lists and Table 1 evaluates), computed once per
+ * graph and cached by the caller (graph-level caching, Section 3).
+ *
+ *   deg[t]   = sum of the weights of the edges into t, + self_loop_fill
+ *              when add_self_loops is non-zero (one implicit self-loop per
+ *              node, added even when the edge list already has one)
+ *   dinv[t]  = deg[t]^-1/2, or 0 when deg[t] == 0
+ *   w_csr[k] = w_e * dinv[col[k]] * dinv[t] for position k of row t, where
+ *              e = perm[k] and w_e = edge_weight[e] (1 when edge_weight is NULL)
+ *
+ *   rowptr, col, perm (device): the output of tfg_build_csr.
+ *   edge_weight (device) fp32 [num_edges] in ORIGINAL edge order, or NULL.
+ *   dinv (device) fp32 [num_nodes], written.
+ *   w_csr (device) fp32 [num_edges] in CSR order, written; may be NULL when
+ *              only dinv is wanted (tfg_gcn_aggregate_sum can form the
+ *              weights on the fly for an unweighted graph).
+ * The implicit self-loop weight self_loop_fill * dinv[t]^2 is not part of
+ * w_csr; tfg_gcn_aggregate_sum adds it.
+ * ---------------------------------------------------------------------- */
+int tfg_gcn_norm(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
+                 const float *edge_weight, int64_t num_nodes, int64_t num_edges,
+                 int add_self_loops, float self_loop_fill, float *dinv, float *w_csr,
+                 tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Message aggregation (Fig. 1) with the reducer of Fig. 5b:
+ *   out[t, :] = REDUCE over positions k of row t of  w_k * x[col[k], :]
+ *   sum; mean = sum / (rowptr[t+1] - rowptr[t]); max.
+ *
+ *   rowptr, col (device): CSR by target (tfg_build_csr).
+ *   w_csr (device) fp32 [num_edges] in CSR order, or NULL for w = 1.
+ *   x (device) [num_nodes, num_features] row-major, x_dtype TFG_F32 or
+ *        TFG_BF16.  16-byte alignment of x and a feature count that is a
+ *        multiple of 4 (fp32) or 8 (bf16) select the vectorised kernels;
+ *        any other layout takes a scalar path with the same results.
+ *   out (device) fp32 [num_nodes, num_features], written (not accumulated).
+ * The sum and mean accumulate in fp32 in a fixed order (deterministic);
+ * max is exact (the maximum of fp32 products w_k * x).
+ * ---------------------------------------------------------------------- */
+int tfg_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float *w_csr,
+                      const void *x, int x_dtype, int64_t num_nodes, int64_t num_features,
+                      float *out, tfg_stream_t stream);
+int tfg_aggregate_mean(const int32_t *rowptr, const int32_t *col, const float *w_csr,
+                       const void *x, int x_dtype, int64_t num_nodes, int64_t num_features,
+                       float *out, tfg_stream_t stream);
+int tfg_aggregate_max(const int32_t *rowptr, const int32_t *col, const float *w_csr,
+                      const void *x, int x_dtype, int64_t num_nodes, int64_t num_features,
+                      float *out, tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * GCN propagation  out = D^-1/2 (A + I) D^-1/2 x  in one pass (GCN, Section
+ * 2.2 / Table 1; the weights are those of tfg_gcn_norm):
+ *   out[t, :] = sum over positions k of row t of  w_k * x[col[k], :]
+ *               + (add_self_loops ? self_loop_fill * dinv[t]^2 * x[t, :] : 0)
+ * with w_k = w_csr[k] when w_csr is given, else dinv[col[k]] * dinv[t]
+ * (an unweighted graph; no per-edge weight array is read).
+ *   dinv (device) fp32 [num_nodes] from tfg_gcn_norm (same add_self_loops
+ *        and self_loop_fill).
+ *   Other arguments as for tfg_aggregate_sum.
+ * ---------------------------------------------------------------------- */
+int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float *dinv,
+                          const float *w_csr, const void *x, int x_dtype, int64_t num_nodes,
+                          int64_t num_features, int add_self_loops, float self_loop_fill,
+                          float *out, tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Edge-softmax (GAT) aggregation -- the map-reduce workflow of Fig. 5a
+ * (Section 2.1.2) fused with the weighted sum it feeds:
+ *   s_src[n, h] = <x[n, h, :], a_src[h, :]>,  s_dst[n, h] likewise with a_dst
+ *   map:    l[k, h] = LeakyReLU(s_src[col[k], h] + s_dst[t, h]; negative_slope)
+ *   reduce: alpha[k, h] = exp(l[k, h]) / sum over row t of exp(l[., h])
+ *           (evaluated with the row maximum subtracted; same value)
+ *   out[t, h, :] = sum over row t of alpha[k, h] * x[col[k], h, :]
+ *
+ *   x (device) fp32 [num_nodes, heads * channels], head h in columns
+ *          h*channels .. h*channels+channels-1.
+ *   a_src, a_dst (device) fp32 [heads * channels], same layout.
+ *   out (device) fp32 [num_nodes, heads * channels], written.
+ *   alpha (device) fp32 [num_edges, heads] in CSR order, or NULL.
+ *   workspace (device) >= tfg_edge_softmax_workspace_size() bytes (node
+ *          scores); contents are scratch.
+ * Rows without incoming edges give 0.
+ * ---------------------------------------------------------------------- */
+int tfg_edge_softmax_workspace_size(int64_t num_nodes, int heads, size_t *bytes);
+int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const float *x,
+                               int64_t num_nodes, int64_t num_edges, int heads, int channels,
+                               const float *a_src, const float *a_dst, float negative_slope,
+                               float *out, float *alpha, void *workspace,
+                               size_t workspace_bytes, tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Graph pooling keyed by node_graph_index (Section 2.1.1 BatchGraph; Fig. 2a
+ * common graph pooling):
+ *   out[g, :] = REDUCE over nodes v with batch[v] == g of x[v, :]
+ *   sum; mean = sum / node count; max.
+ *
+ *   x (device) [num_nodes, num_features], x_dtype TFG_F32 or TFG_BF16.
+ *   batch (device) int64 [num_nodes], non-decreasing, values in
+ *          [0, num_graphs) -- the order a BatchGraph's reindexing produces.
+ *   out (device) fp32 [num_graphs, num_features], written.
+ *   status (device) int32 [1]: 0, TFG_ERR_UNSORTED or TFG_ERR_INDEX_RANGE.
+ * ---------------------------------------------------------------------- */
+int tfg_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t num_nodes,
+                     int64_t num_graphs, int64_t num_features, int reduce, float *out,
+                     int32_t *status, tfg_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TFG_H */

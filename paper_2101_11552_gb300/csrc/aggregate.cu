@@ -1,0 +1,272 @@
+// Fused gather * weight * reduce over a CSR grouped by target: the message
+// aggregation of tf_geometric (Fig. 1) with the reducer of Fig. 5b, which the
+// paper implements as tf.math.unsorted_segment_* over the edge list
+// (Section 2.1.2).  Grouping by target first turns the scatter-reduce into
+// owner-computes row reductions: no atomics, a fixed summation order, and
+// bit-identical results from run to run.
+//
+// Work layout
+//  * A CTA (8 warps) owns kRowsPerCta consecutive target rows.  Its warps take
+//    rows one at a time from a shared counter.  A row is split among
+//    G = 32 / LPR lane groups: each group of LPR lanes covers LPR * VEC
+//    features (16-byte loads when the layout allows) and takes every G-th
+//    edge of the row; the groups' partials are then combined by a butterfly.
+//  * Rows longer than kHeavyDeg (power-law hubs) are set aside and done after
+//    the light rows by the whole CTA: each warp takes one contiguous slice of
+//    the row, and the eight warp partials are combined in warp order through
+//    shared memory.  No global scratch and no inter-CTA waiting.
+//  * Column ids (and weights) of 32 edges are loaded by the 32 lanes at once
+//    and broadcast with shuffles; kUnroll gathers are kept in flight per lane.
+//  * GCN mode without w_csr forms the weight on the fly:  out[t] = dinv[t] *
+//    (sum_k dinv[col[k]] * x[col[k]] + fill * dinv[t] * x[t]), so no per-edge
+//    weight array is read.  With w_csr it adds fill * dinv[t]^2 * x[t] to the
+//    weighted sum.
+#include <math_constants.h>
+
+#include "common.cuh"
+
+namespace tfg {
+namespace {
+
+constexpr int kAggWarps = 8;
+constexpr int kAggThreads = kAggWarps * 32;
+constexpr int kRowsPerCta = 64;
+constexpr int kHeavyDeg = 2048;
+constexpr int kUnroll = 4;
+
+struct AggArgs {
+    const int32_t *rowptr;
+    const int32_t *col;
+    const float *w;     // CSR-order weights or null (sum / mean / max)
+    const float *dinv;  // GCN mode
+    const void *x;
+    float *out;
+    int64_t n;
+    int64_t f;
+    int mean;
+    int add_self;
+    float fill;
+};
+
+enum Kind { kSumLike = 0, kMax = 1, kGcn = 2 };
+
+template <typename XT, int VEC, int LPR, int KIND>
+struct Agg {
+    static constexpr int G = 32 / LPR;
+    static constexpr bool kIsMax = KIND == kMax;
+
+    static __device__ __forceinline__ float identity() { return kIsMax ? -CUDART_INF_F : 0.f; }
+
+    static __device__ __forceinline__ float combine(float a, float b) {
+        return kIsMax ? fmaxf(a, b) : a + b;
+    }
+
+    // Accumulate edges [beg, end) into acc (this lane's VEC features at f0).
+    static __device__ __forceinline__ void edges(const AggArgs &a, int64_t beg, int64_t end,
+                                                 int64_t f0, bool fok, float (&acc)[VEC],
+                                                 int lane) {
+        const XT *x = static_cast<const XT *>(a.x);
+        const int g = lane / LPR;
+        const bool weighted = KIND == kGcn || a.w != nullptr;
+        for (int64_t base = beg; base < end; base += 32) {
+            const int cnt = static_cast<int>(min64(32, end - base));
+            int c = 0;
+            float ww = 1.f;
+            if (lane < cnt) {
+                c = __ldg(a.col + base + lane);
+                if (a.w) ww = __ldg(a.w + base + lane);
+                else if (KIND == kGcn) ww = __ldg(a.dinv + c);
+            }
+            for (int j = 0; j < cnt; j += G * kUnroll) {
+                int src[kUnroll];
+                float wt[kUnroll];
+                bool ok[kUnroll];
+#pragma unroll
+                for (int u = 0; u < kUnroll; ++u) {
+                    const int k = j + u * G + g;
+                    src[u] = __shfl_sync(kFull, c, k & 31);
+                    wt[u] = weighted ? __shfl_sync(kFull, ww, k & 31) : 1.f;
+                    ok[u] = fok && (k < cnt);
+                }
+                float v[kUnroll][VEC];
+#pragma unroll
+                for (int u = 0; u < kUnroll; ++u)
+                    if (ok[u]) VecLoad<XT, VEC>::load(x + static_cast<int64_t>(src[u]) * a.f + f0, v[u]);
+#pragma unroll
+                for (int u = 0; u < kUnroll; ++u) {
+                    if (!ok[u]) continue;
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q) {
+                        if (kIsMax) acc[q] = fmaxf(acc[q], wt[u] * v[u][q]);
+                        else acc[q] = fmaf(wt[u], v[u][q], acc[q]);
+                    }
+                }
+            }
+        }
+    }
+
+    static __device__ __forceinline__ void reduce_groups(float (&acc)[VEC]) {
+#pragma unroll
+        for (int s = LPR; s < 32; s <<= 1)
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] = combine(acc[q], __shfl_xor_sync(kFull, acc[q], s));
+    }
+
+    // Final value of one feature of row t from its reduced accumulator.
+    static __device__ __forceinline__ float finish(const AggArgs &a, int64_t t, int64_t deg,
+                                                   float acc, float xt, float dt) {
+        if (KIND == kGcn) {
+            if (a.w) return a.add_self ? acc + (a.fill * dt) * dt * xt : acc;
+            return a.add_self ? dt * (acc + a.fill * dt * xt) : dt * acc;
+        }
+        if (deg == 0) return 0.f;
+        if (a.mean) return acc / static_cast<float>(deg);
+        return acc;
+    }
+
+    static __device__ void warp_row(const AggArgs &a, int64_t t, int lane) {
+        const int64_t beg = a.rowptr[t], end = a.rowptr[t + 1];
+        const int sub = lane % LPR;
+        const float dt = KIND == kGcn ? __ldg(a.dinv + t) : 1.f;
+        for (int64_t ft = 0; ft < a.f; ft += LPR * VEC) {
+            const int64_t f0 = ft + sub * VEC;
+            const bool fok = f0 < a.f;
+            float acc[VEC];
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] = identity();
+            edges(a, beg, end, f0, fok, acc, lane);
+            reduce_groups(acc);
+            if (lane < LPR && fok) {
+                float xt[VEC];
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) xt[q] = 0.f;
+                if (KIND == kGcn && a.add_self)
+                    VecLoad<XT, VEC>::load(static_cast<const XT *>(a.x) + t * a.f + f0, xt);
+                float *o = a.out + t * a.f + f0;
+                float r[VEC];
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) r[q] = finish(a, t, end - beg, acc[q], xt[q], dt);
+                if constexpr (VEC % 4 == 0) {
+#pragma unroll
+                    for (int q = 0; q < VEC; q += 4)
+                        *reinterpret_cast<float4 *>(o + q) = make_float4(r[q], r[q + 1], r[q + 2], r[q + 3]);
+                } else {
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q) o[q] = r[q];
+                }
+            }
+        }
+    }
+
+    // A hub row done by all warps of the CTA; partials combined in warp order.
+    static __device__ void cta_row(const AggArgs &a, int64_t t, float *s_part) {
+        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, sub = lane % LPR;
+        const int64_t beg = a.rowptr[t], end = a.rowptr[t + 1], deg = end - beg;
+        const int64_t per = ((deg + kAggWarps - 1) / kAggWarps + 31) / 32 * 32;
+        const int64_t wb = min(end, beg + warp * per), we = min(end, wb + per);
+        const float dt = KIND == kGcn ? __ldg(a.dinv + t) : 1.f;
+        constexpr int kSlots = LPR * VEC;
+        for (int64_t ft = 0; ft < a.f; ft += kSlots) {
+            const int64_t f0 = ft + sub * VEC;
+            const bool fok = f0 < a.f;
+            float acc[VEC];
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] = identity();
+            edges(a, wb, we, f0, fok, acc, lane);
+            reduce_groups(acc);
+            if (lane < LPR) {
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) s_part[warp * kSlots + sub * VEC + q] = acc[q];
+            }
+            __syncthreads();
+            for (int i = threadIdx.x; i < kSlots; i += kAggThreads) {
+                const int64_t fi = ft + i;
+                if (fi < a.f) {
+                    float r = s_part[i];
+                    for (int w = 1; w < kAggWarps; ++w) r = combine(r, s_part[w * kSlots + i]);
+                    float xt = 0.f;
+                    if (KIND == kGcn && a.add_self) {
+                        float one[1];
+                        VecLoad<XT, 1>::load(static_cast<const XT *>(a.x) + t * a.f + fi, one);
+                        xt = one[0];
+                    }
+                    a.out[t * a.f + fi] = finish(a, t, deg, r, xt, dt);
+                }
+            }
+            __syncthreads();
+        }
+    }
+};
+
+template <typename XT, int VEC, int LPR, int KIND>
+__global__ void __launch_bounds__(kAggThreads) aggregate_kernel(AggArgs a) {
+    using A = Agg<XT, VEC, LPR, KIND>;
+    __shared__ int s_next, s_nheavy;
+    __shared__ int s_heavy[kRowsPerCta];
+    __shared__ float s_part[kAggWarps * LPR * VEC];
+    const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRowsPerCta;
+    const int nrows = static_cast<int>(min64(kRowsPerCta, a.n - r0));
+    if (threadIdx.x == 0) {
+        s_next = 0;
+        s_nheavy = 0;
+    }
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    for (;;) {
+        int i = 0;
+        if (lane == 0) i = atomicAdd(&s_next, 1);
+        i = __shfl_sync(kFull, i, 0);
+        if (i >= nrows) break;
+        const int64_t t = r0 + i;
+        if (a.rowptr[t + 1] - a.rowptr[t] > kHeavyDeg) {
+            if (lane == 0) s_heavy[atomicAdd(&s_nheavy, 1)] = i;
+            continue;
+        }
+        A::warp_row(a, t, lane);
+    }
+    __syncthreads();
+    const int nh = s_nheavy;
+    for (int h = 0; h < nh; ++h) A::cta_row(a, r0 + s_heavy[h], s_part);
+}
+
+template <typename XT, int VEC, int KIND>
+cudaError_t launch_lpr(const AggArgs &a, int lpr, cudaStream_t s) {
+    const int grid = ceil_div(a.n, kRowsPerCta);
+    switch (lpr) {
+        case 32: aggregate_kernel<XT, VEC, 32, KIND><<<grid, kAggThreads, 0, s>>>(a); break;
+        case 16: aggregate_kernel<XT, VEC, 16, KIND><<<grid, kAggThreads, 0, s>>>(a); break;
+        default: aggregate_kernel<XT, VEC, 8, KIND><<<grid, kAggThreads, 0, s>>>(a); break;
+    }
+    return cudaGetLastError();
+}
+
+template <typename XT, int VEC>
+cudaError_t launch_kind(const AggArgs &a, int kind, int lpr, cudaStream_t s) {
+    switch (kind) {
+        case kMax: return launch_lpr<XT, VEC, kMax>(a, lpr, s);
+        case kGcn: return launch_lpr<XT, VEC, kGcn>(a, lpr, s);
+        default: return launch_lpr<XT, VEC, kSumLike>(a, lpr, s);
+    }
+}
+
+int lanes_per_row(int64_t chunks) { return chunks >= 32 ? 32 : (chunks > 8 ? 16 : 8); }
+
+}  // namespace
+
+cudaError_t launch_aggregate(int mode, const int32_t *rowptr, const int32_t *col, const float *w,
+                             const float *dinv, const void *x, int x_dtype, int64_t n, int64_t f,
+                             int add_self, float fill, float *out, cudaStream_t s) {
+    if (n <= 0) return cudaSuccess;
+    AggArgs a{rowptr, col, w, dinv, x, out, n, f, mode == 1, add_self, fill};
+    const int kind = mode == 2 ? kMax : (mode == 3 ? kGcn : kSumLike);
+    const bool aligned = (reinterpret_cast<uintptr_t>(x) % 16 == 0) &&
+                         (reinterpret_cast<uintptr_t>(out) % 16 == 0);
+    if (x_dtype == TFG_BF16) {
+        if (aligned && f % 8 == 0) return launch_kind<uint16_t, 8>(a, kind, lanes_per_row(f / 8), s);
+        return launch_kind<uint16_t, 1>(a, kind, lanes_per_row(f), s);
+    }
+    if (aligned && f % 4 == 0) return launch_kind<float, 4>(a, kind, lanes_per_row(f / 4), s);
+    return launch_kind<float, 1>(a, kind, lanes_per_row(f), s);
+}
+
+}  // namespace tfg

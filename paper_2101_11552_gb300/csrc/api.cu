@@ -1,0 +1,229 @@
+// C ABI of libtfg: host-side argument checks, then the launchers.
+// Every entry point validates before it touches the GPU, so a rejected call
+// enqueues nothing.  See include/tfg.h for the contract of each call.
+#include <cstdarg>
+#include <cstdio>
+
+#include "common.cuh"
+
+namespace {
+
+thread_local char g_err[512];
+
+int fail(int code, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int ok() {
+    g_err[0] = '\0';
+    return TFG_OK;
+}
+
+int cuda_result(cudaError_t e, const char *where) {
+    if (e != cudaSuccess) return fail(TFG_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+    return ok();
+}
+
+constexpr int64_t kIndexLimit = int64_t(1) << 31;  // CSR ids are int32
+
+int check_counts(const char *fn, int64_t n, int64_t e) {
+    if (n < 0 || e < 0) return fail(TFG_ERR_INVALID_ARG, "%s: negative size (N=%lld, E=%lld)", fn,
+                                    (long long)n, (long long)e);
+    if (n >= kIndexLimit || e >= kIndexLimit)
+        return fail(TFG_ERR_TOO_LARGE, "%s: N and E must be < 2^31 (N=%lld, E=%lld)", fn,
+                    (long long)n, (long long)e);
+    if (e > 0 && n == 0) return fail(TFG_ERR_INVALID_ARG, "%s: edges given but N == 0", fn);
+    return TFG_OK;
+}
+
+int check_features(const char *fn, int64_t n, int64_t f) {
+    if (f < 1 || f > (int64_t(1) << 24))
+        return fail(TFG_ERR_INVALID_ARG, "%s: feature count must be in [1, 2^24] (F=%lld)", fn,
+                    (long long)f);
+    if (n * f >= (int64_t(1) << 46))
+        return fail(TFG_ERR_TOO_LARGE, "%s: N*F too large", fn);
+    return TFG_OK;
+}
+
+int check_dtype(const char *fn, int dtype) {
+    if (dtype != TFG_F32 && dtype != TFG_BF16)
+        return fail(TFG_ERR_INVALID_ARG, "%s: unknown dtype %d", fn, dtype);
+    return TFG_OK;
+}
+
+#define TFG_TRY(expr)                    \
+    do {                                 \
+        int rc_ = (expr);                \
+        if (rc_ != TFG_OK) return rc_;   \
+    } while (0)
+
+#define TFG_NEED(ptr, cond, fn, name)                                                  \
+    do {                                                                               \
+        if ((cond) && (ptr) == nullptr)                                                \
+            return fail(TFG_ERR_INVALID_ARG, "%s: %s must not be NULL", fn, name);    \
+    } while (0)
+
+int aggregate_common(const char *fn, int mode, const int32_t *rowptr, const int32_t *col,
+                     const float *w, const float *dinv, const void *x, int dtype, int64_t n,
+                     int64_t f, int add_self, float fill, float *out, tfg_stream_t stream) {
+    TFG_TRY(check_counts(fn, n, 0));
+    TFG_TRY(check_features(fn, n, f));
+    TFG_TRY(check_dtype(fn, dtype));
+    TFG_NEED(rowptr, true, fn, "rowptr");
+    TFG_NEED(col, n > 0, fn, "col");
+    TFG_NEED(x, n > 0, fn, "x");
+    TFG_NEED(out, n > 0, fn, "out");
+    TFG_NEED(dinv, mode == 3 && n > 0, fn, "dinv");
+    return cuda_result(tfg::launch_aggregate(mode, rowptr, col, w, dinv, x, dtype, n, f, add_self,
+                                             fill, out, reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+}  // namespace
+
+extern "C" {
+
+int tfg_version(void) { return 100; }
+
+const char *tfg_last_error(void) { return g_err; }
+
+int tfg_build_csr_workspace_size(int64_t num_nodes, int64_t num_edges, size_t *bytes) {
+    const char *fn = "tfg_build_csr_workspace_size";
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    TFG_NEED(bytes, true, fn, "bytes");
+    *bytes = tfg::csr_workspace_bytes(num_nodes, num_edges);
+    return ok();
+}
+
+int tfg_build_csr(const int64_t *edge_index, int64_t num_edges, int64_t num_nodes,
+                  int32_t *rowptr, int32_t *col, int32_t *perm, int32_t *in_degree,
+                  void *workspace, size_t workspace_bytes, int32_t *status,
+                  tfg_stream_t stream) {
+    const char *fn = "tfg_build_csr";
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    TFG_NEED(edge_index, num_edges > 0, fn, "edge_index");
+    TFG_NEED(rowptr, true, fn, "rowptr");
+    TFG_NEED(col, num_edges > 0, fn, "col");
+    TFG_NEED(perm, num_edges > 0, fn, "perm");
+    TFG_NEED(in_degree, num_nodes > 0, fn, "in_degree");
+    TFG_NEED(status, true, fn, "status");
+    const size_t need = tfg::csr_workspace_bytes(num_nodes, num_edges);
+    if (num_edges > 0) {
+        if (workspace == nullptr || workspace_bytes < need)
+            return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
+                        workspace ? workspace_bytes : size_t(0));
+        if (reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
+            return fail(TFG_ERR_INVALID_ARG, "%s: workspace must be 256-byte aligned", fn);
+    }
+    return cuda_result(tfg::launch_build_csr(edge_index, num_edges, num_nodes, rowptr, col, perm,
+                                             in_degree, workspace, status,
+                                             reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+int tfg_gcn_norm(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
+                 const float *edge_weight, int64_t num_nodes, int64_t num_edges,
+                 int add_self_loops, float self_loop_fill, float *dinv, float *w_csr,
+                 tfg_stream_t stream) {
+    const char *fn = "tfg_gcn_norm";
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    TFG_NEED(rowptr, true, fn, "rowptr");
+    TFG_NEED(dinv, num_nodes > 0, fn, "dinv");
+    TFG_NEED(col, w_csr != nullptr && num_edges > 0, fn, "col");
+    TFG_NEED(perm, (w_csr != nullptr || edge_weight != nullptr) && num_edges > 0, fn, "perm");
+    return cuda_result(tfg::launch_gcn_norm(rowptr, col, perm, edge_weight, num_nodes,
+                                            add_self_loops, self_loop_fill, dinv, w_csr,
+                                            reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+int tfg_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float *w_csr,
+                      const void *x, int x_dtype, int64_t num_nodes, int64_t num_features,
+                      float *out, tfg_stream_t stream) {
+    return aggregate_common("tfg_aggregate_sum", 0, rowptr, col, w_csr, nullptr, x, x_dtype,
+                            num_nodes, num_features, 0, 0.f, out, stream);
+}
+
+int tfg_aggregate_mean(const int32_t *rowptr, const int32_t *col, const float *w_csr,
+                       const void *x, int x_dtype, int64_t num_nodes, int64_t num_features,
+                       float *out, tfg_stream_t stream) {
+    return aggregate_common("tfg_aggregate_mean", 1, rowptr, col, w_csr, nullptr, x, x_dtype,
+                            num_nodes, num_features, 0, 0.f, out, stream);
+}
+
+int tfg_aggregate_max(const int32_t *rowptr, const int32_t *col, const float *w_csr,
+                      const void *x, int x_dtype, int64_t num_nodes, int64_t num_features,
+                      float *out, tfg_stream_t stream) {
+    return aggregate_common("tfg_aggregate_max", 2, rowptr, col, w_csr, nullptr, x, x_dtype,
+                            num_nodes, num_features, 0, 0.f, out, stream);
+}
+
+int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float *dinv,
+                          const float *w_csr, const void *x, int x_dtype, int64_t num_nodes,
+                          int64_t num_features, int add_self_loops, float self_loop_fill,
+                          float *out, tfg_stream_t stream) {
+    return aggregate_common("tfg_gcn_aggregate_sum", 3, rowptr, col, w_csr, dinv, x, x_dtype,
+                            num_nodes, num_features, add_self_loops, self_loop_fill, out, stream);
+}
+
+int tfg_edge_softmax_workspace_size(int64_t num_nodes, int heads, size_t *bytes) {
+    const char *fn = "tfg_edge_softmax_workspace_size";
+    TFG_TRY(check_counts(fn, num_nodes, 0));
+    if (heads < 1) return fail(TFG_ERR_INVALID_ARG, "%s: heads must be >= 1", fn);
+    TFG_NEED(bytes, true, fn, "bytes");
+    *bytes = tfg::softmax_workspace_bytes(num_nodes, heads);
+    return ok();
+}
+
+int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const float *x,
+                               int64_t num_nodes, int64_t num_edges, int heads, int channels,
+                               const float *a_src, const float *a_dst, float negative_slope,
+                               float *out, float *alpha, void *workspace,
+                               size_t workspace_bytes, tfg_stream_t stream) {
+    const char *fn = "tfg_edge_softmax_aggregate";
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    if (heads < 1 || channels < 1)
+        return fail(TFG_ERR_INVALID_ARG, "%s: heads and channels must be >= 1", fn);
+    TFG_TRY(check_features(fn, num_nodes, int64_t(heads) * channels));
+    TFG_NEED(rowptr, true, fn, "rowptr");
+    TFG_NEED(col, num_nodes > 0, fn, "col");
+    TFG_NEED(x, num_nodes > 0, fn, "x");
+    TFG_NEED(out, num_nodes > 0, fn, "out");
+    TFG_NEED(a_src, true, fn, "a_src");
+    TFG_NEED(a_dst, true, fn, "a_dst");
+    const size_t need = tfg::softmax_workspace_bytes(num_nodes, heads);
+    if (num_nodes > 0 && (workspace == nullptr || workspace_bytes < need))
+        return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
+                    workspace ? workspace_bytes : size_t(0));
+    return cuda_result(tfg::launch_edge_softmax(rowptr, col, x, num_nodes, heads, channels, a_src,
+                                                a_dst, negative_slope, out, alpha, workspace,
+                                                reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+int tfg_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t num_nodes,
+                     int64_t num_graphs, int64_t num_features, int reduce, float *out,
+                     int32_t *status, tfg_stream_t stream) {
+    const char *fn = "tfg_segment_pool";
+    if (num_nodes < 0 || num_graphs < 0)
+        return fail(TFG_ERR_INVALID_ARG, "%s: negative size", fn);
+    if (num_graphs >= kIndexLimit) return fail(TFG_ERR_TOO_LARGE, "%s: too many graphs", fn);
+    TFG_TRY(check_features(fn, num_nodes > num_graphs ? num_nodes : num_graphs, num_features));
+    TFG_TRY(check_dtype(fn, x_dtype));
+    if (reduce != TFG_SUM && reduce != TFG_MEAN && reduce != TFG_MAX)
+        return fail(TFG_ERR_INVALID_ARG, "%s: unknown reducer %d", fn, reduce);
+    TFG_NEED(x, num_nodes > 0, fn, "x");
+    TFG_NEED(batch, num_nodes > 0, fn, "batch");
+    TFG_NEED(out, num_graphs > 0, fn, "out");
+    TFG_NEED(status, true, fn, "status");
+    return cuda_result(tfg::launch_segment_pool(x, x_dtype, batch, num_nodes, num_graphs,
+                                                num_features, reduce, out, status,
+                                                reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+}  // extern "C"

@@ -1,0 +1,76 @@
+// Internal helpers shared by the kernels of libtfg (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/tfg.h"
+
+namespace tfg {
+
+constexpr unsigned kFull = 0xffffffffu;
+
+// First error wins: a kernel that finds bad data records its code once.
+__device__ __forceinline__ void set_status(int32_t *status, int32_t code) {
+    if (status) atomicCAS(status, 0, code);
+}
+
+// bf16 -> fp32 is exact: the 16 stored bits are the high half of the fp32 word.
+__device__ __forceinline__ float bf16_lo(uint32_t packed) { return __uint_as_float(packed << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t packed) { return __uint_as_float(packed & 0xffff0000u); }
+
+// VEC consecutive features of one row, widened to fp32.
+template <typename XT, int VEC> struct VecLoad;
+
+template <> struct VecLoad<float, 4> {
+    static __device__ __forceinline__ void load(const float *p, float (&v)[4]) {
+        float4 q = __ldg(reinterpret_cast<const float4 *>(p));
+        v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+    }
+};
+template <> struct VecLoad<float, 1> {
+    static __device__ __forceinline__ void load(const float *p, float (&v)[1]) { v[0] = __ldg(p); }
+};
+template <> struct VecLoad<uint16_t, 8> {
+    static __device__ __forceinline__ void load(const uint16_t *p, float (&v)[8]) {
+        uint4 q = __ldg(reinterpret_cast<const uint4 *>(p));
+        v[0] = bf16_lo(q.x); v[1] = bf16_hi(q.x);
+        v[2] = bf16_lo(q.y); v[3] = bf16_hi(q.y);
+        v[4] = bf16_lo(q.z); v[5] = bf16_hi(q.z);
+        v[6] = bf16_lo(q.w); v[7] = bf16_hi(q.w);
+    }
+};
+template <> struct VecLoad<uint16_t, 1> {
+    static __device__ __forceinline__ void load(const uint16_t *p, float (&v)[1]) {
+        v[0] = __uint_as_float(static_cast<uint32_t>(__ldg(p)) << 16);
+    }
+};
+
+__host__ __device__ constexpr int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
+__host__ __device__ constexpr int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
+
+}  // namespace tfg
+
+// Host-side launchers implemented in the kernel files; api.cu validates
+// arguments before calling them.  Each returns cudaSuccess or the launch error.
+namespace tfg {
+size_t csr_workspace_bytes(int64_t n, int64_t e);
+cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
+                             int32_t *col, int32_t *perm, int32_t *in_degree, void *ws,
+                             int32_t *status, cudaStream_t s);
+cudaError_t launch_gcn_norm(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
+                            const float *ew, int64_t n, int add_self, float fill, float *dinv,
+                            float *w_csr, cudaStream_t s);
+// mode: 0 = sum, 1 = mean, 2 = max, 3 = gcn sum
+cudaError_t launch_aggregate(int mode, const int32_t *rowptr, const int32_t *col, const float *w,
+                             const float *dinv, const void *x, int x_dtype, int64_t n, int64_t f,
+                             int add_self, float fill, float *out, cudaStream_t s);
+size_t softmax_workspace_bytes(int64_t n, int heads);
+cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const float *x,
+                                int64_t n, int heads, int channels, const float *a_src,
+                                const float *a_dst, float slope, float *out, float *alpha,
+                                void *ws, cudaStream_t s);
+cudaError_t launch_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n,
+                                int64_t g, int64_t f, int reduce, float *out, int32_t *status,
+                                cudaStream_t s);
+}  // namespace tfg

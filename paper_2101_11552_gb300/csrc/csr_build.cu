@@ -1,0 +1,335 @@
+// COO -> CSR grouped by target node: the "reduce by key" grouping of the
+// graph map-reduce framework (tf_geometric Section 2.1.2, Fig. 5b), with the
+// target node as the key.
+//
+// Method: a stable least-significant-digit radix sort of the edges by target
+// id, one pass per digit of ceil(log2 N) bits split into <= 10-bit digits.
+// Each pass is reduce-then-scan:
+//   upsweep   per-tile digit histogram  -> hist[digit][tile]
+//   scan      exclusive scan of hist (digit-major) -> first output slot of
+//             every (digit, tile) pair; digit-major order keeps the sort stable
+//   downsweep each warp ranks its elements with __match_any_sync and writes
+//             them to their slots
+// No kernel waits on another CTA, so nothing can spin.  The first pass reads
+// the int64 edge_index directly and checks every id; the last pass writes
+// col (source) and perm (original edge id) in final order, plus the sorted
+// keys from which rowptr is found by binary search.
+#include "common.cuh"
+
+namespace tfg {
+namespace {
+
+constexpr int kSortWarps = 8;
+constexpr int kSortThreads = kSortWarps * 32;
+constexpr int kItems = 32;                        // per lane
+constexpr int kTile = kSortThreads * kItems;      // 8192 edges per CTA
+constexpr int kMaxDigitBits = 10;
+constexpr int kScanThreads = 256;
+constexpr int kScanItems = 16;
+constexpr int kScanChunk = kScanThreads * kScanItems;
+
+struct SortPlan {
+    int passes;
+    int width;
+};
+
+SortPlan plan_for(int64_t n) {
+    int bits = 1;
+    while ((int64_t(1) << bits) < n) ++bits;
+    int passes = (bits + kMaxDigitBits - 1) / kMaxDigitBits;
+    int width = (bits + passes - 1) / passes;
+    return {passes, width};
+}
+
+size_t align256(size_t b) { return (b + 255) & ~size_t(255); }
+
+// An id outside [0, n) is reported and replaced by 0, so every later index
+// stays in bounds.  The upsweep and downsweep clamp identically, keeping the
+// per-tile counts consistent with the ranks.
+__device__ __forceinline__ uint32_t checked_id(int64_t v, int64_t n, int32_t *status) {
+    if (v < 0 || v >= n) {
+        if (status) set_status(status, TFG_ERR_INDEX_RANGE);
+        return 0u;
+    }
+    return static_cast<uint32_t>(v);
+}
+
+template <bool FIRST>
+__global__ void __launch_bounds__(kSortThreads)
+radix_upsweep(const int64_t *__restrict__ dst64, const uint32_t *__restrict__ key32, int64_t e,
+              int64_t n, int shift, int width, int num_tiles, int32_t *__restrict__ hist,
+              int32_t *status) {
+    extern __shared__ int32_t s_cnt[];
+    const int radix = 1 << width;
+    for (int d = threadIdx.x; d < radix; d += kSortThreads) s_cnt[d] = 0;
+    __syncthreads();
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * kTile;
+    const int64_t stop = min64(e, base + kTile);
+    for (int64_t i = base + threadIdx.x; i < stop; i += kSortThreads) {
+        uint32_t key = FIRST ? checked_id(__ldg(dst64 + i), n, status) : __ldg(key32 + i);
+        atomicAdd(&s_cnt[(key >> shift) & (radix - 1)], 1);
+    }
+    __syncthreads();
+    for (int d = threadIdx.x; d < radix; d += kSortThreads)
+        hist[static_cast<int64_t>(d) * num_tiles + blockIdx.x] = s_cnt[d];
+}
+
+template <bool FIRST>
+__global__ void __launch_bounds__(kSortThreads)
+radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ dst64,
+                const uint32_t *__restrict__ key_in, const int32_t *__restrict__ src_in,
+                const int32_t *__restrict__ eid_in, int64_t e, int64_t n, int shift, int width,
+                int num_tiles, const int32_t *__restrict__ offs, uint32_t *__restrict__ key_out,
+                int32_t *__restrict__ src_out, int32_t *__restrict__ eid_out, int32_t *status) {
+    extern __shared__ int32_t s_base[];  // [kSortWarps][radix]
+    const int radix = 1 << width;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int32_t *mine = s_base + warp * radix;
+    for (int d = lane; d < radix; d += 32) mine[d] = 0;
+    __syncwarp();
+
+    // Phase A: per-warp digit counts over the warp's contiguous sub-tile.
+    const int64_t wbase = static_cast<int64_t>(blockIdx.x) * kTile +
+                          static_cast<int64_t>(warp) * 32 * kItems;
+    uint32_t keys[kItems];
+#pragma unroll
+    for (int r = 0; r < kItems; ++r) {
+        const int64_t idx = wbase + r * 32 + lane;
+        const bool ok = idx < e;
+        uint32_t key = 0;
+        if (ok) key = FIRST ? checked_id(__ldg(dst64 + idx), n, nullptr) : __ldg(key_in + idx);
+        keys[r] = key;
+        const uint32_t dig = ok ? ((key >> shift) & (radix - 1)) : uint32_t(radix);
+        const unsigned peers = __match_any_sync(kFull, dig);
+        if (ok && lane == __ffs(peers) - 1) mine[dig] += __popc(peers);
+        __syncwarp();
+    }
+    __syncthreads();
+
+    // Phase B: warp-major exclusive prefix per digit, seeded by the scanned
+    // global slot of (digit, this tile).
+    for (int d = threadIdx.x; d < radix; d += kSortThreads) {
+        int32_t run = offs[static_cast<int64_t>(d) * num_tiles + blockIdx.x];
+        for (int w = 0; w < kSortWarps; ++w) {
+            const int32_t c = s_base[w * radix + d];
+            s_base[w * radix + d] = run;
+            run += c;
+        }
+    }
+    __syncthreads();
+
+    // Phase C: rank inside the warp in element order and scatter.
+    const unsigned lower = (1u << lane) - 1u;
+#pragma unroll
+    for (int r = 0; r < kItems; ++r) {
+        const int64_t idx = wbase + r * 32 + lane;
+        const bool ok = idx < e;
+        const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
+        const unsigned peers = __match_any_sync(kFull, dig);
+        int32_t pos = 0;
+        if (ok) pos = mine[dig] + __popc(peers & lower);
+        __syncwarp();
+        if (ok && lane == __ffs(peers) - 1) mine[dig] += __popc(peers);
+        __syncwarp();
+        if (ok) {
+            int32_t s, id;
+            if (FIRST) {
+                s = static_cast<int32_t>(checked_id(__ldg(src64 + idx), n, status));
+                id = static_cast<int32_t>(idx);
+            } else {
+                s = __ldg(src_in + idx);
+                id = __ldg(eid_in + idx);
+            }
+            key_out[pos] = keys[r];
+            src_out[pos] = s;
+            eid_out[pos] = id;
+        }
+    }
+}
+
+// ---- exclusive scan of an int32 array (in place), three kernels ----------
+__device__ int32_t block_exclusive_scan(int32_t v, int32_t *total) {
+    __shared__ int32_t warp_sums[kScanThreads / 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int32_t incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int32_t y = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) warp_sums[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        int32_t s = lane < kScanThreads / 32 ? warp_sums[lane] : 0;
+        int32_t si = s;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int32_t y = __shfl_up_sync(kFull, si, o);
+            if (lane >= o) si += y;
+        }
+        if (lane < kScanThreads / 32) warp_sums[lane] = si - s;
+        if (lane == kScanThreads / 32 - 1 && total) *total = si;
+    }
+    __syncthreads();
+    const int32_t r = incl - v + warp_sums[warp];
+    __syncthreads();
+    return r;
+}
+
+__global__ void __launch_bounds__(kScanThreads)
+scan_reduce(const int32_t *__restrict__ data, int64_t m, int32_t *__restrict__ sums) {
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * kScanChunk;
+    int32_t s = 0;
+    for (int i = threadIdx.x; i < kScanChunk; i += kScanThreads) {
+        const int64_t k = base + i;
+        if (k < m) s += data[k];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(kFull, s, o);
+    __shared__ int32_t ws[kScanThreads / 32];
+    if ((threadIdx.x & 31) == 0) ws[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int32_t t = 0;
+        for (int w = 0; w < kScanThreads / 32; ++w) t += ws[w];
+        sums[blockIdx.x] = t;
+    }
+}
+
+__global__ void __launch_bounds__(kScanThreads) scan_top(int32_t *sums, int nb) {
+    __shared__ int32_t carry;
+    __shared__ int32_t tot;
+    if (threadIdx.x == 0) carry = 0;
+    __syncthreads();
+    for (int base = 0; base < nb; base += kScanThreads) {
+        const int k = base + threadIdx.x;
+        const int32_t v = k < nb ? sums[k] : 0;
+        const int32_t ex = block_exclusive_scan(v, &tot);
+        if (k < nb) sums[k] = ex + carry;
+        __syncthreads();
+        if (threadIdx.x == 0) carry += tot;
+        __syncthreads();
+    }
+}
+
+__global__ void __launch_bounds__(kScanThreads)
+scan_down(int32_t *data, int64_t m, const int32_t *__restrict__ sums) {
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * kScanChunk +
+                         static_cast<int64_t>(threadIdx.x) * kScanItems;
+    int32_t v[kScanItems];
+    int32_t local = 0;
+#pragma unroll
+    for (int i = 0; i < kScanItems; ++i) {
+        v[i] = (base + i < m) ? data[base + i] : 0;
+        local += v[i];
+    }
+    int32_t run = block_exclusive_scan(local, nullptr) + sums[blockIdx.x];
+#pragma unroll
+    for (int i = 0; i < kScanItems; ++i) {
+        if (base + i < m) data[base + i] = run;
+        run += v[i];
+    }
+}
+
+// rowptr[k] = first sorted position whose key is >= k, for k in [0, n].
+__global__ void rowptr_from_sorted(const uint32_t *__restrict__ keys, int64_t e, int64_t n,
+                                   int32_t *__restrict__ rowptr) {
+    const int64_t k = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (k > n) return;
+    int64_t lo = 0, hi = e;
+    while (lo < hi) {
+        const int64_t mid = (lo + hi) >> 1;
+        if (static_cast<int64_t>(__ldg(keys + mid)) < k) lo = mid + 1;
+        else hi = mid;
+    }
+    rowptr[k] = static_cast<int32_t>(lo);
+}
+
+__global__ void degree_from_rowptr(const int32_t *__restrict__ rowptr, int64_t n,
+                                   int32_t *__restrict__ deg) {
+    const int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (t < n) deg[t] = rowptr[t + 1] - rowptr[t];
+}
+
+cudaError_t exclusive_scan(int32_t *data, int64_t m, int32_t *sums, cudaStream_t s) {
+    const int nb = ceil_div(m, kScanChunk);
+    scan_reduce<<<nb, kScanThreads, 0, s>>>(data, m, sums);
+    scan_top<<<1, kScanThreads, 0, s>>>(sums, nb);
+    scan_down<<<nb, kScanThreads, 0, s>>>(data, m, sums);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t csr_workspace_bytes(int64_t n, int64_t e) {
+    if (e <= 0) return 256;
+    const SortPlan p = plan_for(n);
+    const int64_t tiles = ceil_div(e, kTile);
+    const int64_t cells = (int64_t(1) << p.width) * tiles;
+    const size_t a = align256(sizeof(int32_t) * 3 * size_t(e));
+    const size_t b = align256(sizeof(int32_t) * (p.passes >= 3 ? 3 : 1) * size_t(e));
+    const size_t h = align256(sizeof(int32_t) * size_t(cells));
+    const size_t sums = align256(sizeof(int32_t) * size_t(ceil_div(cells, kScanChunk)));
+    return a + b + h + sums;
+}
+
+cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
+                             int32_t *col, int32_t *perm, int32_t *in_degree, void *ws,
+                             int32_t *status, cudaStream_t s) {
+    cudaError_t err = cudaMemsetAsync(status, 0, sizeof(int32_t), s);
+    if (err != cudaSuccess) return err;
+    const uint32_t *sorted_keys = nullptr;
+    if (e > 0) {
+        const SortPlan p = plan_for(n);
+        const int tiles = ceil_div(e, kTile);
+        const int radix = 1 << p.width;
+        const int64_t cells = int64_t(radix) * tiles;
+        char *w = static_cast<char *>(ws);
+        struct Buf { uint32_t *key; int32_t *src; int32_t *eid; } buf[2];
+        buf[0].key = reinterpret_cast<uint32_t *>(w);
+        buf[0].src = reinterpret_cast<int32_t *>(buf[0].key + e);
+        buf[0].eid = buf[0].src + e;
+        w += align256(sizeof(int32_t) * 3 * size_t(e));
+        buf[1].key = reinterpret_cast<uint32_t *>(w);
+        buf[1].src = reinterpret_cast<int32_t *>(buf[1].key + e);
+        buf[1].eid = buf[1].src + e;
+        w += align256(sizeof(int32_t) * (p.passes >= 3 ? 3 : 1) * size_t(e));
+        int32_t *hist = reinterpret_cast<int32_t *>(w);
+        w += align256(sizeof(int32_t) * size_t(cells));
+        int32_t *sums = reinterpret_cast<int32_t *>(w);
+
+        const int64_t *src64 = edge_index, *dst64 = edge_index + e;
+        for (int pass = 0; pass < p.passes; ++pass) {
+            const int shift = pass * p.width;
+            const bool first = pass == 0, last = pass == p.passes - 1;
+            const Buf &in = buf[(pass + 1) & 1];
+            Buf out = buf[pass & 1];
+            if (last) { out.src = col; out.eid = perm; }
+            if (first)
+                radix_upsweep<true><<<tiles, kSortThreads, radix * sizeof(int32_t), s>>>(
+                    dst64, nullptr, e, n, shift, p.width, tiles, hist, status);
+            else
+                radix_upsweep<false><<<tiles, kSortThreads, radix * sizeof(int32_t), s>>>(
+                    nullptr, in.key, e, n, shift, p.width, tiles, hist, status);
+            err = exclusive_scan(hist, cells, sums, s);
+            if (err != cudaSuccess) return err;
+            const size_t smem = size_t(kSortWarps) * radix * sizeof(int32_t);
+            if (first)
+                radix_downsweep<true><<<tiles, kSortThreads, smem, s>>>(
+                    src64, dst64, nullptr, nullptr, nullptr, e, n, shift, p.width, tiles, hist,
+                    out.key, out.src, out.eid, status);
+            else
+                radix_downsweep<false><<<tiles, kSortThreads, smem, s>>>(
+                    nullptr, nullptr, in.key, in.src, in.eid, e, n, shift, p.width, tiles, hist,
+                    out.key, out.src, out.eid, status);
+            err = cudaGetLastError();
+            if (err != cudaSuccess) return err;
+            sorted_keys = out.key;
+        }
+    }
+    rowptr_from_sorted<<<ceil_div(n + 1, 256), 256, 0, s>>>(sorted_keys, e, n, rowptr);
+    if (n > 0) degree_from_rowptr<<<ceil_div(n, 256), 256, 0, s>>>(rowptr, n, in_degree);
+    return cudaGetLastError();
+}
+
+}  // namespace tfg

@@ -159,9 +159,13 @@ def ba_pairs(n: int, m: int, rng: np.random.Generator) -> np.ndarray:
 
 def symmetrise(pairs: np.ndarray) -> np.ndarray:
     """Unordered pairs -> directed edge_index [2, 2M]: every (i, j) then every (j, i)."""
-    src = np.concatenate([pairs[:, 0], pairs[:, 1]])
-    dst = np.concatenate([pairs[:, 1], pairs[:, 0]])
-    return np.ascontiguousarray(np.stack([src, dst]).astype(np.int64))
+    m = pairs.shape[0]
+    out = np.empty((2, 2 * m), dtype=np.int64)
+    out[0, :m] = pairs[:, 0]
+    out[0, m:] = pairs[:, 1]
+    out[1, :m] = pairs[:, 1]
+    out[1, m:] = pairs[:, 0]
+    return out
 
 
 def with_self_loops(edge_index: np.ndarray, n: int) -> np.ndarray:
@@ -238,29 +242,49 @@ def dcsbm_pairs(n: int, blocks: int, m: int, rng: np.random.Generator,
         b_prob[s0:s1] = pr
         b_alias[s0:s1] = al + s0
 
-    def draw_global(k):
-        idx = rng.integers(0, n, size=k)
-        return np.where(rng.random(k) < g_prob[idx], idx, g_alias[idx])
+    sizes32 = sizes.astype(np.int32)
+    starts32 = starts.astype(np.int32)
+    block32 = block_of.astype(np.int32)
+    b_alias32 = b_alias.astype(np.int32)
+    g_alias32 = g_alias.astype(np.int32)
+    chunk = 1 << 21          # draw in chunks: bounded temporaries, reused memory
 
-    factor = 1.15
+    def draw_global(k):
+        idx = rng.integers(0, n, size=k, dtype=np.int32)
+        return np.where(rng.random(k, dtype=np.float32) < g_prob[idx], idx, g_alias32[idx])
+
+    def draw_keys(k, out):
+        """Fill out[:k] with the keys of k drawn pairs; return how many were kept."""
+        kept = 0
+        for c0 in range(0, k, chunk):
+            c = min(chunk, k - c0)
+            i = draw_global(c)
+            b = block32[i]
+            loc = starts32[b] + (rng.random(c, dtype=np.float32) * sizes32[b]).astype(np.int32)
+            np.minimum(loc, starts32[b + 1] - 1, out=loc)
+            j_in = np.where(rng.random(c, dtype=np.float32) < b_prob[loc], loc, b_alias32[loc])
+            j = np.where(rng.random(c, dtype=np.float32) < p_in, j_in, draw_global(c))
+            ok = i != j
+            lo = np.minimum(i[ok], j[ok]).astype(np.int64)
+            hi = np.maximum(i[ok], j[ok])
+            out[kept:kept + lo.shape[0]] = lo * n + hi
+            kept += lo.shape[0]
+        return kept
+
+    factor = 1.5
     while True:
         k = int(m * factor) + 1024
-        i = draw_global(k)
-        b = block_of[i]
-        loc = starts[b] + (rng.random(k) * sizes[b]).astype(np.int64)
-        loc = np.minimum(loc, starts[b + 1] - 1)
-        j_in = np.where(rng.random(k) < b_prob[loc], loc, b_alias[loc])
-        j = np.where(rng.random(k) < p_in, j_in, draw_global(k))
-        ok = i != j
-        key = np.minimum(i[ok], j[ok]) * n + np.maximum(i[ok], j[ok])
-        del i, j, b, loc, j_in, ok
+        key = np.empty(k, dtype=np.int64)
+        key = key[:draw_keys(k, key)]
         key.sort()
         key = key[np.concatenate([[True], key[1:] != key[:-1]])]
         if key.shape[0] >= m:
             break
         factor *= 1.25
     key = key[rng.permutation(key.shape[0])[:m]]
-    pairs = np.stack([key // n, key % n], axis=1)
+    pairs = np.empty((m, 2), dtype=np.int64)
+    np.floor_divide(key, n, out=pairs[:, 0])
+    np.remainder(key, n, out=pairs[:, 1])
     return pairs, block_of, sizes
 
 

@@ -1,0 +1,276 @@
+"""Thin Python binding of libtfg (the C ABI in include/tfg.h).
+
+Argument marshalling only: it checks tensor devices, dtypes and shapes,
+allocates output and workspace tensors with PyTorch (device memory), passes
+raw pointers and the current CUDA stream, and turns error codes into
+exceptions.  Every step of the computation runs in the CUDA kernels of
+libtfg.so; there is no CPU fallback.  If the library has not been built, the
+first call raises.
+
+Function names follow the ABI (``tfg_build_csr`` ...).  All tensors must be
+CUDA tensors on the same device; calls are asynchronous on the current stream.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from typing import NamedTuple, Optional
+
+import torch
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtfg.so")
+
+TFG_OK = 0
+TFG_ERR_INVALID_ARG = -1
+TFG_ERR_TOO_LARGE = -2
+TFG_ERR_WORKSPACE = -3
+TFG_ERR_CUDA = -4
+TFG_ERR_INDEX_RANGE = -5
+TFG_ERR_UNSORTED = -6
+TFG_ERR_TIMEOUT = -7
+TFG_F32, TFG_BF16 = 0, 1
+REDUCERS = {"sum": 0, "mean": 1, "max": 2}
+
+_lock = threading.Lock()
+_lib: Optional[ctypes.CDLL] = None
+
+
+class TfgError(RuntimeError):
+    def __init__(self, code: int, message: str):
+        super().__init__(f"libtfg error {code}: {message}")
+        self.code = code
+
+
+def lib() -> ctypes.CDLL:
+    """Load libtfg.so (once).  Raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(
+                    f"{LIB_PATH} is missing: build it first (python -m paper_2101_11552_gb300.build "
+                    "or __graft_entry__.build()); there is no CPU fallback")
+            L = ctypes.CDLL(LIB_PATH)
+            P, I64, I, F, SZ = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float,
+                                ctypes.c_size_t)
+            sigs = {
+                "tfg_version": [],
+                "tfg_build_csr_workspace_size": [I64, I64, ctypes.POINTER(SZ)],
+                "tfg_build_csr": [P, I64, I64, P, P, P, P, P, SZ, P, P],
+                "tfg_gcn_norm": [P, P, P, P, I64, I64, I, F, P, P, P],
+                "tfg_aggregate_sum": [P, P, P, P, I, I64, I64, P, P],
+                "tfg_aggregate_mean": [P, P, P, P, I, I64, I64, P, P],
+                "tfg_aggregate_max": [P, P, P, P, I, I64, I64, P, P],
+                "tfg_gcn_aggregate_sum": [P, P, P, P, P, I, I64, I64, I, F, P, P],
+                "tfg_edge_softmax_workspace_size": [I64, I, ctypes.POINTER(SZ)],
+                "tfg_edge_softmax_aggregate": [P, P, P, I64, I64, I, I, P, P, F, P, P, P, SZ, P],
+                "tfg_segment_pool": [P, I, P, I64, I64, I64, I, P, P, P],
+            }
+            for name, args in sigs.items():
+                fn = getattr(L, name)
+                fn.argtypes = args
+                fn.restype = ctypes.c_int
+            L.tfg_last_error.argtypes = []
+            L.tfg_last_error.restype = ctypes.c_char_p
+            _lib = L
+        return _lib
+
+
+def tfg_version() -> int:
+    return lib().tfg_version()
+
+
+def tfg_last_error() -> str:
+    return lib().tfg_last_error().decode()
+
+
+def _check(rc: int):
+    if rc != TFG_OK:
+        raise TfgError(rc, tfg_last_error())
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(device: torch.device):
+    return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _need_cuda(name: str, t: torch.Tensor, dtype=None, device=None):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+
+
+def _x_dtype(x: torch.Tensor) -> int:
+    if x.dtype == torch.float32:
+        return TFG_F32
+    if x.dtype == torch.bfloat16:
+        return TFG_BF16
+    raise ValueError(f"features must be float32 or bfloat16, got {x.dtype}")
+
+
+class CSR(NamedTuple):
+    rowptr: torch.Tensor     # int32 [N + 1]
+    col: torch.Tensor        # int32 [E]
+    perm: torch.Tensor       # int32 [E]
+    in_degree: torch.Tensor  # int32 [N]
+    status: torch.Tensor     # int32 [1] (device)
+
+
+def check_status(status: torch.Tensor):
+    """Synchronise on the status word and raise if a kernel flagged bad input."""
+    code = int(status.item())
+    if code != 0:
+        raise TfgError(code, "device-side validation failed "
+                             f"({'index out of range' if code == TFG_ERR_INDEX_RANGE else 'unsorted batch'})")
+
+
+def tfg_build_csr_workspace_size(num_nodes: int, num_edges: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().tfg_build_csr_workspace_size(num_nodes, num_edges, ctypes.byref(n)))
+    return n.value
+
+
+def tfg_build_csr(edge_index: torch.Tensor, num_nodes: int,
+                  workspace: Optional[torch.Tensor] = None) -> CSR:
+    """Group the edges of ``edge_index`` (int64 [2, E]) by target node."""
+    _need_cuda("edge_index", edge_index, torch.int64)
+    if edge_index.dim() != 2 or edge_index.shape[0] != 2:
+        raise ValueError("edge_index must have shape [2, E]")
+    dev = edge_index.device
+    e = edge_index.shape[1]
+    rowptr = torch.empty(num_nodes + 1, dtype=torch.int32, device=dev)
+    col = torch.empty(e, dtype=torch.int32, device=dev)
+    perm = torch.empty(e, dtype=torch.int32, device=dev)
+    deg = torch.empty(num_nodes, dtype=torch.int32, device=dev)
+    status = torch.empty(1, dtype=torch.int32, device=dev)
+    need = tfg_build_csr_workspace_size(num_nodes, e)
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+    _check(lib().tfg_build_csr(_ptr(edge_index), e, num_nodes, _ptr(rowptr), _ptr(col), _ptr(perm),
+                               _ptr(deg), _ptr(workspace), workspace.numel(), _ptr(status),
+                               _stream(dev)))
+    return CSR(rowptr, col, perm, deg, status)
+
+
+def tfg_gcn_norm(rowptr: torch.Tensor, col: torch.Tensor, perm: torch.Tensor, num_nodes: int,
+                 edge_weight: Optional[torch.Tensor] = None, add_self_loops: int = 0,
+                 self_loop_fill: float = 1.0, want_w_csr: bool = True):
+    """Return (dinv [N], w_csr [E] or None) of the GCN normalisation of A + I."""
+    _need_cuda("rowptr", rowptr, torch.int32)
+    dev = rowptr.device
+    e = col.numel()
+    if edge_weight is not None:
+        _need_cuda("edge_weight", edge_weight, torch.float32, dev)
+    dinv = torch.empty(num_nodes, dtype=torch.float32, device=dev)
+    w_csr = torch.empty(e, dtype=torch.float32, device=dev) if want_w_csr else None
+    _check(lib().tfg_gcn_norm(_ptr(rowptr), _ptr(col), _ptr(perm), _ptr(edge_weight), num_nodes, e,
+                              int(add_self_loops), float(self_loop_fill), _ptr(dinv), _ptr(w_csr),
+                              _stream(dev)))
+    return dinv, w_csr
+
+
+def _aggregate(fn_name: str, rowptr, col, x, w_csr, out):
+    _need_cuda("rowptr", rowptr, torch.int32)
+    dev = rowptr.device
+    _need_cuda("col", col, torch.int32, dev)
+    _need_cuda("x", x, None, dev)
+    n, f = x.shape
+    if rowptr.numel() != n + 1:
+        raise ValueError("rowptr must have N + 1 entries")
+    if w_csr is not None:
+        _need_cuda("w_csr", w_csr, torch.float32, dev)
+    if out is None:
+        out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    _need_cuda("out", out, torch.float32, dev)
+    _check(getattr(lib(), fn_name)(_ptr(rowptr), _ptr(col), _ptr(w_csr), _ptr(x), _x_dtype(x), n, f,
+                                   _ptr(out), _stream(dev)))
+    return out
+
+
+def tfg_aggregate_sum(rowptr, col, x, w_csr=None, out=None):
+    return _aggregate("tfg_aggregate_sum", rowptr, col, x, w_csr, out)
+
+
+def tfg_aggregate_mean(rowptr, col, x, w_csr=None, out=None):
+    return _aggregate("tfg_aggregate_mean", rowptr, col, x, w_csr, out)
+
+
+def tfg_aggregate_max(rowptr, col, x, w_csr=None, out=None):
+    return _aggregate("tfg_aggregate_max", rowptr, col, x, w_csr, out)
+
+
+def tfg_gcn_aggregate_sum(rowptr, col, dinv, x, w_csr=None, add_self_loops: int = 0,
+                          self_loop_fill: float = 1.0, out=None):
+    _need_cuda("rowptr", rowptr, torch.int32)
+    dev = rowptr.device
+    _need_cuda("col", col, torch.int32, dev)
+    _need_cuda("dinv", dinv, torch.float32, dev)
+    _need_cuda("x", x, None, dev)
+    n, f = x.shape
+    if rowptr.numel() != n + 1:
+        raise ValueError("rowptr must have N + 1 entries")
+    if w_csr is not None:
+        _need_cuda("w_csr", w_csr, torch.float32, dev)
+    if out is None:
+        out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    _need_cuda("out", out, torch.float32, dev)
+    _check(lib().tfg_gcn_aggregate_sum(_ptr(rowptr), _ptr(col), _ptr(dinv), _ptr(w_csr), _ptr(x),
+                                       _x_dtype(x), n, f, int(add_self_loops),
+                                       float(self_loop_fill), _ptr(out), _stream(dev)))
+    return out
+
+
+def tfg_edge_softmax_workspace_size(num_nodes: int, heads: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().tfg_edge_softmax_workspace_size(num_nodes, heads, ctypes.byref(n)))
+    return n.value
+
+
+def tfg_edge_softmax_aggregate(rowptr, col, x, heads: int, channels: int, a_src, a_dst,
+                               negative_slope: float = 0.2, want_alpha: bool = False,
+                               out=None, workspace=None):
+    """Return (out [N, H*C], alpha [E, H] in CSR order or None)."""
+    _need_cuda("rowptr", rowptr, torch.int32)
+    dev = rowptr.device
+    _need_cuda("col", col, torch.int32, dev)
+    _need_cuda("x", x, torch.float32, dev)
+    _need_cuda("a_src", a_src, torch.float32, dev)
+    _need_cuda("a_dst", a_dst, torch.float32, dev)
+    n, f = x.shape
+    if f != heads * channels:
+        raise ValueError("x must have heads * channels columns")
+    e = col.numel()
+    if out is None:
+        out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    alpha = torch.empty(e, heads, dtype=torch.float32, device=dev) if want_alpha else None
+    need = tfg_edge_softmax_workspace_size(n, heads)
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+    _check(lib().tfg_edge_softmax_aggregate(_ptr(rowptr), _ptr(col), _ptr(x), n, e, heads, channels,
+                                            _ptr(a_src), _ptr(a_dst), float(negative_slope),
+                                            _ptr(out), _ptr(alpha), _ptr(workspace),
+                                            workspace.numel(), _stream(dev)))
+    return out, alpha
+
+
+def tfg_segment_pool(x, batch, num_graphs: int, reduce: str = "sum", out=None):
+    """Return (out [G, F], status) -- status is the device status word."""
+    _need_cuda("x", x)
+    dev = x.device
+    _need_cuda("batch", batch, torch.int64, dev)
+    n, f = x.shape
+    if out is None:
+        out = torch.empty(num_graphs, f, dtype=torch.float32, device=dev)
+    status = torch.empty(1, dtype=torch.int32, device=dev)
+    _check(lib().tfg_segment_pool(_ptr(x), _x_dtype(x), _ptr(batch), n, num_graphs, f,
+                                  REDUCERS[reduce], _ptr(out), _ptr(status), _stream(dev)))
+    return out, status

@@ -1,0 +1,103 @@
+"""Full-size dense-community workload (232,965 nodes, 114.6M edges, bf16 F=128).
+
+Exactly the calls and launch configuration the benchmark times.  The CSR,
+in-degrees and dinv are compared whole; the aggregations on sampled rows
+(every hub above the CTA-cooperative threshold that the sample reaches, the
+highest-degree rows and a seeded random sample), which the oracle computes
+one by one from its own stable CSR.  Pooling is compared whole.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2101_11552_gb300 import graphgen as gg
+from paper_2101_11552_gb300 import tfg
+from _helpers import TOL_BF16, TOL_F32, assert_exact_f32, assert_scaled_close, dev, max_scaled_error
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+
+@pytest.fixture(scope="module")
+def c5():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2101_11552_gb300 import build
+    build.build_library()
+    wl = gg.make_c5()
+    ocsr = oracle.build_csr(wl.edge_index, wl.num_nodes)
+    ei = dev(wl.edge_index)
+    csr = tfg.tfg_build_csr(ei, wl.num_nodes)
+    tfg.check_status(csr.status)
+    del ei
+    deg = ocsr[3]
+    rng = np.random.default_rng(7)
+    top = np.argsort(deg)[-64:]
+    low = np.argsort(deg)[:16]
+    rows = np.unique(np.concatenate([top, low, rng.choice(wl.num_nodes, 1500, replace=False),
+                                     [0, wl.num_nodes - 1]])).astype(np.int64)
+    return wl, ocsr, csr, rows
+
+
+def test_c5_csr_bit_exact(c5):
+    wl, ocsr, csr, _ = c5
+    for name, g, w in zip(("rowptr", "col", "perm", "in_degree"), csr[:4], ocsr):
+        assert np.array_equal(g.cpu().numpy(), w), name
+
+
+def test_c5_gcn_bf16_sampled_rows(c5):
+    wl, ocsr, csr, rows = c5
+    n = wl.num_nodes
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 1, 1.0, want_w_csr=False)
+    ref_norm = oracle.gcn_norm(wl.edge_index, n, None, 1, 1.0)
+    np.testing.assert_allclose(dinv.cpu().numpy(), ref_norm["dinv"], rtol=2e-6, atol=0)
+    x = dev(wl.x_bf16.view(np.int16)).view(torch.bfloat16)
+    out = tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, x, None, 1, 1.0)
+    got = out[dev(rows)].cpu().numpy()
+    w_norm = ref_norm["w_norm"]
+    ref, scale = oracle.aggregate_rows(ocsr, n, wl.x_bf16, "sum", rows, w=w_norm,
+                                       self_w=ref_norm["self_w"])
+    assert_scaled_close(got, ref, scale, TOL_BF16, "c5 gcn bf16")
+    # the bf16 bound is loose by design; the fp32 accumulation is far tighter
+    assert max_scaled_error(got, ref, scale) < 1e-5
+
+
+def test_c5_edge_softmax_sampled_rows(c5):
+    wl, ocsr, csr, rows = c5
+    n = wl.num_nodes
+    out, alpha = tfg.tfg_edge_softmax_aggregate(csr.rowptr, csr.col, dev(wl.x), wl.heads,
+                                                wl.channels, dev(wl.a_src), dev(wl.a_dst),
+                                                wl.negative_slope, want_alpha=True)
+    sub = rows[:400]
+    ref, ref_alpha, scale = oracle.edge_softmax_rows(ocsr, n, wl.x, wl.heads, wl.channels,
+                                                     wl.a_src, wl.a_dst, wl.negative_slope, sub)
+    assert_scaled_close(out[dev(sub)].cpu().numpy(), ref, scale, TOL_F32, "c5 softmax")
+    rp = ocsr[0]
+    got_alpha = np.concatenate([alpha[int(rp[r]):int(rp[r + 1])].cpu().numpy() for r in sub])
+    assert_scaled_close(got_alpha, ref_alpha, ref_alpha, TOL_F32, "c5 alpha")
+
+
+def test_c5_max_and_mean_sampled_rows(c5):
+    wl, ocsr, csr, rows = c5
+    n = wl.num_nodes
+    x = dev(wl.x_bf16.view(np.int16)).view(torch.bfloat16)
+    for reduce, fn in (("max", tfg.tfg_aggregate_max), ("mean", tfg.tfg_aggregate_mean)):
+        got = fn(csr.rowptr, csr.col, x)[dev(rows)].cpu().numpy()
+        ref, scale = oracle.aggregate_rows(ocsr, n, wl.x_bf16, reduce, rows)
+        if reduce == "max":
+            assert_exact_f32(got, ref, "c5 max")
+        else:
+            assert_scaled_close(got, ref, scale, TOL_BF16, "c5 mean")
+
+
+def test_c5_community_pool(c5):
+    wl, _, csr, _ = c5
+    x = dev(wl.x)
+    for reduce in ("sum", "mean", "max"):
+        out, status = tfg.tfg_segment_pool(x, dev(wl.batch), wl.num_graphs, reduce)
+        tfg.check_status(status)
+        ref, scale = oracle.segment_pool(wl.x, wl.batch, wl.num_graphs, reduce)
+        if reduce == "max":
+            assert_exact_f32(out.cpu().numpy(), ref, "c5 pool max")
+        else:
+            assert_scaled_close(out.cpu().numpy(), ref, scale, TOL_F32, f"c5 pool {reduce}")

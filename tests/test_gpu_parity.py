@@ -1,0 +1,303 @@
+"""CUDA path vs fp64 oracle, element by element, through the C ABI.
+
+Small and mid-size seeded graphs span several tiles of every kernel and a
+ragged tail, plus the degenerate cases (no edges, one node, isolated nodes,
+duplicate edges, self-loops, a single hub taking half of all edges, feature
+counts that are not a multiple of the vector width).  The four smaller
+workloads run at full size.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2101_11552_gb300 import graphgen as gg
+from paper_2101_11552_gb300 import tfg
+from _helpers import (TOL_BF16, TOL_F32, assert_exact_f32, assert_scaled_close, dev, features,
+                      host_features)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2101_11552_gb300 import build
+    build.build_library()
+
+
+def gpu_csr(ei: np.ndarray, n: int):
+    csr = tfg.tfg_build_csr(dev(ei), n)
+    tfg.check_status(csr.status)
+    return csr
+
+
+def np_(t):
+    return t.cpu().numpy()
+
+
+# ---------------------------------------------------------------------------
+# CSR build: bit-exact
+# ---------------------------------------------------------------------------
+CSR_CASES = [
+    # (n, e, hub, isolated, seed)
+    (1, 5, -1, 0, 0), (5, 0, -1, 0, 1), (2, 1, -1, 0, 2), (7, 40, 0, 2, 3),
+    (1000, 30000, 3, 10, 4),          # 10-bit keys: one radix pass
+    (1025, 9000, -1, 0, 5),           # 11 bits: two passes
+    (70000, 250000, 12, 100, 6),      # several tiles, ragged tail
+    (1_500_000, 120_000, -1, 0, 7),   # 21 bits: three passes
+    (300, 8192 * 3, 5, 0, 8),         # exact multiple of the tile
+]
+
+
+@pytest.mark.parametrize("n,e,hub,iso,seed", CSR_CASES)
+def test_csr_bit_exact(n, e, hub, iso, seed):
+    wl = gg.random_edge_case_graph(n, e, 1, seed, hub=hub, isolated=iso)
+    want = oracle.build_csr(wl.edge_index, n)
+    got = gpu_csr(wl.edge_index, n)
+    for name, g, w in zip(("rowptr", "col", "perm", "in_degree"), got[:4], want):
+        assert np.array_equal(np_(g), w), name
+
+
+def test_csr_empty_graph():
+    got = tfg.tfg_build_csr(torch.zeros(2, 0, dtype=torch.int64, device="cuda"), 0)
+    tfg.check_status(got.status)
+    assert np_(got.rowptr).tolist() == [0]
+
+
+def test_csr_out_of_range_ids_set_status():
+    ei = np.array([[0, 1, 2, 7], [1, 2, -1, 0]], dtype=np.int64)   # 7 >= N, -1 < 0
+    got = tfg.tfg_build_csr(dev(ei), 4)
+    assert int(got.status.item()) == tfg.TFG_ERR_INDEX_RANGE
+    # the clamped ids keep every write in bounds: rowptr still partitions E
+    rp = np_(got.rowptr)
+    assert rp[0] == 0 and rp[-1] == 4 and np.all(np.diff(rp) >= 0)
+
+
+# ---------------------------------------------------------------------------
+# GCN normalisation
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("weighted", [False, True])
+@pytest.mark.parametrize("add_self", [0, 1])
+def test_gcn_norm(weighted, add_self):
+    n, e = 5000, 60000
+    wl = gg.random_edge_case_graph(n, e, 1, 11, hub=4, isolated=30)
+    ew = np.random.default_rng(0).uniform(0.1, 2.0, e).astype(np.float32) if weighted else None
+    csr = gpu_csr(wl.edge_index, n)
+    dinv, w_csr = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n,
+                                   dev(ew) if weighted else None, add_self, 1.0)
+    ref = oracle.gcn_norm(wl.edge_index, n, ew, add_self, 1.0)
+    np.testing.assert_allclose(np_(dinv), ref["dinv"], rtol=2e-6, atol=0)
+    _, _, perm, _ = oracle.build_csr(wl.edge_index, n)
+    np.testing.assert_allclose(np_(w_csr), ref["w_norm"][perm], rtol=4e-6, atol=0)
+
+
+# ---------------------------------------------------------------------------
+# Aggregation: sum / mean / max, fp32 and bf16, weighted and unweighted
+# ---------------------------------------------------------------------------
+AGG_GRAPHS = [
+    (1, 3, -1, 0),          # one node with self-loops
+    (50, 0, -1, 0),         # no edges
+    (300, 4000, 7, 20),     # a hub with ~2000 in-edges (CTA-cooperative path)
+    (4000, 30000, -1, 50),
+    (2000, 60000, 1, 0),    # hub with ~30000 in-edges
+]
+
+
+@pytest.mark.parametrize("reduce", ["sum", "mean", "max"])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("weighted", [False, True])
+@pytest.mark.parametrize("f", [1, 3, 8, 20, 64, 128, 136, 256])
+def test_aggregate(reduce, dtype, weighted, f):
+    for gi, (n, e, hub, iso) in enumerate(AGG_GRAPHS):
+        wl = gg.random_edge_case_graph(n, e, f, 100 + gi + f, hub=hub, isolated=iso)
+        ocsr = oracle.build_csr(wl.edge_index, n)
+        w_coo = (np.random.default_rng(gi).uniform(-1.5, 1.5, e).astype(np.float32)
+                 if weighted else None)
+        csr = gpu_csr(wl.edge_index, n)
+        w_csr = dev(w_coo[ocsr[2]]) if weighted else None
+        x = features(wl, dtype)
+        fn = {"sum": tfg.tfg_aggregate_sum, "mean": tfg.tfg_aggregate_mean,
+              "max": tfg.tfg_aggregate_max}[reduce]
+        got = np_(fn(csr.rowptr, csr.col, x, w_csr))
+        ref, scale = oracle.aggregate(wl.edge_index, n, host_features(wl, dtype), reduce, w=w_coo)
+        what = f"{reduce} {dtype} w={weighted} F={f} graph={gi}"
+        if reduce == "max":
+            assert_exact_f32(got, ref, what)
+        else:
+            assert_scaled_close(got, ref, scale, TOL_F32 if dtype == "f32" else TOL_BF16, what)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("add_self", [0, 1])
+@pytest.mark.parametrize("f", [5, 64, 128])
+def test_gcn_aggregate_on_the_fly(dtype, add_self, f):
+    n, e = 3000, 40000
+    wl = gg.random_edge_case_graph(n, e, f, 7 + f, hub=2, isolated=10)
+    csr = gpu_csr(wl.edge_index, n)
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, add_self, 1.0,
+                               want_w_csr=False)
+    got = np_(tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, features(wl, dtype), None,
+                                        add_self, 1.0))
+    ref, scale = oracle.gcn_aggregate(wl.edge_index, n, host_features(wl, dtype), None, add_self, 1.0)
+    assert_scaled_close(got, ref, scale, TOL_F32 if dtype == "f32" else TOL_BF16,
+                        f"gcn {dtype} self={add_self} F={f}")
+
+
+@pytest.mark.parametrize("add_self", [0, 1])
+def test_gcn_aggregate_weighted(add_self):
+    n, e, f = 2500, 30000, 32
+    wl = gg.random_edge_case_graph(n, e, f, 19, hub=0, isolated=5)
+    ew = np.random.default_rng(4).uniform(0.2, 3.0, e).astype(np.float32)
+    csr = gpu_csr(wl.edge_index, n)
+    dinv, w_csr = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, dev(ew), add_self, 2.0)
+    got = np_(tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, features(wl, "f32"), w_csr,
+                                        add_self, 2.0))
+    ref, scale = oracle.gcn_aggregate(wl.edge_index, n, wl.x, ew, add_self, 2.0)
+    assert_scaled_close(got, ref, scale, TOL_F32, f"weighted gcn self={add_self}")
+
+
+# ---------------------------------------------------------------------------
+# Edge softmax (GAT)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("heads,channels", [(1, 1), (2, 3), (4, 4), (8, 16), (3, 48), (1, 160)])
+def test_edge_softmax(heads, channels):
+    n, e = 3000, 25000
+    f = heads * channels
+    wl = gg.random_edge_case_graph(n, e, f, 31 + f, hub=9, isolated=40)
+    rng = np.random.default_rng(heads * 100 + channels)
+    a_s = rng.standard_normal(f).astype(np.float32)
+    a_d = rng.standard_normal(f).astype(np.float32)
+    csr = gpu_csr(wl.edge_index, n)
+    out, alpha = tfg.tfg_edge_softmax_aggregate(csr.rowptr, csr.col, dev(wl.x), heads, channels,
+                                                dev(a_s), dev(a_d), 0.2, want_alpha=True)
+    ref, ref_alpha, scale = oracle.edge_softmax(wl.edge_index, n, wl.x, heads, channels, a_s, a_d, 0.2)
+    assert_scaled_close(np_(out), ref, scale, TOL_F32, f"softmax H={heads} C={channels}")
+    perm = oracle.build_csr(wl.edge_index, n)[2]
+    want = ref_alpha[perm]
+    assert_scaled_close(np_(alpha), want, want, TOL_F32, "alpha")
+
+
+# ---------------------------------------------------------------------------
+# Segment pooling
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("reduce", ["sum", "mean", "max"])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("f", [1, 7, 128, 264])
+def test_segment_pool(reduce, dtype, f):
+    rng = np.random.default_rng(f)
+    g = 300
+    sizes = rng.integers(0, 40, size=g)
+    sizes[[0, 17, 299]] = 0                    # empty graphs, including the last
+    sizes[5] = 3000                            # one large graph
+    batch = np.repeat(np.arange(g), sizes).astype(np.int64)
+    n = batch.size
+    wl = gg.Workload("pool", n, np.zeros((2, 0), np.int64),
+                     rng.standard_normal((n, f)).astype(np.float32))
+    out, status = tfg.tfg_segment_pool(features(wl, dtype), dev(batch), g, reduce)
+    tfg.check_status(status)
+    ref, scale = oracle.segment_pool(host_features(wl, dtype), batch, g, reduce)
+    if reduce == "max":
+        assert_exact_f32(np_(out), ref, f"pool max {dtype}")
+    else:
+        assert_scaled_close(np_(out), ref, scale, TOL_F32, f"pool {reduce} {dtype} F={f}")
+
+
+def test_segment_pool_bad_batch_sets_status():
+    x = torch.ones(6, 4, device="cuda")
+    _, status = tfg.tfg_segment_pool(x, dev(np.array([0, 0, 2, 1, 1, 2])), 3, "sum")
+    assert int(status.item()) == tfg.TFG_ERR_UNSORTED
+    _, status = tfg.tfg_segment_pool(x, dev(np.array([0, 0, 1, 1, 2, 3])), 3, "sum")
+    assert int(status.item()) == tfg.TFG_ERR_INDEX_RANGE
+
+
+# ---------------------------------------------------------------------------
+# The four smaller workloads at full size
+# ---------------------------------------------------------------------------
+def test_c1_gcn_full():
+    wl = gg.make_c1()
+    n = wl.num_nodes
+    csr = gpu_csr(wl.edge_index, n)
+    want = oracle.build_csr(wl.edge_index, n)
+    assert all(np.array_equal(np_(a), b) for a, b in zip(csr[:4], want))
+    dinv, w_csr = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0)
+    got = np_(tfg.tfg_aggregate_sum(csr.rowptr, csr.col, dev(wl.x), w_csr))
+    ref, scale = oracle.gcn_aggregate(wl.edge_index, n, wl.x, None, 0)
+    assert_scaled_close(got, ref, scale, TOL_F32, "c1")
+    got2 = np_(tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, dev(wl.x)))
+    assert_scaled_close(got2, ref, scale, TOL_F32, "c1 on the fly")
+
+
+def test_c2_sum_mean_max_full():
+    wl = gg.make_c2()
+    n = wl.num_nodes
+    csr = gpu_csr(wl.edge_index, n)
+    x = dev(wl.x)
+    for reduce, fn in (("sum", tfg.tfg_aggregate_sum), ("mean", tfg.tfg_aggregate_mean),
+                       ("max", tfg.tfg_aggregate_max)):
+        got = np_(fn(csr.rowptr, csr.col, x))
+        ref, scale = oracle.aggregate(wl.edge_index, n, wl.x, reduce)
+        if reduce == "max":
+            assert_exact_f32(got, ref, "c2 max")
+        else:
+            assert_scaled_close(got, ref, scale, TOL_F32, f"c2 {reduce}")
+
+
+def test_c3_edge_softmax_full():
+    wl = gg.make_c3()
+    n = wl.num_nodes
+    csr = gpu_csr(wl.edge_index, n)
+    out, alpha = tfg.tfg_edge_softmax_aggregate(csr.rowptr, csr.col, dev(wl.x), wl.heads,
+                                                wl.channels, dev(wl.a_src), dev(wl.a_dst),
+                                                wl.negative_slope, want_alpha=True)
+    ref, ref_alpha, scale = oracle.edge_softmax(wl.edge_index, n, wl.x, wl.heads, wl.channels,
+                                                wl.a_src, wl.a_dst, wl.negative_slope)
+    assert_scaled_close(np_(out), ref, scale, TOL_F32, "c3 out")
+    perm = np_(csr.perm)
+    assert_scaled_close(np_(alpha), ref_alpha[perm], ref_alpha[perm], TOL_F32, "c3 alpha")
+    deg = np.bincount(wl.edge_index[1], minlength=n)
+    assert np.all(np_(out)[deg == 0] == 0.0)
+
+
+def test_c4_batched_gcn_then_pool_full():
+    wl = gg.make_c4()
+    n = wl.num_nodes
+    csr = gpu_csr(wl.edge_index, n)
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
+    h = tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, dev(wl.x))
+    ref_h, scale = oracle.gcn_aggregate(wl.edge_index, n, wl.x, None, 0)
+    assert_scaled_close(np_(h), ref_h, scale, TOL_F32, "c4 gcn")
+    batch = dev(wl.batch)
+    h32 = np_(h)                      # the pooling oracle reads what the GPU pooled
+    for reduce in ("sum", "mean", "max"):
+        out, status = tfg.tfg_segment_pool(h, batch, wl.num_graphs, reduce)
+        tfg.check_status(status)
+        ref, pscale = oracle.segment_pool(h32, wl.batch, wl.num_graphs, reduce)
+        if reduce == "max":
+            assert_exact_f32(np_(out), ref, "c4 pool max")
+        else:
+            assert_scaled_close(np_(out), ref, pscale, TOL_F32, f"c4 pool {reduce}")
+    # batched == per graph (Section 2.1.1): graph g's rows only see graph g
+    offs = np.concatenate([[0], np.cumsum(wl.graph_sizes)])
+    for g in (0, 511, 1023):
+        s0, s1 = offs[g], offs[g + 1]
+        m = (wl.edge_index[1] >= s0) & (wl.edge_index[1] < s1)
+        sub = wl.edge_index[:, m] - s0
+        ref_g, _ = oracle.gcn_aggregate(sub, s1 - s0, wl.x[s0:s1], None, 0)
+        np.testing.assert_allclose(h32[s0:s1], ref_g, rtol=1e-5, atol=1e-5)
+
+
+def test_deterministic_bitwise():
+    wl = gg.random_edge_case_graph(20000, 400000, 128, 5, hub=3, isolated=100)
+    n = wl.num_nodes
+    runs = []
+    for _ in range(2):
+        csr = gpu_csr(wl.edge_index, n)
+        dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 1, 1.0, want_w_csr=False)
+        a = tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, features(wl, "bf16"), None, 1, 1.0)
+        b, al = tfg.tfg_edge_softmax_aggregate(csr.rowptr, csr.col, dev(wl.x), 8, 16,
+                                               dev(np.ones(128, np.float32)),
+                                               dev(np.ones(128, np.float32)), 0.2, want_alpha=True)
+        runs.append([np_(t).tobytes() for t in (csr.col, csr.perm, dinv, a, b, al)])
+    assert runs[0] == runs[1]
