@@ -62,13 +62,22 @@ struct Agg {
     }
 
     // Accumulate edges [beg, end) into acc (this lane's VEC features at f0).
+    // Sums are blocked in two levels -- a partial per 32-edge chunk, a partial
+    // per 32 chunks, then the total -- so no fp32 chain is longer than about
+    // 64 + deg / 1024 additions, even on hub rows.  The order is fixed.
     static __device__ __forceinline__ void edges(const AggArgs &a, int64_t beg, int64_t end,
                                                  int64_t f0, bool fok, float (&acc)[VEC],
                                                  int lane) {
         const XT *x = static_cast<const XT *>(a.x);
         const int g = lane / LPR;
         const bool weighted = KIND == kGcn || a.w != nullptr;
+        float sup[VEC], part[VEC];
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) sup[q] = 0.f;
+        int chunks = 0;
         for (int64_t base = beg; base < end; base += 32) {
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) part[q] = 0.f;
             const int cnt = static_cast<int>(min64(32, end - base));
             int c = 0;
             float ww = 1.f;
@@ -98,10 +107,26 @@ struct Agg {
 #pragma unroll
                     for (int q = 0; q < VEC; ++q) {
                         if (kIsMax) acc[q] = fmaxf(acc[q], wt[u] * v[u][q]);
-                        else acc[q] = fmaf(wt[u], v[u][q], acc[q]);
+                        else part[q] = fmaf(wt[u], v[u][q], part[q]);
                     }
                 }
             }
+            if (!kIsMax) {
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) sup[q] += part[q];
+                if (++chunks == 32) {
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q) {
+                        acc[q] += sup[q];
+                        sup[q] = 0.f;
+                    }
+                    chunks = 0;
+                }
+            }
+        }
+        if (!kIsMax) {
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] += sup[q];
         }
     }
 

@@ -73,14 +73,19 @@ softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict_
             }
         }
 
-        // pass 2: denominator and exp-weighted feature sum
-        float den = 0.f;
-        float acc[VEC];
+        // pass 2: denominator and exp-weighted feature sum, blocked in two
+        // levels (32-edge chunk, 32 chunks, total) to keep fp32 chains short
+        float den = 0.f, den_sup = 0.f;
+        float acc[VEC], sup[VEC], part[VEC];
 #pragma unroll
-        for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
+        for (int q = 0; q < VEC; ++q) acc[q] = sup[q] = 0.f;
+        int chunks = 0;
         for (int64_t base = beg; base < end; base += 32) {
             const int cnt = static_cast<int>(min64(32, end - base));
             const int c = lane < cnt ? __ldg(col + base + lane) : 0;
+            float den_part = 0.f;
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) part[q] = 0.f;
             for (int j = 0; j < cnt; j += kSmUnroll) {
                 int src[kSmUnroll];
                 float p[kSmUnroll];
@@ -98,14 +103,30 @@ softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict_
 #pragma unroll
                 for (int u = 0; u < kSmUnroll; ++u) {
                     if (j + u >= cnt) continue;
-                    den += p[u];
+                    den_part += p[u];
                     if (fok) {
 #pragma unroll
-                        for (int q = 0; q < VEC; ++q) acc[q] = fmaf(p[u], v[u][q], acc[q]);
+                        for (int q = 0; q < VEC; ++q) part[q] = fmaf(p[u], v[u][q], part[q]);
                     }
                 }
             }
+            den_sup += den_part;
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) sup[q] += part[q];
+            if (++chunks == 32) {
+                den += den_sup;
+                den_sup = 0.f;
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) {
+                    acc[q] += sup[q];
+                    sup[q] = 0.f;
+                }
+                chunks = 0;
+            }
         }
+        den += den_sup;
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) acc[q] += sup[q];
         if (fok) {
             float *o = out + t * f + f0;
 #pragma unroll
