@@ -128,7 +128,8 @@ int tfg_gcn_norm(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
  *   out[t, :] = REDUCE over positions k of row t of  w_k * x[col[k], :]
  *   sum; mean = sum / (rowptr[t+1] - rowptr[t]); max.
  *
- *   rowptr, col (device): CSR by target (tfg_build_csr).
+ *   rowptr, col (device): CSR by target (tfg_build_csr).  col may be NULL
+ *        only for a graph without edges; every row is then empty.
  *   w_csr (device) fp32 [num_edges] in CSR order, or NULL for w = 1.
  *   x (device) [num_nodes, num_features] row-major, x_dtype TFG_F32 or
  *        TFG_BF16.  16-byte alignment of x and a feature count that is a
@@ -173,18 +174,22 @@ int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float
  *           (evaluated with the row maximum subtracted; same value)
  *   out[t, h, :] = sum over row t of alpha[k, h] * x[col[k], h, :]
  *
- *   x (device) fp32 [num_nodes, heads * channels], head h in columns
- *          h*channels .. h*channels+channels-1.
+ *   x (device) [num_nodes, heads * channels], x_dtype TFG_F32 or TFG_BF16,
+ *          head h in columns h*channels .. h*channels+channels-1.
+ *   num_edges: rowptr[num_nodes]; col may be NULL when it is 0.
  *   a_src, a_dst (device) fp32 [heads * channels], same layout.
  *   out (device) fp32 [num_nodes, heads * channels], written.
  *   alpha (device) fp32 [num_edges, heads] in CSR order, or NULL.
  *   workspace (device) >= tfg_edge_softmax_workspace_size() bytes (node
  *          scores); contents are scratch.
- * Rows without incoming edges give 0.
+ * Rows without incoming edges give 0.  The row maximum is tracked as a
+ * running maximum in one pass (rescaling the partial sums when it grows),
+ * which gives the same alpha and out as the three-pass workflow.
  * ---------------------------------------------------------------------- */
 int tfg_edge_softmax_workspace_size(int64_t num_nodes, int heads, size_t *bytes);
-int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const float *x,
-                               int64_t num_nodes, int64_t num_edges, int heads, int channels,
+int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const void *x,
+                               int x_dtype, int64_t num_nodes, int64_t num_edges, int heads,
+                               int channels,
                                const float *a_src, const float *a_dst, float negative_slope,
                                float *out, float *alpha, void *workspace,
                                size_t workspace_bytes, tfg_stream_t stream);

@@ -62,22 +62,19 @@ struct Agg {
     }
 
     // Accumulate edges [beg, end) into acc (this lane's VEC features at f0).
-    // Sums are blocked in two levels -- a partial per 32-edge chunk, a partial
-    // per 32 chunks, then the total -- so no fp32 chain is longer than about
-    // 64 + deg / 1024 additions, even on hub rows.  The order is fixed.
+    // Each 32-edge chunk is summed into its own partial before it is added to
+    // acc, so an fp32 chain is at most 32 / G + deg / 32 additions long.  The
+    // order is fixed.  Out-of-range slots contribute an exact zero (weight 0,
+    // value 0) instead of a branch, except for max.
     static __device__ __forceinline__ void edges(const AggArgs &a, int64_t beg, int64_t end,
                                                  int64_t f0, bool fok, float (&acc)[VEC],
                                                  int lane) {
+        using V = VecLoad<XT, VEC>;
         const XT *x = static_cast<const XT *>(a.x);
         const int g = lane / LPR;
         const bool weighted = KIND == kGcn || a.w != nullptr;
-        float sup[VEC], part[VEC];
-#pragma unroll
-        for (int q = 0; q < VEC; ++q) sup[q] = 0.f;
-        int chunks = 0;
+        if (a.col == nullptr) return;   // a graph without edges
         for (int64_t base = beg; base < end; base += 32) {
-#pragma unroll
-            for (int q = 0; q < VEC; ++q) part[q] = 0.f;
             const int cnt = static_cast<int>(min64(32, end - base));
             int c = 0;
             float ww = 1.f;
@@ -86,47 +83,41 @@ struct Agg {
                 if (a.w) ww = __ldg(a.w + base + lane);
                 else if (KIND == kGcn) ww = __ldg(a.dinv + c);
             }
+            float part[VEC];
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) part[q] = 0.f;
             for (int j = 0; j < cnt; j += G * kUnroll) {
-                int src[kUnroll];
+                typename V::Raw raw[kUnroll];
                 float wt[kUnroll];
                 bool ok[kUnroll];
 #pragma unroll
                 for (int u = 0; u < kUnroll; ++u) {
                     const int k = j + u * G + g;
-                    src[u] = __shfl_sync(kFull, c, k & 31);
+                    const int src = __shfl_sync(kFull, c, k & 31);
                     wt[u] = weighted ? __shfl_sync(kFull, ww, k & 31) : 1.f;
                     ok[u] = fok && (k < cnt);
+                    raw[u] = ok[u] ? V::raw(x + static_cast<int64_t>(src) * a.f + f0) : V::zero();
+                    if (!kIsMax && !ok[u]) wt[u] = 0.f;
                 }
-                float v[kUnroll][VEC];
-#pragma unroll
-                for (int u = 0; u < kUnroll; ++u)
-                    if (ok[u]) VecLoad<XT, VEC>::load(x + static_cast<int64_t>(src[u]) * a.f + f0, v[u]);
 #pragma unroll
                 for (int u = 0; u < kUnroll; ++u) {
-                    if (!ok[u]) continue;
+                    float v[VEC];
+                    V::widen(raw[u], v);
+                    if (kIsMax) {
+                        if (ok[u]) {
 #pragma unroll
-                    for (int q = 0; q < VEC; ++q) {
-                        if (kIsMax) acc[q] = fmaxf(acc[q], wt[u] * v[u][q]);
-                        else part[q] = fmaf(wt[u], v[u][q], part[q]);
+                            for (int q = 0; q < VEC; ++q) acc[q] = fmaxf(acc[q], wt[u] * v[q]);
+                        }
+                    } else {
+#pragma unroll
+                        for (int q = 0; q < VEC; ++q) part[q] = fmaf(wt[u], v[q], part[q]);
                     }
                 }
             }
             if (!kIsMax) {
 #pragma unroll
-                for (int q = 0; q < VEC; ++q) sup[q] += part[q];
-                if (++chunks == 32) {
-#pragma unroll
-                    for (int q = 0; q < VEC; ++q) {
-                        acc[q] += sup[q];
-                        sup[q] = 0.f;
-                    }
-                    chunks = 0;
-                }
+                for (int q = 0; q < VEC; ++q) acc[q] += part[q];
             }
-        }
-        if (!kIsMax) {
-#pragma unroll
-            for (int q = 0; q < VEC; ++q) acc[q] += sup[q];
         }
     }
 
@@ -224,7 +215,7 @@ struct Agg {
 };
 
 template <typename XT, int VEC, int LPR, int KIND>
-__global__ void __launch_bounds__(kAggThreads) aggregate_kernel(AggArgs a) {
+__global__ void __launch_bounds__(kAggThreads, VEC >= 8 ? 3 : 4) aggregate_kernel(AggArgs a) {
     using A = Agg<XT, VEC, LPR, KIND>;
     __shared__ int s_next, s_nheavy;
     __shared__ int s_heavy[kRowsPerCta];

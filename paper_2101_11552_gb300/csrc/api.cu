@@ -74,7 +74,6 @@ int aggregate_common(const char *fn, int mode, const int32_t *rowptr, const int3
     TFG_TRY(check_features(fn, n, f));
     TFG_TRY(check_dtype(fn, dtype));
     TFG_NEED(rowptr, true, fn, "rowptr");
-    TFG_NEED(col, n > 0, fn, "col");
     TFG_NEED(x, n > 0, fn, "x");
     TFG_NEED(out, n > 0, fn, "out");
     TFG_NEED(dinv, mode == 3 && n > 0, fn, "dinv");
@@ -179,8 +178,9 @@ int tfg_edge_softmax_workspace_size(int64_t num_nodes, int heads, size_t *bytes)
     return ok();
 }
 
-int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const float *x,
-                               int64_t num_nodes, int64_t num_edges, int heads, int channels,
+int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const void *x,
+                               int x_dtype, int64_t num_nodes, int64_t num_edges, int heads,
+                               int channels,
                                const float *a_src, const float *a_dst, float negative_slope,
                                float *out, float *alpha, void *workspace,
                                size_t workspace_bytes, tfg_stream_t stream) {
@@ -189,8 +189,9 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
     if (heads < 1 || channels < 1)
         return fail(TFG_ERR_INVALID_ARG, "%s: heads and channels must be >= 1", fn);
     TFG_TRY(check_features(fn, num_nodes, int64_t(heads) * channels));
+    TFG_TRY(check_dtype(fn, x_dtype));
     TFG_NEED(rowptr, true, fn, "rowptr");
-    TFG_NEED(col, num_nodes > 0, fn, "col");
+    TFG_NEED(col, num_edges > 0, fn, "col");
     TFG_NEED(x, num_nodes > 0, fn, "x");
     TFG_NEED(out, num_nodes > 0, fn, "out");
     TFG_NEED(a_src, true, fn, "a_src");
@@ -199,8 +200,9 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
     if (num_nodes > 0 && (workspace == nullptr || workspace_bytes < need))
         return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
                     workspace ? workspace_bytes : size_t(0));
-    return cuda_result(tfg::launch_edge_softmax(rowptr, col, x, num_nodes, heads, channels, a_src,
-                                                a_dst, negative_slope, out, alpha, workspace,
+    return cuda_result(tfg::launch_edge_softmax(rowptr, num_edges > 0 ? col : nullptr, x, x_dtype,
+                                                num_nodes, heads, channels, a_src, a_dst,
+                                                negative_slope, out, alpha, workspace,
                                                 reinterpret_cast<cudaStream_t>(stream)),
                        fn);
 }
@@ -214,6 +216,8 @@ int tfg_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n
     if (num_graphs >= kIndexLimit) return fail(TFG_ERR_TOO_LARGE, "%s: too many graphs", fn);
     TFG_TRY(check_features(fn, num_nodes > num_graphs ? num_nodes : num_graphs, num_features));
     TFG_TRY(check_dtype(fn, x_dtype));
+    if (num_features > int64_t(65535) * 8)
+        return fail(TFG_ERR_TOO_LARGE, "%s: at most %d features", fn, 65535 * 8);
     if (reduce != TFG_SUM && reduce != TFG_MEAN && reduce != TFG_MAX)
         return fail(TFG_ERR_INVALID_ARG, "%s: unknown reducer %d", fn, reduce);
     TFG_NEED(x, num_nodes > 0, fn, "x");

@@ -19,31 +19,50 @@ __device__ __forceinline__ void set_status(int32_t *status, int32_t code) {
 __device__ __forceinline__ float bf16_lo(uint32_t packed) { return __uint_as_float(packed << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t packed) { return __uint_as_float(packed & 0xffff0000u); }
 
-// VEC consecutive features of one row, widened to fp32.
+// VEC consecutive features of one row: a raw load (kept packed in registers
+// while the load is in flight) and its widening to fp32.
 template <typename XT, int VEC> struct VecLoad;
 
 template <> struct VecLoad<float, 4> {
-    static __device__ __forceinline__ void load(const float *p, float (&v)[4]) {
-        float4 q = __ldg(reinterpret_cast<const float4 *>(p));
+    using Raw = float4;
+    static __device__ __forceinline__ Raw raw(const float *p) {
+        return __ldg(reinterpret_cast<const float4 *>(p));
+    }
+    static __device__ __forceinline__ Raw zero() { return make_float4(0.f, 0.f, 0.f, 0.f); }
+    static __device__ __forceinline__ void widen(const Raw &q, float (&v)[4]) {
         v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
     }
+    static __device__ __forceinline__ void load(const float *p, float (&v)[4]) { widen(raw(p), v); }
 };
 template <> struct VecLoad<float, 1> {
+    using Raw = float;
+    static __device__ __forceinline__ Raw raw(const float *p) { return __ldg(p); }
+    static __device__ __forceinline__ Raw zero() { return 0.f; }
+    static __device__ __forceinline__ void widen(const Raw &q, float (&v)[1]) { v[0] = q; }
     static __device__ __forceinline__ void load(const float *p, float (&v)[1]) { v[0] = __ldg(p); }
 };
 template <> struct VecLoad<uint16_t, 8> {
-    static __device__ __forceinline__ void load(const uint16_t *p, float (&v)[8]) {
-        uint4 q = __ldg(reinterpret_cast<const uint4 *>(p));
+    using Raw = uint4;
+    static __device__ __forceinline__ Raw raw(const uint16_t *p) {
+        return __ldg(reinterpret_cast<const uint4 *>(p));
+    }
+    static __device__ __forceinline__ Raw zero() { return make_uint4(0u, 0u, 0u, 0u); }
+    static __device__ __forceinline__ void widen(const Raw &q, float (&v)[8]) {
         v[0] = bf16_lo(q.x); v[1] = bf16_hi(q.x);
         v[2] = bf16_lo(q.y); v[3] = bf16_hi(q.y);
         v[4] = bf16_lo(q.z); v[5] = bf16_hi(q.z);
         v[6] = bf16_lo(q.w); v[7] = bf16_hi(q.w);
     }
+    static __device__ __forceinline__ void load(const uint16_t *p, float (&v)[8]) { widen(raw(p), v); }
 };
 template <> struct VecLoad<uint16_t, 1> {
-    static __device__ __forceinline__ void load(const uint16_t *p, float (&v)[1]) {
-        v[0] = __uint_as_float(static_cast<uint32_t>(__ldg(p)) << 16);
+    using Raw = uint32_t;
+    static __device__ __forceinline__ Raw raw(const uint16_t *p) {
+        return static_cast<uint32_t>(__ldg(p)) << 16;
     }
+    static __device__ __forceinline__ Raw zero() { return 0u; }
+    static __device__ __forceinline__ void widen(const Raw &q, float (&v)[1]) { v[0] = __uint_as_float(q); }
+    static __device__ __forceinline__ void load(const uint16_t *p, float (&v)[1]) { widen(raw(p), v); }
 };
 
 __host__ __device__ constexpr int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
@@ -66,10 +85,10 @@ cudaError_t launch_aggregate(int mode, const int32_t *rowptr, const int32_t *col
                              const float *dinv, const void *x, int x_dtype, int64_t n, int64_t f,
                              int add_self, float fill, float *out, cudaStream_t s);
 size_t softmax_workspace_bytes(int64_t n, int heads);
-cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const float *x,
-                                int64_t n, int heads, int channels, const float *a_src,
-                                const float *a_dst, float slope, float *out, float *alpha,
-                                void *ws, cudaStream_t s);
+cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const void *x,
+                                int x_dtype, int64_t n, int heads, int channels,
+                                const float *a_src, const float *a_dst, float slope, float *out,
+                                float *alpha, void *ws, cudaStream_t s);
 cudaError_t launch_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n,
                                 int64_t g, int64_t f, int reduce, float *out, int32_t *status,
                                 cudaStream_t s);

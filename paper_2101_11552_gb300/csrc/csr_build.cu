@@ -74,26 +74,47 @@ radix_upsweep(const int64_t *__restrict__ dst64, const uint32_t *__restrict__ ke
         hist[static_cast<int64_t>(d) * num_tiles + blockIdx.x] = s_cnt[d];
 }
 
+// Downsweep: 32 warps share one 8192-edge tile, 8 elements per lane.
+// Elements are ranked inside the tile (stable: warp-major, then round, then
+// lane = original order), staged in shared memory in digit order, and then
+// written out by consecutive threads, so each digit's run of the tile leaves
+// as coalesced stores.  The key array and each value array are staged in
+// turn through one value buffer to fit the tile in shared memory.
+constexpr int kDsWarps = 32;
+constexpr int kDsThreads = kDsWarps * 32;
+constexpr int kDsItems = kTile / kDsThreads;   // 8 per lane
+
+size_t downsweep_smem(int radix) {
+    return sizeof(uint32_t) * 2 * kTile + sizeof(uint16_t) * kDsWarps * radix +
+           sizeof(int32_t) * 2 * radix;
+}
+
 template <bool FIRST>
-__global__ void __launch_bounds__(kSortThreads)
+__global__ void __launch_bounds__(kDsThreads, 1)
 radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ dst64,
                 const uint32_t *__restrict__ key_in, const int32_t *__restrict__ src_in,
                 const int32_t *__restrict__ eid_in, int64_t e, int64_t n, int shift, int width,
                 int num_tiles, const int32_t *__restrict__ offs, uint32_t *__restrict__ key_out,
                 int32_t *__restrict__ src_out, int32_t *__restrict__ eid_out, int32_t *status) {
-    extern __shared__ int32_t s_base[];  // [kSortWarps][radix]
+    extern __shared__ __align__(16) unsigned char smem[];
     const int radix = 1 << width;
+    uint32_t *s_key = reinterpret_cast<uint32_t *>(smem);
+    int32_t *s_val = reinterpret_cast<int32_t *>(s_key + kTile);
+    uint16_t *s_cnt = reinterpret_cast<uint16_t *>(s_val + kTile);   // [warp][digit]
+    int32_t *s_tstart = reinterpret_cast<int32_t *>(s_cnt + kDsWarps * radix);
+    int32_t *s_gbase = s_tstart + radix;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    int32_t *mine = s_base + warp * radix;
+    const int64_t tile0 = static_cast<int64_t>(blockIdx.x) * kTile;
+    const int count = static_cast<int>(min64(kTile, e - tile0));
+    uint16_t *mine = s_cnt + warp * radix;
     for (int d = lane; d < radix; d += 32) mine[d] = 0;
     __syncwarp();
 
     // Phase A: per-warp digit counts over the warp's contiguous sub-tile.
-    const int64_t wbase = static_cast<int64_t>(blockIdx.x) * kTile +
-                          static_cast<int64_t>(warp) * 32 * kItems;
-    uint32_t keys[kItems];
+    const int64_t wbase = tile0 + static_cast<int64_t>(warp) * 32 * kDsItems;
+    uint32_t keys[kDsItems];
 #pragma unroll
-    for (int r = 0; r < kItems; ++r) {
+    for (int r = 0; r < kDsItems; ++r) {
         const int64_t idx = wbase + r * 32 + lane;
         const bool ok = idx < e;
         uint32_t key = 0;
@@ -101,49 +122,81 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
         keys[r] = key;
         const uint32_t dig = ok ? ((key >> shift) & (radix - 1)) : uint32_t(radix);
         const unsigned peers = __match_any_sync(kFull, dig);
-        if (ok && lane == __ffs(peers) - 1) mine[dig] += __popc(peers);
+        if (ok && lane == __ffs(peers) - 1) mine[dig] += static_cast<uint16_t>(__popc(peers));
         __syncwarp();
     }
     __syncthreads();
 
-    // Phase B: warp-major exclusive prefix per digit, seeded by the scanned
-    // global slot of (digit, this tile).
-    for (int d = threadIdx.x; d < radix; d += kSortThreads) {
-        int32_t run = offs[static_cast<int64_t>(d) * num_tiles + blockIdx.x];
-        for (int w = 0; w < kSortWarps; ++w) {
-            const int32_t c = s_base[w * radix + d];
-            s_base[w * radix + d] = run;
+    // Phase B: per digit, warp-major exclusive prefix (in place) and tile
+    // total; then an exclusive scan of the totals over digits.
+    for (int d = threadIdx.x; d < radix; d += kDsThreads) {
+        int run = 0;
+        for (int w = 0; w < kDsWarps; ++w) {
+            const int c = s_cnt[w * radix + d];
+            s_cnt[w * radix + d] = static_cast<uint16_t>(run);
             run += c;
+        }
+        s_tstart[d] = run;
+        s_gbase[d] = offs[static_cast<int64_t>(d) * num_tiles + blockIdx.x];
+    }
+    __syncthreads();
+    if (warp == 0) {   // exclusive scan of s_tstart[0 .. radix) by one warp
+        int carry = 0;
+        for (int base = 0; base < radix; base += 32) {
+            const int v = s_tstart[base + lane];
+            int incl = v;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(kFull, incl, o);
+                if (lane >= o) incl += y;
+            }
+            s_tstart[base + lane] = carry + incl - v;
+            carry += __shfl_sync(kFull, incl, 31);
         }
     }
     __syncthreads();
 
-    // Phase C: rank inside the warp in element order and scatter.
+    // Phase C: tile-local slot of every element (stable), keys staged.
     const unsigned lower = (1u << lane) - 1u;
+    uint32_t slots[kDsItems / 2];   // two 13-bit tile slots per register
 #pragma unroll
-    for (int r = 0; r < kItems; ++r) {
+    for (int r = 0; r < kDsItems; ++r) {
         const int64_t idx = wbase + r * 32 + lane;
         const bool ok = idx < e;
         const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
         const unsigned peers = __match_any_sync(kFull, dig);
-        int32_t pos = 0;
-        if (ok) pos = mine[dig] + __popc(peers & lower);
+        uint32_t slot = 0;
+        if (ok) slot = static_cast<uint32_t>(s_tstart[dig] + mine[dig] + __popc(peers & lower));
         __syncwarp();
-        if (ok && lane == __ffs(peers) - 1) mine[dig] += __popc(peers);
+        if (ok && lane == __ffs(peers) - 1) mine[dig] += static_cast<uint16_t>(__popc(peers));
         __syncwarp();
-        if (ok) {
-            int32_t s, id;
-            if (FIRST) {
-                s = static_cast<int32_t>(checked_id(__ldg(src64 + idx), n, status));
-                id = static_cast<int32_t>(idx);
-            } else {
-                s = __ldg(src_in + idx);
-                id = __ldg(eid_in + idx);
-            }
-            key_out[pos] = keys[r];
-            src_out[pos] = s;
-            eid_out[pos] = id;
+        if (ok) s_key[slot] = keys[r];
+        if (r & 1) slots[r / 2] |= slot << 16;
+        else slots[r / 2] = slot;
+    }
+
+    // Phase D: keys and the two value arrays leave in digit order.
+    for (int which = 0; which < 2; ++which) {
+#pragma unroll
+        for (int r = 0; r < kDsItems; ++r) {
+            const int64_t idx = wbase + r * 32 + lane;
+            if (idx >= e) continue;
+            int32_t v;
+            if (which == 0) v = FIRST ? static_cast<int32_t>(checked_id(__ldg(src64 + idx), n, status))
+                                      : __ldg(src_in + idx);
+            else v = FIRST ? static_cast<int32_t>(idx) : __ldg(eid_in + idx);
+            s_val[(slots[r / 2] >> (16 * (r & 1))) & 0xffffu] = v;
         }
+        __syncthreads();
+        int32_t *dst = which == 0 ? src_out : eid_out;
+        for (int i = threadIdx.x; i < count; i += kDsThreads) {
+            const uint32_t k = s_key[i];
+            const int d = static_cast<int>((k >> shift) & (radix - 1));
+            const int64_t pos = static_cast<int64_t>(s_gbase[d]) + (i - s_tstart[d]);
+            if (which == 0) key_out[pos] = k;
+            dst[pos] = s_val[i];
+        }
+        __syncthreads();
     }
 }
 
@@ -299,6 +352,11 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
         int32_t *sums = reinterpret_cast<int32_t *>(w);
 
         const int64_t *src64 = edge_index, *dst64 = edge_index + e;
+        const int smem_max = static_cast<int>(downsweep_smem(1 << kMaxDigitBits));
+        err = cudaFuncSetAttribute(radix_downsweep<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
+        if (err == cudaSuccess)
+            err = cudaFuncSetAttribute(radix_downsweep<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
+        if (err != cudaSuccess) return err;
         for (int pass = 0; pass < p.passes; ++pass) {
             const int shift = pass * p.width;
             const bool first = pass == 0, last = pass == p.passes - 1;
@@ -313,13 +371,13 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
                     nullptr, in.key, e, n, shift, p.width, tiles, hist, status);
             err = exclusive_scan(hist, cells, sums, s);
             if (err != cudaSuccess) return err;
-            const size_t smem = size_t(kSortWarps) * radix * sizeof(int32_t);
+            const size_t smem = downsweep_smem(radix);
             if (first)
-                radix_downsweep<true><<<tiles, kSortThreads, smem, s>>>(
+                radix_downsweep<true><<<tiles, kDsThreads, smem, s>>>(
                     src64, dst64, nullptr, nullptr, nullptr, e, n, shift, p.width, tiles, hist,
                     out.key, out.src, out.eid, status);
             else
-                radix_downsweep<false><<<tiles, kSortThreads, smem, s>>>(
+                radix_downsweep<false><<<tiles, kDsThreads, smem, s>>>(
                     nullptr, nullptr, in.key, in.src, in.eid, e, n, shift, p.width, tiles, hist,
                     out.key, out.src, out.eid, status);
             err = cudaGetLastError();

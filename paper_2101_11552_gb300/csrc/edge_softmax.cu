@@ -7,13 +7,17 @@
 //   map          alpha = exp(l - m) / den
 //   aggregate    out[t,h,:] = sum over row t of alpha * x[src,h,:]
 //
-// One warp owns a target row; lane L covers features f0 = 32*VEC*tile +
-// L*VEC (all of them inside head f0 / C).  Pass 1 finds the row maximum of
-// each head, pass 2 accumulates exp(l - m) and exp(l - m) * x in fp32, and
-// the result is divided by the denominator once.  With alpha requested a
-// third pass writes the normalised weights.  Every lane of a head computes
-// the same logits from the same inputs in the same order, so the values are
-// consistent across lanes and deterministic.
+// The paper's workflow runs map, reduce and map as separate passes over the
+// edges.  Here one warp owns a target row and makes a single pass with the
+// running-maximum form of the softmax: when an edge raises the row maximum m
+// of a head, the running denominator and weighted sum are rescaled by
+// exp(m_old - m_new), which leaves alpha and out mathematically unchanged.
+// A row is split among G = 32 / LPR lane groups (each group covers LPR * VEC
+// features and takes every G-th edge); the groups' (m, den, acc) triples are
+// merged by a butterfly at the end.  Sums are blocked per 32-edge chunk to
+// keep fp32 chains short.  Every lane of a head evaluates the same logits in
+// the same order, so the lanes agree and results are deterministic.  With
+// alpha requested, a second pass over the row writes the normalised weights.
 #include <math_constants.h>
 
 #include "common.cuh"
@@ -24,20 +28,22 @@ namespace {
 constexpr int kSmThreads = 256;
 constexpr int kSmUnroll = 4;
 
-__global__ void node_scores(const float *__restrict__ x, int64_t n, int heads, int channels,
+template <typename XT>
+__global__ void node_scores(const XT *__restrict__ x, int64_t n, int heads, int channels,
                             const float *__restrict__ a_src, const float *__restrict__ a_dst,
                             float *__restrict__ s_src, float *__restrict__ s_dst) {
     const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (i >= n * heads) return;
     const int64_t v = i / heads;
     const int h = static_cast<int>(i % heads);
-    const float *xr = x + v * heads * channels + static_cast<int64_t>(h) * channels;
+    const XT *xr = x + v * heads * channels + static_cast<int64_t>(h) * channels;
     const float *as = a_src + h * channels, *ad = a_dst + h * channels;
     float a = 0.f, b = 0.f;
     for (int c = 0; c < channels; ++c) {
-        const float xv = __ldg(xr + c);
-        a = fmaf(xv, __ldg(as + c), a);
-        b = fmaf(xv, __ldg(ad + c), b);
+        float xv[1];
+        VecLoad<XT, 1>::load(xr + c, xv);
+        a = fmaf(xv[0], __ldg(as + c), a);
+        b = fmaf(xv[0], __ldg(ad + c), b);
     }
     s_src[i] = a;
     s_dst[i] = b;
@@ -45,96 +51,100 @@ __global__ void node_scores(const float *__restrict__ x, int64_t n, int heads, i
 
 __device__ __forceinline__ float leaky(float v, float slope) { return v > 0.f ? v : slope * v; }
 
-template <int VEC>
-__global__ void __launch_bounds__(kSmThreads)
+// exp(m_old - m_new), with exp(-inf - anything) = 0 (an empty group has m = -inf).
+__device__ __forceinline__ float rescale(float m_old, float m_new) {
+    return m_old == -CUDART_INF_F ? 0.f : __expf(m_old - m_new);
+}
+
+template <typename XT, int VEC, int LPR>
+__global__ void __launch_bounds__(kSmThreads, 3)
 softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,
-                  const float *__restrict__ x, int64_t n, int heads, int channels, float slope,
+                  const XT *__restrict__ x, int64_t n, int heads, int channels, float slope,
                   const float *__restrict__ s_src, const float *__restrict__ s_dst,
                   float *__restrict__ out, float *__restrict__ alpha) {
+    using V = VecLoad<XT, VEC>;
+    constexpr int G = 32 / LPR;
     const int64_t t = (static_cast<int64_t>(blockIdx.x) * kSmThreads + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
+    const int lane = threadIdx.x & 31, g = lane / LPR, sub = lane % LPR;
     if (t >= n) return;
     const int64_t f = static_cast<int64_t>(heads) * channels;
-    const int64_t beg = rowptr[t], end = rowptr[t + 1];
-    for (int64_t ft = 0; ft < f; ft += 32 * VEC) {
-        const int64_t f0 = ft + lane * VEC;
+    const int64_t beg = rowptr[t], end = col ? rowptr[t + 1] : rowptr[t];
+    for (int64_t ft = 0; ft < f; ft += LPR * VEC) {
+        const int64_t f0 = ft + sub * VEC;
         const bool fok = f0 < f;
         const int h = fok ? static_cast<int>(f0 / channels) : 0;
         const float sd = __ldg(s_dst + t * heads + h);
 
-        // pass 1: per-head maximum of the logits of this row
-        float m = -CUDART_INF_F;
-        for (int64_t base = beg; base < end; base += 32) {
-            const int cnt = static_cast<int>(min64(32, end - base));
-            const int c = lane < cnt ? __ldg(col + base + lane) : 0;
-            for (int j = 0; j < cnt; ++j) {
-                const int src = __shfl_sync(kFull, c, j);
-                m = fmaxf(m, leaky(__ldg(s_src + static_cast<int64_t>(src) * heads + h) + sd, slope));
-            }
-        }
-
-        // pass 2: denominator and exp-weighted feature sum, blocked in two
-        // levels (32-edge chunk, 32 chunks, total) to keep fp32 chains short
-        float den = 0.f, den_sup = 0.f;
-        float acc[VEC], sup[VEC], part[VEC];
+        float m = -CUDART_INF_F, den = 0.f;
+        float acc[VEC];
 #pragma unroll
-        for (int q = 0; q < VEC; ++q) acc[q] = sup[q] = 0.f;
-        int chunks = 0;
+        for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
         for (int64_t base = beg; base < end; base += 32) {
             const int cnt = static_cast<int>(min64(32, end - base));
             const int c = lane < cnt ? __ldg(col + base + lane) : 0;
-            float den_part = 0.f;
+            float den_part = 0.f, part[VEC];
 #pragma unroll
             for (int q = 0; q < VEC; ++q) part[q] = 0.f;
-            for (int j = 0; j < cnt; j += kSmUnroll) {
-                int src[kSmUnroll];
-                float p[kSmUnroll];
-                float v[kSmUnroll][VEC];
+            for (int j = 0; j < cnt; j += G * kSmUnroll) {
+                float l[kSmUnroll];
+                typename V::Raw raw[kSmUnroll];
 #pragma unroll
                 for (int u = 0; u < kSmUnroll; ++u) {
-                    src[u] = __shfl_sync(kFull, c, (j + u) & 31);
-                    p[u] = 0.f;
-                    if (j + u < cnt) {
-                        const float l = leaky(__ldg(s_src + static_cast<int64_t>(src[u]) * heads + h) + sd, slope);
-                        p[u] = __expf(l - m);
-                        if (fok) VecLoad<float, VEC>::load(x + static_cast<int64_t>(src[u]) * f + f0, v[u]);
-                    }
+                    const int k = j + u * G + g;
+                    const int src = __shfl_sync(kFull, c, k & 31);
+                    const bool ok = k < cnt;
+                    l[u] = ok ? leaky(__ldg(s_src + static_cast<int64_t>(src) * heads + h) + sd, slope)
+                              : -CUDART_INF_F;
+                    raw[u] = (ok && fok) ? V::raw(x + static_cast<int64_t>(src) * f + f0) : V::zero();
                 }
 #pragma unroll
                 for (int u = 0; u < kSmUnroll; ++u) {
-                    if (j + u >= cnt) continue;
-                    den_part += p[u];
-                    if (fok) {
+                    if (l[u] == -CUDART_INF_F) continue;   // empty slot
+                    if (l[u] > m) {                        // new running maximum
+                        const float sc = rescale(m, l[u]);
+                        den *= sc;
+                        den_part *= sc;
 #pragma unroll
-                        for (int q = 0; q < VEC; ++q) part[q] = fmaf(p[u], v[u][q], part[q]);
+                        for (int q = 0; q < VEC; ++q) {
+                            acc[q] *= sc;
+                            part[q] *= sc;
+                        }
+                        m = l[u];
                     }
+                    const float p = __expf(l[u] - m);
+                    den_part += p;
+                    float v[VEC];
+                    V::widen(raw[u], v);
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q) part[q] = fmaf(p, v[q], part[q]);
                 }
             }
-            den_sup += den_part;
+            den += den_part;
 #pragma unroll
-            for (int q = 0; q < VEC; ++q) sup[q] += part[q];
-            if (++chunks == 32) {
-                den += den_sup;
-                den_sup = 0.f;
-#pragma unroll
-                for (int q = 0; q < VEC; ++q) {
-                    acc[q] += sup[q];
-                    sup[q] = 0.f;
-                }
-                chunks = 0;
-            }
+            for (int q = 0; q < VEC; ++q) acc[q] += part[q];
         }
-        den += den_sup;
+        // merge the G groups: (m, den, acc) in a fixed butterfly order
 #pragma unroll
-        for (int q = 0; q < VEC; ++q) acc[q] += sup[q];
-        if (fok) {
+        for (int s = LPR; s < 32; s <<= 1) {
+            const float mo = __shfl_xor_sync(kFull, m, s);
+            const float dn = __shfl_xor_sync(kFull, den, s);
+            const float mm = fmaxf(m, mo);
+            const float a = rescale(m, mm), b = rescale(mo, mm);
+            den = den * a + dn * b;
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) {
+                const float ao = __shfl_xor_sync(kFull, acc[q], s);
+                acc[q] = acc[q] * a + ao * b;
+            }
+            m = mm;
+        }
+        if (lane < LPR && fok) {
             float *o = out + t * f + f0;
 #pragma unroll
             for (int q = 0; q < VEC; ++q) o[q] = end > beg ? acc[q] / den : 0.f;
         }
-
-        // pass 3 (optional): normalised attention weights, one writer per head
-        if (alpha && fok && (f0 % channels) == 0) {
+        // normalised attention weights, one writer per (edge, head)
+        if (alpha && lane < LPR && fok && (f0 % channels) == 0) {
             for (int64_t k = beg; k < end; ++k) {
                 const int src = __ldg(col + k);
                 const float l = leaky(__ldg(s_src + static_cast<int64_t>(src) * heads + h) + sd, slope);
@@ -146,31 +156,56 @@ softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict_
 
 size_t align256(size_t b) { return (b + 255) & ~size_t(255); }
 
+template <typename XT, int VEC>
+void launch_main(const int32_t *rowptr, const int32_t *col, const void *x, int64_t n, int heads,
+                 int channels, float slope, const float *s_src, const float *s_dst, float *out,
+                 float *alpha, cudaStream_t s) {
+    const int64_t chunks = static_cast<int64_t>(heads) * channels / VEC;
+    const int grid = ceil_div(n * 32, kSmThreads);
+    const XT *xp = static_cast<const XT *>(x);
+    if (chunks >= 32)
+        softmax_aggregate<XT, VEC, 32><<<grid, kSmThreads, 0, s>>>(rowptr, col, xp, n, heads, channels,
+                                                                   slope, s_src, s_dst, out, alpha);
+    else if (chunks > 8)
+        softmax_aggregate<XT, VEC, 16><<<grid, kSmThreads, 0, s>>>(rowptr, col, xp, n, heads, channels,
+                                                                   slope, s_src, s_dst, out, alpha);
+    else
+        softmax_aggregate<XT, VEC, 8><<<grid, kSmThreads, 0, s>>>(rowptr, col, xp, n, heads, channels,
+                                                                  slope, s_src, s_dst, out, alpha);
+}
+
 }  // namespace
 
 size_t softmax_workspace_bytes(int64_t n, int heads) {
     return 2 * align256(sizeof(float) * size_t(n > 0 ? n : 1) * size_t(heads));
 }
 
-cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const float *x,
-                                int64_t n, int heads, int channels, const float *a_src,
-                                const float *a_dst, float slope, float *out, float *alpha,
-                                void *ws, cudaStream_t s) {
+cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const void *x,
+                                int x_dtype, int64_t n, int heads, int channels,
+                                const float *a_src, const float *a_dst, float slope, float *out,
+                                float *alpha, void *ws, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     float *s_src = static_cast<float *>(ws);
     float *s_dst = reinterpret_cast<float *>(static_cast<char *>(ws) +
                                              align256(sizeof(float) * size_t(n) * size_t(heads)));
-    node_scores<<<ceil_div(n * heads, 256), 256, 0, s>>>(x, n, heads, channels, a_src, a_dst,
-                                                        s_src, s_dst);
-    const bool vec = (channels % 4 == 0) && (reinterpret_cast<uintptr_t>(x) % 16 == 0) &&
-                     (reinterpret_cast<uintptr_t>(out) % 16 == 0);
-    const int grid = ceil_div(n * 32, kSmThreads);
-    if (vec)
-        softmax_aggregate<4><<<grid, kSmThreads, 0, s>>>(rowptr, col, x, n, heads, channels, slope,
-                                                         s_src, s_dst, out, alpha);
-    else
-        softmax_aggregate<1><<<grid, kSmThreads, 0, s>>>(rowptr, col, x, n, heads, channels, slope,
-                                                         s_src, s_dst, out, alpha);
+    const int sgrid = ceil_div(n * heads, 256);
+    const bool aligned = (reinterpret_cast<uintptr_t>(x) % 16 == 0) &&
+                         (reinterpret_cast<uintptr_t>(out) % 16 == 0);
+    if (x_dtype == TFG_BF16) {
+        node_scores<uint16_t><<<sgrid, 256, 0, s>>>(static_cast<const uint16_t *>(x), n, heads,
+                                                    channels, a_src, a_dst, s_src, s_dst);
+        if (aligned && channels % 8 == 0)
+            launch_main<uint16_t, 8>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+        else
+            launch_main<uint16_t, 1>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+    } else {
+        node_scores<float><<<sgrid, 256, 0, s>>>(static_cast<const float *>(x), n, heads, channels,
+                                                 a_src, a_dst, s_src, s_dst);
+        if (aligned && channels % 4 == 0)
+            launch_main<float, 4>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+        else
+            launch_main<float, 1>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+    }
     return cudaGetLastError();
 }
 

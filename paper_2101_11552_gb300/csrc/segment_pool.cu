@@ -3,18 +3,27 @@
 // leaves the nodes of each graph contiguous and the batch vector sorted.
 // This is the sorted-key reduction the paper builds from tf.math.segment_*.
 //
-// A CTA owns one (graph, feature tile).  It finds the graph's node range by
-// binary search on the sorted batch vector, its 256 threads form
-// 256 / LPR node groups that stride over the range, and the group partials
-// are combined in group order through shared memory (deterministic).
+// One (graph, feature tile) is reduced by S CTAs forming a thread-block
+// cluster (S = 1 for small graphs, up to 8 for large ones).  Each CTA finds
+// the graph's node range by binary search on the sorted batch vector and
+// takes one contiguous S-th of it; its 256 threads form 256 / LPR node groups
+// striding over that part, and the group partials are combined in group
+// order in shared memory.  CTA rank 0 of the cluster then reads the other
+// CTAs' partials through distributed shared memory, in rank order, and
+// writes the result.  The combination order is fixed, so results are
+// deterministic, and no global scratch is needed.
+#include <cooperative_groups.h>
 #include <math_constants.h>
 
 #include "common.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace tfg {
 namespace {
 
 constexpr int kPoolThreads = 256;
+constexpr int kMaxCluster = 8;
 
 __global__ void check_batch(const int64_t *__restrict__ batch, int64_t n, int64_t g,
                             int32_t *status) {
@@ -35,7 +44,13 @@ __device__ __forceinline__ int64_t lower_bound(const int64_t *batch, int64_t n, 
     return lo;
 }
 
-template <typename XT, int VEC, int LPR, int RED>
+template <int RED>
+__device__ __forceinline__ float pool_op(float a, float b) {
+    return RED == TFG_MAX ? fmaxf(a, b) : a + b;
+}
+
+// grid = (graphs, feature tiles, S); cluster = (1, 1, S) when S > 1.
+template <typename XT, int VEC, int LPR, int RED, bool CLUSTER>
 __global__ void __launch_bounds__(kPoolThreads)
 pool_kernel(const XT *__restrict__ x, const int64_t *__restrict__ batch, int64_t n, int64_t f,
             float *__restrict__ out) {
@@ -43,11 +58,15 @@ pool_kernel(const XT *__restrict__ x, const int64_t *__restrict__ batch, int64_t
     constexpr int kSlots = LPR * VEC;
     __shared__ int64_t s_range[2];
     __shared__ float s_part[kGroups * kSlots];
+    __shared__ float s_red[kSlots];
     const int64_t gid = blockIdx.x;
+    const int split = blockIdx.z, nsplit = gridDim.z;
     if (threadIdx.x == 0) s_range[0] = lower_bound(batch, n, gid);
     if (threadIdx.x == 32) s_range[1] = lower_bound(batch, n, gid + 1);
     __syncthreads();
     const int64_t beg = s_range[0], end = max(s_range[0], s_range[1]);
+    const int64_t len = (end - beg + nsplit - 1) / nsplit;
+    const int64_t pb = min(end, beg + split * len), pe = min(end, pb + len);
     const int grp = threadIdx.x / LPR, sub = threadIdx.x % LPR;
     const int64_t ft = static_cast<int64_t>(blockIdx.y) * kSlots;
     const int64_t f0 = ft + sub * VEC;
@@ -56,52 +75,103 @@ pool_kernel(const XT *__restrict__ x, const int64_t *__restrict__ batch, int64_t
 #pragma unroll
     for (int q = 0; q < VEC; ++q) acc[q] = RED == TFG_MAX ? -CUDART_INF_F : 0.f;
     if (fok) {
-        for (int64_t v = beg + grp; v < end; v += kGroups) {
+        for (int64_t v = pb + grp; v < pe; v += kGroups) {
             float val[VEC];
             VecLoad<XT, VEC>::load(x + v * f + f0, val);
 #pragma unroll
-            for (int q = 0; q < VEC; ++q) acc[q] = RED == TFG_MAX ? fmaxf(acc[q], val[q]) : acc[q] + val[q];
+            for (int q = 0; q < VEC; ++q) acc[q] = pool_op<RED>(acc[q], val[q]);
         }
     }
 #pragma unroll
     for (int q = 0; q < VEC; ++q) s_part[grp * kSlots + sub * VEC + q] = acc[q];
     __syncthreads();
     for (int i = threadIdx.x; i < kSlots; i += kPoolThreads) {
-        const int64_t fi = ft + i;
-        if (fi >= f) continue;
         float r = s_part[i];
-        for (int k = 1; k < kGroups; ++k)
-            r = RED == TFG_MAX ? fmaxf(r, s_part[k * kSlots + i]) : r + s_part[k * kSlots + i];
-        const int64_t cnt = end - beg;
-        if (cnt == 0) r = 0.f;
-        else if (RED == TFG_MEAN) r = r / static_cast<float>(cnt);
-        out[gid * f + fi] = r;
+        for (int k = 1; k < kGroups; ++k) r = pool_op<RED>(r, s_part[k * kSlots + i]);
+        s_red[i] = r;
+    }
+    const int64_t cnt = end - beg;
+    if constexpr (CLUSTER) {
+        cg::cluster_group cluster = cg::this_cluster();
+        cluster.sync();   // every CTA's partial is in its shared memory
+        if (cluster.block_rank() == 0) {
+            for (int i = threadIdx.x; i < kSlots; i += kPoolThreads) {
+                float r = s_red[i];
+                for (int q = 1; q < nsplit; ++q) r = pool_op<RED>(r, cluster.map_shared_rank(s_red, q)[i]);
+                const int64_t fi = ft + i;
+                if (fi < f) {
+                    if (cnt == 0) r = 0.f;
+                    else if (RED == TFG_MEAN) r = r / static_cast<float>(cnt);
+                    out[gid * f + fi] = r;
+                }
+            }
+        }
+        cluster.sync();   // keep partials alive until rank 0 has read them
+    } else {
+        __syncthreads();
+        for (int i = threadIdx.x; i < kSlots; i += kPoolThreads) {
+            const int64_t fi = ft + i;
+            if (fi >= f) continue;
+            float r = s_red[i];
+            if (cnt == 0) r = 0.f;
+            else if (RED == TFG_MEAN) r = r / static_cast<float>(cnt);
+            out[gid * f + fi] = r;
+        }
     }
 }
 
-template <typename XT, int VEC, int RED>
-void launch_lpr(const void *x, const int64_t *batch, int64_t n, int64_t g, int64_t f, float *out,
-                int lpr, cudaStream_t s) {
-    const dim3 grid(static_cast<unsigned>(g), ceil_div(f, int64_t(lpr) * VEC));
+template <typename XT, int VEC, int LPR, int RED>
+cudaError_t launch_split(const void *x, const int64_t *batch, int64_t n, int64_t g, int64_t f,
+                         float *out, int nsplit, cudaStream_t s) {
     const XT *xp = static_cast<const XT *>(x);
+    const dim3 grid(static_cast<unsigned>(g), ceil_div(f, int64_t(LPR) * VEC), nsplit);
+    if (nsplit == 1) {
+        pool_kernel<XT, VEC, LPR, RED, false><<<grid, kPoolThreads, 0, s>>>(xp, batch, n, f, out);
+        return cudaGetLastError();
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(kPoolThreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = nsplit;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, pool_kernel<XT, VEC, LPR, RED, true>, xp, batch, n, f, out);
+}
+
+template <typename XT, int VEC, int RED>
+cudaError_t launch_lpr(const void *x, const int64_t *batch, int64_t n, int64_t g, int64_t f,
+                       float *out, int lpr, int nsplit, cudaStream_t s) {
     switch (lpr) {
-        case 32: pool_kernel<XT, VEC, 32, RED><<<grid, kPoolThreads, 0, s>>>(xp, batch, n, f, out); break;
-        case 16: pool_kernel<XT, VEC, 16, RED><<<grid, kPoolThreads, 0, s>>>(xp, batch, n, f, out); break;
-        default: pool_kernel<XT, VEC, 8, RED><<<grid, kPoolThreads, 0, s>>>(xp, batch, n, f, out); break;
+        case 32: return launch_split<XT, VEC, 32, RED>(x, batch, n, g, f, out, nsplit, s);
+        case 16: return launch_split<XT, VEC, 16, RED>(x, batch, n, g, f, out, nsplit, s);
+        default: return launch_split<XT, VEC, 8, RED>(x, batch, n, g, f, out, nsplit, s);
     }
 }
 
 template <typename XT, int VEC>
-void launch_red(const void *x, const int64_t *batch, int64_t n, int64_t g, int64_t f, int reduce,
-                float *out, int lpr, cudaStream_t s) {
+cudaError_t launch_red(const void *x, const int64_t *batch, int64_t n, int64_t g, int64_t f,
+                       int reduce, float *out, int lpr, int nsplit, cudaStream_t s) {
     switch (reduce) {
-        case TFG_MEAN: launch_lpr<XT, VEC, TFG_MEAN>(x, batch, n, g, f, out, lpr, s); break;
-        case TFG_MAX: launch_lpr<XT, VEC, TFG_MAX>(x, batch, n, g, f, out, lpr, s); break;
-        default: launch_lpr<XT, VEC, TFG_SUM>(x, batch, n, g, f, out, lpr, s); break;
+        case TFG_MEAN: return launch_lpr<XT, VEC, TFG_MEAN>(x, batch, n, g, f, out, lpr, nsplit, s);
+        case TFG_MAX: return launch_lpr<XT, VEC, TFG_MAX>(x, batch, n, g, f, out, lpr, nsplit, s);
+        default: return launch_lpr<XT, VEC, TFG_SUM>(x, batch, n, g, f, out, lpr, nsplit, s);
     }
 }
 
 int lanes_for(int64_t chunks) { return chunks >= 32 ? 32 : (chunks > 8 ? 16 : 8); }
+
+// CTAs per graph: one per ~1024 nodes of an average graph, at most a portable cluster.
+int splits_for(int64_t n, int64_t g) {
+    const int64_t avg = g > 0 ? n / g : 0;
+    int64_t s = avg / 1024;
+    return static_cast<int>(s < 1 ? 1 : (s > kMaxCluster ? kMaxCluster : s));
+}
 
 }  // namespace
 
@@ -111,16 +181,18 @@ cudaError_t launch_segment_pool(const void *x, int x_dtype, const int64_t *batch
     cudaError_t err = cudaMemsetAsync(status, 0, sizeof(int32_t), s);
     if (err != cudaSuccess) return err;
     if (n > 0) check_batch<<<ceil_div(n, 256), 256, 0, s>>>(batch, n, g, status);
-    if (g <= 0) return cudaGetLastError();
+    err = cudaGetLastError();
+    if (err != cudaSuccess || g <= 0) return err;
+    const int nsplit = splits_for(n, g);
     const bool aligned = reinterpret_cast<uintptr_t>(x) % 16 == 0;
     if (x_dtype == TFG_BF16) {
-        if (aligned && f % 8 == 0) launch_red<uint16_t, 8>(x, batch, n, g, f, reduce, out, lanes_for(f / 8), s);
-        else launch_red<uint16_t, 1>(x, batch, n, g, f, reduce, out, lanes_for(f), s);
-    } else {
-        if (aligned && f % 4 == 0) launch_red<float, 4>(x, batch, n, g, f, reduce, out, lanes_for(f / 4), s);
-        else launch_red<float, 1>(x, batch, n, g, f, reduce, out, lanes_for(f), s);
+        if (aligned && f % 8 == 0)
+            return launch_red<uint16_t, 8>(x, batch, n, g, f, reduce, out, lanes_for(f / 8), nsplit, s);
+        return launch_red<uint16_t, 1>(x, batch, n, g, f, reduce, out, lanes_for(f), nsplit, s);
     }
-    return cudaGetLastError();
+    if (aligned && f % 4 == 0)
+        return launch_red<float, 4>(x, batch, n, g, f, reduce, out, lanes_for(f / 4), nsplit, s);
+    return launch_red<float, 1>(x, batch, n, g, f, reduce, out, lanes_for(f), nsplit, s);
 }
 
 }  // namespace tfg

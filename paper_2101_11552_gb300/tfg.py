@@ -64,7 +64,7 @@ def lib() -> ctypes.CDLL:
                 "tfg_aggregate_max": [P, P, P, P, I, I64, I64, P, P],
                 "tfg_gcn_aggregate_sum": [P, P, P, P, P, I, I64, I64, I, F, P, P],
                 "tfg_edge_softmax_workspace_size": [I64, I, ctypes.POINTER(SZ)],
-                "tfg_edge_softmax_aggregate": [P, P, P, I64, I64, I, I, P, P, F, P, P, P, SZ, P],
+                "tfg_edge_softmax_aggregate": [P, P, P, I, I64, I64, I, I, P, P, F, P, P, P, SZ, P],
                 "tfg_segment_pool": [P, I, P, I64, I64, I64, I, P, P, P],
             }
             for name, args in sigs.items():
@@ -242,7 +242,7 @@ def tfg_edge_softmax_aggregate(rowptr, col, x, heads: int, channels: int, a_src,
     _need_cuda("rowptr", rowptr, torch.int32)
     dev = rowptr.device
     _need_cuda("col", col, torch.int32, dev)
-    _need_cuda("x", x, torch.float32, dev)
+    _need_cuda("x", x, None, dev)
     _need_cuda("a_src", a_src, torch.float32, dev)
     _need_cuda("a_dst", a_dst, torch.float32, dev)
     n, f = x.shape
@@ -255,7 +255,8 @@ def tfg_edge_softmax_aggregate(rowptr, col, x, heads: int, channels: int, a_src,
     need = tfg_edge_softmax_workspace_size(n, heads)
     if workspace is None:
         workspace = torch.empty(need, dtype=torch.uint8, device=dev)
-    _check(lib().tfg_edge_softmax_aggregate(_ptr(rowptr), _ptr(col), _ptr(x), n, e, heads, channels,
+    _check(lib().tfg_edge_softmax_aggregate(_ptr(rowptr), _ptr(col), _ptr(x), _x_dtype(x), n, e,
+                                            heads, channels,
                                             _ptr(a_src), _ptr(a_dst), float(negative_slope),
                                             _ptr(out), _ptr(alpha), _ptr(workspace),
                                             workspace.numel(), _stream(dev)))

@@ -90,9 +90,11 @@ def test_gcn_norm_rejects(lib):
 
 def test_edge_softmax_rejects(lib):
     f = lib.tfg_edge_softmax_aggregate
-    assert f(FAKE, FAKE, FAKE, 10, 20, 0, 4, FAKE, FAKE, 0.2, FAKE, None, FAKE, 1 << 20, None) == -1
-    assert f(FAKE, FAKE, FAKE, 10, 20, 2, 4, None, FAKE, 0.2, FAKE, None, FAKE, 1 << 20, None) == -1
-    assert f(FAKE, FAKE, FAKE, 10, 20, 2, 4, FAKE, FAKE, 0.2, FAKE, None, FAKE, 8, None) == -3
+    assert f(FAKE, FAKE, FAKE, 0, 10, 20, 0, 4, FAKE, FAKE, 0.2, FAKE, None, FAKE, 1 << 20, None) == -1
+    assert f(FAKE, FAKE, FAKE, 0, 10, 20, 2, 4, None, FAKE, 0.2, FAKE, None, FAKE, 1 << 20, None) == -1
+    assert f(FAKE, FAKE, FAKE, 0, 10, 20, 2, 4, FAKE, FAKE, 0.2, FAKE, None, FAKE, 8, None) == -3
+    assert f(FAKE, FAKE, FAKE, 9, 10, 20, 2, 4, FAKE, FAKE, 0.2, FAKE, None, FAKE, 1 << 20, None) == -1
+    assert f(FAKE, None, FAKE, 0, 10, 20, 2, 4, FAKE, FAKE, 0.2, FAKE, None, FAKE, 1 << 20, None) == -1
 
 
 def test_segment_pool_rejects(lib):

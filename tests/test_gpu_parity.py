@@ -161,8 +161,10 @@ def test_gcn_aggregate_weighted(add_self):
 # ---------------------------------------------------------------------------
 # Edge softmax (GAT)
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("heads,channels", [(1, 1), (2, 3), (4, 4), (8, 16), (3, 48), (1, 160)])
-def test_edge_softmax(heads, channels):
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("heads,channels", [(1, 1), (2, 3), (4, 4), (8, 16), (3, 48), (1, 160),
+                                            (2, 8), (16, 8)])
+def test_edge_softmax(heads, channels, dtype):
     n, e = 3000, 25000
     f = heads * channels
     wl = gg.random_edge_case_graph(n, e, f, 31 + f, hub=9, isolated=40)
@@ -170,10 +172,12 @@ def test_edge_softmax(heads, channels):
     a_s = rng.standard_normal(f).astype(np.float32)
     a_d = rng.standard_normal(f).astype(np.float32)
     csr = gpu_csr(wl.edge_index, n)
-    out, alpha = tfg.tfg_edge_softmax_aggregate(csr.rowptr, csr.col, dev(wl.x), heads, channels,
-                                                dev(a_s), dev(a_d), 0.2, want_alpha=True)
-    ref, ref_alpha, scale = oracle.edge_softmax(wl.edge_index, n, wl.x, heads, channels, a_s, a_d, 0.2)
-    assert_scaled_close(np_(out), ref, scale, TOL_F32, f"softmax H={heads} C={channels}")
+    out, alpha = tfg.tfg_edge_softmax_aggregate(csr.rowptr, csr.col, features(wl, dtype), heads,
+                                                channels, dev(a_s), dev(a_d), 0.2, want_alpha=True)
+    ref, ref_alpha, scale = oracle.edge_softmax(wl.edge_index, n, host_features(wl, dtype), heads,
+                                                channels, a_s, a_d, 0.2)
+    # the oracle reads the same bf16 values, so fp32 arithmetic is the only error
+    assert_scaled_close(np_(out), ref, scale, TOL_F32, f"softmax {dtype} H={heads} C={channels}")
     perm = oracle.build_csr(wl.edge_index, n)[2]
     want = ref_alpha[perm]
     assert_scaled_close(np_(alpha), want, want, TOL_F32, "alpha")
@@ -202,6 +206,25 @@ def test_segment_pool(reduce, dtype, f):
         assert_exact_f32(np_(out), ref, f"pool max {dtype}")
     else:
         assert_scaled_close(np_(out), ref, scale, TOL_F32, f"pool {reduce} {dtype} F={f}")
+
+
+@pytest.mark.parametrize("reduce", ["sum", "mean", "max"])
+def test_segment_pool_large_graphs_cluster_path(reduce):
+    """Graphs of thousands of nodes: several CTAs per graph combine through
+    distributed shared memory."""
+    rng = np.random.default_rng(3)
+    sizes = rng.integers(6000, 12000, size=9)
+    sizes[4] = 0
+    batch = np.repeat(np.arange(9), sizes).astype(np.int64)
+    n, f = batch.size, 128
+    x = rng.standard_normal((n, f)).astype(np.float32)
+    out, status = tfg.tfg_segment_pool(dev(x), dev(batch), 9, reduce)
+    tfg.check_status(status)
+    ref, scale = oracle.segment_pool(x, batch, 9, reduce)
+    if reduce == "max":
+        assert_exact_f32(np_(out), ref, "cluster pool max")
+    else:
+        assert_scaled_close(np_(out), ref, scale, TOL_F32, f"cluster pool {reduce}")
 
 
 def test_segment_pool_bad_batch_sets_status():
