@@ -47,16 +47,25 @@ def needs_build() -> bool:
     return any(os.path.getmtime(p) > t for p in _deps())
 
 
-def build_library(force: bool = False, verbose: bool = False, ptxas_info: bool = False) -> str:
-    """Build libtfg.so if needed and return its path."""
-    if not force and not needs_build():
+def build_library(force: bool = False, verbose: bool = False, ptxas_info: bool = False,
+                  defines: tuple = (), lib_path: str | None = None) -> str:
+    """Build libtfg.so if needed and return its path.
+
+    ``defines`` (e.g. ("TFG_NO_PACKED_FMA",)) and ``lib_path`` build a variant
+    of the library elsewhere, for side-by-side timing; the default build
+    defines nothing.
+    """
+    out_path = lib_path or LIB_PATH
+    obj_dir = OBJ_DIR if not defines else os.path.join(OBJ_DIR, "_".join(defines))
+    if not force and not defines and lib_path is None and not needs_build():
         return LIB_PATH
     nvcc = _nvcc()
-    os.makedirs(OBJ_DIR, exist_ok=True)
+    os.makedirs(obj_dir, exist_ok=True)
     extra = ["-Xptxas", "-v"] if ptxas_info else []
+    extra += [f"-D{d}" for d in defines]
 
     def compile_one(src: str) -> str:
-        obj = os.path.join(OBJ_DIR, os.path.basename(src) + ".o")
+        obj = os.path.join(obj_dir, os.path.basename(src) + ".o")
         cmd = [nvcc, *ARCH, *NVCC_FLAGS, *extra, "-c", src, "-o", obj]
         res = subprocess.run(cmd, capture_output=True, text=True)
         if res.returncode != 0:
@@ -68,13 +77,13 @@ def build_library(force: bool = False, verbose: bool = False, ptxas_info: bool =
     srcs = sources()
     with ThreadPoolExecutor(max_workers=min(len(srcs), os.cpu_count() or 4)) as ex:
         objs = list(ex.map(compile_one, srcs))
-    tmp = LIB_PATH + ".tmp"
+    tmp = out_path + ".tmp"
     cmd = [nvcc, *ARCH, "-shared", "-o", tmp, *objs]
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError(f"link failed:\n{res.stdout}\n{res.stderr}")
-    os.replace(tmp, LIB_PATH)
-    return LIB_PATH
+    os.replace(tmp, out_path)
+    return out_path
 
 
 if __name__ == "__main__":

@@ -61,16 +61,62 @@ struct Agg {
         return kIsMax ? fmaxf(a, b) : a + b;
     }
 
+    // part[q] += w * v[q] for one gathered vector (pairs through fma2).
+    static __device__ __forceinline__ void axpy(float (&part)[VEC], float w,
+                                                const typename VecLoad<XT, VEC>::Raw &raw) {
+        float v[VEC];
+        VecLoad<XT, VEC>::widen(raw, v);
+        if constexpr (VEC % 2 == 0) {
+            const float2 w2 = make_float2(w, w);
+#pragma unroll
+            for (int q = 0; q < VEC; q += 2) {
+                const float2 r = fma2(make_float2(v[q], v[q + 1]), w2, make_float2(part[q], part[q + 1]));
+                part[q] = r.x;
+                part[q + 1] = r.y;
+            }
+        } else {
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) part[q] = fmaf(w, v[q], part[q]);
+        }
+    }
+
+    // One 32-edge chunk of a sum: group g takes edges g, g + G, ...  FULL
+    // chunks need no bounds checks; in a partial chunk the slots past cnt get
+    // weight 0 and read row 0 (always valid), contributing an exact zero.
+    // Lanes whose features lie past F read the row's first features instead
+    // (in bounds); their partials are never stored.
+    template <bool FULL>
+    static __device__ __forceinline__ void sum_chunk(const XT *xf, uint32_t fs, int c, float ww,
+                                                     int cnt, int g, bool weighted,
+                                                     float (&part)[VEC]) {
+        using V = VecLoad<XT, VEC>;
+        for (int j = 0; j < (FULL ? 32 : cnt); j += G * kUnroll) {
+            typename V::Raw raw[kUnroll];
+            float wt[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int k = j + u * G + g;
+                const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31));
+                wt[u] = weighted ? __shfl_sync(kFull, ww, k & 31) : 1.f;
+                if (!FULL && k >= cnt) wt[u] = 0.f;
+                raw[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
+            }
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) axpy(part, wt[u], raw[u]);
+        }
+    }
+
     // Accumulate edges [beg, end) into acc (this lane's VEC features at f0).
     // Each 32-edge chunk is summed into its own partial before it is added to
     // acc, so an fp32 chain is at most 32 / G + deg / 32 additions long.  The
-    // order is fixed.  Out-of-range slots contribute an exact zero (weight 0,
-    // value 0) instead of a branch, except for max.
+    // order is fixed, so results are deterministic.
     static __device__ __forceinline__ void edges(const AggArgs &a, int64_t beg, int64_t end,
                                                  int64_t f0, bool fok, float (&acc)[VEC],
                                                  int lane) {
         using V = VecLoad<XT, VEC>;
         const XT *x = static_cast<const XT *>(a.x);
+        const XT *xf = x + (fok ? f0 : 0);
+        const uint32_t fs = static_cast<uint32_t>(a.f);
         const int g = lane / LPR;
         const bool weighted = KIND == kGcn || a.w != nullptr;
         if (a.col == nullptr) return;   // a graph without edges
@@ -83,38 +129,34 @@ struct Agg {
                 if (a.w) ww = __ldg(a.w + base + lane);
                 else if (KIND == kGcn) ww = __ldg(a.dinv + c);
             }
-            float part[VEC];
+            if constexpr (kIsMax) {
+                for (int j = 0; j < cnt; j += G * kUnroll) {
+                    typename V::Raw raw[kUnroll];
+                    float wt[kUnroll];
+                    bool ok[kUnroll];
 #pragma unroll
-            for (int q = 0; q < VEC; ++q) part[q] = 0.f;
-            for (int j = 0; j < cnt; j += G * kUnroll) {
-                typename V::Raw raw[kUnroll];
-                float wt[kUnroll];
-                bool ok[kUnroll];
+                    for (int u = 0; u < kUnroll; ++u) {
+                        const int k = j + u * G + g;
+                        const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31));
+                        wt[u] = weighted ? __shfl_sync(kFull, ww, k & 31) : 1.f;
+                        ok[u] = fok && (k < cnt);
+                        raw[u] = ok[u] ? V::raw(xf + static_cast<uint64_t>(src) * fs) : V::zero();
+                    }
 #pragma unroll
-                for (int u = 0; u < kUnroll; ++u) {
-                    const int k = j + u * G + g;
-                    const int src = __shfl_sync(kFull, c, k & 31);
-                    wt[u] = weighted ? __shfl_sync(kFull, ww, k & 31) : 1.f;
-                    ok[u] = fok && (k < cnt);
-                    raw[u] = ok[u] ? V::raw(x + static_cast<int64_t>(src) * a.f + f0) : V::zero();
-                    if (!kIsMax && !ok[u]) wt[u] = 0.f;
-                }
+                    for (int u = 0; u < kUnroll; ++u) {
+                        if (!ok[u]) continue;
+                        float v[VEC];
+                        V::widen(raw[u], v);
 #pragma unroll
-                for (int u = 0; u < kUnroll; ++u) {
-                    float v[VEC];
-                    V::widen(raw[u], v);
-                    if (kIsMax) {
-                        if (ok[u]) {
-#pragma unroll
-                            for (int q = 0; q < VEC; ++q) acc[q] = fmaxf(acc[q], wt[u] * v[q]);
-                        }
-                    } else {
-#pragma unroll
-                        for (int q = 0; q < VEC; ++q) part[q] = fmaf(wt[u], v[q], part[q]);
+                        for (int q = 0; q < VEC; ++q) acc[q] = fmaxf(acc[q], wt[u] * v[q]);
                     }
                 }
-            }
-            if (!kIsMax) {
+            } else {
+                float part[VEC];
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) part[q] = 0.f;
+                if (cnt == 32) sum_chunk<true>(xf, fs, c, ww, cnt, g, weighted, part);
+                else sum_chunk<false>(xf, fs, c, ww, cnt, g, weighted, part);
 #pragma unroll
                 for (int q = 0; q < VEC; ++q) acc[q] += part[q];
             }

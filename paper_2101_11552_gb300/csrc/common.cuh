@@ -65,6 +65,23 @@ template <> struct VecLoad<uint16_t, 1> {
     static __device__ __forceinline__ void load(const uint16_t *p, float (&v)[1]) { widen(raw(p), v); }
 };
 
+// acc += a * b on a pair of fp32 lanes: one packed fma.rn.f32x2 on sm_100+
+// (each half is an ordinary correctly rounded fp32 fma, so the result is
+// bit-identical to two fmaf calls).  TFG_NO_PACKED_FMA selects the scalar form.
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+#if !defined(TFG_NO_PACKED_FMA)
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+        "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+#else
+    return make_float2(fmaf(a.x, b.x, c.x), fmaf(a.y, b.y, c.y));
+#endif
+}
+
 __host__ __device__ constexpr int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 __host__ __device__ constexpr int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
 

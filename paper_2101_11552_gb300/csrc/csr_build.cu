@@ -21,8 +21,7 @@ namespace {
 
 constexpr int kSortWarps = 8;
 constexpr int kSortThreads = kSortWarps * 32;
-constexpr int kItems = 32;                        // per lane
-constexpr int kTile = kSortThreads * kItems;      // 8192 edges per CTA
+constexpr int kTile = 4096;                       // edges per CTA tile
 constexpr int kMaxDigitBits = 10;
 constexpr int kScanThreads = 256;
 constexpr int kScanItems = 16;
@@ -74,13 +73,14 @@ radix_upsweep(const int64_t *__restrict__ dst64, const uint32_t *__restrict__ ke
         hist[static_cast<int64_t>(d) * num_tiles + blockIdx.x] = s_cnt[d];
 }
 
-// Downsweep: 32 warps share one 8192-edge tile, 8 elements per lane.
+// Downsweep: 16 warps share one 4096-edge tile, 8 elements per lane.
 // Elements are ranked inside the tile (stable: warp-major, then round, then
 // lane = original order), staged in shared memory in digit order, and then
 // written out by consecutive threads, so each digit's run of the tile leaves
 // as coalesced stores.  The key array and each value array are staged in
-// turn through one value buffer to fit the tile in shared memory.
-constexpr int kDsWarps = 32;
+// turn through one value buffer; two CTAs fit on an SM, so one CTA's
+// global loads overlap the other's shared-memory phases.
+constexpr int kDsWarps = 16;
 constexpr int kDsThreads = kDsWarps * 32;
 constexpr int kDsItems = kTile / kDsThreads;   // 8 per lane
 
@@ -90,7 +90,7 @@ size_t downsweep_smem(int radix) {
 }
 
 template <bool FIRST>
-__global__ void __launch_bounds__(kDsThreads, 1)
+__global__ void __launch_bounds__(kDsThreads, 2)
 radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ dst64,
                 const uint32_t *__restrict__ key_in, const int32_t *__restrict__ src_in,
                 const int32_t *__restrict__ eid_in, int64_t e, int64_t n, int shift, int width,
@@ -143,14 +143,15 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     if (warp == 0) {   // exclusive scan of s_tstart[0 .. radix) by one warp
         int carry = 0;
         for (int base = 0; base < radix; base += 32) {
-            const int v = s_tstart[base + lane];
+            const bool in = base + lane < radix;   // radix may be < 32
+            const int v = in ? s_tstart[base + lane] : 0;
             int incl = v;
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
                 const int y = __shfl_up_sync(kFull, incl, o);
                 if (lane >= o) incl += y;
             }
-            s_tstart[base + lane] = carry + incl - v;
+            if (in) s_tstart[base + lane] = carry + incl - v;
             carry += __shfl_sync(kFull, incl, 31);
         }
     }
@@ -158,7 +159,7 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
 
     // Phase C: tile-local slot of every element (stable), keys staged.
     const unsigned lower = (1u << lane) - 1u;
-    uint32_t slots[kDsItems / 2];   // two 13-bit tile slots per register
+    uint32_t slots[kDsItems / 2];   // two 12-bit tile slots per register
 #pragma unroll
     for (int r = 0; r < kDsItems; ++r) {
         const int64_t idx = wbase + r * 32 + lane;

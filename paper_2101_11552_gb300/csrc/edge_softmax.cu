@@ -154,7 +154,171 @@ softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict_
     }
 }
 
+// Fast form for the common layout: H divides 32, every lane's VEC features
+// lie in one head, and one feature tile covers the row (F <= LPR * VEC).
+// Two passes over the row, no data-dependent branches:
+//  * score lanes: lane (se, sh) = (lane / H, lane % H) evaluates the logit of
+//    edge slot se and head sh -- each (edge, head) logit and exponential is
+//    computed once.  Pass 1 takes the row maximum per head (butterfly over
+//    the lanes of a head); pass 2 forms p = exp(l - m) and the denominator.
+//  * feature lanes: group g = lane / LPR gathers every G-th edge, fetches the
+//    p of its (edge, head) from the score lane holding it with one shuffle,
+//    and accumulates p * x into fp32 per-chunk partials.
+template <typename XT, int VEC, int LPR, int H>
+__global__ void __launch_bounds__(kSmThreads, 3)
+softmax_fast(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,
+             const XT *__restrict__ x, int64_t n, int channels, float slope,
+             const float *__restrict__ s_src, const float *__restrict__ s_dst,
+             float *__restrict__ out, float *__restrict__ alpha) {
+    using V = VecLoad<XT, VEC>;
+    constexpr int G = 32 / LPR;     // edges per feature step
+    constexpr int ES = 32 / H;      // edges per score step
+    constexpr int R = 32 / ES;      // score steps per 32-edge chunk (= H)
+    static_assert(ES % G == 0, "score step must hold whole feature steps");
+    const int64_t t = (static_cast<int64_t>(blockIdx.x) * kSmThreads + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (t >= n) return;
+    const int se = lane / H, sh = lane % H;
+    const int g = lane / LPR, sub = lane % LPR;
+    const int f = H * channels;
+    const int f0 = sub * VEC;
+    const bool fok = f0 < f;
+    const int fh = fok ? f0 / channels : 0;
+    const XT *xf = x + (fok ? f0 : 0);
+    const uint32_t fs = static_cast<uint32_t>(f);
+    const int64_t beg = rowptr[t], end = col ? rowptr[t + 1] : rowptr[t];
+    const float sd = __ldg(s_dst + t * H + sh);
+
+    // pass 1: row maximum of every head
+    float m = -CUDART_INF_F;
+    for (int64_t base = beg; base < end; base += 32) {
+        const int cnt = static_cast<int>(min64(32, end - base));
+        const int c = lane < cnt ? __ldg(col + base + lane) : 0;
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const int k = r * ES + se;
+            const int src = __shfl_sync(kFull, c, k);
+            if (k < cnt) m = fmaxf(m, leaky(__ldg(s_src + static_cast<int64_t>(src) * H + sh) + sd, slope));
+        }
+    }
+#pragma unroll
+    for (int o = H; o < 32; o <<= 1) m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
+
+    // pass 2: p, denominator, and the p-weighted feature sum
+    float den = 0.f, acc[VEC];
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
+    for (int64_t base = beg; base < end; base += 32) {
+        const int cnt = static_cast<int>(min64(32, end - base));
+        const int c = lane < cnt ? __ldg(col + base + lane) : 0;
+        float p[R];
+        float den_part = 0.f;
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const int k = r * ES + se;
+            const int src = __shfl_sync(kFull, c, k);
+            p[r] = 0.f;
+            if (k < cnt)
+                p[r] = __expf(leaky(__ldg(s_src + static_cast<int64_t>(src) * H + sh) + sd, slope) - m);
+            den_part += p[r];
+        }
+        den += den_part;
+        float part[VEC];
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) part[q] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 32; e += G * kSmUnroll) {
+            if (e >= cnt) break;   // warp-uniform
+            typename V::Raw raw[kSmUnroll];
+            float pw[kSmUnroll];
+#pragma unroll
+            for (int u = 0; u < kSmUnroll; ++u) {
+                const int k0 = e + u * G;              // edge of group 0 in this step
+                const int k = k0 + g;
+                const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31));
+                // p of (edge k, head fh) sits in lane (k % ES) * H + fh, register k / ES
+                pw[u] = __shfl_sync(kFull, p[k0 / ES], ((k0 % ES) + g) * H + fh);
+                raw[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
+            }
+#pragma unroll
+            for (int u = 0; u < kSmUnroll; ++u) {
+                float v[VEC];
+                V::widen(raw[u], v);
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) part[q] = fmaf(pw[u], v[q], part[q]);
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) acc[q] += part[q];
+    }
+#pragma unroll
+    for (int o = H; o < 32; o <<= 1) den += __shfl_xor_sync(kFull, den, o);
+#pragma unroll
+    for (int o = LPR; o < 32; o <<= 1)
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) acc[q] += __shfl_xor_sync(kFull, acc[q], o);
+    const float dh = __shfl_sync(kFull, den, fh);   // lane fh holds head fh's denominator
+    if (lane < LPR && fok) {
+        float *o = out + t * f + f0;
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) o[q] = end > beg ? acc[q] / dh : 0.f;
+    }
+    if (alpha) {
+        for (int64_t base = beg; base < end; base += 32) {
+            const int cnt = static_cast<int>(min64(32, end - base));
+            const int c = lane < cnt ? __ldg(col + base + lane) : 0;
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                const int k = r * ES + se;
+                const int src = __shfl_sync(kFull, c, k);
+                if (k < cnt) {
+                    const float l = leaky(__ldg(s_src + static_cast<int64_t>(src) * H + sh) + sd, slope);
+                    alpha[(base + k) * H + sh] = __expf(l - m) / den;
+                }
+            }
+        }
+    }
+}
+
 size_t align256(size_t b) { return (b + 255) & ~size_t(255); }
+
+// Launch the fast form when the layout allows it; false means "use the generic one".
+template <typename XT, int VEC, int LPR>
+bool launch_fast_lpr(const int32_t *rowptr, const int32_t *col, const void *x, int64_t n, int heads,
+                     int channels, float slope, const float *s_src, const float *s_dst, float *out,
+                     float *alpha, cudaStream_t s) {
+    constexpr int G = 32 / LPR;
+    const int grid = ceil_div(n * 32, kSmThreads);
+    const XT *xp = static_cast<const XT *>(x);
+#define TFG_FAST(HH)                                                                              \
+    if (heads == HH) {                                                                            \
+        if constexpr ((32 / HH) % G == 0) {                                                       \
+            softmax_fast<XT, VEC, LPR, HH><<<grid, kSmThreads, 0, s>>>(rowptr, col, xp, n, channels, \
+                                                                       slope, s_src, s_dst, out, alpha); \
+            return true;                                                                          \
+        }                                                                                         \
+        return false;                                                                             \
+    }
+    TFG_FAST(1)
+    TFG_FAST(2)
+    TFG_FAST(4)
+    TFG_FAST(8)
+    TFG_FAST(16)
+#undef TFG_FAST
+    return false;
+}
+
+template <typename XT, int VEC>
+bool launch_fast(const int32_t *rowptr, const int32_t *col, const void *x, int64_t n, int heads,
+                 int channels, float slope, const float *s_src, const float *s_dst, float *out,
+                 float *alpha, cudaStream_t s) {
+    const int64_t f = static_cast<int64_t>(heads) * channels;
+    if (channels % VEC != 0 || f > 32 * VEC) return false;
+    const int64_t chunks = f / VEC;
+    if (chunks > 16) return launch_fast_lpr<XT, VEC, 32>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+    if (chunks > 8) return launch_fast_lpr<XT, VEC, 16>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+    return launch_fast_lpr<XT, VEC, 8>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+}
 
 template <typename XT, int VEC>
 void launch_main(const int32_t *rowptr, const int32_t *col, const void *x, int64_t n, int heads,
@@ -194,17 +358,21 @@ cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const
     if (x_dtype == TFG_BF16) {
         node_scores<uint16_t><<<sgrid, 256, 0, s>>>(static_cast<const uint16_t *>(x), n, heads,
                                                     channels, a_src, a_dst, s_src, s_dst);
-        if (aligned && channels % 8 == 0)
-            launch_main<uint16_t, 8>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
-        else
+        if (aligned && channels % 8 == 0) {
+            if (!launch_fast<uint16_t, 8>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s))
+                launch_main<uint16_t, 8>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+        } else {
             launch_main<uint16_t, 1>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+        }
     } else {
         node_scores<float><<<sgrid, 256, 0, s>>>(static_cast<const float *>(x), n, heads, channels,
                                                  a_src, a_dst, s_src, s_dst);
-        if (aligned && channels % 4 == 0)
-            launch_main<float, 4>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
-        else
+        if (aligned && channels % 4 == 0) {
+            if (!launch_fast<float, 4>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s))
+                launch_main<float, 4>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+        } else {
             launch_main<float, 1>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+        }
     }
     return cudaGetLastError();
 }
