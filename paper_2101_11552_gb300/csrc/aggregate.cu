@@ -6,8 +6,10 @@
 // bit-identical results from run to run.
 //
 // Work layout
-//  * A CTA (8 warps) owns kRowsPerCta consecutive target rows.  Its warps take
-//    rows one at a time from a shared counter.  A row is split among
+//  * A CTA (8 warps) owns a contiguous range of target rows holding an equal
+//    share of edges + rows (a merge-path split of rowptr), so a hub row does
+//    not leave one CTA running long after the others.  Its warps take rows
+//    one at a time from a shared counter.  A row is split among
 //    G = 32 / LPR lane groups: each group of LPR lanes covers LPR * VEC
 //    features (16-byte loads when the layout allows) and takes every G-th
 //    edge of the row; the groups' partials are then combined by a butterfly.
@@ -30,9 +32,16 @@ namespace {
 
 constexpr int kAggWarps = 8;
 constexpr int kAggThreads = kAggWarps * 32;
-constexpr int kRowsPerCta = 64;
-constexpr int kHeavyDeg = 2048;
-constexpr int kUnroll = 4;
+// Tuning knobs (compile-time; the defaults are the measured best on GB300).
+#ifndef TFG_HEAVY_DEG
+#define TFG_HEAVY_DEG 2048
+#endif
+#ifndef TFG_AGG_UNROLL
+#define TFG_AGG_UNROLL 4
+#endif
+constexpr int kHeavyDeg = TFG_HEAVY_DEG;
+constexpr int kMaxHeavy = 64;   // hub rows a CTA sets aside; more are done warp by warp
+constexpr int kUnroll = TFG_AGG_UNROLL;
 
 struct AggArgs {
     const int32_t *rowptr;
@@ -260,10 +269,11 @@ template <typename XT, int VEC, int LPR, int KIND>
 __global__ void __launch_bounds__(kAggThreads, VEC >= 8 ? 3 : 4) aggregate_kernel(AggArgs a) {
     using A = Agg<XT, VEC, LPR, KIND>;
     __shared__ int s_next, s_nheavy;
-    __shared__ int s_heavy[kRowsPerCta];
+    __shared__ int64_t s_heavy[kMaxHeavy];
     __shared__ float s_part[kAggWarps * LPR * VEC];
-    const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRowsPerCta;
-    const int nrows = static_cast<int>(min64(kRowsPerCta, a.n - r0));
+    int64_t r0, r1;
+    balanced_rows(a.rowptr, a.n, gridDim.x, blockIdx.x, r0, r1);
+    const int64_t nrows = r1 - r0;
     if (threadIdx.x == 0) {
         s_next = 0;
         s_nheavy = 0;
@@ -276,20 +286,26 @@ __global__ void __launch_bounds__(kAggThreads, VEC >= 8 ? 3 : 4) aggregate_kerne
         i = __shfl_sync(kFull, i, 0);
         if (i >= nrows) break;
         const int64_t t = r0 + i;
-        if (a.rowptr[t + 1] - a.rowptr[t] > kHeavyDeg) {
-            if (lane == 0) s_heavy[atomicAdd(&s_nheavy, 1)] = i;
-            continue;
+        if (a.col != nullptr && a.rowptr[t + 1] - a.rowptr[t] > kHeavyDeg) {
+            int slot = 0;
+            if (lane == 0) slot = atomicAdd(&s_nheavy, 1);
+            slot = __shfl_sync(kFull, slot, 0);
+            if (slot < kMaxHeavy) {
+                if (lane == 0) s_heavy[slot] = t;
+                continue;
+            }
         }
         A::warp_row(a, t, lane);
     }
     __syncthreads();
-    const int nh = s_nheavy;
-    for (int h = 0; h < nh; ++h) A::cta_row(a, r0 + s_heavy[h], s_part);
+    const int nh = min(s_nheavy, kMaxHeavy);
+    for (int h = 0; h < nh; ++h) A::cta_row(a, s_heavy[h], s_part);
 }
 
 template <typename XT, int VEC, int KIND>
 cudaError_t launch_lpr(const AggArgs &a, int lpr, cudaStream_t s) {
-    const int grid = ceil_div(a.n, kRowsPerCta);
+    // E is not known on the host; the kernel reads rowptr[N] for the split.
+    const int grid = balanced_grid(a.n, 0, 1);
     switch (lpr) {
         case 32: aggregate_kernel<XT, VEC, 32, KIND><<<grid, kAggThreads, 0, s>>>(a); break;
         case 16: aggregate_kernel<XT, VEC, 16, KIND><<<grid, kAggThreads, 0, s>>>(a); break;

@@ -84,6 +84,23 @@ int aggregate_common(const char *fn, int mode, const int32_t *rowptr, const int3
 
 }  // namespace
 
+namespace tfg {
+int balanced_grid(int64_t n, int64_t e, int64_t min_work) {
+    thread_local int sms = 0, sms_dev = -1;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) dev = 0;
+    if (sms == 0 || sms_dev != dev) {
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
+            sms = 148;
+        sms_dev = dev;
+    }
+    const int64_t by_work = (n + e + min_work - 1) / min_work;
+    const int64_t cap = int64_t(sms) * 16;
+    const int64_t g = by_work < cap ? by_work : cap;
+    return static_cast<int>(g < 1 ? 1 : g);
+}
+}  // namespace tfg
+
 extern "C" {
 
 int tfg_version(void) { return 100; }
@@ -201,7 +218,7 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
         return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
                     workspace ? workspace_bytes : size_t(0));
     return cuda_result(tfg::launch_edge_softmax(rowptr, num_edges > 0 ? col : nullptr, x, x_dtype,
-                                                num_nodes, heads, channels, a_src, a_dst,
+                                                num_nodes, num_edges, heads, channels, a_src, a_dst,
                                                 negative_slope, out, alpha, workspace,
                                                 reinterpret_cast<cudaStream_t>(stream)),
                        fn);

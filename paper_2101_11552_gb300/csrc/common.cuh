@@ -85,7 +85,36 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
 __host__ __device__ constexpr int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 __host__ __device__ constexpr int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
 
+// Work-balanced row ranges.  A CTA b of nb owns the rows t whose merge-path
+// coordinate rowptr[t] + t (edges before t plus rows before t) falls in
+// [b * W, (b + 1) * W), W = ceil((E + N) / nb): every CTA gets about the same
+// number of edges plus rows, whatever the degree distribution, and every row
+// belongs to exactly one CTA.  rowptr[t] + t is strictly increasing in t.
+__device__ __forceinline__ int64_t first_row_at(const int32_t *rowptr, int64_t n, int64_t target) {
+    int64_t lo = 0, hi = n;   // first t in [0, n] with rowptr[t] + t >= target
+    while (lo < hi) {
+        const int64_t mid = (lo + hi) >> 1;
+        if (static_cast<int64_t>(__ldg(rowptr + mid)) + mid < target) lo = mid + 1;
+        else hi = mid;
+    }
+    return lo;
+}
+
+__device__ __forceinline__ void balanced_rows(const int32_t *rowptr, int64_t n, int64_t nb,
+                                              int64_t b, int64_t &r0, int64_t &r1) {
+    const int64_t total = static_cast<int64_t>(__ldg(rowptr + n)) + n;
+    const int64_t w = (total + nb - 1) / nb;
+    r0 = first_row_at(rowptr, n, b * w);
+    r1 = b + 1 == nb ? n : first_row_at(rowptr, n, (b + 1) * w);
+}
+
 }  // namespace tfg
+
+// Number of CTAs for a balanced launch over E edges and N rows: enough for
+// several resident CTAs per SM, and at least min_work units of work each.
+namespace tfg {
+int balanced_grid(int64_t n, int64_t e, int64_t min_work);
+}
 
 // Host-side launchers implemented in the kernel files; api.cu validates
 // arguments before calling them.  Each returns cudaSuccess or the launch error.
@@ -103,7 +132,7 @@ cudaError_t launch_aggregate(int mode, const int32_t *rowptr, const int32_t *col
                              int add_self, float fill, float *out, cudaStream_t s);
 size_t softmax_workspace_bytes(int64_t n, int heads);
 cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const void *x,
-                                int x_dtype, int64_t n, int heads, int channels,
+                                int x_dtype, int64_t n, int64_t e, int heads, int channels,
                                 const float *a_src, const float *a_dst, float slope, float *out,
                                 float *alpha, void *ws, cudaStream_t s);
 cudaError_t launch_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n,

@@ -26,7 +26,10 @@ namespace tfg {
 namespace {
 
 constexpr int kSmThreads = 256;
-constexpr int kSmUnroll = 4;
+#ifndef TFG_SM_UNROLL
+#define TFG_SM_UNROLL 4   // gathers in flight per lane (tuning knob)
+#endif
+constexpr int kSmUnroll = TFG_SM_UNROLL;
 
 template <typename XT>
 __global__ void node_scores(const XT *__restrict__ x, int64_t n, int heads, int channels,
@@ -57,16 +60,16 @@ __device__ __forceinline__ float rescale(float m_old, float m_new) {
 }
 
 template <typename XT, int VEC, int LPR>
-__global__ void __launch_bounds__(kSmThreads, 3)
-softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,
-                  const XT *__restrict__ x, int64_t n, int heads, int channels, float slope,
-                  const float *__restrict__ s_src, const float *__restrict__ s_dst,
-                  float *__restrict__ out, float *__restrict__ alpha) {
+__device__ __forceinline__ void generic_row(const int32_t *__restrict__ rowptr,
+                                            const int32_t *__restrict__ col,
+                                            const XT *__restrict__ x, int heads, int channels,
+                                            float slope, const float *__restrict__ s_src,
+                                            const float *__restrict__ s_dst,
+                                            float *__restrict__ out, float *__restrict__ alpha,
+                                            int64_t t, int lane) {
     using V = VecLoad<XT, VEC>;
     constexpr int G = 32 / LPR;
-    const int64_t t = (static_cast<int64_t>(blockIdx.x) * kSmThreads + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31, g = lane / LPR, sub = lane % LPR;
-    if (t >= n) return;
+    const int g = lane / LPR, sub = lane % LPR;
     const int64_t f = static_cast<int64_t>(heads) * channels;
     const int64_t beg = rowptr[t], end = col ? rowptr[t + 1] : rowptr[t];
     for (int64_t ft = 0; ft < f; ft += LPR * VEC) {
@@ -165,19 +168,17 @@ softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict_
 //    p of its (edge, head) from the score lane holding it with one shuffle,
 //    and accumulates p * x into fp32 per-chunk partials.
 template <typename XT, int VEC, int LPR, int H>
-__global__ void __launch_bounds__(kSmThreads, 3)
-softmax_fast(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,
-             const XT *__restrict__ x, int64_t n, int channels, float slope,
-             const float *__restrict__ s_src, const float *__restrict__ s_dst,
-             float *__restrict__ out, float *__restrict__ alpha) {
+__device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
+                                         const int32_t *__restrict__ col,
+                                         const XT *__restrict__ x, int channels, float slope,
+                                         const float *__restrict__ s_src,
+                                         const float *__restrict__ s_dst, float *__restrict__ out,
+                                         float *__restrict__ alpha, int64_t t, int lane) {
     using V = VecLoad<XT, VEC>;
     constexpr int G = 32 / LPR;     // edges per feature step
     constexpr int ES = 32 / H;      // edges per score step
     constexpr int R = 32 / ES;      // score steps per 32-edge chunk (= H)
     static_assert(ES % G == 0, "score step must hold whole feature steps");
-    const int64_t t = (static_cast<int64_t>(blockIdx.x) * kSmThreads + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    if (t >= n) return;
     const int se = lane / H, sh = lane % H;
     const int g = lane / LPR, sub = lane % LPR;
     const int f = H * channels;
@@ -280,15 +281,60 @@ softmax_fast(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col
     }
 }
 
+// Each CTA owns a work-balanced range of rows (edges + rows split evenly
+// across CTAs); its warps take rows one at a time from a shared counter.
+template <typename RowFn>
+__device__ __forceinline__ void for_each_row(const int32_t *rowptr, int64_t n, RowFn fn) {
+    __shared__ int s_next;
+    int64_t r0, r1;
+    balanced_rows(rowptr, n, gridDim.x, blockIdx.x, r0, r1);
+    if (threadIdx.x == 0) s_next = 0;
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    for (;;) {
+        int i = 0;
+        if (lane == 0) i = atomicAdd(&s_next, 1);
+        i = __shfl_sync(kFull, i, 0);
+        if (i >= r1 - r0) break;
+        fn(r0 + i, lane);
+    }
+}
+
+template <typename XT, int VEC, int LPR>
+__global__ void __launch_bounds__(kSmThreads, 3)
+softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,
+                  const XT *__restrict__ x, int64_t n, int heads, int channels, float slope,
+                  const float *__restrict__ s_src, const float *__restrict__ s_dst,
+                  float *__restrict__ out, float *__restrict__ alpha) {
+    for_each_row(rowptr, n, [&](int64_t t, int lane) {
+        generic_row<XT, VEC, LPR>(rowptr, col, x, heads, channels, slope, s_src, s_dst, out,
+                                  alpha, t, lane);
+    });
+}
+
+template <typename XT, int VEC, int LPR, int H>
+__global__ void __launch_bounds__(kSmThreads, 3)
+softmax_fast(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,
+             const XT *__restrict__ x, int64_t n, int channels, float slope,
+             const float *__restrict__ s_src, const float *__restrict__ s_dst,
+             float *__restrict__ out, float *__restrict__ alpha) {
+    for_each_row(rowptr, n, [&](int64_t t, int lane) {
+        fast_row<XT, VEC, LPR, H>(rowptr, col, x, channels, slope, s_src, s_dst, out, alpha, t,
+                                  lane);
+    });
+}
+
+constexpr int64_t kSmMinWork = 2048;   // edges + rows per CTA, at least
+
 size_t align256(size_t b) { return (b + 255) & ~size_t(255); }
 
 // Launch the fast form when the layout allows it; false means "use the generic one".
 template <typename XT, int VEC, int LPR>
-bool launch_fast_lpr(const int32_t *rowptr, const int32_t *col, const void *x, int64_t n, int heads,
-                     int channels, float slope, const float *s_src, const float *s_dst, float *out,
-                     float *alpha, cudaStream_t s) {
+bool launch_fast_lpr(const int32_t *rowptr, const int32_t *col, const void *x, int64_t n, int64_t e,
+                     int heads, int channels, float slope, const float *s_src, const float *s_dst,
+                     float *out, float *alpha, cudaStream_t s) {
     constexpr int G = 32 / LPR;
-    const int grid = ceil_div(n * 32, kSmThreads);
+    const int grid = balanced_grid(n, e, kSmMinWork);
     const XT *xp = static_cast<const XT *>(x);
 #define TFG_FAST(HH)                                                                              \
     if (heads == HH) {                                                                            \
@@ -309,23 +355,23 @@ bool launch_fast_lpr(const int32_t *rowptr, const int32_t *col, const void *x, i
 }
 
 template <typename XT, int VEC>
-bool launch_fast(const int32_t *rowptr, const int32_t *col, const void *x, int64_t n, int heads,
-                 int channels, float slope, const float *s_src, const float *s_dst, float *out,
-                 float *alpha, cudaStream_t s) {
+bool launch_fast(const int32_t *rowptr, const int32_t *col, const void *x, int64_t n, int64_t e,
+                 int heads, int channels, float slope, const float *s_src, const float *s_dst,
+                 float *out, float *alpha, cudaStream_t s) {
     const int64_t f = static_cast<int64_t>(heads) * channels;
     if (channels % VEC != 0 || f > 32 * VEC) return false;
     const int64_t chunks = f / VEC;
-    if (chunks > 16) return launch_fast_lpr<XT, VEC, 32>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
-    if (chunks > 8) return launch_fast_lpr<XT, VEC, 16>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
-    return launch_fast_lpr<XT, VEC, 8>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+    if (chunks > 16) return launch_fast_lpr<XT, VEC, 32>(rowptr, col, x, n, e, heads, channels, slope, s_src, s_dst, out, alpha, s);
+    if (chunks > 8) return launch_fast_lpr<XT, VEC, 16>(rowptr, col, x, n, e, heads, channels, slope, s_src, s_dst, out, alpha, s);
+    return launch_fast_lpr<XT, VEC, 8>(rowptr, col, x, n, e, heads, channels, slope, s_src, s_dst, out, alpha, s);
 }
 
 template <typename XT, int VEC>
-void launch_main(const int32_t *rowptr, const int32_t *col, const void *x, int64_t n, int heads,
-                 int channels, float slope, const float *s_src, const float *s_dst, float *out,
-                 float *alpha, cudaStream_t s) {
+void launch_main(const int32_t *rowptr, const int32_t *col, const void *x, int64_t n, int64_t e,
+                 int heads, int channels, float slope, const float *s_src, const float *s_dst,
+                 float *out, float *alpha, cudaStream_t s) {
     const int64_t chunks = static_cast<int64_t>(heads) * channels / VEC;
-    const int grid = ceil_div(n * 32, kSmThreads);
+    const int grid = balanced_grid(n, e, kSmMinWork);
     const XT *xp = static_cast<const XT *>(x);
     if (chunks >= 32)
         softmax_aggregate<XT, VEC, 32><<<grid, kSmThreads, 0, s>>>(rowptr, col, xp, n, heads, channels,
@@ -345,7 +391,7 @@ size_t softmax_workspace_bytes(int64_t n, int heads) {
 }
 
 cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const void *x,
-                                int x_dtype, int64_t n, int heads, int channels,
+                                int x_dtype, int64_t n, int64_t e, int heads, int channels,
                                 const float *a_src, const float *a_dst, float slope, float *out,
                                 float *alpha, void *ws, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
@@ -359,19 +405,19 @@ cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const
         node_scores<uint16_t><<<sgrid, 256, 0, s>>>(static_cast<const uint16_t *>(x), n, heads,
                                                     channels, a_src, a_dst, s_src, s_dst);
         if (aligned && channels % 8 == 0) {
-            if (!launch_fast<uint16_t, 8>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s))
-                launch_main<uint16_t, 8>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+            if (!launch_fast<uint16_t, 8>(rowptr, col, x, n, e, heads, channels, slope, s_src, s_dst, out, alpha, s))
+                launch_main<uint16_t, 8>(rowptr, col, x, n, e, heads, channels, slope, s_src, s_dst, out, alpha, s);
         } else {
-            launch_main<uint16_t, 1>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+            launch_main<uint16_t, 1>(rowptr, col, x, n, e, heads, channels, slope, s_src, s_dst, out, alpha, s);
         }
     } else {
         node_scores<float><<<sgrid, 256, 0, s>>>(static_cast<const float *>(x), n, heads, channels,
                                                  a_src, a_dst, s_src, s_dst);
         if (aligned && channels % 4 == 0) {
-            if (!launch_fast<float, 4>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s))
-                launch_main<float, 4>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+            if (!launch_fast<float, 4>(rowptr, col, x, n, e, heads, channels, slope, s_src, s_dst, out, alpha, s))
+                launch_main<float, 4>(rowptr, col, x, n, e, heads, channels, slope, s_src, s_dst, out, alpha, s);
         } else {
-            launch_main<float, 1>(rowptr, col, x, n, heads, channels, slope, s_src, s_dst, out, alpha, s);
+            launch_main<float, 1>(rowptr, col, x, n, e, heads, channels, slope, s_src, s_dst, out, alpha, s);
         }
     }
     return cudaGetLastError();
