@@ -37,11 +37,14 @@ constexpr int kAggThreads = kAggWarps * 32;
 #define TFG_HEAVY_DEG 2048
 #endif
 #ifndef TFG_AGG_UNROLL
-#define TFG_AGG_UNROLL 4
+#define TFG_AGG_UNROLL 8
 #endif
 constexpr int kHeavyDeg = TFG_HEAVY_DEG;
 constexpr int kMaxHeavy = 64;   // hub rows a CTA sets aside; more are done warp by warp
-constexpr int kUnroll = TFG_AGG_UNROLL;
+// gathers in flight per lane: deeper for the 16-byte bf16 sum path (measured
+// faster there), 4 elsewhere (keeps the other variants free of spills)
+template <int VEC, bool IS_MAX>
+constexpr int unroll_for() { return (VEC >= 8 && !IS_MAX) ? TFG_AGG_UNROLL : 4; }
 
 struct AggArgs {
     const int32_t *rowptr;
@@ -63,6 +66,7 @@ template <typename XT, int VEC, int LPR, int KIND>
 struct Agg {
     static constexpr int G = 32 / LPR;
     static constexpr bool kIsMax = KIND == kMax;
+    static constexpr int kUnroll = unroll_for<VEC, kIsMax>();
 
     static __device__ __forceinline__ float identity() { return kIsMax ? -CUDART_INF_F : 0.f; }
 

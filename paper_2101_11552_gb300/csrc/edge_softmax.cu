@@ -27,9 +27,31 @@ namespace {
 
 constexpr int kSmThreads = 256;
 #ifndef TFG_SM_UNROLL
-#define TFG_SM_UNROLL 4   // gathers in flight per lane (tuning knob)
+#define TFG_SM_UNROLL 8   // gathers in flight per lane (tuning knob)
 #endif
-constexpr int kSmUnroll = TFG_SM_UNROLL;
+constexpr int kSmUnroll = TFG_SM_UNROLL;   // fast kernel
+constexpr int kGenUnroll = 4;               // generic kernel
+
+// Compensated dot product (the "Dot2" scheme of Ogita, Rump and Oishi,
+// "Accurate sum and dot product", SIAM J. Sci. Comput. 2005): each product
+// is split exactly into p + e with one fma, each running sum into s + e with
+// the error-free two-sum, and the collected errors are added at the end.  The
+// result is as accurate as a dot product in twice the working precision,
+// rounded once -- node scores feed every logit, so their error would become a
+// relative error in every attention weight.
+struct Dot2 {
+    float s = 0.f, c = 0.f;
+    __device__ __forceinline__ void add(float a, float b) {
+        const float p = a * b;
+        const float pe = fmaf(a, b, -p);       // a * b = p + pe exactly
+        const float t = s + p;
+        const float z = t - s;
+        const float se = (s - (t - z)) + (p - z);  // s + p = t + se exactly
+        s = t;
+        c += pe + se;
+    }
+    __device__ __forceinline__ float value() const { return s + c; }
+};
 
 template <typename XT>
 __global__ void node_scores(const XT *__restrict__ x, int64_t n, int heads, int channels,
@@ -41,15 +63,15 @@ __global__ void node_scores(const XT *__restrict__ x, int64_t n, int heads, int 
     const int h = static_cast<int>(i % heads);
     const XT *xr = x + v * heads * channels + static_cast<int64_t>(h) * channels;
     const float *as = a_src + h * channels, *ad = a_dst + h * channels;
-    float a = 0.f, b = 0.f;
+    Dot2 a, b;
     for (int c = 0; c < channels; ++c) {
         float xv[1];
         VecLoad<XT, 1>::load(xr + c, xv);
-        a = fmaf(xv[0], __ldg(as + c), a);
-        b = fmaf(xv[0], __ldg(ad + c), b);
+        a.add(xv[0], __ldg(as + c));
+        b.add(xv[0], __ldg(ad + c));
     }
-    s_src[i] = a;
-    s_dst[i] = b;
+    s_src[i] = a.value();
+    s_dst[i] = b.value();
 }
 
 __device__ __forceinline__ float leaky(float v, float slope) { return v > 0.f ? v : slope * v; }
@@ -88,11 +110,11 @@ __device__ __forceinline__ void generic_row(const int32_t *__restrict__ rowptr,
             float den_part = 0.f, part[VEC];
 #pragma unroll
             for (int q = 0; q < VEC; ++q) part[q] = 0.f;
-            for (int j = 0; j < cnt; j += G * kSmUnroll) {
-                float l[kSmUnroll];
-                typename V::Raw raw[kSmUnroll];
+            for (int j = 0; j < cnt; j += G * kGenUnroll) {
+                float l[kGenUnroll];
+                typename V::Raw raw[kGenUnroll];
 #pragma unroll
-                for (int u = 0; u < kSmUnroll; ++u) {
+                for (int u = 0; u < kGenUnroll; ++u) {
                     const int k = j + u * G + g;
                     const int src = __shfl_sync(kFull, c, k & 31);
                     const bool ok = k < cnt;
@@ -101,7 +123,7 @@ __device__ __forceinline__ void generic_row(const int32_t *__restrict__ rowptr,
                     raw[u] = (ok && fok) ? V::raw(x + static_cast<int64_t>(src) * f + f0) : V::zero();
                 }
 #pragma unroll
-                for (int u = 0; u < kSmUnroll; ++u) {
+                for (int u = 0; u < kGenUnroll; ++u) {
                     if (l[u] == -CUDART_INF_F) continue;   // empty slot
                     if (l[u] > m) {                        // new running maximum
                         const float sc = rescale(m, l[u]);
