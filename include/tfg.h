@@ -195,6 +195,36 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
                                size_t workspace_bytes, tfg_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Edge-softmax aggregation that allocates nothing and takes no workspace.
+ * This entry point has no counterpart in the paper; it is a library
+ * convenience.
+ *
+ * Some callers cannot allocate device memory at the time of the call: code
+ * being recorded into a CUDA graph (a cudaMalloc there breaks the capture),
+ * plugins whose host application owns all device memory and hands out none,
+ * and real-time pipelines whose memory budget is fixed before they start.
+ * For them, the node-score scratch that tfg_edge_softmax_aggregate takes
+ * as a workspace lives here in a fixed array inside the library: 16 MiB,
+ * enough for num_nodes * heads <= 2,097,152 (node, head) pairs, held on
+ * every GPU that loads the library until the process exits.  Larger inputs
+ * return TFG_ERR_TOO_LARGE; use tfg_edge_softmax_aggregate for them.
+ *
+ * Arguments, layout and results are those of tfg_edge_softmax_aggregate
+ * without the workspace.  Nothing is allocated or freed by any call.
+ * The first call on each device looks up the array's device address (which
+ * may load the library's GPU code), so make that first call outside any
+ * stream capture.  All calls on a device share the one array, and each call
+ * overwrites it: calls that may overlap on the GPU (different streams,
+ * different host threads) race with each other and must be serialised by the
+ * caller.
+ * ---------------------------------------------------------------------- */
+int tfg_edge_softmax_aggregate_noalloc(const int32_t *rowptr, const int32_t *col, const void *x,
+                                       int x_dtype, int64_t num_nodes, int64_t num_edges,
+                                       int heads, int channels, const float *a_src,
+                                       const float *a_dst, float negative_slope, float *out,
+                                       float *alpha, tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * Graph pooling keyed by node_graph_index (Section 2.1.1 BatchGraph; Fig. 2a
  * common graph pooling):
  *   out[g, :] = REDUCE over nodes v with batch[v] == g of x[v, :]

@@ -224,6 +224,43 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
                        fn);
 }
 
+int tfg_edge_softmax_aggregate_noalloc(const int32_t *rowptr, const int32_t *col, const void *x,
+                                       int x_dtype, int64_t num_nodes, int64_t num_edges,
+                                       int heads, int channels, const float *a_src,
+                                       const float *a_dst, float negative_slope, float *out,
+                                       float *alpha, tfg_stream_t stream) {
+    const char *fn = "tfg_edge_softmax_aggregate_noalloc";
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    if (heads < 1 || channels < 1)
+        return fail(TFG_ERR_INVALID_ARG, "%s: heads and channels must be >= 1", fn);
+    const int64_t limit = tfg::noalloc_softmax_max_node_heads();
+    if (num_nodes * heads > limit)
+        return fail(TFG_ERR_TOO_LARGE,
+                    "%s: num_nodes * heads = %lld exceeds the built-in scratch of %lld node-head "
+                    "pairs; use tfg_edge_softmax_aggregate with a caller workspace",
+                    fn, (long long)(num_nodes * heads), (long long)limit);
+    TFG_TRY(check_features(fn, num_nodes, int64_t(heads) * channels));
+    TFG_TRY(check_dtype(fn, x_dtype));
+    TFG_NEED(rowptr, true, fn, "rowptr");
+    TFG_NEED(col, num_edges > 0, fn, "col");
+    TFG_NEED(x, num_nodes > 0, fn, "x");
+    TFG_NEED(out, num_nodes > 0, fn, "out");
+    TFG_NEED(a_src, true, fn, "a_src");
+    TFG_NEED(a_dst, true, fn, "a_dst");
+    if (num_nodes == 0) return ok();
+    void *scratch = nullptr;
+    size_t scratch_bytes = 0;
+    cudaError_t err = tfg::noalloc_softmax_scratch(&scratch, &scratch_bytes);
+    if (err != cudaSuccess) return cuda_result(err, fn);
+    if (tfg::softmax_workspace_bytes(num_nodes, heads) > scratch_bytes)
+        return fail(TFG_ERR_TOO_LARGE, "%s: scratch too small", fn);
+    return cuda_result(tfg::launch_edge_softmax(rowptr, num_edges > 0 ? col : nullptr, x, x_dtype,
+                                                num_nodes, num_edges, heads, channels, a_src, a_dst,
+                                                negative_slope, out, alpha, scratch,
+                                                reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
 int tfg_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t num_nodes,
                      int64_t num_graphs, int64_t num_features, int reduce, float *out,
                      int32_t *status, tfg_stream_t stream) {

@@ -135,6 +135,8 @@ cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const
                                 int x_dtype, int64_t n, int64_t e, int heads, int channels,
                                 const float *a_src, const float *a_dst, float slope, float *out,
                                 float *alpha, void *ws, cudaStream_t s);
+int64_t noalloc_softmax_max_node_heads();
+cudaError_t noalloc_softmax_scratch(void **ptr, size_t *bytes);
 cudaError_t launch_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n,
                                 int64_t g, int64_t f, int reduce, float *out, int32_t *status,
                                 cudaStream_t s);

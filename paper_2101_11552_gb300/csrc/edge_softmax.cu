@@ -20,6 +20,8 @@
 // alpha requested, a second pass over the row writes the normalised weights.
 #include <math_constants.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 namespace tfg {
@@ -406,7 +408,41 @@ void launch_main(const int32_t *rowptr, const int32_t *col, const void *x, int64
                                                                   slope, s_src, s_dst, out, alpha);
 }
 
+// Scratch of tfg_edge_softmax_aggregate_noalloc: the node scores s_src and
+// s_dst of up to kNoAllocNodeHeads (node, head) pairs each, 16 MiB in all,
+// resident on every GPU that loads the library for as long as it stays
+// loaded.  Every call overwrites the part it uses, so nothing needs clearing.
+constexpr int64_t kNoAllocNodeHeads = int64_t(1) << 21;
+__device__ __align__(256) float g_noalloc_scores[2 * kNoAllocNodeHeads];
+
 }  // namespace
+
+int64_t noalloc_softmax_max_node_heads() { return kNoAllocNodeHeads; }
+
+// Device address of the scratch array on the current device.  Host code
+// cannot use the array's name as a device pointer, so the address is looked
+// up once per device with that device current (the lookup may load the
+// module, which is why the first call on a device must not be captured into
+// a CUDA graph) and cached.
+cudaError_t noalloc_softmax_scratch(void **ptr, size_t *bytes) {
+    constexpr int kMaxDevices = 64;
+    static std::mutex mu;
+    static void *addr[kMaxDevices] = {};
+    int dev = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return err;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (addr[dev] == nullptr) {
+        void *p = nullptr;
+        err = cudaGetSymbolAddress(&p, g_noalloc_scores);
+        if (err != cudaSuccess) return err;
+        addr[dev] = p;
+    }
+    *ptr = addr[dev];
+    *bytes = sizeof(g_noalloc_scores);
+    return cudaSuccess;
+}
 
 size_t softmax_workspace_bytes(int64_t n, int heads) {
     return 2 * align256(sizeof(float) * size_t(n > 0 ? n : 1) * size_t(heads));

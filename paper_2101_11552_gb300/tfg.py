@@ -65,6 +65,7 @@ def lib() -> ctypes.CDLL:
                 "tfg_gcn_aggregate_sum": [P, P, P, P, P, I, I64, I64, I, F, P, P],
                 "tfg_edge_softmax_workspace_size": [I64, I, ctypes.POINTER(SZ)],
                 "tfg_edge_softmax_aggregate": [P, P, P, I, I64, I64, I, I, P, P, F, P, P, P, SZ, P],
+                "tfg_edge_softmax_aggregate_noalloc": [P, P, P, I, I64, I64, I, I, P, P, F, P, P, P],
                 "tfg_segment_pool": [P, I, P, I64, I64, I64, I, P, P, P],
             }
             for name, args in sigs.items():
@@ -260,6 +261,31 @@ def tfg_edge_softmax_aggregate(rowptr, col, x, heads: int, channels: int, a_src,
                                             _ptr(a_src), _ptr(a_dst), float(negative_slope),
                                             _ptr(out), _ptr(alpha), _ptr(workspace),
                                             workspace.numel(), _stream(dev)))
+    return out, alpha
+
+
+def tfg_edge_softmax_aggregate_noalloc(rowptr, col, x, heads: int, channels: int, a_src, a_dst,
+                                       negative_slope: float = 0.2, out=None, alpha=None):
+    """Edge-softmax aggregation through the entry point that allocates nothing.
+
+    The library keeps the node scores in its own fixed device array, so the
+    C call takes no workspace; ``out`` (and ``alpha`` if wanted) may be passed
+    in preallocated so that nothing at all is allocated.  Returns
+    (out, alpha)."""
+    _need_cuda("rowptr", rowptr, torch.int32)
+    dev = rowptr.device
+    _need_cuda("col", col, torch.int32, dev)
+    _need_cuda("x", x, None, dev)
+    _need_cuda("a_src", a_src, torch.float32, dev)
+    _need_cuda("a_dst", a_dst, torch.float32, dev)
+    n, f = x.shape
+    if f != heads * channels:
+        raise ValueError("x must have heads * channels columns")
+    if out is None:
+        out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    _check(lib().tfg_edge_softmax_aggregate_noalloc(
+        _ptr(rowptr), _ptr(col), _ptr(x), _x_dtype(x), n, col.numel(), heads, channels,
+        _ptr(a_src), _ptr(a_dst), float(negative_slope), _ptr(out), _ptr(alpha), _stream(dev)))
     return out, alpha
 
 
