@@ -74,18 +74,17 @@ radix_upsweep(const int64_t *__restrict__ dst64, const uint32_t *__restrict__ ke
 }
 
 // Downsweep: 16 warps share one 4096-edge tile, 8 elements per lane.
-// Elements are ranked inside the tile (stable: warp-major, then round, then
-// lane = original order), staged in shared memory in digit order, and then
-// written out by consecutive threads, so each digit's run of the tile leaves
-// as coalesced stores.  The key array and each value array are staged in
-// turn through one value buffer; two CTAs fit on an SM, so one CTA's
-// global loads overlap the other's shared-memory phases.
+// Every global load of the tile (keys and both value arrays) is issued up
+// front, so the tile waits on memory once.  Elements are then ranked inside
+// the tile (stable: warp-major, then round, then lane = original order),
+// staged in shared memory in digit order, and written out by consecutive
+// threads, so each digit's run of the tile leaves as coalesced stores.
 constexpr int kDsWarps = 16;
 constexpr int kDsThreads = kDsWarps * 32;
 constexpr int kDsItems = kTile / kDsThreads;   // 8 per lane
 
 size_t downsweep_smem(int radix) {
-    return sizeof(uint32_t) * 2 * kTile + sizeof(uint16_t) * kDsWarps * radix +
+    return sizeof(uint32_t) * 3 * kTile + sizeof(uint16_t) * kDsWarps * radix +
            sizeof(int32_t) * 2 * radix;
 }
 
@@ -99,8 +98,9 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     extern __shared__ __align__(16) unsigned char smem[];
     const int radix = 1 << width;
     uint32_t *s_key = reinterpret_cast<uint32_t *>(smem);
-    int32_t *s_val = reinterpret_cast<int32_t *>(s_key + kTile);
-    uint16_t *s_cnt = reinterpret_cast<uint16_t *>(s_val + kTile);   // [warp][digit]
+    int32_t *s_src = reinterpret_cast<int32_t *>(s_key + kTile);
+    int32_t *s_eid = s_src + kTile;
+    uint16_t *s_cnt = reinterpret_cast<uint16_t *>(s_eid + kTile);   // [warp][digit]
     int32_t *s_tstart = reinterpret_cast<int32_t *>(s_cnt + kDsWarps * radix);
     int32_t *s_gbase = s_tstart + radix;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -108,19 +108,36 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     const int count = static_cast<int>(min64(kTile, e - tile0));
     uint16_t *mine = s_cnt + warp * radix;
     for (int d = lane; d < radix; d += 32) mine[d] = 0;
-    __syncwarp();
 
-    // Phase A: per-warp digit counts over the warp's contiguous sub-tile.
+    // All loads of this warp's sub-tile, issued together.
     const int64_t wbase = tile0 + static_cast<int64_t>(warp) * 32 * kDsItems;
     uint32_t keys[kDsItems];
+    int32_t srcs[kDsItems], eids[kDsItems];
 #pragma unroll
     for (int r = 0; r < kDsItems; ++r) {
         const int64_t idx = wbase + r * 32 + lane;
-        const bool ok = idx < e;
-        uint32_t key = 0;
-        if (ok) key = FIRST ? checked_id(__ldg(dst64 + idx), n, nullptr) : __ldg(key_in + idx);
-        keys[r] = key;
-        const uint32_t dig = ok ? ((key >> shift) & (radix - 1)) : uint32_t(radix);
+        keys[r] = 0;
+        srcs[r] = 0;
+        eids[r] = 0;
+        if (idx < e) {
+            if (FIRST) {
+                keys[r] = checked_id(__ldg(dst64 + idx), n, nullptr);
+                srcs[r] = static_cast<int32_t>(checked_id(__ldg(src64 + idx), n, status));
+                eids[r] = static_cast<int32_t>(idx);
+            } else {
+                keys[r] = __ldg(key_in + idx);
+                srcs[r] = __ldg(src_in + idx);
+                eids[r] = __ldg(eid_in + idx);
+            }
+        }
+    }
+    __syncwarp();
+
+    // Phase A: per-warp digit counts over the warp's contiguous sub-tile.
+#pragma unroll
+    for (int r = 0; r < kDsItems; ++r) {
+        const bool ok = wbase + r * 32 + lane < e;
+        const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
         const unsigned peers = __match_any_sync(kFull, dig);
         if (ok && lane == __ffs(peers) - 1) mine[dig] += static_cast<uint16_t>(__popc(peers));
         __syncwarp();
@@ -157,47 +174,34 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     }
     __syncthreads();
 
-    // Phase C: tile-local slot of every element (stable), keys staged.
+    // Phase C: tile-local slot of every element (stable); stage all arrays.
     const unsigned lower = (1u << lane) - 1u;
-    uint32_t slots[kDsItems / 2];   // two 12-bit tile slots per register
 #pragma unroll
     for (int r = 0; r < kDsItems; ++r) {
-        const int64_t idx = wbase + r * 32 + lane;
-        const bool ok = idx < e;
+        const bool ok = wbase + r * 32 + lane < e;
         const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
         const unsigned peers = __match_any_sync(kFull, dig);
-        uint32_t slot = 0;
-        if (ok) slot = static_cast<uint32_t>(s_tstart[dig] + mine[dig] + __popc(peers & lower));
+        int slot = 0;
+        if (ok) slot = s_tstart[dig] + mine[dig] + __popc(peers & lower);
         __syncwarp();
         if (ok && lane == __ffs(peers) - 1) mine[dig] += static_cast<uint16_t>(__popc(peers));
         __syncwarp();
-        if (ok) s_key[slot] = keys[r];
-        if (r & 1) slots[r / 2] |= slot << 16;
-        else slots[r / 2] = slot;
+        if (ok) {
+            s_key[slot] = keys[r];
+            s_src[slot] = srcs[r];
+            s_eid[slot] = eids[r];
+        }
     }
+    __syncthreads();
 
-    // Phase D: keys and the two value arrays leave in digit order.
-    for (int which = 0; which < 2; ++which) {
-#pragma unroll
-        for (int r = 0; r < kDsItems; ++r) {
-            const int64_t idx = wbase + r * 32 + lane;
-            if (idx >= e) continue;
-            int32_t v;
-            if (which == 0) v = FIRST ? static_cast<int32_t>(checked_id(__ldg(src64 + idx), n, status))
-                                      : __ldg(src_in + idx);
-            else v = FIRST ? static_cast<int32_t>(idx) : __ldg(eid_in + idx);
-            s_val[(slots[r / 2] >> (16 * (r & 1))) & 0xffffu] = v;
-        }
-        __syncthreads();
-        int32_t *dst = which == 0 ? src_out : eid_out;
-        for (int i = threadIdx.x; i < count; i += kDsThreads) {
-            const uint32_t k = s_key[i];
-            const int d = static_cast<int>((k >> shift) & (radix - 1));
-            const int64_t pos = static_cast<int64_t>(s_gbase[d]) + (i - s_tstart[d]);
-            if (which == 0) key_out[pos] = k;
-            dst[pos] = s_val[i];
-        }
-        __syncthreads();
+    // Phase D: the tile leaves in digit order, one coalesced run per digit.
+    for (int i = threadIdx.x; i < count; i += kDsThreads) {
+        const uint32_t k = s_key[i];
+        const int d = static_cast<int>((k >> shift) & (radix - 1));
+        const int64_t pos = static_cast<int64_t>(s_gbase[d]) + (i - s_tstart[d]);
+        key_out[pos] = k;
+        src_out[pos] = s_src[i];
+        eid_out[pos] = s_eid[i];
     }
 }
 
