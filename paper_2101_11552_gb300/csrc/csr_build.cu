@@ -4,12 +4,15 @@
 //
 // Method: a stable least-significant-digit radix sort of the edges by target
 // id, one pass per digit of ceil(log2 N) bits split into <= 10-bit digits.
-// Each pass is reduce-then-scan:
-//   upsweep   per-tile digit histogram  -> hist[digit][tile]
-//   scan      exclusive scan of hist (digit-major) -> first output slot of
-//             every (digit, tile) pair; digit-major order keeps the sort stable
-//   downsweep each warp ranks its elements with __match_any_sync and writes
-//             them to their slots
+// Each pass is reduce-then-scan over 4096-edge tiles:
+//   upsweep   per-tile digit histogram -> cnt[tile][digit] (tile-major)
+//   colscan   offs[tile][digit] = (edges of all smaller digits)
+//                               + (edges of this digit in earlier tiles):
+//             the first output slot of every (tile, digit) run; taking the
+//             tiles in order inside a digit keeps the sort stable
+//   downsweep ranks each tile's elements in original order, stages the tile
+//             in shared memory in digit order and writes each digit's run
+//             with coalesced stores
 // No kernel waits on another CTA, so nothing can spin.  The first pass reads
 // the int64 edge_index directly and checks every id; the last pass writes
 // col (source) and perm (original edge id) in final order, plus the sorted
@@ -19,13 +22,10 @@
 namespace tfg {
 namespace {
 
-constexpr int kSortWarps = 8;
-constexpr int kSortThreads = kSortWarps * 32;
 constexpr int kTile = 4096;                       // edges per CTA tile
 constexpr int kMaxDigitBits = 10;
-constexpr int kScanThreads = 256;
-constexpr int kScanItems = 16;
-constexpr int kScanChunk = kScanThreads * kScanItems;
+constexpr int kUpThreads = 256;
+constexpr int kColChunk = 128;                    // tiles per column-scan chunk
 
 struct SortPlan {
     int passes;
@@ -54,38 +54,92 @@ __device__ __forceinline__ uint32_t checked_id(int64_t v, int64_t n, int32_t *st
 }
 
 template <bool FIRST>
-__global__ void __launch_bounds__(kSortThreads)
+__global__ void __launch_bounds__(kUpThreads)
 radix_upsweep(const int64_t *__restrict__ dst64, const uint32_t *__restrict__ key32, int64_t e,
-              int64_t n, int shift, int width, int num_tiles, int32_t *__restrict__ hist,
-              int32_t *status) {
+              int64_t n, int shift, int width, int32_t *__restrict__ cnt, int32_t *status) {
     extern __shared__ int32_t s_cnt[];
     const int radix = 1 << width;
-    for (int d = threadIdx.x; d < radix; d += kSortThreads) s_cnt[d] = 0;
+    for (int d = threadIdx.x; d < radix; d += kUpThreads) s_cnt[d] = 0;
     __syncthreads();
     const int64_t base = static_cast<int64_t>(blockIdx.x) * kTile;
     const int64_t stop = min64(e, base + kTile);
-    for (int64_t i = base + threadIdx.x; i < stop; i += kSortThreads) {
+    for (int64_t i = base + threadIdx.x; i < stop; i += kUpThreads) {
         uint32_t key = FIRST ? checked_id(__ldg(dst64 + i), n, status) : __ldg(key32 + i);
         atomicAdd(&s_cnt[(key >> shift) & (radix - 1)], 1);
     }
     __syncthreads();
-    for (int d = threadIdx.x; d < radix; d += kSortThreads)
-        hist[static_cast<int64_t>(d) * num_tiles + blockIdx.x] = s_cnt[d];
+    for (int d = threadIdx.x; d < radix; d += kUpThreads)
+        cnt[static_cast<int64_t>(blockIdx.x) * radix + d] = s_cnt[d];
 }
 
-// Downsweep: 16 warps share one 4096-edge tile, 8 elements per lane.
-// Every global load of the tile (keys and both value arrays) is issued up
-// front, so the tile waits on memory once.  Elements are then ranked inside
-// the tile (stable: warp-major, then round, then lane = original order),
-// staged in shared memory in digit order, and written out by consecutive
-// threads, so each digit's run of the tile leaves as coalesced stores.
+// ---- column scan of cnt[tiles][radix] ------------------------------------
+// blockDim = radix; thread d owns digit column d (loads coalesce across d).
+__global__ void colscan_partial(const int32_t *__restrict__ cnt, int tiles, int radix,
+                                int32_t *__restrict__ part) {
+    const int d = threadIdx.x;
+    const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kColChunk;
+    const int64_t t1 = min64(tiles, t0 + kColChunk);
+    int32_t s = 0;
+    for (int64_t t = t0; t < t1; ++t) s += cnt[t * radix + d];
+    part[static_cast<int64_t>(blockIdx.x) * radix + d] = s;
+}
+
+// One CTA: per digit, exclusive prefix over chunks; then digit bases.
+__global__ void colscan_top(int32_t *part, int chunks, int radix) {
+    extern __shared__ int32_t s_tot[];   // [radix]
+    for (int d = threadIdx.x; d < radix; d += blockDim.x) {
+        int32_t run = 0;
+        for (int c = 0; c < chunks; ++c) {
+            const int32_t v = part[static_cast<int64_t>(c) * radix + d];
+            part[static_cast<int64_t>(c) * radix + d] = run;
+            run += v;
+        }
+        s_tot[d] = run;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {   // digit bases: at most 1024 digits, once per pass
+        int32_t run = 0;
+        for (int d = 0; d < radix; ++d) {
+            const int32_t v = s_tot[d];
+            s_tot[d] = run;
+            run += v;
+        }
+    }
+    __syncthreads();
+    for (int d = threadIdx.x; d < radix; d += blockDim.x)
+        for (int c = 0; c < chunks; ++c) part[static_cast<int64_t>(c) * radix + d] += s_tot[d];
+}
+
+__global__ void colscan_down(int32_t *cnt, int tiles, int radix, const int32_t *__restrict__ part) {
+    const int d = threadIdx.x;
+    const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kColChunk;
+    const int64_t t1 = min64(tiles, t0 + kColChunk);
+    int32_t run = part[static_cast<int64_t>(blockIdx.x) * radix + d];
+    for (int64_t t = t0; t < t1; ++t) {
+        const int32_t v = cnt[t * radix + d];
+        cnt[t * radix + d] = run;
+        run += v;
+    }
+}
+
+// ---- downsweep ------------------------------------------------------------
+// 16 warps share one 4096-edge tile, 8 elements per lane.  Every global load
+// of the tile is issued up front, so the tile waits on memory once.
+//   A  per-warp digit counts with shared-memory atomics (order-free)
+//   B  per digit: warp-major exclusive prefix and tile total; block scan of
+//      the totals over digits -> each digit's first slot in the tile
+//   C  stable slots: per round, peers with equal digits are found with
+//      __match_any_sync, their leader claims a block of slots with one
+//      returning atomic, and each lane adds its rank among the peers
+//   D  the tile leaves in digit order, consecutive threads writing
+//      consecutive positions of each digit's run
 constexpr int kDsWarps = 16;
 constexpr int kDsThreads = kDsWarps * 32;
 constexpr int kDsItems = kTile / kDsThreads;   // 8 per lane
 
 size_t downsweep_smem(int radix) {
-    return sizeof(uint32_t) * 3 * kTile + sizeof(uint16_t) * kDsWarps * radix +
-           sizeof(int32_t) * 2 * radix;
+    return sizeof(uint32_t) * 3 * kTile + sizeof(int32_t) * kDsWarps * radix +
+           sizeof(int32_t) * 2 * radix + sizeof(int32_t) * 32;
 }
 
 template <bool FIRST>
@@ -93,21 +147,24 @@ __global__ void __launch_bounds__(kDsThreads, 2)
 radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ dst64,
                 const uint32_t *__restrict__ key_in, const int32_t *__restrict__ src_in,
                 const int32_t *__restrict__ eid_in, int64_t e, int64_t n, int shift, int width,
-                int num_tiles, const int32_t *__restrict__ offs, uint32_t *__restrict__ key_out,
+                const int32_t *__restrict__ offs, uint32_t *__restrict__ key_out,
                 int32_t *__restrict__ src_out, int32_t *__restrict__ eid_out, int32_t *status) {
     extern __shared__ __align__(16) unsigned char smem[];
     const int radix = 1 << width;
     uint32_t *s_key = reinterpret_cast<uint32_t *>(smem);
     int32_t *s_src = reinterpret_cast<int32_t *>(s_key + kTile);
     int32_t *s_eid = s_src + kTile;
-    uint16_t *s_cnt = reinterpret_cast<uint16_t *>(s_eid + kTile);   // [warp][digit]
-    int32_t *s_tstart = reinterpret_cast<int32_t *>(s_cnt + kDsWarps * radix);
-    int32_t *s_gbase = s_tstart + radix;
+    int32_t *s_cnt = s_eid + kTile;                 // [warp][digit]
+    int32_t *s_tstart = s_cnt + kDsWarps * radix;  // [digit]
+    int32_t *s_gbase = s_tstart + radix;           // [digit]
+    int32_t *s_chunk = s_gbase + radix;            // [32] chunk totals of the digit scan
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t tile0 = static_cast<int64_t>(blockIdx.x) * kTile;
     const int count = static_cast<int>(min64(kTile, e - tile0));
-    uint16_t *mine = s_cnt + warp * radix;
+    int32_t *mine = s_cnt + warp * radix;
     for (int d = lane; d < radix; d += 32) mine[d] = 0;
+    for (int d = threadIdx.x; d < radix; d += kDsThreads)
+        s_gbase[d] = offs[static_cast<int64_t>(blockIdx.x) * radix + d];
 
     // All loads of this warp's sub-tile, issued together.
     const int64_t wbase = tile0 + static_cast<int64_t>(warp) * 32 * kDsItems;
@@ -133,60 +190,67 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     }
     __syncwarp();
 
-    // Phase A: per-warp digit counts over the warp's contiguous sub-tile.
+    // A: per-warp digit counts.
 #pragma unroll
-    for (int r = 0; r < kDsItems; ++r) {
-        const bool ok = wbase + r * 32 + lane < e;
-        const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
-        const unsigned peers = __match_any_sync(kFull, dig);
-        if (ok && lane == __ffs(peers) - 1) mine[dig] += static_cast<uint16_t>(__popc(peers));
-        __syncwarp();
-    }
+    for (int r = 0; r < kDsItems; ++r)
+        if (wbase + r * 32 + lane < e) atomicAdd(&mine[(keys[r] >> shift) & (radix - 1)], 1);
     __syncthreads();
 
-    // Phase B: per digit, warp-major exclusive prefix (in place) and tile
-    // total; then an exclusive scan of the totals over digits.
+    // B: warp-major prefix per digit, tile totals, then a block scan over digits.
     for (int d = threadIdx.x; d < radix; d += kDsThreads) {
-        int run = 0;
+        int32_t c[kDsWarps];
+#pragma unroll
+        for (int w = 0; w < kDsWarps; ++w) c[w] = s_cnt[w * radix + d];
+        int32_t run = 0;
+#pragma unroll
         for (int w = 0; w < kDsWarps; ++w) {
-            const int c = s_cnt[w * radix + d];
-            s_cnt[w * radix + d] = static_cast<uint16_t>(run);
-            run += c;
+            s_cnt[w * radix + d] = run;
+            run += c[w];
         }
         s_tstart[d] = run;
-        s_gbase[d] = offs[static_cast<int64_t>(d) * num_tiles + blockIdx.x];
     }
     __syncthreads();
-    if (warp == 0) {   // exclusive scan of s_tstart[0 .. radix) by one warp
-        int carry = 0;
-        for (int base = 0; base < radix; base += 32) {
-            const bool in = base + lane < radix;   // radix may be < 32
-            const int v = in ? s_tstart[base + lane] : 0;
-            int incl = v;
+    const int chunks = (radix + 31) / 32;   // <= 32
+    for (int ch = warp; ch < chunks; ch += kDsWarps) {   // scan of each 32-digit chunk
+        const int d = ch * 32 + lane;
+        const int32_t v = d < radix ? s_tstart[d] : 0;
+        int32_t incl = v;
 #pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int y = __shfl_up_sync(kFull, incl, o);
-                if (lane >= o) incl += y;
-            }
-            if (in) s_tstart[base + lane] = carry + incl - v;
-            carry += __shfl_sync(kFull, incl, 31);
+        for (int o = 1; o < 32; o <<= 1) {
+            const int32_t y = __shfl_up_sync(kFull, incl, o);
+            if (lane >= o) incl += y;
         }
+        if (d < radix) s_tstart[d] = incl - v;
+        if (lane == 31) s_chunk[ch] = incl;
     }
+    __syncthreads();
+    if (warp == 0) {   // exclusive scan of the chunk totals
+        const int32_t v = lane < chunks ? s_chunk[lane] : 0;
+        int32_t incl = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int32_t y = __shfl_up_sync(kFull, incl, o);
+            if (lane >= o) incl += y;
+        }
+        if (lane < chunks) s_chunk[lane] = incl - v;
+    }
+    __syncthreads();
+    for (int d = threadIdx.x; d < radix; d += kDsThreads) s_tstart[d] += s_chunk[d >> 5];
     __syncthreads();
 
-    // Phase C: tile-local slot of every element (stable); stage all arrays.
+    // C: stable slot of every element; stage key, source and edge id.
     const unsigned lower = (1u << lane) - 1u;
 #pragma unroll
     for (int r = 0; r < kDsItems; ++r) {
         const bool ok = wbase + r * 32 + lane < e;
         const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
         const unsigned peers = __match_any_sync(kFull, dig);
-        int slot = 0;
-        if (ok) slot = s_tstart[dig] + mine[dig] + __popc(peers & lower);
-        __syncwarp();
-        if (ok && lane == __ffs(peers) - 1) mine[dig] += static_cast<uint16_t>(__popc(peers));
-        __syncwarp();
+        const int leader = __ffs(peers) - 1;
+        int32_t base = 0;
+        if (ok && lane == leader) base = atomicAdd(&mine[dig], __popc(peers));
+        base = __shfl_sync(kFull, base, leader);
         if (ok) {
+            const int slot = s_tstart[dig] + base + __popc(peers & lower);
             s_key[slot] = keys[r];
             s_src[slot] = srcs[r];
             s_eid[slot] = eids[r];
@@ -194,98 +258,18 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     }
     __syncthreads();
 
-    // Phase D: the tile leaves in digit order, one coalesced run per digit.
-    for (int i = threadIdx.x; i < count; i += kDsThreads) {
-        const uint32_t k = s_key[i];
-        const int d = static_cast<int>((k >> shift) & (radix - 1));
-        const int64_t pos = static_cast<int64_t>(s_gbase[d]) + (i - s_tstart[d]);
-        key_out[pos] = k;
-        src_out[pos] = s_src[i];
-        eid_out[pos] = s_eid[i];
-    }
-}
-
-// ---- exclusive scan of an int32 array (in place), three kernels ----------
-__device__ int32_t block_exclusive_scan(int32_t v, int32_t *total) {
-    __shared__ int32_t warp_sums[kScanThreads / 32];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    int32_t incl = v;
+    // D: write the tile out, one coalesced run per digit.
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int32_t y = __shfl_up_sync(kFull, incl, o);
-        if (lane >= o) incl += y;
-    }
-    if (lane == 31) warp_sums[warp] = incl;
-    __syncthreads();
-    if (warp == 0) {
-        int32_t s = lane < kScanThreads / 32 ? warp_sums[lane] : 0;
-        int32_t si = s;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int32_t y = __shfl_up_sync(kFull, si, o);
-            if (lane >= o) si += y;
+    for (int j = 0; j < kDsItems; ++j) {
+        const int i = threadIdx.x + j * kDsThreads;
+        if (i < count) {
+            const uint32_t k = s_key[i];
+            const int d = static_cast<int>((k >> shift) & (radix - 1));
+            const int64_t pos = static_cast<int64_t>(s_gbase[d]) + (i - s_tstart[d]);
+            key_out[pos] = k;
+            src_out[pos] = s_src[i];
+            eid_out[pos] = s_eid[i];
         }
-        if (lane < kScanThreads / 32) warp_sums[lane] = si - s;
-        if (lane == kScanThreads / 32 - 1 && total) *total = si;
-    }
-    __syncthreads();
-    const int32_t r = incl - v + warp_sums[warp];
-    __syncthreads();
-    return r;
-}
-
-__global__ void __launch_bounds__(kScanThreads)
-scan_reduce(const int32_t *__restrict__ data, int64_t m, int32_t *__restrict__ sums) {
-    const int64_t base = static_cast<int64_t>(blockIdx.x) * kScanChunk;
-    int32_t s = 0;
-    for (int i = threadIdx.x; i < kScanChunk; i += kScanThreads) {
-        const int64_t k = base + i;
-        if (k < m) s += data[k];
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(kFull, s, o);
-    __shared__ int32_t ws[kScanThreads / 32];
-    if ((threadIdx.x & 31) == 0) ws[threadIdx.x >> 5] = s;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        int32_t t = 0;
-        for (int w = 0; w < kScanThreads / 32; ++w) t += ws[w];
-        sums[blockIdx.x] = t;
-    }
-}
-
-__global__ void __launch_bounds__(kScanThreads) scan_top(int32_t *sums, int nb) {
-    __shared__ int32_t carry;
-    __shared__ int32_t tot;
-    if (threadIdx.x == 0) carry = 0;
-    __syncthreads();
-    for (int base = 0; base < nb; base += kScanThreads) {
-        const int k = base + threadIdx.x;
-        const int32_t v = k < nb ? sums[k] : 0;
-        const int32_t ex = block_exclusive_scan(v, &tot);
-        if (k < nb) sums[k] = ex + carry;
-        __syncthreads();
-        if (threadIdx.x == 0) carry += tot;
-        __syncthreads();
-    }
-}
-
-__global__ void __launch_bounds__(kScanThreads)
-scan_down(int32_t *data, int64_t m, const int32_t *__restrict__ sums) {
-    const int64_t base = static_cast<int64_t>(blockIdx.x) * kScanChunk +
-                         static_cast<int64_t>(threadIdx.x) * kScanItems;
-    int32_t v[kScanItems];
-    int32_t local = 0;
-#pragma unroll
-    for (int i = 0; i < kScanItems; ++i) {
-        v[i] = (base + i < m) ? data[base + i] : 0;
-        local += v[i];
-    }
-    int32_t run = block_exclusive_scan(local, nullptr) + sums[blockIdx.x];
-#pragma unroll
-    for (int i = 0; i < kScanItems; ++i) {
-        if (base + i < m) data[base + i] = run;
-        run += v[i];
     }
 }
 
@@ -309,26 +293,18 @@ __global__ void degree_from_rowptr(const int32_t *__restrict__ rowptr, int64_t n
     if (t < n) deg[t] = rowptr[t + 1] - rowptr[t];
 }
 
-cudaError_t exclusive_scan(int32_t *data, int64_t m, int32_t *sums, cudaStream_t s) {
-    const int nb = ceil_div(m, kScanChunk);
-    scan_reduce<<<nb, kScanThreads, 0, s>>>(data, m, sums);
-    scan_top<<<1, kScanThreads, 0, s>>>(sums, nb);
-    scan_down<<<nb, kScanThreads, 0, s>>>(data, m, sums);
-    return cudaGetLastError();
-}
-
 }  // namespace
 
 size_t csr_workspace_bytes(int64_t n, int64_t e) {
     if (e <= 0) return 256;
     const SortPlan p = plan_for(n);
     const int64_t tiles = ceil_div(e, kTile);
-    const int64_t cells = (int64_t(1) << p.width) * tiles;
+    const int64_t radix = int64_t(1) << p.width;
     const size_t a = align256(sizeof(int32_t) * 3 * size_t(e));
     const size_t b = align256(sizeof(int32_t) * (p.passes >= 3 ? 3 : 1) * size_t(e));
-    const size_t h = align256(sizeof(int32_t) * size_t(cells));
-    const size_t sums = align256(sizeof(int32_t) * size_t(ceil_div(cells, kScanChunk)));
-    return a + b + h + sums;
+    const size_t h = align256(sizeof(int32_t) * size_t(radix * tiles));
+    const size_t part = align256(sizeof(int32_t) * size_t(radix * ceil_div(tiles, kColChunk)));
+    return a + b + h + part;
 }
 
 cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
@@ -341,7 +317,7 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
         const SortPlan p = plan_for(n);
         const int tiles = ceil_div(e, kTile);
         const int radix = 1 << p.width;
-        const int64_t cells = int64_t(radix) * tiles;
+        const int chunks = ceil_div(tiles, kColChunk);
         char *w = static_cast<char *>(ws);
         struct Buf { uint32_t *key; int32_t *src; int32_t *eid; } buf[2];
         buf[0].key = reinterpret_cast<uint32_t *>(w);
@@ -352,9 +328,9 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
         buf[1].src = reinterpret_cast<int32_t *>(buf[1].key + e);
         buf[1].eid = buf[1].src + e;
         w += align256(sizeof(int32_t) * (p.passes >= 3 ? 3 : 1) * size_t(e));
-        int32_t *hist = reinterpret_cast<int32_t *>(w);
-        w += align256(sizeof(int32_t) * size_t(cells));
-        int32_t *sums = reinterpret_cast<int32_t *>(w);
+        int32_t *cnt = reinterpret_cast<int32_t *>(w);
+        w += align256(sizeof(int32_t) * size_t(int64_t(radix) * tiles));
+        int32_t *part = reinterpret_cast<int32_t *>(w);
 
         const int64_t *src64 = edge_index, *dst64 = edge_index + e;
         const int smem_max = static_cast<int>(downsweep_smem(1 << kMaxDigitBits));
@@ -369,22 +345,23 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
             Buf out = buf[pass & 1];
             if (last) { out.src = col; out.eid = perm; }
             if (first)
-                radix_upsweep<true><<<tiles, kSortThreads, radix * sizeof(int32_t), s>>>(
-                    dst64, nullptr, e, n, shift, p.width, tiles, hist, status);
+                radix_upsweep<true><<<tiles, kUpThreads, radix * sizeof(int32_t), s>>>(
+                    dst64, nullptr, e, n, shift, p.width, cnt, status);
             else
-                radix_upsweep<false><<<tiles, kSortThreads, radix * sizeof(int32_t), s>>>(
-                    nullptr, in.key, e, n, shift, p.width, tiles, hist, status);
-            err = exclusive_scan(hist, cells, sums, s);
-            if (err != cudaSuccess) return err;
+                radix_upsweep<false><<<tiles, kUpThreads, radix * sizeof(int32_t), s>>>(
+                    nullptr, in.key, e, n, shift, p.width, cnt, status);
+            colscan_partial<<<chunks, radix, 0, s>>>(cnt, tiles, radix, part);
+            colscan_top<<<1, radix, radix * sizeof(int32_t), s>>>(part, chunks, radix);
+            colscan_down<<<chunks, radix, 0, s>>>(cnt, tiles, radix, part);
             const size_t smem = downsweep_smem(radix);
             if (first)
                 radix_downsweep<true><<<tiles, kDsThreads, smem, s>>>(
-                    src64, dst64, nullptr, nullptr, nullptr, e, n, shift, p.width, tiles, hist,
-                    out.key, out.src, out.eid, status);
+                    src64, dst64, nullptr, nullptr, nullptr, e, n, shift, p.width, cnt, out.key,
+                    out.src, out.eid, status);
             else
                 radix_downsweep<false><<<tiles, kDsThreads, smem, s>>>(
-                    nullptr, nullptr, in.key, in.src, in.eid, e, n, shift, p.width, tiles, hist,
-                    out.key, out.src, out.eid, status);
+                    nullptr, nullptr, in.key, in.src, in.eid, e, n, shift, p.width, cnt, out.key,
+                    out.src, out.eid, status);
             err = cudaGetLastError();
             if (err != cudaSuccess) return err;
             sorted_keys = out.key;
