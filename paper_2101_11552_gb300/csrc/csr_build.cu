@@ -5,9 +5,9 @@
 // Method: a stable least-significant-digit radix sort of the edges by target
 // id, one pass per digit of ceil(log2 N) bits split into <= 10-bit digits.
 // Each pass is reduce-then-scan over 4096-edge tiles:
-//   upsweep   per-tile digit histogram -> cnt[tile][digit] (tile-major)
-//   colscan   offs[tile][digit] = (edges of all smaller digits)
-//                               + (edges of this digit in earlier tiles):
+//   upsweep   per-tile digit histogram -> cnt[digit][tile] (digit-major)
+//   scan      exclusive scan of cnt in that order: offs[digit][tile] = (edges
+//             of all smaller digits) + (edges of this digit in earlier tiles),
 //             the first output slot of every (tile, digit) run; taking the
 //             tiles in order inside a digit keeps the sort stable
 //   downsweep ranks each tile's elements in original order, stages the tile
@@ -25,7 +25,9 @@ namespace {
 constexpr int kTile = 4096;                       // edges per CTA tile
 constexpr int kMaxDigitBits = 10;
 constexpr int kUpThreads = 256;
-constexpr int kColChunk = 128;                    // tiles per column-scan chunk
+constexpr int kScanThreads = 256;
+constexpr int kScanItems = 16;
+constexpr int kScanChunk = kScanThreads * kScanItems;
 
 struct SortPlan {
     int passes;
@@ -56,7 +58,8 @@ __device__ __forceinline__ uint32_t checked_id(int64_t v, int64_t n, int32_t *st
 template <bool FIRST>
 __global__ void __launch_bounds__(kUpThreads)
 radix_upsweep(const int64_t *__restrict__ dst64, const uint32_t *__restrict__ key32, int64_t e,
-              int64_t n, int shift, int width, int32_t *__restrict__ cnt, int32_t *status) {
+              int64_t n, int shift, int width, int num_tiles, int32_t *__restrict__ cnt,
+              int32_t *status) {
     extern __shared__ int32_t s_cnt[];
     const int radix = 1 << width;
     for (int d = threadIdx.x; d < radix; d += kUpThreads) s_cnt[d] = 0;
@@ -69,57 +72,115 @@ radix_upsweep(const int64_t *__restrict__ dst64, const uint32_t *__restrict__ ke
     }
     __syncthreads();
     for (int d = threadIdx.x; d < radix; d += kUpThreads)
-        cnt[static_cast<int64_t>(blockIdx.x) * radix + d] = s_cnt[d];
+        cnt[static_cast<int64_t>(d) * num_tiles + blockIdx.x] = s_cnt[d];
 }
 
-// ---- column scan of cnt[tiles][radix] ------------------------------------
-// blockDim = radix; thread d owns digit column d (loads coalesce across d).
-__global__ void colscan_partial(const int32_t *__restrict__ cnt, int tiles, int radix,
-                                int32_t *__restrict__ part) {
-    const int d = threadIdx.x;
-    const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kColChunk;
-    const int64_t t1 = min64(tiles, t0 + kColChunk);
+// ---- exclusive scan of an int32 array (in place), three kernels ----------
+__device__ int32_t block_exclusive_scan(int32_t v, int32_t *total) {
+    __shared__ int32_t warp_sums[kScanThreads / 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int32_t incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int32_t y = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) warp_sums[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        const int32_t s = lane < kScanThreads / 32 ? warp_sums[lane] : 0;
+        int32_t si = s;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int32_t y = __shfl_up_sync(kFull, si, o);
+            if (lane >= o) si += y;
+        }
+        if (lane < kScanThreads / 32) warp_sums[lane] = si - s;
+        if (lane == kScanThreads / 32 - 1 && total) *total = si;
+    }
+    __syncthreads();
+    const int32_t r = incl - v + warp_sums[warp];
+    __syncthreads();
+    return r;
+}
+
+__global__ void __launch_bounds__(kScanThreads)
+scan_reduce(const int32_t *__restrict__ data, int64_t m, int32_t *__restrict__ sums) {
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * kScanChunk;
     int32_t s = 0;
-    for (int64_t t = t0; t < t1; ++t) s += cnt[t * radix + d];
-    part[static_cast<int64_t>(blockIdx.x) * radix + d] = s;
+#pragma unroll
+    for (int i = 0; i < kScanItems; ++i) {
+        const int64_t k = base + i * kScanThreads + threadIdx.x;
+        if (k < m) s += data[k];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(kFull, s, o);
+    __shared__ int32_t ws[kScanThreads / 32];
+    if ((threadIdx.x & 31) == 0) ws[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int32_t t = 0;
+        for (int w = 0; w < kScanThreads / 32; ++w) t += ws[w];
+        sums[blockIdx.x] = t;
+    }
 }
 
-// One CTA: per digit, exclusive prefix over chunks; then digit bases.
-__global__ void colscan_top(int32_t *part, int chunks, int radix) {
-    extern __shared__ int32_t s_tot[];   // [radix]
-    for (int d = threadIdx.x; d < radix; d += blockDim.x) {
-        int32_t run = 0;
-        for (int c = 0; c < chunks; ++c) {
-            const int32_t v = part[static_cast<int64_t>(c) * radix + d];
-            part[static_cast<int64_t>(c) * radix + d] = run;
-            run += v;
-        }
-        s_tot[d] = run;
-    }
+__global__ void __launch_bounds__(kScanThreads) scan_top(int32_t *sums, int nb) {
+    __shared__ int32_t carry;
+    __shared__ int32_t tot;
+    if (threadIdx.x == 0) carry = 0;
     __syncthreads();
-    if (threadIdx.x == 0) {   // digit bases: at most 1024 digits, once per pass
-        int32_t run = 0;
-        for (int d = 0; d < radix; ++d) {
-            const int32_t v = s_tot[d];
-            s_tot[d] = run;
-            run += v;
-        }
+    for (int base = 0; base < nb; base += kScanThreads) {
+        const int k = base + threadIdx.x;
+        const int32_t v = k < nb ? sums[k] : 0;
+        const int32_t ex = block_exclusive_scan(v, &tot);
+        if (k < nb) sums[k] = ex + carry;
+        __syncthreads();
+        if (threadIdx.x == 0) carry += tot;
+        __syncthreads();
     }
-    __syncthreads();
-    for (int d = threadIdx.x; d < radix; d += blockDim.x)
-        for (int c = 0; c < chunks; ++c) part[static_cast<int64_t>(c) * radix + d] += s_tot[d];
 }
 
-__global__ void colscan_down(int32_t *cnt, int tiles, int radix, const int32_t *__restrict__ part) {
-    const int d = threadIdx.x;
-    const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kColChunk;
-    const int64_t t1 = min64(tiles, t0 + kColChunk);
-    int32_t run = part[static_cast<int64_t>(blockIdx.x) * radix + d];
-    for (int64_t t = t0; t < t1; ++t) {
-        const int32_t v = cnt[t * radix + d];
-        cnt[t * radix + d] = run;
-        run += v;
+// Each thread scans kScanItems consecutive values; loads are staged through
+// shared memory so the global reads and writes stay coalesced.
+__global__ void __launch_bounds__(kScanThreads)
+scan_down(int32_t *data, int64_t m, const int32_t *__restrict__ sums) {
+    __shared__ int32_t s_v[kScanChunk + kScanChunk / 32];   // padded against bank conflicts
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * kScanChunk;
+    auto at = [](int i) { return i + (i >> 5); };
+#pragma unroll
+    for (int i = 0; i < kScanItems; ++i) {
+        const int j = i * kScanThreads + threadIdx.x;
+        s_v[at(j)] = base + j < m ? data[base + j] : 0;
     }
+    __syncthreads();
+    int32_t v[kScanItems];
+    int32_t local = 0;
+#pragma unroll
+    for (int i = 0; i < kScanItems; ++i) {
+        v[i] = s_v[at(threadIdx.x * kScanItems + i)];
+        local += v[i];
+    }
+    int32_t run = block_exclusive_scan(local, nullptr) + sums[blockIdx.x];
+#pragma unroll
+    for (int i = 0; i < kScanItems; ++i) {
+        s_v[at(threadIdx.x * kScanItems + i)] = run;
+        run += v[i];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < kScanItems; ++i) {
+        const int j = i * kScanThreads + threadIdx.x;
+        if (base + j < m) data[base + j] = s_v[at(j)];
+    }
+}
+
+cudaError_t exclusive_scan(int32_t *data, int64_t m, int32_t *sums, cudaStream_t s) {
+    const int nb = ceil_div(m, kScanChunk);
+    scan_reduce<<<nb, kScanThreads, 0, s>>>(data, m, sums);
+    scan_top<<<1, kScanThreads, 0, s>>>(sums, nb);
+    scan_down<<<nb, kScanThreads, 0, s>>>(data, m, sums);
+    return cudaGetLastError();
 }
 
 // ---- downsweep ------------------------------------------------------------
@@ -147,7 +208,7 @@ __global__ void __launch_bounds__(kDsThreads, 2)
 radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ dst64,
                 const uint32_t *__restrict__ key_in, const int32_t *__restrict__ src_in,
                 const int32_t *__restrict__ eid_in, int64_t e, int64_t n, int shift, int width,
-                const int32_t *__restrict__ offs, uint32_t *__restrict__ key_out,
+                int num_tiles, const int32_t *__restrict__ offs, uint32_t *__restrict__ key_out,
                 int32_t *__restrict__ src_out, int32_t *__restrict__ eid_out, int32_t *status) {
     extern __shared__ __align__(16) unsigned char smem[];
     const int radix = 1 << width;
@@ -164,7 +225,7 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     int32_t *mine = s_cnt + warp * radix;
     for (int d = lane; d < radix; d += 32) mine[d] = 0;
     for (int d = threadIdx.x; d < radix; d += kDsThreads)
-        s_gbase[d] = offs[static_cast<int64_t>(blockIdx.x) * radix + d];
+        s_gbase[d] = offs[static_cast<int64_t>(d) * num_tiles + blockIdx.x];
 
     // All loads of this warp's sub-tile, issued together.
     const int64_t wbase = tile0 + static_cast<int64_t>(warp) * 32 * kDsItems;
@@ -303,8 +364,8 @@ size_t csr_workspace_bytes(int64_t n, int64_t e) {
     const size_t a = align256(sizeof(int32_t) * 3 * size_t(e));
     const size_t b = align256(sizeof(int32_t) * (p.passes >= 3 ? 3 : 1) * size_t(e));
     const size_t h = align256(sizeof(int32_t) * size_t(radix * tiles));
-    const size_t part = align256(sizeof(int32_t) * size_t(radix * ceil_div(tiles, kColChunk)));
-    return a + b + h + part;
+    const size_t sums = align256(sizeof(int32_t) * size_t(ceil_div(radix * tiles, kScanChunk)));
+    return a + b + h + sums;
 }
 
 cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
@@ -317,7 +378,6 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
         const SortPlan p = plan_for(n);
         const int tiles = ceil_div(e, kTile);
         const int radix = 1 << p.width;
-        const int chunks = ceil_div(tiles, kColChunk);
         char *w = static_cast<char *>(ws);
         struct Buf { uint32_t *key; int32_t *src; int32_t *eid; } buf[2];
         buf[0].key = reinterpret_cast<uint32_t *>(w);
@@ -330,7 +390,7 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
         w += align256(sizeof(int32_t) * (p.passes >= 3 ? 3 : 1) * size_t(e));
         int32_t *cnt = reinterpret_cast<int32_t *>(w);
         w += align256(sizeof(int32_t) * size_t(int64_t(radix) * tiles));
-        int32_t *part = reinterpret_cast<int32_t *>(w);
+        int32_t *sums = reinterpret_cast<int32_t *>(w);
 
         const int64_t *src64 = edge_index, *dst64 = edge_index + e;
         const int smem_max = static_cast<int>(downsweep_smem(1 << kMaxDigitBits));
@@ -346,22 +406,21 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
             if (last) { out.src = col; out.eid = perm; }
             if (first)
                 radix_upsweep<true><<<tiles, kUpThreads, radix * sizeof(int32_t), s>>>(
-                    dst64, nullptr, e, n, shift, p.width, cnt, status);
+                    dst64, nullptr, e, n, shift, p.width, tiles, cnt, status);
             else
                 radix_upsweep<false><<<tiles, kUpThreads, radix * sizeof(int32_t), s>>>(
-                    nullptr, in.key, e, n, shift, p.width, cnt, status);
-            colscan_partial<<<chunks, radix, 0, s>>>(cnt, tiles, radix, part);
-            colscan_top<<<1, radix, radix * sizeof(int32_t), s>>>(part, chunks, radix);
-            colscan_down<<<chunks, radix, 0, s>>>(cnt, tiles, radix, part);
+                    nullptr, in.key, e, n, shift, p.width, tiles, cnt, status);
+            err = exclusive_scan(cnt, int64_t(radix) * tiles, sums, s);
+            if (err != cudaSuccess) return err;
             const size_t smem = downsweep_smem(radix);
             if (first)
                 radix_downsweep<true><<<tiles, kDsThreads, smem, s>>>(
-                    src64, dst64, nullptr, nullptr, nullptr, e, n, shift, p.width, cnt, out.key,
-                    out.src, out.eid, status);
+                    src64, dst64, nullptr, nullptr, nullptr, e, n, shift, p.width, tiles, cnt,
+                    out.key, out.src, out.eid, status);
             else
                 radix_downsweep<false><<<tiles, kDsThreads, smem, s>>>(
-                    nullptr, nullptr, in.key, in.src, in.eid, e, n, shift, p.width, cnt, out.key,
-                    out.src, out.eid, status);
+                    nullptr, nullptr, in.key, in.src, in.eid, e, n, shift, p.width, tiles, cnt,
+                    out.key, out.src, out.eid, status);
             err = cudaGetLastError();
             if (err != cudaSuccess) return err;
             sorted_keys = out.key;
