@@ -413,7 +413,7 @@ void launch_main(const int32_t *rowptr, const int32_t *col, const void *x, int64
 // resident on every GPU that loads the library for as long as it stays
 // loaded.  Every call overwrites the part it uses, so nothing needs clearing.
 constexpr int64_t kNoAllocNodeHeads = int64_t(1) << 21;
-__device__ __align__(256) float g_noalloc_scores[2 * kNoAllocNodeHeads];
+static __device__ __align__(256) float g_noalloc_scores[2 * kNoAllocNodeHeads];
 
 }  // namespace
 
