@@ -39,6 +39,9 @@ constexpr int kAggThreads = kAggWarps * 32;
 #ifndef TFG_AGG_UNROLL
 #define TFG_AGG_UNROLL 8
 #endif
+#ifndef TFG_AGG_MINB
+#define TFG_AGG_MINB 3   // resident CTAs per SM asked of the compiler, 16-byte bf16 path
+#endif
 constexpr int kHeavyDeg = TFG_HEAVY_DEG;
 constexpr int kMaxHeavy = 64;   // hub rows a CTA sets aside; more are done warp by warp
 // gathers in flight per lane: deeper for the 16-byte bf16 sum path (measured
@@ -270,7 +273,7 @@ struct Agg {
 };
 
 template <typename XT, int VEC, int LPR, int KIND>
-__global__ void __launch_bounds__(kAggThreads, VEC >= 8 ? 3 : 4) aggregate_kernel(AggArgs a) {
+__global__ void __launch_bounds__(kAggThreads, VEC >= 8 ? TFG_AGG_MINB : 4) aggregate_kernel(AggArgs a) {
     using A = Agg<XT, VEC, LPR, KIND>;
     __shared__ int s_next, s_nheavy;
     __shared__ int64_t s_heavy[kMaxHeavy];

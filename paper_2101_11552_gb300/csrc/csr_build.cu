@@ -188,10 +188,12 @@ cudaError_t exclusive_scan(int32_t *data, int64_t m, int32_t *sums, cudaStream_t
 // of the tile is issued up front, so the tile waits on memory once.
 //   A  per-warp digit counts with shared-memory atomics (order-free)
 //   B  per digit: warp-major exclusive prefix and tile total; block scan of
-//      the totals over digits -> each digit's first slot in the tile
+//      the totals over digits -> each digit's first slot in the tile, folded
+//      into every warp's counter; per digit, global base minus tile start
 //   C  stable slots: per round, peers with equal digits are found with
 //      __match_any_sync, their leader claims a block of slots with one
-//      returning atomic, and each lane adds its rank among the peers
+//      returning atomic, and each lane adds its rank among the peers; the
+//      element (key, source, edge id) is staged as one 16-byte record
 //   D  the tile leaves in digit order, consecutive threads writing
 //      consecutive positions of each digit's run
 constexpr int kDsWarps = 16;
@@ -199,7 +201,7 @@ constexpr int kDsThreads = kDsWarps * 32;
 constexpr int kDsItems = kTile / kDsThreads;   // 8 per lane
 
 size_t downsweep_smem(int radix) {
-    return sizeof(uint32_t) * 3 * kTile + sizeof(int32_t) * kDsWarps * radix +
+    return sizeof(uint4) * kTile + sizeof(int32_t) * kDsWarps * radix +
            sizeof(int32_t) * 2 * radix + sizeof(int32_t) * 32;
 }
 
@@ -212,20 +214,18 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
                 int32_t *__restrict__ src_out, int32_t *__restrict__ eid_out, int32_t *status) {
     extern __shared__ __align__(16) unsigned char smem[];
     const int radix = 1 << width;
-    uint32_t *s_key = reinterpret_cast<uint32_t *>(smem);
-    int32_t *s_src = reinterpret_cast<int32_t *>(s_key + kTile);
-    int32_t *s_eid = s_src + kTile;
-    int32_t *s_cnt = s_eid + kTile;                 // [warp][digit]
-    int32_t *s_tstart = s_cnt + kDsWarps * radix;  // [digit]
-    int32_t *s_gbase = s_tstart + radix;           // [digit]
-    int32_t *s_chunk = s_gbase + radix;            // [32] chunk totals of the digit scan
+    uint4 *s_elem = reinterpret_cast<uint4 *>(smem);                      // [tile]
+    int32_t *s_cnt = reinterpret_cast<int32_t *>(s_elem + kTile);          // [warp][digit]
+    int32_t *s_tstart = s_cnt + kDsWarps * radix;                          // [digit]
+    int32_t *s_delta = s_tstart + radix;                                   // [digit]
+    int32_t *s_chunk = s_delta + radix;                                    // [32]
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t tile0 = static_cast<int64_t>(blockIdx.x) * kTile;
     const int count = static_cast<int>(min64(kTile, e - tile0));
     int32_t *mine = s_cnt + warp * radix;
     for (int d = lane; d < radix; d += 32) mine[d] = 0;
     for (int d = threadIdx.x; d < radix; d += kDsThreads)
-        s_gbase[d] = offs[static_cast<int64_t>(d) * num_tiles + blockIdx.x];
+        s_delta[d] = offs[static_cast<int64_t>(d) * num_tiles + blockIdx.x];   // global base for now
 
     // All loads of this warp's sub-tile, issued together.
     const int64_t wbase = tile0 + static_cast<int64_t>(warp) * 32 * kDsItems;
@@ -296,10 +296,15 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
         if (lane < chunks) s_chunk[lane] = incl - v;
     }
     __syncthreads();
-    for (int d = threadIdx.x; d < radix; d += kDsThreads) s_tstart[d] += s_chunk[d >> 5];
+    for (int d = threadIdx.x; d < radix; d += kDsThreads) {
+        const int32_t ts = s_tstart[d] + s_chunk[d >> 5];
+        s_delta[d] -= ts;   // global position of tile slot i of digit d = delta[d] + i
+#pragma unroll
+        for (int w = 0; w < kDsWarps; ++w) s_cnt[w * radix + d] += ts;
+    }
     __syncthreads();
 
-    // C: stable slot of every element; stage key, source and edge id.
+    // C: stable slot of every element; stage (key, source, edge id).
     const unsigned lower = (1u << lane) - 1u;
 #pragma unroll
     for (int r = 0; r < kDsItems; ++r) {
@@ -310,12 +315,9 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
         int32_t base = 0;
         if (ok && lane == leader) base = atomicAdd(&mine[dig], __popc(peers));
         base = __shfl_sync(kFull, base, leader);
-        if (ok) {
-            const int slot = s_tstart[dig] + base + __popc(peers & lower);
-            s_key[slot] = keys[r];
-            s_src[slot] = srcs[r];
-            s_eid[slot] = eids[r];
-        }
+        if (ok)
+            s_elem[base + __popc(peers & lower)] =
+                make_uint4(keys[r], static_cast<uint32_t>(srcs[r]), static_cast<uint32_t>(eids[r]), 0u);
     }
     __syncthreads();
 
@@ -324,12 +326,12 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     for (int j = 0; j < kDsItems; ++j) {
         const int i = threadIdx.x + j * kDsThreads;
         if (i < count) {
-            const uint32_t k = s_key[i];
-            const int d = static_cast<int>((k >> shift) & (radix - 1));
-            const int64_t pos = static_cast<int64_t>(s_gbase[d]) + (i - s_tstart[d]);
-            key_out[pos] = k;
-            src_out[pos] = s_src[i];
-            eid_out[pos] = s_eid[i];
+            const uint4 v = s_elem[i];
+            const int d = static_cast<int>((v.x >> shift) & (radix - 1));
+            const int64_t pos = static_cast<int64_t>(s_delta[d]) + i;
+            key_out[pos] = v.x;
+            src_out[pos] = static_cast<int32_t>(v.y);
+            eid_out[pos] = static_cast<int32_t>(v.z);
         }
     }
 }

@@ -269,8 +269,19 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
             for (int u = 0; u < kSmUnroll; ++u) {
                 float v[VEC];
                 V::widen(raw[u], v);
+                if constexpr (VEC % 2 == 0) {
+                    const float2 w2 = make_float2(pw[u], pw[u]);
 #pragma unroll
-                for (int q = 0; q < VEC; ++q) part[q] = fmaf(pw[u], v[q], part[q]);
+                    for (int q = 0; q < VEC; q += 2) {
+                        const float2 r2 = fma2(make_float2(v[q], v[q + 1]), w2,
+                                               make_float2(part[q], part[q + 1]));
+                        part[q] = r2.x;
+                        part[q + 1] = r2.y;
+                    }
+                } else {
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q) part[q] = fmaf(pw[u], v[q], part[q]);
+                }
             }
         }
 #pragma unroll
