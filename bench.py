@@ -97,7 +97,7 @@ def combine_ranks(elapsed_s: float, units: int, world: int, dist=None):
 
 
 KERNEL_SOURCES = {
-    "build_csr": "csr_build.cu", "gcn_norm": "gcn_norm.cu", "gcn_aggregate": "aggregate.cu",
+    "build_csr": "csr_build.cu", "gcn_norm": "gcn_norm.cu", "gcn_aggregate": "agg.cuh",
     "edge_softmax": "edge_softmax.cu", "pool_mean": "segment_pool.cu", "pool_max": "segment_pool.cu",
 }
 
@@ -237,6 +237,114 @@ def cpu_desc(s) -> str:
 
 
 # ---------------------------------------------------------------------------
+def _event_ms(fn, stream, reps: int) -> float:
+    """Mean device time of fn() over reps launches (after 3 untimed), CUDA events
+    on the launching stream."""
+    import torch
+    for _ in range(3):
+        fn()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    t0.record(stream)
+    for _ in range(reps):
+        fn()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    return t0.elapsed_time(t1) / reps
+
+
+def next_rows(L, wl, bufs, stream, hbm_peak):
+    """The rows built beyond the timed step, each measured on its own (not part
+    of the headline value): APPNP K = 10 on the same graph and bf16 features,
+    Transformer-style (dot-product) attention with bf16 q, k, v of the same
+    8 x 16 layout, the fused Mean-Max pool on the GCN output, and device
+    BatchGraph construction on 1,024 molecule-sized graphs."""
+    import torch
+    from paper_2101_11552_gb300 import graphgen as gg
+    from paper_2101_11552_gb300 import tfg
+    P = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
+    dev = bufs["xb"].device
+    sp = ctypes.c_void_p(stream.cuda_stream)
+    n, f = wl.num_nodes, bufs["xb"].shape[1]
+    e = wl.edge_index.shape[1]
+    g = wl.num_graphs
+    rows = {}
+
+    def check(rc):
+        if rc != 0:
+            raise RuntimeError(f"libtfg error {rc}: {tfg.tfg_last_error()}")
+
+    hops, alpha = 10, 0.1
+    out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    ws = torch.empty(max(tfg.tfg_propagate_workspace_size(n, f, hops), 1), dtype=torch.uint8,
+                     device=dev)
+    ms = _event_ms(lambda: check(L.tfg_appnp_propagate(
+        P(bufs["rowptr"]), P(bufs["col"]), P(bufs["dinv"]), None, P(bufs["xb"]), tfg.TFG_BF16,
+        n, f, hops, alpha, 1, 1.0, P(out), P(ws), ws.numel(), sp)), stream, 5)
+    # per hop: col 4E + rowptr + dinv + gathered rows once + x0 row (bf16) + out row;
+    # hop 0 gathers bf16 x0, later hops fp32 iterates
+    hop_bytes = 4 * e + 4 * (n + 1) + 4 * n + 2 * n * f + 4 * n * f
+    abytes = hop_bytes * hops + 2 * n * f + 4 * n * f * (hops - 1)
+    rows["appnp_k10"] = {"ms": round(ms, 4), "hops": hops, "alpha": alpha,
+                         "edge_features_per_s": hops * (e + n) * f / (ms * 1e-3),
+                         "gbs": round(abytes / (ms * 1e-3) / 1e9, 1),
+                         "frac": round(abytes / (ms * 1e-3) / 1e9 / hbm_peak, 4),
+                         "algorithmic_bytes": abytes}
+
+    heads, ch = wl.heads, wl.channels
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1305)
+    qkv = [torch.randn(n, f, generator=gen, device=dev).to(torch.bfloat16) for _ in range(3)]
+    att = torch.empty(n, f, dtype=torch.float32, device=dev)
+    ms = _event_ms(lambda: check(L.tfg_dot_edge_softmax_aggregate(
+        P(bufs["rowptr"]), P(bufs["col"]), *[P(t) for t in qkv], tfg.TFG_BF16, n, e, heads, ch,
+        1.0 / ch ** 0.5, P(att), None, sp)), stream, 10)
+    # col 4E + rowptr + q rows + k and v rows (each row once) + out
+    abytes = 4 * e + 4 * (n + 1) + 3 * 2 * n * f + 4 * n * f
+    rows["dot_softmax"] = {"ms": round(ms, 4), "heads": heads, "channels": ch,
+                           "edge_features_per_s": e * f / (ms * 1e-3),
+                           "gbs": round(abytes / (ms * 1e-3) / 1e9, 1),
+                           "frac": round(abytes / (ms * 1e-3) / 1e9 / hbm_peak, 4),
+                           "algorithmic_bytes": abytes}
+    del qkv, att
+
+    pooled = torch.empty(g, 2 * f, dtype=torch.float32, device=dev)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    ms = _event_ms(lambda: check(L.tfg_segment_pool_meanmax(
+        P(bufs["h"]), tfg.TFG_F32, P(bufs["batch"]), n, g, f, P(pooled), P(st), sp)), stream, 20)
+    abytes = 4 * n * f + 8 * n + 8 * g * f
+    rows["pool_meanmax"] = {"ms": round(ms, 4), "edge_features_per_s": 2 * n * f / (ms * 1e-3),
+                            "gbs": round(abytes / (ms * 1e-3) / 1e9, 1),
+                            "frac": round(abytes / (ms * 1e-3) / 1e9 / hbm_peak, 4),
+                            "algorithmic_bytes": abytes}
+
+    mol = gg.make_c4()
+    sizes = np.asarray(mol.graph_sizes, np.int64)
+    offs = np.concatenate([[0], np.cumsum(sizes)[:-1]])
+    src_graph = mol.batch[mol.edge_index[0]]
+    local = mol.edge_index - offs[src_graph][None, :]
+    ecount = np.bincount(src_graph, minlength=len(sizes)).astype(np.int64)
+    d_sizes, d_ecount = torch.from_numpy(sizes).to(dev), torch.from_numpy(ecount).to(dev)
+    d_local = torch.from_numpy(np.ascontiguousarray(local)).to(dev)
+    mn, me, mg = int(sizes.sum()), local.shape[1], len(sizes)
+    o_ei = torch.empty(2, me, dtype=torch.int64, device=dev)
+    o_b = torch.empty(mn, dtype=torch.int64, device=dev)
+    o_off = torch.empty(mg + 1, dtype=torch.int64, device=dev)
+    wsb = torch.empty(tfg.tfg_batch_graphs_workspace_size(mg), dtype=torch.uint8, device=dev)
+    ms = _event_ms(lambda: check(L.tfg_batch_graphs(
+        mg, P(d_sizes), P(d_ecount), P(d_local), me, mn, P(o_ei), P(o_b), P(o_off), P(wsb),
+        wsb.numel(), P(st), sp)), stream, 50)
+    torch.cuda.synchronize()
+    if int(st.item()) != 0 or not torch.equal(o_ei.cpu(), torch.from_numpy(mol.edge_index)):
+        raise RuntimeError("BatchGraph construction disagrees with the generator's batched graph")
+    abytes = 2 * 16 * me + 8 * mn + 16 * mg
+    rows["batch_graphs"] = {"ms": round(ms, 4), "graphs": mg, "nodes": mn, "edges": me,
+                            "gbs": round(abytes / (ms * 1e-3) / 1e9, 1),
+                            "note": "1,024 molecule-sized graphs (20-200 nodes): launch-bound"}
+    return rows
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -485,6 +593,8 @@ def main():
                 "d2h_bytes_per_step": d2h, "steps": args.e2e_steps},
         "clocks": clocks.summary(),
     }
+    line["next_rows"] = next_rows(L, wl, dict(rowptr=rowptr, col=col, dinv=dinv, xb=xb, h=h,
+                                              batch=batch), stream, hbm_peak)
     if world == 1 and not args.no_cpu_baseline:
         cu, ct, s = time_oracle(wl, args.cpu_budget)
         line["cpu_baseline"] = {"value": cu / ct, "unit": UNIT, "cores": 1, "kind": "oracle",

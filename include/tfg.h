@@ -166,6 +166,43 @@ int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float
                           float *out, tfg_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Multi-hop propagation: APPNP and SGC, node-level models the paper lists
+ * beside GCN and GAT (Section 3) and evaluates in Table 1.  With Ahat the
+ * GCN-normalised adjacency of tfg_gcn_aggregate_sum:
+ *   h_0 = x0,   h_{k+1} = (1 - alpha) * Ahat h_k + alpha * x0,   out = h_K
+ * (K = num_hops).  APPNP (Klicpera et al.) is the power iteration for
+ * personalised PageRank with teleport probability alpha; alpha = 0 gives
+ * SGC's Ahat^K x0 (Wu et al.), also offered as tfg_sgc_propagate.
+ *
+ *   rowptr, col, dinv, w_csr, add_self_loops, self_loop_fill: as for
+ *        tfg_gcn_aggregate_sum (w_csr NULL forms the weights from dinv).
+ *   x0 (device) [num_nodes, num_features] row-major, TFG_F32 or TFG_BF16;
+ *        read by every hop (the teleport term), never written.
+ *   num_hops K in [0, 1024]; K = 0 copies x0 (widened to fp32) into out.
+ *   alpha in [0, 1] (finite).
+ *   out (device) fp32 [num_nodes, num_features], written.
+ *   workspace (device) >= tfg_propagate_workspace_size() bytes, 16-byte
+ *        aligned (N * F fp32 values when K >= 2, else 0 bytes and it may be
+ *        NULL); contents are scratch.
+ * Each hop is one fused launch: GCN gather-sum, self-loop term and the
+ * teleport epilogue  alpha * x0[t] + (1 - alpha) * (...)  (one fp32 fma),
+ * accumulated in fp32 in a fixed order; iterates between hops are fp32.
+ * out, workspace and x0 must not overlap.
+ * ---------------------------------------------------------------------- */
+int tfg_propagate_workspace_size(int64_t num_nodes, int64_t num_features, int64_t num_hops,
+                                 size_t *bytes);
+int tfg_appnp_propagate(const int32_t *rowptr, const int32_t *col, const float *dinv,
+                        const float *w_csr, const void *x0, int x_dtype, int64_t num_nodes,
+                        int64_t num_features, int64_t num_hops, float alpha, int add_self_loops,
+                        float self_loop_fill, float *out, void *workspace,
+                        size_t workspace_bytes, tfg_stream_t stream);
+int tfg_sgc_propagate(const int32_t *rowptr, const int32_t *col, const float *dinv,
+                      const float *w_csr, const void *x0, int x_dtype, int64_t num_nodes,
+                      int64_t num_features, int64_t num_hops, int add_self_loops,
+                      float self_loop_fill, float *out, void *workspace, size_t workspace_bytes,
+                      tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * Edge-softmax (GAT) aggregation -- the map-reduce workflow of Fig. 5a
  * (Section 2.1.2) fused with the weighted sum it feeds:
  *   s_src[n, h] = <x[n, h, :], a_src[h, :]>,  s_dst[n, h] likewise with a_dst
@@ -193,6 +230,36 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
                                const float *a_src, const float *a_dst, float negative_slope,
                                float *out, float *alpha, void *workspace,
                                size_t workspace_bytes, tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Dot-product (Transformer-style) edge-softmax aggregation: the attention
+ * form of tf_geometric's own GAT (Section 3 calls it Transformer-based), on
+ * the map-reduce workflow of Fig. 5a:
+ *   map:    l[k, h] = scale * <q[t, h, :], k[col[k], h, :]>  (position k of row t)
+ *   reduce: alpha[k, h] = exp(l[k, h]) / sum over row t of exp(l[., h])
+ *           (evaluated with the row maximum subtracted; same value)
+ *   out[t, h, :] = sum over row t of alpha[k, h] * v[col[k], h, :]
+ * An empty row gives out = 0.
+ *
+ *   rowptr, col (device): CSR by target (tfg_build_csr).
+ *   q, k, v (device) [num_nodes, heads * channels] row-major, head-major
+ *        within a row ([h0c0 .. h0c(C-1), h1c0, ...]), all three of type
+ *        x_dtype (TFG_F32 or TFG_BF16).  q is read at targets, k and v at
+ *        sources.
+ *   channels <= 256.  scale: finite multiplier of the dot product
+ *        (1 / sqrt(channels) for the Transformer form).
+ *   out (device) fp32 [num_nodes, heads * channels], written.
+ *   alpha (device) fp32 [num_edges, heads] in CSR order, or NULL.
+ * One pass per row with the running-maximum softmax, fp32 accumulation in a
+ * fixed order (deterministic).  16-byte aligned rows with channels a power
+ * of two times 4 (fp32) or 8 (bf16), up to 128 / 256, take the vectorised
+ * kernel; any other layout a general one with the same definition.
+ * No workspace.
+ * ---------------------------------------------------------------------- */
+int tfg_dot_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const void *q,
+                                   const void *k, const void *v, int x_dtype, int64_t num_nodes,
+                                   int64_t num_edges, int heads, int channels, float scale,
+                                   float *out, float *alpha, tfg_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * Edge-softmax aggregation that allocates nothing and takes no workspace.
@@ -239,6 +306,46 @@ int tfg_edge_softmax_aggregate_noalloc(const int32_t *rowptr, const int32_t *col
 int tfg_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t num_nodes,
                      int64_t num_graphs, int64_t num_features, int reduce, float *out,
                      int32_t *status, tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Mean-Max graph pooling in one pass: out[g, 0:F] = mean and out[g, F:2F] =
+ * max over the nodes of graph g -- the concatenated readout of the Mean-Max
+ * Pool model evaluated in Table 2 (Section 4.1), built from the common graph
+ * pooling of Fig. 2a.  Arguments as for tfg_segment_pool, with out
+ * (device) fp32 [num_graphs, 2 * num_features].  Empty graphs give 0 in
+ * both halves.
+ * ---------------------------------------------------------------------- */
+int tfg_segment_pool_meanmax(const void *x, int x_dtype, const int64_t *batch,
+                             int64_t num_nodes, int64_t num_graphs, int64_t num_features,
+                             float *out, int32_t *status, tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * BatchGraph construction on the device: the reindexing trick of Section
+ * 2.1.1 (Fig. 4).  Graph g's j-th node becomes node node_offsets[g] + j,
+ * where node_offsets[g] is the number of nodes in graphs 0 .. g-1; every
+ * edge of graph g is shifted by node_offsets[g]; batch[v] (node_graph_index)
+ * is the graph of node v.
+ *
+ *   node_counts, edge_counts (device) int64 [num_graphs]: nodes and edges of
+ *          each graph.
+ *   edge_index (device) int64 [2, total_edges]: the graphs' own edge lists
+ *          (local node ids 0 .. n_g - 1), stacked in graph order, sources
+ *          row then targets row.
+ *   total_edges, total_nodes: the sums of the counts (sizes of the outputs).
+ *   out_edge_index (device) int64 [2, total_edges]: the batched edge list.
+ *   batch (device) int64 [total_nodes], non-decreasing graph ids.
+ *   node_offsets (device) int64 [num_graphs + 1]; the last entry is the total.
+ *   workspace (device) >= tfg_batch_graphs_workspace_size() bytes.
+ *   status (device) int32 [1]: TFG_ERR_INDEX_RANGE when a count is negative,
+ *          a local id lies outside its graph, or the counts do not sum to the
+ *          declared totals (bad ids are replaced by 0 of their graph).
+ * ---------------------------------------------------------------------- */
+int tfg_batch_graphs_workspace_size(int64_t num_graphs, size_t *bytes);
+int tfg_batch_graphs(int64_t num_graphs, const int64_t *node_counts, const int64_t *edge_counts,
+                     const int64_t *edge_index, int64_t total_edges, int64_t total_nodes,
+                     int64_t *out_edge_index, int64_t *batch, int64_t *node_offsets,
+                     void *workspace, size_t workspace_bytes, int32_t *status,
+                     tfg_stream_t stream);
 
 #ifdef __cplusplus
 }

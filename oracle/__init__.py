@@ -72,6 +72,9 @@ def _load(plant: Optional[str] = None) -> ctypes.CDLL:
                 "oracle_edge_softmax": [I64, I64, P, P, I, I, P, P, D, P, P, P],
                 "oracle_edge_softmax_rows": [I64, P, P, P, I, I, P, P, D, P, I64, P, P, P],
                 "oracle_segment_pool": [I, I64, I64, I64, P, P, P, P],
+                "oracle_appnp": [I64, I64, P, P, P, P, I64, I64, D, P, P],
+                "oracle_dot_softmax": [I64, I64, P, P, P, P, I, I, D, P, P, P],
+                "oracle_dot_softmax_rows": [I64, P, P, P, P, P, I, I, D, P, I64, P, P, P],
             }
             for fn, args in sigs.items():
                 getattr(lib, fn).argtypes = args
@@ -194,6 +197,64 @@ class _Oracle:
             self._p(alpha), self._p(ab)))
         return out[:len(rows)], alpha[:total], ab[:len(rows)]
 
+    # -- dot-product (Transformer-style) attention ----------------------
+    def dot_softmax(self, edge_index, n, q, k, v, heads, channels, scale=None):
+        """Scaled query-key logits, softmax over each target's in-edges per
+        head, attention-weighted sum of values.  scale defaults to 1/sqrt(C).
+        Returns (out [N, H*C], alpha [E, H] in COO order, error scale)."""
+        ei = np.ascontiguousarray(edge_index, dtype=np.int64)
+        e = ei.shape[1]
+        q, k, v = widen(q), widen(k), widen(v)
+        f = q.shape[1]
+        assert f == heads * channels and k.shape == q.shape and v.shape == q.shape
+        sc = 1.0 / np.sqrt(channels) if scale is None else float(scale)
+        out = np.zeros((max(n, 1), f))
+        ab = np.zeros((max(n, 1), f))
+        alpha = np.zeros((max(e, 1), heads))
+        self._check(self.lib.oracle_dot_softmax(n, e, self._p(ei), self._p(q), self._p(k),
+                                                self._p(v), heads, channels, sc, self._p(out),
+                                                self._p(alpha), self._p(ab)))
+        return out[:n], alpha[:e], ab[:n]
+
+    def dot_softmax_rows(self, csr, n, q, k, v, heads, channels, scale, rows):
+        rowptr, col, _, _ = csr
+        q, k, v = widen(q), widen(k), widen(v)
+        f = q.shape[1]
+        rows = np.ascontiguousarray(rows, np.int64)
+        total = int(sum(rowptr[r + 1] - rowptr[r] for r in rows))
+        out = np.zeros((max(len(rows), 1), f))
+        ab = np.zeros((max(len(rows), 1), f))
+        alpha = np.zeros((max(total, 1), heads))
+        self._check(self.lib.oracle_dot_softmax_rows(
+            n, self._p(rowptr), self._p(np.ascontiguousarray(col)), self._p(q), self._p(k),
+            self._p(v), heads, channels, float(scale), self._p(rows), len(rows), self._p(out),
+            self._p(alpha), self._p(ab)))
+        return out[:len(rows)], alpha[:total], ab[:len(rows)]
+
+    # -- multi-hop propagation (APPNP / SGC) ----------------------------
+    def appnp(self, edge_index, n, x0, num_hops, alpha, edge_weight=None, add_self_loops=0,
+              fill=1.0):
+        """K steps of h <- (1 - alpha) Ahat h + alpha x0 from h = x0 (APPNP, the
+        propagation model of Section 3 / Table 1; alpha = 0 is SGC).  Ahat is the
+        GCN normalisation of gcn_norm.  Returns (h_K, error scale), both [N, F]."""
+        ei = np.ascontiguousarray(edge_index, dtype=np.int64)
+        e = ei.shape[1]
+        nrm = self.gcn_norm(ei, n, edge_weight, add_self_loops, fill)
+        x0 = widen(x0)
+        f = x0.shape[1]
+        w = np.ascontiguousarray(nrm["w_norm"], np.float64)
+        sw = None if nrm["self_w"] is None else np.ascontiguousarray(nrm["self_w"], np.float64)
+        out = np.zeros((max(n, 1), f))
+        ab = np.zeros((max(n, 1), f))
+        self._check(self.lib.oracle_appnp(n, e, self._p(ei), self._p(w), self._p(sw),
+                                          self._p(x0), f, int(num_hops), float(alpha),
+                                          self._p(out), self._p(ab)))
+        return out[:n], ab[:n]
+
+    def sgc(self, edge_index, n, x0, num_hops, edge_weight=None, add_self_loops=0, fill=1.0):
+        """Ahat^K x0 (SGC propagation: APPNP with alpha = 0)."""
+        return self.appnp(edge_index, n, x0, num_hops, 0.0, edge_weight, add_self_loops, fill)
+
     # -- pooling --------------------------------------------------------
     def segment_pool(self, x, batch, num_graphs, reduce):
         x = widen(x)
@@ -204,6 +265,39 @@ class _Oracle:
         self._check(self.lib.oracle_segment_pool(REDUCE[reduce], n, f, num_graphs, self._p(b),
                                                  self._p(x), self._p(out), self._p(ab)))
         return out[:num_graphs], ab[:num_graphs]
+
+
+def batch_graphs(node_counts, edge_counts, edge_index):
+    """BatchGraph by the reindexing trick (Section 2.1.1, Fig. 4), one graph
+    at a time: node j of graph g becomes offset_g + j with offset_g the number
+    of nodes in graphs 0 .. g-1; graph g's edges (the next edge_counts[g]
+    columns of the stacked local edge list) are shifted by offset_g.
+    Returns (edge_index [2, E], batch [N], offsets [G + 1])."""
+    node_counts = [int(c) for c in node_counts]
+    edge_counts = [int(c) for c in edge_counts]
+    ei = np.asarray(edge_index, dtype=np.int64)
+    out = np.empty_like(ei)
+    batch = []
+    offsets = [0]
+    col = 0
+    for g, (n_g, e_g) in enumerate(zip(node_counts, edge_counts)):
+        off = offsets[-1]
+        for k in range(col, col + e_g):
+            s, d = int(ei[0, k]), int(ei[1, k])
+            if not (0 <= s < n_g and 0 <= d < n_g):
+                raise OracleError(-5)
+            out[0, k], out[1, k] = off + s, off + d
+        col += e_g
+        batch.extend([g] * n_g)
+        offsets.append(off + n_g)
+    return out, np.asarray(batch, dtype=np.int64), np.asarray(offsets, dtype=np.int64)
+
+
+def segment_pool_meanmax(x, batch, num_graphs):
+    """Mean-Max Pool readout (Table 2): [mean | max] per graph."""
+    mean, amean = default.segment_pool(x, batch, num_graphs, "mean")
+    mx, amax = default.segment_pool(x, batch, num_graphs, "max")
+    return np.concatenate([mean, mx], axis=1), np.concatenate([amean, amax], axis=1)
 
 
 def widen(x: np.ndarray) -> np.ndarray:
@@ -245,6 +339,10 @@ aggregate_rows = default.aggregate_rows
 edge_softmax = default.edge_softmax
 edge_softmax_rows = default.edge_softmax_rows
 segment_pool = default.segment_pool
+appnp = default.appnp
+dot_softmax = default.dot_softmax
+dot_softmax_rows = default.dot_softmax_rows
+sgc = default.sgc
 
 
 def planted(plant: str) -> _Oracle:

@@ -405,3 +405,177 @@ int oracle_segment_pool(int reduce, int64_t n, int64_t f, int64_t g, const int64
     free(count);
     return OK;
 }
+
+/* ---------------------------------------------------------------------------
+ * Multi-hop propagation: APPNP and SGC, two of the node-level models the
+ * paper lists (Section 3) and evaluates (Table 1).  APPNP (Klicpera et al.)
+ * runs K steps of
+ *     h_0 = x0,   h_{k+1}[t] = (1 - alpha) * (sum over edges e into t of
+ *                   w_e * h_k[src_e]  +  self_w[t] * h_k[t])  +  alpha * x0[t]
+ * with w, self_w the GCN-normalised weights of oracle_gcn_norm; SGC
+ * (Wu et al.) is alpha = 0.  Each step loops over the edges in their
+ * original order, fp64 throughout.  absout runs the same recursion on
+ * absolute values (|w|, |self_w|, |x0|): the scale of the rounding error of
+ * an fp32 evaluation.  out/absout are [n, f].
+ * ------------------------------------------------------------------------- */
+int oracle_appnp(int64_t n, int64_t e, const int64_t *edge_index, const double *w,
+                 const double *self_w, const double *x0, int64_t f, int64_t hops, double alpha,
+                 double *out, double *absout)
+{
+    if (n < 0 || e < 0 || f < 0 || hops < 0 || !w) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+    for (int64_t i = 0; i < e; ++i)
+        if (src[i] < 0 || src[i] >= n || dst[i] < 0 || dst[i] >= n) return E_RANGE;
+    const size_t cells = (size_t)(n * f > 0 ? n * f : 1);
+    double *th = (double *)calloc(cells, sizeof(double));
+    double *ta = (double *)calloc(cells, sizeof(double));
+    if (!th || !ta) { free(th); free(ta); return E_ARG; }
+    for (int64_t k = 0; k < n * f; ++k) { out[k] = x0[k]; absout[k] = fabs(x0[k]); }
+    for (int64_t hop = 0; hop < hops; ++hop) {
+        for (int64_t k = 0; k < n * f; ++k) { th[k] = 0.0; ta[k] = 0.0; }
+        for (int64_t i = 0; i < e; ++i) {
+            const int64_t s = src[i], t = dst[i];
+            for (int64_t c = 0; c < f; ++c) {
+                th[t * f + c] += w[i] * out[s * f + c];
+                ta[t * f + c] += fabs(w[i]) * absout[s * f + c];
+            }
+        }
+        if (self_w)
+            for (int64_t t = 0; t < n; ++t)
+                for (int64_t c = 0; c < f; ++c) {
+                    th[t * f + c] += self_w[t] * out[t * f + c];
+                    ta[t * f + c] += fabs(self_w[t]) * absout[t * f + c];
+                }
+        for (int64_t k = 0; k < n * f; ++k) {
+#ifdef ORACLE_PLANT_APPNP_TELEPORT_FROM_H
+            const double tele = out[k];                  /* planted: teleport to h_k, not x0 */
+#else
+            const double tele = x0[k];
+#endif
+            out[k] = (1.0 - alpha) * th[k] + alpha * tele;
+            absout[k] = (1.0 - alpha) * ta[k] + alpha * fabs(x0[k]);
+        }
+    }
+    free(th);
+    free(ta);
+    return OK;
+}
+
+/* ---------------------------------------------------------------------------
+ * Dot-product (Transformer-style) attention, the GAT form the paper says
+ * tf_geometric uses (Section 3), on the workflow of Fig. 5a:
+ *   map        l[e,h] = scale * sum_c q[dst_e,h,c] k[src_e,h,c]
+ *   reduce     m[t,h] = max over edges into t of l[e,h]          (stability)
+ *              den[t,h] = sum over edges into t of exp(l[e,h] - m[t,h])
+ *   map        alpha[e,h] = exp(l[e,h] - m[dst_e,h]) / den[dst_e,h]
+ *   aggregate  out[t,h,:] = sum over edges into t of alpha[e,h] v[src_e,h,:]
+ * q, k, v are [n, H*C], head-major within a row; alpha is [e, H] in COO
+ * order; targets without incoming edges give 0.
+ * absout[t, h*C+c] = sum of alpha[e,h] |v[src_e,h,c]|.
+ * ------------------------------------------------------------------------- */
+static double dot_logit(const double *q, const double *k, int64_t t, int64_t s, int64_t f,
+                        int hh, int c, double scale)
+{
+    double d = 0.0;
+    for (int cc = 0; cc < c; ++cc) {
+#ifdef ORACLE_PLANT_DOT_KEY_AT_TARGET
+        d += q[t * f + hh * c + cc] * k[t * f + hh * c + cc];   /* planted: key of the target */
+        (void)s;
+#else
+        d += q[t * f + hh * c + cc] * k[s * f + hh * c + cc];
+#endif
+    }
+    return scale * d;
+}
+
+int oracle_dot_softmax(int64_t n, int64_t e, const int64_t *edge_index, const double *q,
+                       const double *k, const double *v, int h, int c, double scale,
+                       double *out, double *alpha, double *absout)
+{
+    if (n < 0 || e < 0 || h <= 0 || c <= 0) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+    for (int64_t i = 0; i < e; ++i)
+        if (src[i] < 0 || src[i] >= n || dst[i] < 0 || dst[i] >= n) return E_RANGE;
+    int64_t f = (int64_t)h * c;
+    size_t nh = (size_t)(n > 0 ? n : 1) * (size_t)h;
+    double *mx = (double *)calloc(nh, sizeof(double));
+    double *den = (double *)calloc(nh, sizeof(double));
+    char *seen = (char *)calloc(nh, 1);
+    double *logit = (double *)calloc((size_t)(e > 0 ? e : 1) * (size_t)h, sizeof(double));
+    if (!mx || !den || !seen || !logit) {
+        free(mx); free(den); free(seen); free(logit);
+        return E_ARG;
+    }
+    /* map: scaled query-key products; reduce: per-target max */
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            double l = dot_logit(q, k, dst[i], src[i], f, hh, c, scale);
+            logit[i * h + hh] = l;
+            size_t kk = (size_t)dst[i] * h + hh;
+            if (!seen[kk] || l > mx[kk]) mx[kk] = l;
+            seen[kk] = 1;
+        }
+    /* reduce: segment sum of exp -> softmax denominator */
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh)
+            den[(size_t)dst[i] * h + hh] += exp(logit[i * h + hh] - mx[(size_t)dst[i] * h + hh]);
+    /* map: divide; then the attention-weighted sum of values */
+    for (int64_t kk = 0; kk < n * f; ++kk) { out[kk] = 0.0; absout[kk] = 0.0; }
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            size_t kk = (size_t)dst[i] * h + hh;
+            double al = exp(logit[i * h + hh] - mx[kk]) / den[kk];
+            if (alpha) alpha[i * h + hh] = al;
+            for (int cc = 0; cc < c; ++cc) {
+                double m = al * v[src[i] * f + hh * c + cc];
+                out[dst[i] * f + hh * c + cc] += m;
+                absout[dst[i] * f + hh * c + cc] += fabs(m);
+            }
+        }
+    free(mx); free(den); free(seen); free(logit);
+    return OK;
+}
+
+/* The same passes for the listed target rows only, through the oracle's
+ * stable CSR; alpha_rows packs each listed row's [deg, H] block in CSR order. */
+int oracle_dot_softmax_rows(int64_t n, const int32_t *rowptr, const int32_t *col,
+                            const double *q, const double *k, const double *v, int h, int c,
+                            double scale, const int64_t *rows, int64_t nrows, double *out,
+                            double *alpha_rows, double *absout)
+{
+    if (h <= 0 || c <= 0) return E_ARG;
+    int64_t f = (int64_t)h * c;
+    int64_t apos = 0;
+    for (int64_t r = 0; r < nrows; ++r) {
+        int64_t t = rows[r];
+        if (t < 0 || t >= n) return E_RANGE;
+        int64_t k0 = rowptr[t], k1 = rowptr[t + 1], deg = k1 - k0;
+        double *o = out + r * f, *ab = absout + r * f;
+        for (int64_t x = 0; x < f; ++x) { o[x] = 0.0; ab[x] = 0.0; }
+        if (deg == 0) continue;
+        double *lg = (double *)malloc(sizeof(double) * (size_t)deg);
+        if (!lg) return E_ARG;
+        for (int hh = 0; hh < h; ++hh) {
+            double mx = 0.0, den = 0.0;
+            for (int64_t p = k0; p < k1; ++p) {
+                double l = dot_logit(q, k, t, col[p], f, hh, c, scale);
+                lg[p - k0] = l;
+                if (p == k0 || l > mx) mx = l;
+            }
+            for (int64_t p = k0; p < k1; ++p) den += exp(lg[p - k0] - mx);
+            for (int64_t p = k0; p < k1; ++p) {
+                int64_t s = col[p];
+                double al = exp(lg[p - k0] - mx) / den;
+                if (alpha_rows) alpha_rows[(apos + (p - k0)) * h + hh] = al;
+                for (int cc = 0; cc < c; ++cc) {
+                    double m = al * v[s * f + hh * c + cc];
+                    o[hh * c + cc] += m;
+                    ab[hh * c + cc] += fabs(m);
+                }
+            }
+        }
+        apos += deg;
+        free(lg);
+    }
+    return OK;
+}

@@ -1,0 +1,344 @@
+// Fused gather * weight * reduce over a CSR grouped by target: the message
+// aggregation of tf_geometric (Fig. 1) with the reducer of Fig. 5b, which the
+// paper implements as tf.math.unsorted_segment_* over the edge list
+// (Section 2.1.2).  Grouping by target first turns the scatter-reduce into
+// owner-computes row reductions: no atomics, a fixed summation order, and
+// bit-identical results from run to run.
+//
+// Work layout
+//  * A CTA (8 warps) owns a contiguous range of target rows holding an equal
+//    share of edges + rows (a merge-path split of rowptr), so a hub row does
+//    not leave one CTA running long after the others.  Its warps take rows
+//    one at a time from a shared counter.  A row is split among
+//    G = 32 / LPR lane groups: each group of LPR lanes covers LPR * VEC
+//    features (16-byte loads when the layout allows) and takes every G-th
+//    edge of the row; the groups' partials are then combined by a butterfly.
+//  * Rows longer than kHeavyDeg (power-law hubs) are set aside and done after
+//    the light rows by the whole CTA: each warp takes one contiguous slice of
+//    the row, and the eight warp partials are combined in warp order through
+//    shared memory.  No global scratch and no inter-CTA waiting.
+//  * Column ids (and weights) of 32 edges are loaded by the 32 lanes at once
+//    and broadcast with shuffles; kUnroll gathers are kept in flight per lane.
+//  * GCN mode without w_csr forms the weight on the fly:  out[t] = dinv[t] *
+//    (sum_k dinv[col[k]] * x[col[k]] + fill * dinv[t] * x[t]), so no per-edge
+//    weight array is read.  With w_csr it adds fill * dinv[t]^2 * x[t] to the
+//    weighted sum.
+//  * APPNP mode (one propagation step, Klicpera et al., the APPNP model the
+//    paper lists in Section 3 and Table 1) is GCN mode with an epilogue:
+//    out[t] = (1 - alpha) * gcn(h)[t] + alpha * x0[t], x0 read in its own
+//    storage type X0T.  alpha = 0 is one SGC step.
+//
+// Shared by aggregate.cu (one-hop entry points) and propagate.cu (multi-hop);
+// each translation unit instantiates the variants it launches.
+#pragma once
+#include <math_constants.h>
+
+#include "common.cuh"
+
+namespace tfg {
+namespace {
+
+constexpr int kAggWarps = 8;
+constexpr int kAggThreads = kAggWarps * 32;
+// Tuning knobs (compile-time; the defaults are the measured best on GB300).
+#ifndef TFG_HEAVY_DEG
+#define TFG_HEAVY_DEG 2048
+#endif
+#ifndef TFG_AGG_UNROLL
+#define TFG_AGG_UNROLL 4
+#endif
+#ifndef TFG_AGG_MINB
+#define TFG_AGG_MINB 4   // resident CTAs per SM asked of the compiler, 16-byte bf16 path
+#endif
+constexpr int kHeavyDeg = TFG_HEAVY_DEG;
+constexpr int kMaxHeavy = 64;   // hub rows a CTA sets aside; more are done warp by warp
+// gathers in flight per lane: deeper for the 16-byte bf16 sum path (measured
+// faster there), 4 elsewhere (keeps the other variants free of spills)
+template <int VEC, bool IS_MAX>
+constexpr int unroll_for() { return (VEC >= 8 && !IS_MAX) ? TFG_AGG_UNROLL : 4; }
+
+struct AggArgs {
+    const int32_t *rowptr;
+    const int32_t *col;
+    const float *w;     // CSR-order weights or null (sum / mean / max)
+    const float *dinv;  // GCN mode
+    const void *x;
+    float *out;
+    int64_t n;
+    int64_t f;
+    int mean;
+    int add_self;
+    float fill;
+    const void *x0;     // APPNP mode: the teleport features x0 [N, F]
+    float alpha;        // APPNP mode: teleport weight
+    float beta;         // APPNP mode: 1 - alpha, rounded once on the host
+};
+
+enum Kind { kSumLike = 0, kMax = 1, kGcn = 2, kAppnp = 3 };
+
+template <typename XT, int VEC, int LPR, int KIND, typename X0T = XT>
+struct Agg {
+    static constexpr int G = 32 / LPR;
+    static constexpr bool kIsMax = KIND == kMax;
+    static constexpr bool kGcnLike = KIND == kGcn || KIND == kAppnp;
+    static constexpr int kUnroll = unroll_for<VEC, kIsMax>();
+
+    static __device__ __forceinline__ float identity() { return kIsMax ? -CUDART_INF_F : 0.f; }
+
+    static __device__ __forceinline__ float combine(float a, float b) {
+        return kIsMax ? fmaxf(a, b) : a + b;
+    }
+
+    // part[q] += w * v[q] for one gathered vector (pairs through fma2).
+    static __device__ __forceinline__ void axpy(float (&part)[VEC], float w,
+                                                const typename VecLoad<XT, VEC>::Raw &raw) {
+        float v[VEC];
+        VecLoad<XT, VEC>::widen(raw, v);
+        if constexpr (VEC % 2 == 0) {
+            const float2 w2 = make_float2(w, w);
+#pragma unroll
+            for (int q = 0; q < VEC; q += 2) {
+                const float2 r = fma2(make_float2(v[q], v[q + 1]), w2, make_float2(part[q], part[q + 1]));
+                part[q] = r.x;
+                part[q + 1] = r.y;
+            }
+        } else {
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) part[q] = fmaf(w, v[q], part[q]);
+        }
+    }
+
+    // One 32-edge chunk of a sum: group g takes edges g, g + G, ...  FULL
+    // chunks need no bounds checks; in a partial chunk the slots past cnt get
+    // weight 0 and read row 0 (always valid), contributing an exact zero.
+    // Lanes whose features lie past F read the row's first features instead
+    // (in bounds); their partials are never stored.
+    template <bool FULL>
+    static __device__ __forceinline__ void sum_chunk(const XT *xf, uint32_t fs, int c, float ww,
+                                                     int cnt, int g, bool weighted,
+                                                     float (&part)[VEC]) {
+        using V = VecLoad<XT, VEC>;
+        for (int j = 0; j < (FULL ? 32 : cnt); j += G * kUnroll) {
+            typename V::Raw raw[kUnroll];
+            float wt[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int k = j + u * G + g;
+                const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31));
+                wt[u] = weighted ? __shfl_sync(kFull, ww, k & 31) : 1.f;
+                if (!FULL && k >= cnt) wt[u] = 0.f;
+                raw[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
+            }
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) axpy(part, wt[u], raw[u]);
+        }
+    }
+
+    // Accumulate edges [beg, end) into acc (this lane's VEC features at f0).
+    // Each 32-edge chunk is summed into its own partial before it is added to
+    // acc, so an fp32 chain is at most 32 / G + deg / 32 additions long.  The
+    // order is fixed, so results are deterministic.
+    static __device__ __forceinline__ void edges(const AggArgs &a, int64_t beg, int64_t end,
+                                                 int64_t f0, bool fok, float (&acc)[VEC],
+                                                 int lane) {
+        using V = VecLoad<XT, VEC>;
+        const XT *x = static_cast<const XT *>(a.x);
+        const XT *xf = x + (fok ? f0 : 0);
+        const uint32_t fs = static_cast<uint32_t>(a.f);
+        const int g = lane / LPR;
+        const bool weighted = kGcnLike || a.w != nullptr;
+        if (a.col == nullptr) return;   // a graph without edges
+        for (int64_t base = beg; base < end; base += 32) {
+            const int cnt = static_cast<int>(min64(32, end - base));
+            int c = 0;
+            float ww = 1.f;
+            if (lane < cnt) {
+                c = __ldg(a.col + base + lane);
+                if (a.w) ww = __ldg(a.w + base + lane);
+                else if (kGcnLike) ww = __ldg(a.dinv + c);
+            }
+            if constexpr (kIsMax) {
+                for (int j = 0; j < cnt; j += G * kUnroll) {
+                    typename V::Raw raw[kUnroll];
+                    float wt[kUnroll];
+                    bool ok[kUnroll];
+#pragma unroll
+                    for (int u = 0; u < kUnroll; ++u) {
+                        const int k = j + u * G + g;
+                        const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31));
+                        wt[u] = weighted ? __shfl_sync(kFull, ww, k & 31) : 1.f;
+                        ok[u] = fok && (k < cnt);
+                        raw[u] = ok[u] ? V::raw(xf + static_cast<uint64_t>(src) * fs) : V::zero();
+                    }
+#pragma unroll
+                    for (int u = 0; u < kUnroll; ++u) {
+                        if (!ok[u]) continue;
+                        float v[VEC];
+                        V::widen(raw[u], v);
+#pragma unroll
+                        for (int q = 0; q < VEC; ++q) acc[q] = fmaxf(acc[q], wt[u] * v[q]);
+                    }
+                }
+            } else {
+                float part[VEC];
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) part[q] = 0.f;
+                if (cnt == 32) sum_chunk<true>(xf, fs, c, ww, cnt, g, weighted, part);
+                else sum_chunk<false>(xf, fs, c, ww, cnt, g, weighted, part);
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) acc[q] += part[q];
+            }
+        }
+    }
+
+    static __device__ __forceinline__ void reduce_groups(float (&acc)[VEC]) {
+#pragma unroll
+        for (int s = LPR; s < 32; s <<= 1)
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] = combine(acc[q], __shfl_xor_sync(kFull, acc[q], s));
+    }
+
+    // Final value of one feature of row t from its reduced accumulator.
+    static __device__ __forceinline__ float finish(const AggArgs &a, int64_t t, int64_t deg,
+                                                   float acc, float xt, float dt, float x0t) {
+        if (kGcnLike) {
+            float r;
+            if (a.w) r = a.add_self ? acc + (a.fill * dt) * dt * xt : acc;
+            else r = a.add_self ? dt * (acc + a.fill * dt * xt) : dt * acc;
+            if (KIND == kAppnp) r = fmaf(a.alpha, x0t, a.beta * r);
+            return r;
+        }
+        if (deg == 0) return 0.f;
+        if (a.mean) return acc / static_cast<float>(deg);
+        return acc;
+    }
+
+    static __device__ void warp_row(const AggArgs &a, int64_t t, int lane) {
+        const int64_t beg = a.rowptr[t], end = a.rowptr[t + 1];
+        const int sub = lane % LPR;
+        const float dt = kGcnLike ? __ldg(a.dinv + t) : 1.f;
+        for (int64_t ft = 0; ft < a.f; ft += LPR * VEC) {
+            const int64_t f0 = ft + sub * VEC;
+            const bool fok = f0 < a.f;
+            float acc[VEC];
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] = identity();
+            edges(a, beg, end, f0, fok, acc, lane);
+            reduce_groups(acc);
+            if (lane < LPR && fok) {
+                float xt[VEC], x0t[VEC];
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) xt[q] = x0t[q] = 0.f;
+                if (kGcnLike && a.add_self)
+                    VecLoad<XT, VEC>::load(static_cast<const XT *>(a.x) + t * a.f + f0, xt);
+                if (KIND == kAppnp)
+                    VecLoad<X0T, VEC>::load(static_cast<const X0T *>(a.x0) + t * a.f + f0, x0t);
+                float *o = a.out + t * a.f + f0;
+                float r[VEC];
+#pragma unroll
+                for (int q = 0; q < VEC; ++q)
+                    r[q] = finish(a, t, end - beg, acc[q], xt[q], dt, x0t[q]);
+                if constexpr (VEC % 4 == 0) {
+#pragma unroll
+                    for (int q = 0; q < VEC; q += 4)
+                        *reinterpret_cast<float4 *>(o + q) = make_float4(r[q], r[q + 1], r[q + 2], r[q + 3]);
+                } else {
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q) o[q] = r[q];
+                }
+            }
+        }
+    }
+
+    // A hub row done by all warps of the CTA; partials combined in warp order.
+    static __device__ void cta_row(const AggArgs &a, int64_t t, float *s_part) {
+        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, sub = lane % LPR;
+        const int64_t beg = a.rowptr[t], end = a.rowptr[t + 1], deg = end - beg;
+        const int64_t per = ((deg + kAggWarps - 1) / kAggWarps + 31) / 32 * 32;
+        const int64_t wb = min(end, beg + warp * per), we = min(end, wb + per);
+        const float dt = kGcnLike ? __ldg(a.dinv + t) : 1.f;
+        constexpr int kSlots = LPR * VEC;
+        for (int64_t ft = 0; ft < a.f; ft += kSlots) {
+            const int64_t f0 = ft + sub * VEC;
+            const bool fok = f0 < a.f;
+            float acc[VEC];
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] = identity();
+            edges(a, wb, we, f0, fok, acc, lane);
+            reduce_groups(acc);
+            if (lane < LPR) {
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) s_part[warp * kSlots + sub * VEC + q] = acc[q];
+            }
+            __syncthreads();
+            for (int i = threadIdx.x; i < kSlots; i += kAggThreads) {
+                const int64_t fi = ft + i;
+                if (fi < a.f) {
+                    float r = s_part[i];
+                    for (int w = 1; w < kAggWarps; ++w) r = combine(r, s_part[w * kSlots + i]);
+                    float one[1] = {0.f}, x0t[1] = {0.f};
+                    if (kGcnLike && a.add_self)
+                        VecLoad<XT, 1>::load(static_cast<const XT *>(a.x) + t * a.f + fi, one);
+                    if (KIND == kAppnp)
+                        VecLoad<X0T, 1>::load(static_cast<const X0T *>(a.x0) + t * a.f + fi, x0t);
+                    a.out[t * a.f + fi] = finish(a, t, deg, r, one[0], dt, x0t[0]);
+                }
+            }
+            __syncthreads();
+        }
+    }
+};
+
+template <typename XT, int VEC, int LPR, int KIND, typename X0T>
+__global__ void __launch_bounds__(kAggThreads, VEC >= 8 ? TFG_AGG_MINB : 4) aggregate_kernel(AggArgs a) {
+    using A = Agg<XT, VEC, LPR, KIND, X0T>;
+    __shared__ int s_next, s_nheavy;
+    __shared__ int64_t s_heavy[kMaxHeavy];
+    __shared__ float s_part[kAggWarps * LPR * VEC];
+    int64_t r0, r1;
+    balanced_rows(a.rowptr, a.n, gridDim.x, blockIdx.x, r0, r1);
+    const int64_t nrows = r1 - r0;
+    if (threadIdx.x == 0) {
+        s_next = 0;
+        s_nheavy = 0;
+    }
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    for (;;) {
+        int i = 0;
+        if (lane == 0) i = atomicAdd(&s_next, 1);
+        i = __shfl_sync(kFull, i, 0);
+        if (i >= nrows) break;
+        const int64_t t = r0 + i;
+        if (a.col != nullptr && a.rowptr[t + 1] - a.rowptr[t] > kHeavyDeg) {
+            int slot = 0;
+            if (lane == 0) slot = atomicAdd(&s_nheavy, 1);
+            slot = __shfl_sync(kFull, slot, 0);
+            if (slot < kMaxHeavy) {
+                if (lane == 0) s_heavy[slot] = t;
+                continue;
+            }
+        }
+        A::warp_row(a, t, lane);
+    }
+    __syncthreads();
+    const int nh = min(s_nheavy, kMaxHeavy);
+    for (int h = 0; h < nh; ++h) A::cta_row(a, s_heavy[h], s_part);
+}
+
+template <typename XT, int VEC, int KIND, typename X0T = XT>
+cudaError_t launch_lpr(const AggArgs &a, int lpr, cudaStream_t s) {
+    // E is not known on the host; the kernel reads rowptr[N] for the split.
+    const int grid = balanced_grid(a.n, 0, 1);
+    switch (lpr) {
+        case 32: aggregate_kernel<XT, VEC, 32, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
+        case 16: aggregate_kernel<XT, VEC, 16, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
+        default: aggregate_kernel<XT, VEC, 8, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
+    }
+    return cudaGetLastError();
+}
+
+inline int lanes_per_row(int64_t chunks) { return chunks >= 32 ? 32 : (chunks > 8 ? 16 : 8); }
+
+}  // namespace
+}  // namespace tfg

@@ -82,6 +82,37 @@ int aggregate_common(const char *fn, int mode, const int32_t *rowptr, const int3
                        fn);
 }
 
+constexpr int kMaxHops = 1024;
+
+int propagate_common(const char *fn, const int32_t *rowptr, const int32_t *col, const float *dinv,
+                     const float *w, const void *x0, int dtype, int64_t n, int64_t f, int64_t hops,
+                     float alpha, int add_self, float fill, float *out, void *ws, size_t ws_bytes,
+                     tfg_stream_t stream) {
+    TFG_TRY(check_counts(fn, n, 0));
+    TFG_TRY(check_features(fn, n, f));
+    TFG_TRY(check_dtype(fn, dtype));
+    if (hops < 0 || hops > kMaxHops)
+        return fail(TFG_ERR_INVALID_ARG, "%s: num_hops must be in [0, %d]", fn, kMaxHops);
+    if (!(alpha >= 0.f && alpha <= 1.f))
+        return fail(TFG_ERR_INVALID_ARG, "%s: alpha must be in [0, 1]", fn);
+    TFG_NEED(rowptr, hops > 0, fn, "rowptr");
+    TFG_NEED(dinv, hops > 0 && n > 0, fn, "dinv");
+    TFG_NEED(x0, n > 0, fn, "x0");
+    TFG_NEED(out, n > 0, fn, "out");
+    const size_t need = tfg::propagate_workspace_bytes(n, f, hops);
+    if (need > 0) {
+        if (ws == nullptr || ws_bytes < need)
+            return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
+                        ws ? ws_bytes : size_t(0));
+        if (reinterpret_cast<uintptr_t>(ws) % 16 != 0)
+            return fail(TFG_ERR_INVALID_ARG, "%s: workspace must be 16-byte aligned", fn);
+    }
+    return cuda_result(tfg::launch_propagate(rowptr, col, w, dinv, x0, dtype, n, f, hops, alpha,
+                                             add_self, fill, out, ws,
+                                             reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
 }  // namespace
 
 namespace tfg {
@@ -186,6 +217,38 @@ int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float
                             num_nodes, num_features, add_self_loops, self_loop_fill, out, stream);
 }
 
+int tfg_propagate_workspace_size(int64_t num_nodes, int64_t num_features, int64_t num_hops,
+                                 size_t *bytes) {
+    const char *fn = "tfg_propagate_workspace_size";
+    TFG_TRY(check_counts(fn, num_nodes, 0));
+    TFG_TRY(check_features(fn, num_nodes, num_features));
+    if (num_hops < 0 || num_hops > kMaxHops)
+        return fail(TFG_ERR_INVALID_ARG, "%s: num_hops must be in [0, %d]", fn, kMaxHops);
+    TFG_NEED(bytes, true, fn, "bytes");
+    *bytes = tfg::propagate_workspace_bytes(num_nodes, num_features, num_hops);
+    return ok();
+}
+
+int tfg_appnp_propagate(const int32_t *rowptr, const int32_t *col, const float *dinv,
+                        const float *w_csr, const void *x0, int x_dtype, int64_t num_nodes,
+                        int64_t num_features, int64_t num_hops, float alpha, int add_self_loops,
+                        float self_loop_fill, float *out, void *workspace,
+                        size_t workspace_bytes, tfg_stream_t stream) {
+    return propagate_common("tfg_appnp_propagate", rowptr, col, dinv, w_csr, x0, x_dtype,
+                            num_nodes, num_features, num_hops, alpha, add_self_loops,
+                            self_loop_fill, out, workspace, workspace_bytes, stream);
+}
+
+int tfg_sgc_propagate(const int32_t *rowptr, const int32_t *col, const float *dinv,
+                      const float *w_csr, const void *x0, int x_dtype, int64_t num_nodes,
+                      int64_t num_features, int64_t num_hops, int add_self_loops,
+                      float self_loop_fill, float *out, void *workspace, size_t workspace_bytes,
+                      tfg_stream_t stream) {
+    return propagate_common("tfg_sgc_propagate", rowptr, col, dinv, w_csr, x0, x_dtype,
+                            num_nodes, num_features, num_hops, 0.f, add_self_loops,
+                            self_loop_fill, out, workspace, workspace_bytes, stream);
+}
+
 int tfg_edge_softmax_workspace_size(int64_t num_nodes, int heads, size_t *bytes) {
     const char *fn = "tfg_edge_softmax_workspace_size";
     TFG_TRY(check_counts(fn, num_nodes, 0));
@@ -224,6 +287,34 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
                        fn);
 }
 
+int tfg_dot_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const void *q,
+                                   const void *k, const void *v, int x_dtype, int64_t num_nodes,
+                                   int64_t num_edges, int heads, int channels, float scale,
+                                   float *out, float *alpha, tfg_stream_t stream) {
+    const char *fn = "tfg_dot_edge_softmax_aggregate";
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    if (heads < 1 || channels < 1)
+        return fail(TFG_ERR_INVALID_ARG, "%s: heads and channels must be >= 1", fn);
+    if (channels > tfg::dot_softmax_max_channels())
+        return fail(TFG_ERR_TOO_LARGE, "%s: at most %d channels per head", fn,
+                    tfg::dot_softmax_max_channels());
+    TFG_TRY(check_features(fn, num_nodes, int64_t(heads) * channels));
+    TFG_TRY(check_dtype(fn, x_dtype));
+    if (!(scale == scale) || scale == INFINITY || scale == -INFINITY)
+        return fail(TFG_ERR_INVALID_ARG, "%s: scale must be finite", fn);
+    TFG_NEED(rowptr, true, fn, "rowptr");
+    TFG_NEED(col, num_edges > 0, fn, "col");
+    TFG_NEED(q, num_nodes > 0, fn, "q");
+    TFG_NEED(k, num_nodes > 0, fn, "k");
+    TFG_NEED(v, num_nodes > 0, fn, "v");
+    TFG_NEED(out, num_nodes > 0, fn, "out");
+    return cuda_result(tfg::launch_dot_softmax(rowptr, num_edges > 0 ? col : nullptr, q, k, v,
+                                               x_dtype, num_nodes, num_edges, heads, channels,
+                                               scale, out, alpha,
+                                               reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
 int tfg_edge_softmax_aggregate_noalloc(const int32_t *rowptr, const int32_t *col, const void *x,
                                        int x_dtype, int64_t num_nodes, int64_t num_edges,
                                        int heads, int channels, const float *a_src,
@@ -257,6 +348,64 @@ int tfg_edge_softmax_aggregate_noalloc(const int32_t *rowptr, const int32_t *col
     return cuda_result(tfg::launch_edge_softmax(rowptr, num_edges > 0 ? col : nullptr, x, x_dtype,
                                                 num_nodes, num_edges, heads, channels, a_src, a_dst,
                                                 negative_slope, out, alpha, scratch,
+                                                reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+int tfg_segment_pool_meanmax(const void *x, int x_dtype, const int64_t *batch,
+                             int64_t num_nodes, int64_t num_graphs, int64_t num_features,
+                             float *out, int32_t *status, tfg_stream_t stream) {
+    const char *fn = "tfg_segment_pool_meanmax";
+    if (num_nodes < 0 || num_graphs < 0)
+        return fail(TFG_ERR_INVALID_ARG, "%s: negative size", fn);
+    if (num_graphs >= kIndexLimit) return fail(TFG_ERR_TOO_LARGE, "%s: too many graphs", fn);
+    TFG_TRY(check_features(fn, num_nodes > num_graphs ? num_nodes : num_graphs, num_features));
+    TFG_TRY(check_dtype(fn, x_dtype));
+    if (num_features > int64_t(65535) * 8)
+        return fail(TFG_ERR_TOO_LARGE, "%s: at most %d features", fn, 65535 * 8);
+    TFG_NEED(x, num_nodes > 0, fn, "x");
+    TFG_NEED(batch, num_nodes > 0, fn, "batch");
+    TFG_NEED(out, num_graphs > 0, fn, "out");
+    TFG_NEED(status, true, fn, "status");
+    return cuda_result(tfg::launch_segment_pool(x, x_dtype, batch, num_nodes, num_graphs,
+                                                num_features, 3 /* mean | max */, out, status,
+                                                reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+int tfg_batch_graphs_workspace_size(int64_t num_graphs, size_t *bytes) {
+    const char *fn = "tfg_batch_graphs_workspace_size";
+    if (num_graphs < 0) return fail(TFG_ERR_INVALID_ARG, "%s: negative size", fn);
+    TFG_NEED(bytes, true, fn, "bytes");
+    *bytes = tfg::batch_graphs_workspace_bytes(num_graphs);
+    return ok();
+}
+
+int tfg_batch_graphs(int64_t num_graphs, const int64_t *node_counts, const int64_t *edge_counts,
+                     const int64_t *edge_index, int64_t total_edges, int64_t total_nodes,
+                     int64_t *out_edge_index, int64_t *batch, int64_t *node_offsets,
+                     void *workspace, size_t workspace_bytes, int32_t *status,
+                     tfg_stream_t stream) {
+    const char *fn = "tfg_batch_graphs";
+    TFG_TRY(check_counts(fn, total_nodes, total_edges));
+    if (num_graphs < 0) return fail(TFG_ERR_INVALID_ARG, "%s: negative graph count", fn);
+    if (num_graphs >= kIndexLimit) return fail(TFG_ERR_TOO_LARGE, "%s: too many graphs", fn);
+    if (num_graphs == 0 && (total_nodes > 0 || total_edges > 0))
+        return fail(TFG_ERR_INVALID_ARG, "%s: nodes or edges given for zero graphs", fn);
+    TFG_NEED(node_counts, num_graphs > 0, fn, "node_counts");
+    TFG_NEED(edge_counts, num_graphs > 0, fn, "edge_counts");
+    TFG_NEED(edge_index, total_edges > 0, fn, "edge_index");
+    TFG_NEED(out_edge_index, total_edges > 0, fn, "out_edge_index");
+    TFG_NEED(batch, total_nodes > 0, fn, "batch");
+    TFG_NEED(node_offsets, true, fn, "node_offsets");
+    TFG_NEED(status, true, fn, "status");
+    const size_t need = tfg::batch_graphs_workspace_bytes(num_graphs);
+    if (workspace == nullptr || workspace_bytes < need)
+        return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
+                    workspace ? workspace_bytes : size_t(0));
+    return cuda_result(tfg::launch_batch_graphs(num_graphs, node_counts, edge_counts, edge_index,
+                                                total_edges, total_nodes, out_edge_index, batch,
+                                                node_offsets, workspace, status,
                                                 reinterpret_cast<cudaStream_t>(stream)),
                        fn);
 }

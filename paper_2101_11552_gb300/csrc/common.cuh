@@ -55,6 +55,18 @@ template <> struct VecLoad<uint16_t, 8> {
     }
     static __device__ __forceinline__ void load(const uint16_t *p, float (&v)[8]) { widen(raw(p), v); }
 };
+template <> struct VecLoad<uint16_t, 4> {
+    using Raw = uint2;
+    static __device__ __forceinline__ Raw raw(const uint16_t *p) {
+        return __ldg(reinterpret_cast<const uint2 *>(p));
+    }
+    static __device__ __forceinline__ Raw zero() { return make_uint2(0u, 0u); }
+    static __device__ __forceinline__ void widen(const Raw &q, float (&v)[4]) {
+        v[0] = bf16_lo(q.x); v[1] = bf16_hi(q.x);
+        v[2] = bf16_lo(q.y); v[3] = bf16_hi(q.y);
+    }
+    static __device__ __forceinline__ void load(const uint16_t *p, float (&v)[4]) { widen(raw(p), v); }
+};
 template <> struct VecLoad<uint16_t, 1> {
     using Raw = uint32_t;
     static __device__ __forceinline__ Raw raw(const uint16_t *p) {
@@ -130,11 +142,26 @@ cudaError_t launch_gcn_norm(const int32_t *rowptr, const int32_t *col, const int
 cudaError_t launch_aggregate(int mode, const int32_t *rowptr, const int32_t *col, const float *w,
                              const float *dinv, const void *x, int x_dtype, int64_t n, int64_t f,
                              int add_self, float fill, float *out, cudaStream_t s);
+size_t propagate_workspace_bytes(int64_t n, int64_t f, int64_t hops);
+cudaError_t launch_propagate(const int32_t *rowptr, const int32_t *col, const float *w,
+                             const float *dinv, const void *x0, int x_dtype, int64_t n, int64_t f,
+                             int64_t hops, float alpha, int add_self, float fill, float *out,
+                             void *ws, cudaStream_t s);
+int dot_softmax_max_channels();
+cudaError_t launch_dot_softmax(const int32_t *rowptr, const int32_t *col, const void *q,
+                               const void *k, const void *v, int x_dtype, int64_t n, int64_t e,
+                               int heads, int channels, float scale, float *out, float *alpha,
+                               cudaStream_t s);
 size_t softmax_workspace_bytes(int64_t n, int heads);
 cudaError_t launch_edge_softmax(const int32_t *rowptr, const int32_t *col, const void *x,
                                 int x_dtype, int64_t n, int64_t e, int heads, int channels,
                                 const float *a_src, const float *a_dst, float slope, float *out,
                                 float *alpha, void *ws, cudaStream_t s);
+size_t batch_graphs_workspace_bytes(int64_t g);
+cudaError_t launch_batch_graphs(int64_t g, const int64_t *node_counts, const int64_t *edge_counts,
+                                const int64_t *edge_index, int64_t e, int64_t n,
+                                int64_t *out_edge_index, int64_t *batch, int64_t *node_offsets,
+                                void *ws, int32_t *status, cudaStream_t s);
 int64_t noalloc_softmax_max_node_heads();
 cudaError_t noalloc_softmax_scratch(void **ptr, size_t *bytes);
 cudaError_t launch_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n,

@@ -192,8 +192,8 @@ cudaError_t exclusive_scan(int32_t *data, int64_t m, int32_t *sums, cudaStream_t
 //      into every warp's counter; per digit, global base minus tile start
 //   C  stable slots: per round, peers with equal digits are found with
 //      __match_any_sync, their leader claims a block of slots with one
-//      returning atomic, and each lane adds its rank among the peers; the
-//      element (key, source, edge id) is staged as one 16-byte record
+//      returning atomic, and each lane adds its rank among the peers; key,
+//      source and edge id are staged in three arrays
 //   D  the tile leaves in digit order, consecutive threads writing
 //      consecutive positions of each digit's run
 constexpr int kDsWarps = 16;
@@ -201,7 +201,7 @@ constexpr int kDsThreads = kDsWarps * 32;
 constexpr int kDsItems = kTile / kDsThreads;   // 8 per lane
 
 size_t downsweep_smem(int radix) {
-    return sizeof(uint4) * kTile + sizeof(int32_t) * kDsWarps * radix +
+    return sizeof(uint32_t) * 3 * kTile + sizeof(int32_t) * kDsWarps * radix +
            sizeof(int32_t) * 2 * radix + sizeof(int32_t) * 32;
 }
 
@@ -214,8 +214,10 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
                 int32_t *__restrict__ src_out, int32_t *__restrict__ eid_out, int32_t *status) {
     extern __shared__ __align__(16) unsigned char smem[];
     const int radix = 1 << width;
-    uint4 *s_elem = reinterpret_cast<uint4 *>(smem);                      // [tile]
-    int32_t *s_cnt = reinterpret_cast<int32_t *>(s_elem + kTile);          // [warp][digit]
+    uint32_t *s_key = reinterpret_cast<uint32_t *>(smem);                 // [tile]
+    int32_t *s_src = reinterpret_cast<int32_t *>(s_key + kTile);           // [tile]
+    int32_t *s_eid = s_src + kTile;                                        // [tile]
+    int32_t *s_cnt = s_eid + kTile;                                        // [warp][digit]
     int32_t *s_tstart = s_cnt + kDsWarps * radix;                          // [digit]
     int32_t *s_delta = s_tstart + radix;                                   // [digit]
     int32_t *s_chunk = s_delta + radix;                                    // [32]
@@ -315,9 +317,12 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
         int32_t base = 0;
         if (ok && lane == leader) base = atomicAdd(&mine[dig], __popc(peers));
         base = __shfl_sync(kFull, base, leader);
-        if (ok)
-            s_elem[base + __popc(peers & lower)] =
-                make_uint4(keys[r], static_cast<uint32_t>(srcs[r]), static_cast<uint32_t>(eids[r]), 0u);
+        if (ok) {
+            const int slot = base + __popc(peers & lower);
+            s_key[slot] = keys[r];
+            s_src[slot] = srcs[r];
+            s_eid[slot] = eids[r];
+        }
     }
     __syncthreads();
 
@@ -326,12 +331,12 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     for (int j = 0; j < kDsItems; ++j) {
         const int i = threadIdx.x + j * kDsThreads;
         if (i < count) {
-            const uint4 v = s_elem[i];
-            const int d = static_cast<int>((v.x >> shift) & (radix - 1));
+            const uint32_t k = s_key[i];
+            const int d = static_cast<int>((k >> shift) & (radix - 1));
             const int64_t pos = static_cast<int64_t>(s_delta[d]) + i;
-            key_out[pos] = v.x;
-            src_out[pos] = static_cast<int32_t>(v.y);
-            eid_out[pos] = static_cast<int32_t>(v.z);
+            key_out[pos] = k;
+            src_out[pos] = s_src[i];
+            eid_out[pos] = s_eid[i];
         }
     }
 }

@@ -44,21 +44,41 @@ __device__ __forceinline__ int64_t lower_bound(const int64_t *batch, int64_t n, 
     return lo;
 }
 
+// Reducer ids of the kernel: TFG_SUM, TFG_MEAN, TFG_MAX, and kMeanMax, which
+// keeps a sum and a max per feature in one pass and writes [mean | max]
+// (the Mean-Max Pool readout of Table 2).
+constexpr int kMeanMax = 3;
+
+// op of accumulator a (0 = the sum/mean/max itself; for kMeanMax 0 = sum, 1 = max)
 template <int RED>
-__device__ __forceinline__ float pool_op(float a, float b) {
-    return RED == TFG_MAX ? fmaxf(a, b) : a + b;
+__device__ __forceinline__ float pool_op(int a, float x, float y) {
+    const bool is_max = RED == TFG_MAX || (RED == kMeanMax && a == 1);
+    return is_max ? fmaxf(x, y) : x + y;
+}
+template <int RED>
+__device__ __forceinline__ float pool_init(int a) {
+    const bool is_max = RED == TFG_MAX || (RED == kMeanMax && a == 1);
+    return is_max ? -CUDART_INF_F : 0.f;
+}
+template <int RED>
+__device__ __forceinline__ float pool_final(int a, float r, int64_t cnt) {
+    if (cnt == 0) return 0.f;
+    const bool is_mean = RED == TFG_MEAN || (RED == kMeanMax && a == 0);
+    return is_mean ? r / static_cast<float>(cnt) : r;
 }
 
 // grid = (graphs, feature tiles, S); cluster = (1, 1, S) when S > 1.
+// out is [G, NA * F]: accumulator a of feature f goes to column a * F + f.
 template <typename XT, int VEC, int LPR, int RED, bool CLUSTER>
 __global__ void __launch_bounds__(kPoolThreads)
 pool_kernel(const XT *__restrict__ x, const int64_t *__restrict__ batch, int64_t n, int64_t f,
             float *__restrict__ out) {
+    constexpr int NA = RED == kMeanMax ? 2 : 1;
     constexpr int kGroups = kPoolThreads / LPR;
     constexpr int kSlots = LPR * VEC;
     __shared__ int64_t s_range[2];
-    __shared__ float s_part[kGroups * kSlots];
-    __shared__ float s_red[kSlots];
+    __shared__ float s_part[NA][kGroups * kSlots];
+    __shared__ float s_red[NA][kSlots];
     const int64_t gid = blockIdx.x;
     const int split = blockIdx.z, nsplit = gridDim.z;
     if (threadIdx.x == 0) s_range[0] = lower_bound(batch, n, gid);
@@ -71,38 +91,48 @@ pool_kernel(const XT *__restrict__ x, const int64_t *__restrict__ batch, int64_t
     const int64_t ft = static_cast<int64_t>(blockIdx.y) * kSlots;
     const int64_t f0 = ft + sub * VEC;
     const bool fok = f0 < f;
-    float acc[VEC];
+    float acc[NA][VEC];
 #pragma unroll
-    for (int q = 0; q < VEC; ++q) acc[q] = RED == TFG_MAX ? -CUDART_INF_F : 0.f;
+    for (int a = 0; a < NA; ++a)
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) acc[a][q] = pool_init<RED>(a);
     if (fok) {
         for (int64_t v = pb + grp; v < pe; v += kGroups) {
             float val[VEC];
             VecLoad<XT, VEC>::load(x + v * f + f0, val);
 #pragma unroll
-            for (int q = 0; q < VEC; ++q) acc[q] = pool_op<RED>(acc[q], val[q]);
+            for (int a = 0; a < NA; ++a)
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) acc[a][q] = pool_op<RED>(a, acc[a][q], val[q]);
         }
     }
 #pragma unroll
-    for (int q = 0; q < VEC; ++q) s_part[grp * kSlots + sub * VEC + q] = acc[q];
+    for (int a = 0; a < NA; ++a)
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) s_part[a][grp * kSlots + sub * VEC + q] = acc[a][q];
     __syncthreads();
     for (int i = threadIdx.x; i < kSlots; i += kPoolThreads) {
-        float r = s_part[i];
-        for (int k = 1; k < kGroups; ++k) r = pool_op<RED>(r, s_part[k * kSlots + i]);
-        s_red[i] = r;
+#pragma unroll
+        for (int a = 0; a < NA; ++a) {
+            float r = s_part[a][i];
+            for (int k = 1; k < kGroups; ++k) r = pool_op<RED>(a, r, s_part[a][k * kSlots + i]);
+            s_red[a][i] = r;
+        }
     }
     const int64_t cnt = end - beg;
+    const int64_t ostride = NA * f;
     if constexpr (CLUSTER) {
         cg::cluster_group cluster = cg::this_cluster();
         cluster.sync();   // every CTA's partial is in its shared memory
         if (cluster.block_rank() == 0) {
             for (int i = threadIdx.x; i < kSlots; i += kPoolThreads) {
-                float r = s_red[i];
-                for (int q = 1; q < nsplit; ++q) r = pool_op<RED>(r, cluster.map_shared_rank(s_red, q)[i]);
                 const int64_t fi = ft + i;
-                if (fi < f) {
-                    if (cnt == 0) r = 0.f;
-                    else if (RED == TFG_MEAN) r = r / static_cast<float>(cnt);
-                    out[gid * f + fi] = r;
+#pragma unroll
+                for (int a = 0; a < NA; ++a) {
+                    float r = s_red[a][i];
+                    for (int q = 1; q < nsplit; ++q)
+                        r = pool_op<RED>(a, r, cluster.map_shared_rank(&s_red[a][0], q)[i]);
+                    if (fi < f) out[gid * ostride + a * f + fi] = pool_final<RED>(a, r, cnt);
                 }
             }
         }
@@ -112,10 +142,9 @@ pool_kernel(const XT *__restrict__ x, const int64_t *__restrict__ batch, int64_t
         for (int i = threadIdx.x; i < kSlots; i += kPoolThreads) {
             const int64_t fi = ft + i;
             if (fi >= f) continue;
-            float r = s_red[i];
-            if (cnt == 0) r = 0.f;
-            else if (RED == TFG_MEAN) r = r / static_cast<float>(cnt);
-            out[gid * f + fi] = r;
+#pragma unroll
+            for (int a = 0; a < NA; ++a)
+                out[gid * ostride + a * f + fi] = pool_final<RED>(a, s_red[a][i], cnt);
         }
     }
 }
@@ -160,6 +189,7 @@ cudaError_t launch_red(const void *x, const int64_t *batch, int64_t n, int64_t g
     switch (reduce) {
         case TFG_MEAN: return launch_lpr<XT, VEC, TFG_MEAN>(x, batch, n, g, f, out, lpr, nsplit, s);
         case TFG_MAX: return launch_lpr<XT, VEC, TFG_MAX>(x, batch, n, g, f, out, lpr, nsplit, s);
+        case kMeanMax: return launch_lpr<XT, VEC, kMeanMax>(x, batch, n, g, f, out, lpr, nsplit, s);
         default: return launch_lpr<XT, VEC, TFG_SUM>(x, batch, n, g, f, out, lpr, nsplit, s);
     }
 }

@@ -13,6 +13,7 @@ CUDA tensors on the same device; calls are asynchronous on the current stream.
 from __future__ import annotations
 
 import ctypes
+import math
 import os
 import threading
 from typing import NamedTuple, Optional
@@ -63,10 +64,17 @@ def lib() -> ctypes.CDLL:
                 "tfg_aggregate_mean": [P, P, P, P, I, I64, I64, P, P],
                 "tfg_aggregate_max": [P, P, P, P, I, I64, I64, P, P],
                 "tfg_gcn_aggregate_sum": [P, P, P, P, P, I, I64, I64, I, F, P, P],
+                "tfg_propagate_workspace_size": [I64, I64, I64, ctypes.POINTER(SZ)],
+                "tfg_appnp_propagate": [P, P, P, P, P, I, I64, I64, I64, F, I, F, P, P, SZ, P],
+                "tfg_sgc_propagate": [P, P, P, P, P, I, I64, I64, I64, I, F, P, P, SZ, P],
                 "tfg_edge_softmax_workspace_size": [I64, I, ctypes.POINTER(SZ)],
                 "tfg_edge_softmax_aggregate": [P, P, P, I, I64, I64, I, I, P, P, F, P, P, P, SZ, P],
+                "tfg_dot_edge_softmax_aggregate": [P, P, P, P, P, I, I64, I64, I, I, F, P, P, P],
                 "tfg_edge_softmax_aggregate_noalloc": [P, P, P, I, I64, I64, I, I, P, P, F, P, P, P],
                 "tfg_segment_pool": [P, I, P, I64, I64, I64, I, P, P, P],
+                "tfg_segment_pool_meanmax": [P, I, P, I64, I64, I64, P, P, P],
+                "tfg_batch_graphs_workspace_size": [I64, ctypes.POINTER(SZ)],
+                "tfg_batch_graphs": [I64, P, P, P, I64, I64, P, P, P, P, SZ, P, P],
             }
             for name, args in sigs.items():
                 fn = getattr(L, name)
@@ -230,6 +238,54 @@ def tfg_gcn_aggregate_sum(rowptr, col, dinv, x, w_csr=None, add_self_loops: int 
     return out
 
 
+def tfg_propagate_workspace_size(num_nodes: int, num_features: int, num_hops: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().tfg_propagate_workspace_size(num_nodes, num_features, num_hops, ctypes.byref(n)))
+    return n.value
+
+
+def tfg_appnp_propagate(rowptr, col, dinv, x0, num_hops: int, alpha: float, w_csr=None,
+                        add_self_loops: int = 0, self_loop_fill: float = 1.0, out=None,
+                        workspace=None):
+    """h_{k+1} = (1 - alpha) Ahat h_k + alpha x0, h_0 = x0; returns h_K (fp32)."""
+    return _propagate("tfg_appnp_propagate", rowptr, col, dinv, x0, num_hops, alpha, w_csr,
+                      add_self_loops, self_loop_fill, out, workspace)
+
+
+def tfg_sgc_propagate(rowptr, col, dinv, x0, num_hops: int, w_csr=None, add_self_loops: int = 0,
+                      self_loop_fill: float = 1.0, out=None, workspace=None):
+    """Ahat^K x0 (fp32)."""
+    return _propagate("tfg_sgc_propagate", rowptr, col, dinv, x0, num_hops, None, w_csr,
+                      add_self_loops, self_loop_fill, out, workspace)
+
+
+def _propagate(name, rowptr, col, dinv, x0, num_hops, alpha, w_csr, add_self_loops,
+               self_loop_fill, out, workspace):
+    _need_cuda("rowptr", rowptr, torch.int32)
+    dev = rowptr.device
+    _need_cuda("col", col, torch.int32, dev)
+    _need_cuda("dinv", dinv, torch.float32, dev)
+    _need_cuda("x0", x0, None, dev)
+    n, f = x0.shape
+    if rowptr.numel() != n + 1:
+        raise ValueError("rowptr must have N + 1 entries")
+    if w_csr is not None:
+        _need_cuda("w_csr", w_csr, torch.float32, dev)
+    if out is None:
+        out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    _need_cuda("out", out, torch.float32, dev)
+    nb = tfg_propagate_workspace_size(n, f, num_hops)
+    if workspace is None or workspace.numel() < nb:
+        workspace = torch.empty(max(nb, 1), dtype=torch.uint8, device=dev)
+    head = [_ptr(rowptr), _ptr(col), _ptr(dinv), _ptr(w_csr), _ptr(x0), _x_dtype(x0), n, f,
+            int(num_hops)]
+    tail = [int(add_self_loops), float(self_loop_fill), _ptr(out), _ptr(workspace),
+            workspace.numel(), _stream(dev)]
+    fn = getattr(lib(), name)
+    _check(fn(*head, *([] if alpha is None else [float(alpha)]), *tail))
+    return out
+
+
 def tfg_edge_softmax_workspace_size(num_nodes: int, heads: int) -> int:
     n = ctypes.c_size_t(0)
     _check(lib().tfg_edge_softmax_workspace_size(num_nodes, heads, ctypes.byref(n)))
@@ -261,6 +317,35 @@ def tfg_edge_softmax_aggregate(rowptr, col, x, heads: int, channels: int, a_src,
                                             _ptr(a_src), _ptr(a_dst), float(negative_slope),
                                             _ptr(out), _ptr(alpha), _ptr(workspace),
                                             workspace.numel(), _stream(dev)))
+    return out, alpha
+
+
+def tfg_dot_edge_softmax_aggregate(rowptr, col, q, k, v, heads: int, channels: int,
+                                   scale: Optional[float] = None, want_alpha: bool = False,
+                                   out=None, alpha=None):
+    """Transformer-style attention over in-edges; scale defaults to 1/sqrt(channels).
+    Returns (out [N, H*C] fp32, alpha [E, H] or None)."""
+    _need_cuda("rowptr", rowptr, torch.int32)
+    dev = rowptr.device
+    _need_cuda("col", col, torch.int32, dev)
+    _need_cuda("q", q, None, dev)
+    _need_cuda("k", k, q.dtype, dev)
+    _need_cuda("v", v, q.dtype, dev)
+    n, f = q.shape
+    if k.shape != q.shape or v.shape != q.shape:
+        raise ValueError("q, k and v must have the same shape")
+    if f != heads * channels:
+        raise ValueError("feature width must equal heads * channels")
+    e = col.numel()
+    if scale is None:
+        scale = 1.0 / math.sqrt(channels)
+    if out is None:
+        out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    if want_alpha and alpha is None:
+        alpha = torch.empty(e, heads, dtype=torch.float32, device=dev)
+    _check(lib().tfg_dot_edge_softmax_aggregate(
+        _ptr(rowptr), _ptr(col), _ptr(q), _ptr(k), _ptr(v), _x_dtype(q), n, e, heads, channels,
+        float(scale), _ptr(out), _ptr(alpha), _stream(dev)))
     return out, alpha
 
 
@@ -301,3 +386,50 @@ def tfg_segment_pool(x, batch, num_graphs: int, reduce: str = "sum", out=None):
     _check(lib().tfg_segment_pool(_ptr(x), _x_dtype(x), _ptr(batch), n, num_graphs, f,
                                   REDUCERS[reduce], _ptr(out), _ptr(status), _stream(dev)))
     return out, status
+
+
+def tfg_segment_pool_meanmax(x, batch, num_graphs: int, out=None):
+    """Return (out [G, 2F] = [mean | max], status)."""
+    _need_cuda("x", x)
+    dev = x.device
+    _need_cuda("batch", batch, torch.int64, dev)
+    n, f = x.shape
+    if out is None:
+        out = torch.empty(num_graphs, 2 * f, dtype=torch.float32, device=dev)
+    status = torch.empty(1, dtype=torch.int32, device=dev)
+    _check(lib().tfg_segment_pool_meanmax(_ptr(x), _x_dtype(x), _ptr(batch), n, num_graphs, f,
+                                          _ptr(out), _ptr(status), _stream(dev)))
+    return out, status
+
+
+def tfg_batch_graphs_workspace_size(num_graphs: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().tfg_batch_graphs_workspace_size(num_graphs, ctypes.byref(n)))
+    return n.value
+
+
+class BatchGraph(NamedTuple):
+    edge_index: torch.Tensor    # int64 [2, E]
+    batch: torch.Tensor         # int64 [N]
+    node_offsets: torch.Tensor  # int64 [G + 1]
+    status: torch.Tensor        # int32 [1] (device)
+
+
+def tfg_batch_graphs(node_counts: torch.Tensor, edge_counts: torch.Tensor,
+                     edge_index: torch.Tensor, total_nodes: int) -> BatchGraph:
+    """Combine graphs into one BatchGraph on the device (reindexing trick)."""
+    _need_cuda("node_counts", node_counts, torch.int64)
+    dev = node_counts.device
+    _need_cuda("edge_counts", edge_counts, torch.int64, dev)
+    _need_cuda("edge_index", edge_index, torch.int64, dev)
+    g = node_counts.numel()
+    e = edge_index.shape[1]
+    out_ei = torch.empty(2, e, dtype=torch.int64, device=dev)
+    batch = torch.empty(total_nodes, dtype=torch.int64, device=dev)
+    offs = torch.empty(g + 1, dtype=torch.int64, device=dev)
+    status = torch.empty(1, dtype=torch.int32, device=dev)
+    ws = torch.empty(tfg_batch_graphs_workspace_size(g), dtype=torch.uint8, device=dev)
+    _check(lib().tfg_batch_graphs(g, _ptr(node_counts), _ptr(edge_counts), _ptr(edge_index), e,
+                                  total_nodes, _ptr(out_ei), _ptr(batch), _ptr(offs), _ptr(ws),
+                                  ws.numel(), _ptr(status), _stream(dev)))
+    return BatchGraph(out_ei, batch, offs, status)

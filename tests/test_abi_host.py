@@ -104,3 +104,76 @@ def test_segment_pool_rejects(lib):
     assert f(FAKE, 0, None, 10, 3, 4, 0, FAKE, FAKE, None) == -1        # batch
     assert f(FAKE, 0, FAKE, -1, 3, 4, 0, FAKE, FAKE, None) == -1
     assert f(FAKE, 5, FAKE, 10, 3, 4, 0, FAKE, FAKE, None) == -1        # dtype
+
+
+def test_segment_pool_meanmax_rejects(lib):
+    f = lib.tfg_segment_pool_meanmax
+    assert f(FAKE, 0, FAKE, 10, 3, 4, FAKE, None, None) == -1            # status
+    assert f(FAKE, 0, None, 10, 3, 4, FAKE, FAKE, None) == -1            # batch
+    assert f(FAKE, 0, FAKE, 10, 3, 4, None, FAKE, None) == -1            # out
+    assert f(FAKE, 5, FAKE, 10, 3, 4, FAKE, FAKE, None) == -1            # dtype
+    assert f(FAKE, 0, FAKE, 10, -3, 4, FAKE, FAKE, None) == -1
+    assert f(FAKE, 0, FAKE, 10, 3, 0, FAKE, FAKE, None) == -1            # F = 0
+
+
+def test_batch_graphs_rejects(lib):
+    n = ctypes.c_size_t(0)
+    assert lib.tfg_batch_graphs_workspace_size(5, ctypes.byref(n)) == 0 and n.value >= 8 * 6
+    assert lib.tfg_batch_graphs_workspace_size(-1, ctypes.byref(n)) == -1
+    f = lib.tfg_batch_graphs
+    ok = (FAKE, FAKE, FAKE, 10, 7, FAKE, FAKE, FAKE, FAKE, 1 << 12, FAKE, None)
+    assert f(-1, *ok) == -1
+    assert f(0, *ok) == -1                                               # nodes for zero graphs
+    assert f(1 << 31, *ok) == -2
+    assert f(3, FAKE, FAKE, FAKE, 10, 7, FAKE, FAKE, FAKE, FAKE, 16, FAKE, None) == -3
+    assert "workspace" in err(lib)
+    assert f(3, FAKE, FAKE, FAKE, 10, 7, FAKE, FAKE, FAKE, None, 1 << 12, FAKE, None) == -3
+    assert f(3, None, FAKE, FAKE, 10, 7, FAKE, FAKE, FAKE, FAKE, 1 << 12, FAKE, None) == -1
+    assert f(3, FAKE, FAKE, None, 10, 7, FAKE, FAKE, FAKE, FAKE, 1 << 12, FAKE, None) == -1
+    assert f(3, FAKE, FAKE, FAKE, 10, 7, FAKE, FAKE, None, FAKE, 1 << 12, FAKE, None) == -1
+    assert f(3, FAKE, FAKE, FAKE, 10, 7, FAKE, FAKE, FAKE, FAKE, 1 << 12, None, None) == -1
+    assert f(3, FAKE, FAKE, FAKE, -10, 7, FAKE, FAKE, FAKE, FAKE, 1 << 12, FAKE, None) == -1
+
+
+def test_propagate_rejects(lib):
+    n = ctypes.c_size_t(0)
+    assert lib.tfg_propagate_workspace_size(100, 8, 1, ctypes.byref(n)) == 0 and n.value == 0
+    assert lib.tfg_propagate_workspace_size(100, 8, 3, ctypes.byref(n)) == 0 and n.value >= 3200
+    assert lib.tfg_propagate_workspace_size(100, 8, -1, ctypes.byref(n)) == -1
+    f = lib.tfg_appnp_propagate
+    args = lambda **kw: [kw.get(k, v) for k, v in dict(
+        rowptr=FAKE, col=FAKE, dinv=FAKE, w=None, x0=FAKE, dt=0, n=10, f=4, k=3, a=0.1, sl=1,
+        fill=1.0, out=FAKE, ws=FAKE, wsb=1 << 12, st=None).items()]
+    assert f(*args(k=-1)) == -1
+    assert f(*args(k=1025)) == -1
+    assert f(*args(a=1.5)) == -1
+    assert f(*args(a=float("nan"))) == -1
+    assert f(*args(dinv=None)) == -1
+    assert f(*args(x0=None)) == -1
+    assert f(*args(out=None)) == -1
+    assert f(*args(dt=4)) == -1
+    assert f(*args(f=0)) == -1
+    assert f(*args(ws=None)) == -3
+    assert f(*args(wsb=64)) == -3
+    assert "workspace" in err(lib)
+    assert f(*args(ws=ctypes.c_void_p(0x1004))) == -1           # unaligned workspace
+    sgc = lib.tfg_sgc_propagate
+    assert sgc(FAKE, FAKE, None, None, FAKE, 0, 10, 4, 2, 1, 1.0, FAKE, FAKE, 1 << 12, None) == -1
+
+
+def test_dot_softmax_rejects(lib):
+    f = lib.tfg_dot_edge_softmax_aggregate
+    ok = dict(rp=FAKE, col=FAKE, q=FAKE, k=FAKE, v=FAKE, dt=0, n=10, e=20, h=2, c=8, s=0.25,
+              out=FAKE, al=None, st=None)
+    call = lambda **kw: f(*[kw.get(key, val) for key, val in ok.items()])  # noqa: E731
+    assert call(h=0) == -1
+    assert call(c=257) == -2
+    assert call(dt=3) == -1
+    assert call(s=float("inf")) == -1
+    assert call(s=float("nan")) == -1
+    assert call(q=None) == -1
+    assert call(k=None) == -1
+    assert call(v=None) == -1
+    assert call(col=None) == -1
+    assert call(out=None) == -1
+    assert call(e=-1) == -1

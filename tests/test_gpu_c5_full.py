@@ -105,3 +105,57 @@ def test_c5_community_pool(c5):
             assert_exact_f32(out.cpu().numpy(), ref, "c5 pool max")
         else:
             assert_scaled_close(out.cpu().numpy(), ref, scale, TOL_F32, f"c5 pool {reduce}")
+
+
+def test_c5_appnp_sqrt_degree_fixed_point(c5):
+    """On a symmetric graph with self-loops Ahat sqrt(d) = sqrt(d), so
+    x0 = sqrt(d) v^T is a fixed point of every APPNP step; the error scale
+    |Ahat|^k |x0| is |x0| itself."""
+    wl, ocsr, csr, _ = c5
+    n = wl.num_nodes
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 1, 1.0, want_w_csr=False)
+    d = ocsr[3].astype(np.float64) + 1.0
+    v = np.random.default_rng(21).standard_normal(128)
+    x0 = (np.sqrt(d)[:, None] * v[None, :]).astype(np.float32)
+    out = tfg.tfg_appnp_propagate(csr.rowptr, csr.col, dinv, dev(x0), 10, 0.1, add_self_loops=1)
+    got = out.cpu().numpy()
+    assert_scaled_close(got, x0.astype(np.float64), np.abs(x0).astype(np.float64), TOL_F32,
+                        "c5 appnp fixed point")
+
+
+def test_c5_appnp_one_hop_sampled_rows_and_sgc_chain(c5):
+    wl, ocsr, csr, rows = c5
+    n = wl.num_nodes
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 1, 1.0, want_w_csr=False)
+    x = dev(wl.x_bf16.view(np.int16)).view(torch.bfloat16)
+    alpha = 0.1
+    out = tfg.tfg_appnp_propagate(csr.rowptr, csr.col, dinv, x, 1, alpha, add_self_loops=1)
+    nrm = oracle.gcn_norm(wl.edge_index, n, None, 1, 1.0)
+    agg, scale = oracle.aggregate_rows(ocsr, n, wl.x_bf16, "sum", rows, w=nrm["w_norm"],
+                                       self_w=nrm["self_w"])
+    x0 = oracle.widen(wl.x_bf16)[rows]
+    ref = (1 - alpha) * agg + alpha * x0
+    sc = (1 - alpha) * scale + alpha * np.abs(x0)
+    assert_scaled_close(out[dev(rows)].cpu().numpy(), ref, sc, TOL_F32, "c5 appnp 1 hop")
+    sgc = tfg.tfg_sgc_propagate(csr.rowptr, csr.col, dinv, x, 2, add_self_loops=1)
+    h = tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, x, None, 1, 1.0)
+    h = tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, h, None, 1, 1.0)
+    assert torch.equal(sgc, h)
+
+
+def test_c5_dot_softmax_sampled_rows(c5):
+    """Transformer-style attention at full size: q, k, v bf16 [N, 8 x 16]."""
+    wl, ocsr, csr, rows = c5
+    n = wl.num_nodes
+    rng = np.random.default_rng(1305)
+    bits = [gg.bf16_bits_rne(rng.standard_normal((n, 128), dtype=np.float32)) for _ in range(3)]
+    q, k, v = (dev(b.view(np.int16)).view(torch.bfloat16) for b in bits)
+    out, alpha = tfg.tfg_dot_edge_softmax_aggregate(csr.rowptr, csr.col, q, k, v, 8, 16,
+                                                    want_alpha=True)
+    sub = rows[:400]
+    ref, ref_alpha, scale = oracle.dot_softmax_rows(ocsr, n, *bits, 8, 16, 0.25, sub)
+    got = out[dev(sub)].cpu().numpy()
+    assert_scaled_close(got, ref, scale, TOL_F32, "c5 dot softmax")
+    rp = ocsr[0]
+    got_alpha = np.concatenate([alpha[int(rp[r]):int(rp[r + 1])].cpu().numpy() for r in sub])
+    assert_scaled_close(got_alpha, ref_alpha, alpha_scale(ref_alpha), TOL_F32, "c5 dot alpha")

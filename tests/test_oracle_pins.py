@@ -302,6 +302,26 @@ def test_batch_reindex_example():
     assert list(batch) == [0, 0, 0, 0, 1, 1, 2, 2, 2]
 
 
+def test_oracle_batch_graphs_worked_example():
+    """The oracle's own reindexing reproduces the paper's example and agrees
+    with the generator's stacking (two independent implementations)."""
+    g = _golden("batch_reindex.json")
+    sizes = g["graph_sizes"]
+    rng = np.random.default_rng(2)
+    parts = [gg.symmetrise(gg.er_pairs(s, s - 1, rng)) if s > 1 else np.zeros((2, 0), np.int64)
+             for s in sizes]
+    stacked = np.concatenate(parts, axis=1)
+    ei, batch, offs = oracle.batch_graphs(sizes, [p.shape[1] for p in parts], stacked)
+    assert list(offs[:-1]) == g["offsets"] and offs[-1] == sum(sizes)
+    for item in g["one_based"]:
+        assert item["node"] + offs[item["graph"] - 1] == item["index"]
+    ref_ei, ref_batch, ref_offs = gg.batch_graphs(parts, sizes)
+    assert np.array_equal(ei, ref_ei) and np.array_equal(batch, ref_batch)
+    assert np.array_equal(offs[:-1], ref_offs)
+    with pytest.raises(oracle.OracleError):
+        oracle.batch_graphs([2, 2], [1, 0], np.array([[0], [2]]))   # node 2 outside graph 0
+
+
 def pin_batched_equals_per_graph(o):
     """Applying the aggregation to a BatchGraph equals applying it per graph
     and concatenating (Section 2.1.1); pooling equals per-graph full reductions."""
@@ -369,6 +389,158 @@ def test_bf16_widening_is_exact():
 
 
 # ---------------------------------------------------------------------------
+# Dot-product (Transformer-style) attention
+# ---------------------------------------------------------------------------
+def pin_dot_star(o):
+    g = _golden("dot_star.json")
+    ei = np.array(g["edge_index"], dtype=np.int64)
+    q = np.zeros((4, 2))
+    q[0] = g["q0"]
+    k = np.zeros((4, 2))
+    for s, m in zip((1, 2, 3), g["key_logs"]):
+        k[s, 0] = 2.0 * math.log(m)
+    v = np.array(g["v"])
+    out, alpha, _ = o.dot_softmax(ei, 4, q, k, v, g["heads"], g["channels"], g["scale"])
+    np.testing.assert_allclose(alpha[:, 0], g["alpha"], rtol=0, atol=g["abs_tol"])
+    np.testing.assert_allclose(out[0], g["out0"], rtol=0, atol=g["abs_tol"])
+    np.testing.assert_array_equal(out[1:], 0.0)
+
+
+def test_dot_star():
+    pin_dot_star(oracle.default)
+
+
+def pin_dot_limits(o):
+    """q = 0 makes every logit 0, so the result is the mean of the value rows
+    over in-edges (the dense row-normalised adjacency times v); a single
+    in-edge gives its source's value row with weight 1; weights sum to 1 per
+    (target, head); shifting every key of a head by one vector changes each
+    target's logits by a constant and leaves the result unchanged; heads
+    are independent."""
+    n, e, h, c = 50, 400, 3, 4
+    wl = gg.random_edge_case_graph(n, e, h * c, 71, hub=2, isolated=4)
+    ei = wl.edge_index
+    rng = np.random.default_rng(71)
+    q = rng.standard_normal((n, h * c))
+    k = rng.standard_normal((n, h * c))
+    v = rng.standard_normal((n, h * c))
+    out, _, _ = o.dot_softmax(ei, n, np.zeros_like(q), k, v, h, c)
+    cnt = oracle.dense_adjacency(ei, n, None)
+    deg = cnt.sum(axis=1)
+    mean = np.where(deg[:, None] > 0, (cnt @ v) / np.maximum(deg, 1)[:, None], 0.0)
+    np.testing.assert_allclose(out, mean, rtol=1e-12, atol=1e-12)
+    out, alpha, _ = o.dot_softmax(ei, n, q, k, v, h, c)
+    sums = np.zeros((n, h))
+    np.add.at(sums, ei[1], alpha)
+    np.testing.assert_allclose(sums[deg > 0], 1.0, rtol=1e-13)
+    shift = np.tile(rng.standard_normal(c), h)
+    out2, _, _ = o.dot_softmax(ei, n, q, k + shift[None, :], v, h, c)
+    np.testing.assert_allclose(out2, out, rtol=1e-10, atol=1e-12)
+    one = np.array([[3, 7], [5, 9]])       # 3 -> 5, 7 -> 9
+    out1, al1, _ = o.dot_softmax(one, 10, q[:10], k[:10], v[:10], h, c)
+    np.testing.assert_allclose(out1[5], v[3], rtol=1e-15)
+    np.testing.assert_allclose(al1, 1.0, rtol=1e-15)
+    # head 1 alone: the same numbers as a one-head problem on its columns
+    cols = slice(c, 2 * c)
+    out_h, al_h, _ = o.dot_softmax(ei, n, q[:, cols], k[:, cols], v[:, cols], 1, c)
+    np.testing.assert_allclose(out[:, cols], out_h, rtol=1e-13, atol=1e-13)
+    np.testing.assert_allclose(alpha[:, 1], al_h[:, 0], rtol=1e-13)
+
+
+def test_dot_limits():
+    pin_dot_limits(oracle.default)
+
+
+def test_dot_rows_match_full():
+    n, e, h, c = 80, 900, 2, 8
+    wl = gg.random_edge_case_graph(n, e, h * c, 72, hub=1, isolated=6)
+    rng = np.random.default_rng(72)
+    q, k, v = (rng.standard_normal((n, h * c)) for _ in range(3))
+    out, alpha, ab = oracle.dot_softmax(wl.edge_index, n, q, k, v, h, c, 0.3)
+    csr = oracle.build_csr(wl.edge_index, n)
+    rows = np.arange(n)
+    out_r, alpha_r, ab_r = oracle.dot_softmax_rows(csr, n, q, k, v, h, c, 0.3, rows)
+    np.testing.assert_allclose(out_r, out, rtol=1e-13, atol=1e-14)
+    np.testing.assert_allclose(ab_r, ab, rtol=1e-13, atol=1e-14)
+    np.testing.assert_allclose(alpha_r, alpha[csr[2]], rtol=1e-13)
+
+
+# ---------------------------------------------------------------------------
+# Multi-hop propagation (APPNP / SGC)
+# ---------------------------------------------------------------------------
+def pin_appnp_hand_example(o):
+    """Path 0-1-2 with implicit self-loops: d = (2, 3, 2), so Ahat has 1/2 at
+    the ends of the diagonal, 1/3 in the middle and 1/sqrt(6) off it.  Two
+    APPNP steps from x0 = I with alpha = 0.1 give 0.81 Ahat^2 + 0.09 Ahat + 0.1 I;
+    entry (0, 0) is 0.81 (1/4 + 1/6) + 0.09 / 2 + 0.1 = 0.4825 and entry (0, 2)
+    is 0.81 / 6 = 0.135."""
+    ei = np.array([[0, 1, 1, 2], [1, 0, 2, 1]])
+    out, _ = o.appnp(ei, 3, np.eye(3), 2, 0.1, add_self_loops=1)
+    assert abs(out[0, 0] - 0.4825) < 1e-15
+    assert abs(out[0, 2] - 0.135) < 1e-15
+    assert abs(out[1, 1] - (0.81 * (1 / 6 + 1 / 9 + 1 / 6) + 0.09 / 3 + 0.1)) < 1e-15
+    assert abs(out[0, 1] - (0.81 * (1 / (2 * math.sqrt(6)) + 1 / (3 * math.sqrt(6)))
+                            + 0.09 / math.sqrt(6))) < 1e-15
+
+
+def test_appnp_hand_example():
+    pin_appnp_hand_example(oracle.default)
+
+
+def pin_appnp_dense_closed_form(o):
+    """h_K = ((1-a) Ahat)^K x0 + a * sum_{j<K} ((1-a) Ahat)^j x0, with Ahat the
+    numpy dense GCN matrix (an independent route); SGC is a = 0."""
+    for seed in range(5):
+        n = [1, 6, 20, 40, 64][seed]
+        e = [2, 14, 90, 160, 0][seed]
+        wl = gg.random_edge_case_graph(n, e, 5, 40 + seed, hub=0 if n > 2 else -1,
+                                       isolated=min(2, n - 1))
+        ew = np.random.default_rng(seed).uniform(0.2, 2.0, size=e)
+        xd = wl.x.astype(np.float64)
+        for selfl, alpha, k in ((1, 0.1, 4), (0, 0.25, 3), (1, 0.0, 3), (1, 1.0, 2), (0, 0.5, 0)):
+            a_hat = oracle.dense_gcn_matrix(wl.edge_index, n, ew, selfl, 1.0)
+            m = (1.0 - alpha) * a_hat
+            ref = np.linalg.matrix_power(m, k) @ xd
+            for j in range(k):
+                ref = ref + alpha * (np.linalg.matrix_power(m, j) @ xd)
+            out, _ = o.appnp(wl.edge_index, n, wl.x, k, alpha, ew, add_self_loops=selfl, fill=1.0)
+            np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_appnp_dense_closed_form():
+    pin_appnp_dense_closed_form(oracle.default)
+
+
+def pin_appnp_limits(o):
+    """K = 0 and alpha = 1 return x0; many steps reach the personalised
+    PageRank fixed point alpha (I - (1 - alpha) Ahat)^-1 x0 of APPNP; on a
+    symmetric graph with self-loops x0 = sqrt(d) is a fixed point of every
+    step (Ahat sqrt(d) = sqrt(d)); the error scale equals the value when all
+    weights and features are non-negative."""
+    ei = _undirected_random(30, 70, 3)
+    x0 = np.random.default_rng(3).standard_normal((30, 4))
+    for k, alpha in ((0, 0.3), (5, 1.0)):
+        out, _ = o.appnp(ei, 30, x0, k, alpha, add_self_loops=1)
+        np.testing.assert_array_equal(out, x0)
+    alpha = 0.2
+    out, _ = o.appnp(ei, 30, x0, 300, alpha, add_self_loops=1)
+    a_hat = oracle.dense_gcn_matrix(ei, 30, None, 1, 1.0)
+    ppr = alpha * np.linalg.solve(np.eye(30) - (1 - alpha) * a_hat, x0)
+    np.testing.assert_allclose(out, ppr, rtol=1e-10, atol=1e-12)
+    d = np.bincount(ei[1], minlength=30) + 1.0
+    sq = np.sqrt(d)[:, None] * np.array([[1.0, -2.0]])
+    out, _ = o.appnp(ei, 30, sq, 6, 0.15, add_self_loops=1)
+    np.testing.assert_allclose(out, sq, rtol=1e-12)
+    pos = np.abs(x0)
+    out, ab = o.appnp(ei, 30, pos, 4, 0.1, add_self_loops=1)
+    np.testing.assert_allclose(ab, out, rtol=1e-14)
+
+
+def test_appnp_limits():
+    pin_appnp_limits(oracle.default)
+
+
+# ---------------------------------------------------------------------------
 # Planted mistakes: each one must trip at least one pin
 # ---------------------------------------------------------------------------
 PLANTS = {
@@ -380,6 +552,8 @@ PLANTS = {
     "MEAN_PLUS_ONE": [pin_ones_give_in_degree, pin_softmax_normalised_and_mean_limit],
     "NO_LEAKY": [pin_star_softmax],
     "POOL_SKIP_LAST": [pin_pool_counts],
+    "APPNP_TELEPORT_FROM_H": [pin_appnp_hand_example, pin_appnp_dense_closed_form],
+    "DOT_KEY_AT_TARGET": [pin_dot_star],
 }
 
 
