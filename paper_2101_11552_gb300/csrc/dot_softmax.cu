@@ -31,7 +31,14 @@ namespace tfg {
 namespace {
 
 constexpr int kDotThreads = 256;
-constexpr int kDotUnroll = 4;              // edges gathered per lane per step
+// Tuning knobs (compile-time; the defaults are the measured best on GB300).
+#ifndef TFG_DOT_UNROLL
+#define TFG_DOT_UNROLL 4   // edges gathered per lane per step (key + value rows)
+#endif
+#ifndef TFG_DOT_MINB
+#define TFG_DOT_MINB 2     // resident CTAs per SM asked of the compiler, 16-byte bf16 path
+#endif
+constexpr int kDotUnroll = TFG_DOT_UNROLL;
 constexpr int64_t kDotMinWork = 2048;      // edges + rows per CTA, at least
 constexpr int kDotMaxChannels = 256;
 
@@ -67,6 +74,41 @@ __device__ __forceinline__ void dot_rows(const int32_t *rowptr, int64_t n, RowFn
         i = __shfl_sync(kFull, i, 0);
         if (i >= r1 - r0) break;
         fn(r0 + i, lane);
+    }
+}
+
+// This lane's share of a head's dot product: two interleaved fp32 chains
+// through the packed fma (even and odd channels), added at the end.
+template <int VEC>
+__device__ __forceinline__ float lane_dot(const float (&q)[VEC], const float (&k)[VEC]) {
+    if constexpr (VEC % 2 == 0) {
+        float2 d = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int i = 0; i < VEC; i += 2)
+            d = fma2(make_float2(q[i], q[i + 1]), make_float2(k[i], k[i + 1]), d);
+        return d.x + d.y;
+    } else {
+        float d = 0.f;
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) d = fmaf(q[i], k[i], d);
+        return d;
+    }
+}
+
+// part += p * v through the packed fma.
+template <int VEC>
+__device__ __forceinline__ void axpy_vec(float (&part)[VEC], float p, const float (&v)[VEC]) {
+    if constexpr (VEC % 2 == 0) {
+        const float2 p2 = make_float2(p, p);
+#pragma unroll
+        for (int i = 0; i < VEC; i += 2) {
+            const float2 r = fma2(make_float2(v[i], v[i + 1]), p2, make_float2(part[i], part[i + 1]));
+            part[i] = r.x;
+            part[i + 1] = r.y;
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) part[i] = fmaf(p, v[i], part[i]);
     }
 }
 
@@ -116,9 +158,7 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh, int64_t t
                 for (int u = 0; u < kDotUnroll; ++u) {
                     float kv[VEC];
                     V::widen(rk[u], kv);
-                    float d = 0.f;
-#pragma unroll
-                    for (int q = 0; q < VEC; ++q) d = fmaf(qv[q], kv[q], d);
+                    float d = lane_dot(qv, kv);
                     for (int o = 1; o < lh; o <<= 1) d += __shfl_xor_sync(kFull, d, o);
                     l[u] = ok[u] ? d * a.scale : -CUDART_INF_F;
                     mc = fmaxf(mc, l[u]);
@@ -140,8 +180,7 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh, int64_t t
                     den_part += p;
                     float vv[VEC];
                     V::widen(rv[u], vv);
-#pragma unroll
-                    for (int q = 0; q < VEC; ++q) part[q] = fmaf(p, vv[q], part[q]);
+                    axpy_vec(part, p, vv);
                 }
             }
             den += den_part;
@@ -177,9 +216,7 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh, int64_t t
                 const int64_t src = ok ? __ldg(a.col + k) : 0;
                 float kv[VEC];
                 V::load(kp + src * f + fl, kv);
-                float d = 0.f;
-#pragma unroll
-                for (int q = 0; q < VEC; ++q) d = fmaf(qv[q], kv[q], d);
+                float d = lane_dot(qv, kv);
                 for (int o = 1; o < lh; o <<= 1) d += __shfl_xor_sync(kFull, d, o);
                 if (ok && fok && sub % lh == 0)
                     a.alpha[k * a.heads + h] = __expf(d * a.scale - m) / den;
@@ -284,7 +321,7 @@ __device__ __forceinline__ void dot_general_row(const DotArgs &a, int64_t t, int
 // 16-byte bf16 rows hold twice the features per gather: two resident CTAs
 // per SM leave the registers for kDotUnroll key + value gathers in flight.
 template <typename XT, int VEC, int LPR>
-__global__ void __launch_bounds__(kDotThreads, VEC >= 8 ? 2 : 3) dot_fast(DotArgs a, int lh) {
+__global__ void __launch_bounds__(kDotThreads, VEC >= 8 ? TFG_DOT_MINB : 3) dot_fast(DotArgs a, int lh) {
     dot_rows(a.rowptr, a.n, [&](int64_t t, int lane) { dot_fast_row<XT, VEC, LPR>(a, lh, t, lane); });
 }
 

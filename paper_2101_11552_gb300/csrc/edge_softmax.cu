@@ -183,11 +183,13 @@ __device__ __forceinline__ void generic_row(const int32_t *__restrict__ rowptr,
 
 // Fast form for the common layout: H divides 32, every lane's VEC features
 // lie in one head, and one feature tile covers the row (F <= LPR * VEC).
-// Two passes over the row, no data-dependent branches:
+// One pass over the row in 32-edge chunks:
 //  * score lanes: lane (se, sh) = (lane / H, lane % H) evaluates the logit of
 //    edge slot se and head sh -- each (edge, head) logit and exponential is
-//    computed once.  Pass 1 takes the row maximum per head (butterfly over
-//    the lanes of a head); pass 2 forms p = exp(l - m) and the denominator.
+//    computed once.  The chunk's maximum per head (butterfly over the lanes
+//    of a head) updates the running maximum m; when m rises, the sums so far
+//    are rescaled by exp(m_old - m_new) (a warp-uniform branch, taken a few
+//    times per row).  p = exp(l - m) then feeds the denominator.
 //  * feature lanes: group g = lane / LPR gathers every G-th edge, fetches the
 //    p of its (edge, head) from the score lane holding it with one shuffle,
 //    and accumulates p * x into fp32 per-chunk partials.
@@ -214,37 +216,42 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
     const int64_t beg = rowptr[t], end = col ? rowptr[t + 1] : rowptr[t];
     const float sd = __ldg(s_dst + t * H + sh);
 
-    // pass 1: row maximum of every head
-    float m = -CUDART_INF_F;
-    for (int64_t base = beg; base < end; base += 32) {
-        const int cnt = static_cast<int>(min64(32, end - base));
-        const int c = lane < cnt ? __ldg(col + base + lane) : 0;
-#pragma unroll
-        for (int r = 0; r < R; ++r) {
-            const int k = r * ES + se;
-            const int src = __shfl_sync(kFull, c, k);
-            if (k < cnt) m = fmaxf(m, leaky(__ldg(s_src + static_cast<int64_t>(src) * H + sh) + sd, slope));
-        }
-    }
-#pragma unroll
-    for (int o = H; o < 32; o <<= 1) m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
-
-    // pass 2: p, denominator, and the p-weighted feature sum
-    float den = 0.f, acc[VEC];
+    // one pass over the row, 32 edges at a time: the score lanes form the
+    // chunk's logits, the running maximum m of each head absorbs the chunk's
+    // maximum (earlier sums are rescaled by exp(m_old - m_new) when it rises),
+    // then p = exp(l - m) weights the chunk's gathered rows
+    float m = -CUDART_INF_F, den = 0.f, acc[VEC];
 #pragma unroll
     for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
     for (int64_t base = beg; base < end; base += 32) {
         const int cnt = static_cast<int>(min64(32, end - base));
         const int c = lane < cnt ? __ldg(col + base + lane) : 0;
         float p[R];
-        float den_part = 0.f;
+        float cm = -CUDART_INF_F;
 #pragma unroll
         for (int r = 0; r < R; ++r) {
             const int k = r * ES + se;
             const int src = __shfl_sync(kFull, c, k);
-            p[r] = 0.f;
-            if (k < cnt)
-                p[r] = __expf(leaky(__ldg(s_src + static_cast<int64_t>(src) * H + sh) + sd, slope) - m);
+            p[r] = k < cnt ? leaky(__ldg(s_src + static_cast<int64_t>(src) * H + sh) + sd, slope)
+                           : -CUDART_INF_F;
+            cm = fmaxf(cm, p[r]);
+        }
+#pragma unroll
+        for (int o = H; o < 32; o <<= 1) cm = fmaxf(cm, __shfl_xor_sync(kFull, cm, o));
+        const bool rises = cm > m;
+        if (__any_sync(kFull, rises)) {   // warp-uniform; rare after the first chunks
+            const float sc = rises ? (m == -CUDART_INF_F ? 0.f : __expf(m - cm)) : 1.f;
+            den *= sc;
+            const float fsc = __shfl_sync(kFull, sc, fh);   // lane fh scores head fh
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] *= fsc;
+            m = fmaxf(m, cm);
+        }
+        float den_part = 0.f;
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const int k = r * ES + se;
+            p[r] = k < cnt ? __expf(p[r] - m) : 0.f;
             den_part += p[r];
         }
         den += den_part;
