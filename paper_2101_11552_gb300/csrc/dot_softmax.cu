@@ -33,7 +33,7 @@ namespace {
 constexpr int kDotThreads = 256;
 // Tuning knobs (compile-time; the defaults are the measured best on GB300).
 #ifndef TFG_DOT_UNROLL
-#define TFG_DOT_UNROLL 4   // edges gathered per lane per step (key + value rows)
+#define TFG_DOT_UNROLL 8   // edges gathered per lane per step (key + value rows)
 #endif
 #ifndef TFG_DOT_MINB
 #define TFG_DOT_MINB 2     // resident CTAs per SM asked of the compiler, 16-byte bf16 path

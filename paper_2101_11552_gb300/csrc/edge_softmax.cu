@@ -226,6 +226,14 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
     for (int64_t base = beg; base < end; base += 32) {
         const int cnt = static_cast<int>(min64(32, end - base));
         const int c = lane < cnt ? __ldg(col + base + lane) : 0;
+        // the first step's row gathers need only the column ids: issue them
+        // before the scores so that their latency overlaps the score work
+        typename V::Raw raw0[kSmUnroll];
+#pragma unroll
+        for (int u = 0; u < kSmUnroll; ++u) {
+            const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, (u * G + g) & 31));
+            raw0[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
+        }
         float p[R];
         float cm = -CUDART_INF_F;
 #pragma unroll
@@ -267,10 +275,14 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
             for (int u = 0; u < kSmUnroll; ++u) {
                 const int k0 = e + u * G;              // edge of group 0 in this step
                 const int k = k0 + g;
-                const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31));
                 // p of (edge k, head fh) sits in lane (k % ES) * H + fh, register k / ES
                 pw[u] = __shfl_sync(kFull, p[k0 / ES], ((k0 % ES) + g) * H + fh);
-                raw[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
+                if (e == 0) {
+                    raw[u] = raw0[u];
+                } else {
+                    const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31));
+                    raw[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
+                }
             }
 #pragma unroll
             for (int u = 0; u < kSmUnroll; ++u) {
