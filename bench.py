@@ -254,6 +254,29 @@ def _event_ms(fn, stream, reps: int) -> float:
     return t0.elapsed_time(t1) / reps
 
 
+def cold_l2_ms(fns: dict, stream, reps: int = 5) -> dict:
+    """Each call timed alone right after a write of 256 MB (twice the L2), so
+    that its node features and edge arrays come from HBM: the cold-L2
+    counterpart of the per-call times inside the step."""
+    import torch
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=torch.cuda.current_device())
+    out = {}
+    for name, fn in fns.items():
+        fn()
+        ts = []
+        for _ in range(reps):
+            flush.fill_(1)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        out[name] = round(statistics.median(ts), 4)
+    return out
+
+
 def next_rows(L, wl, bufs, stream, hbm_peak):
     """The rows built beyond the timed step, each measured on its own (not part
     of the headline value): APPNP K = 10 on the same graph and bf16 features,
@@ -593,6 +616,15 @@ def main():
                 "d2h_bytes_per_step": d2h, "steps": args.e2e_steps},
         "clocks": clocks.summary(),
     }
+    line["kernels_cold_l2_ms"] = cold_l2_ms({
+        "gcn_aggregate": lambda: check(L.tfg_gcn_aggregate_sum(
+            P(rowptr), P(col), P(dinv), None, P(xb), tfg.TFG_BF16, n, f, 1, 1.0, P(h), sp)),
+        "edge_softmax": lambda: check(L.tfg_edge_softmax_aggregate(
+            P(rowptr), P(col), P(xb), tfg.TFG_BF16, n, e, heads, ch, P(a_src), P(a_dst), 0.2,
+            P(att), None, P(ws_sm), ws_sm.numel(), sp)),
+        "pool_mean": lambda: check(L.tfg_segment_pool(
+            P(h), tfg.TFG_F32, P(batch), n, g, f, tfg.REDUCERS["mean"], P(pool_mean), st1, sp)),
+    }, stream)
     line["next_rows"] = next_rows(L, wl, dict(rowptr=rowptr, col=col, dinv=dinv, xb=xb, h=h,
                                               batch=batch), stream, hbm_peak)
     if world == 1 and not args.no_cpu_baseline:

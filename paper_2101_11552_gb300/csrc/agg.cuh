@@ -121,13 +121,19 @@ struct Agg {
         for (int j = 0; j < (FULL ? 32 : cnt); j += G * kUnroll) {
             typename V::Raw raw[kUnroll];
             float wt[kUnroll];
+            // all row gathers first (they need only the column ids), then the
+            // weights, whose loads may still be in flight
 #pragma unroll
             for (int u = 0; u < kUnroll; ++u) {
                 const int k = j + u * G + g;
                 const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31));
+                raw[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
+            }
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int k = j + u * G + g;
                 wt[u] = weighted ? __shfl_sync(kFull, ww, k & 31) : 1.f;
                 if (!FULL && k >= cnt) wt[u] = 0.f;
-                raw[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
             }
 #pragma unroll
             for (int u = 0; u < kUnroll; ++u) axpy(part, wt[u], raw[u]);
