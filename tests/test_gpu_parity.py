@@ -163,7 +163,10 @@ def test_gcn_aggregate_weighted(add_self):
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("heads,channels", [(1, 1), (2, 3), (4, 4), (8, 16), (3, 48), (1, 160),
-                                            (2, 8), (16, 8)])
+                                            (2, 8), (16, 8),
+                                            # head-per-lane kernel: C of one or two 16-byte vectors
+                                            (1, 4), (8, 4), (1, 8), (4, 8), (8, 8), (1, 16),
+                                            (2, 16), (4, 16)])
 def test_edge_softmax(heads, channels, dtype):
     n, e = 3000, 25000
     f = heads * channels
