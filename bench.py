@@ -374,7 +374,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["tfg", "reference"], default="tfg")
-    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--pairs", type=int, default=57_300_000, help=argparse.SUPPRESS)
@@ -471,7 +471,13 @@ def main():
         if rc != 0:
             raise RuntimeError(f"libtfg error {rc}: {tfg.tfg_last_error()}")
 
-    def step(ev=None):
+    main_io = dict(edge=edge, xb=xb, batch=batch, a_src=a_src, a_dst=a_dst, h=h, att=att,
+                   pool_mean=pool_mean, pool_max=pool_max)
+
+    def step(ev=None, io=None):
+        io = main_io if io is None else io
+        edge, xb, batch, a_src, a_dst = (io[k] for k in ("edge", "xb", "batch", "a_src", "a_dst"))
+        h, att, pool_mean, pool_max = (io[k] for k in ("h", "att", "pool_mean", "pool_max"))
         if ev is not None:
             ev[0].record(stream)
         check(L.tfg_build_csr(P(edge), e, n, P(rowptr), P(col), P(perm), P(indeg), P(ws_csr),
@@ -542,29 +548,58 @@ def main():
     h2d = sum(t.numel() * t.element_size() for t in (hp_edge, hp_xb, hp_batch, hp_as, hp_ad))
     d2h = sum(t.numel() * t.element_size() for t in (ho_h, ho_att, ho_pm, ho_px))
 
-    def e2e_step():
-        edge.copy_(hp_edge, non_blocking=True)
-        xb.copy_(hp_xb, non_blocking=True)
-        batch.copy_(hp_batch, non_blocking=True)
-        a_src.copy_(hp_as, non_blocking=True)
-        a_dst.copy_(hp_ad, non_blocking=True)
-        step()
-        ho_h.copy_(h, non_blocking=True)
-        ho_att.copy_(att, non_blocking=True)
-        ho_pm.copy_(pool_mean, non_blocking=True)
-        ho_px.copy_(pool_max, non_blocking=True)
+    # Every step copies its inputs in and its results out; the copies of one
+    # step overlap the kernels of its neighbours: inputs and outputs are
+    # double-buffered on the device, host->device copies run on one stream,
+    # device->host copies on another, and events order each buffer's reuse.
+    other_io = {k: torch.empty_like(v) for k, v in main_io.items()}
+    io_sets = (main_io, other_io)
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev_loaded = [torch.cuda.Event() for _ in range(2)]
+    ev_computed = [torch.cuda.Event() for _ in range(2)]
+    ev_drained = [torch.cuda.Event() for _ in range(2)]
+    host_in = dict(edge=hp_edge, xb=hp_xb, batch=hp_batch, a_src=hp_as, a_dst=hp_ad)
+    host_out = dict(h=ho_h, att=ho_att, pool_mean=ho_pm, pool_max=ho_px)
 
-    for _ in range(2):
-        e2e_step()
+    def load(i):
+        b = i % 2
+        with torch.cuda.stream(s_in):
+            if i >= 2:
+                s_in.wait_event(ev_computed[b])      # step i - 2 is done with these inputs
+            for k, t in host_in.items():
+                io_sets[b][k].copy_(t, non_blocking=True)
+            ev_loaded[b].record(s_in)
+
+    def e2e_run(k: int, start_ev=None, stop_ev=None):
+        if start_ev is not None:
+            start_ev.record(stream)
+            s_in.wait_event(start_ev)
+        load(0)
+        for i in range(k):
+            b = i % 2
+            if i + 1 < k:
+                load(i + 1)
+            stream.wait_event(ev_loaded[b])
+            if i >= 2:
+                stream.wait_event(ev_drained[b])     # results of step i - 2 have left
+            step(io=io_sets[b])
+            ev_computed[b].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_computed[b])
+                for key, t in host_out.items():
+                    t.copy_(io_sets[b][key], non_blocking=True)
+                ev_drained[b].record(s_out)
+        stream.wait_event(ev_drained[(k - 1) % 2])
+        if stop_ev is not None:
+            stop_ev.record(stream)
+
+    e2e_run(2)
     torch.cuda.synchronize()
     if pg:
         dist.barrier()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.e2e_steps):
-        e2e_step()
-    e1.record(stream)
+    e2e_run(args.e2e_steps, e0, e1)
     torch.cuda.synchronize()
     e2e_t, e2e_units = combine_ranks(e0.elapsed_time(e1) / 1e3,
                                      units_per_step(n, e, f) * args.e2e_steps, world, pg)

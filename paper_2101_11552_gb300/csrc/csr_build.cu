@@ -186,13 +186,15 @@ cudaError_t exclusive_scan(int32_t *data, int64_t m, int32_t *sums, cudaStream_t
 // ---- downsweep ------------------------------------------------------------
 // 16 warps share one 4096-edge tile, 8 elements per lane.  Every global load
 // of the tile is issued up front, so the tile waits on memory once.
-//   A  per-warp digit counts with shared-memory atomics (order-free)
+//   A  per round of 32 elements, lanes holding equal digits are found with
+//      one ballot per digit bit; the group's leader advances the warp's
+//      private counter of that digit, and each element keeps its rank among
+//      the warp's elements of its digit so far (a byte, 8 per lane packed in
+//      two registers)
 //   B  per digit: warp-major exclusive prefix and tile total; block scan of
-//      the totals over digits -> each digit's first slot in the tile, folded
-//      into every warp's counter; per digit, global base minus tile start
-//   C  stable slots: per round, peers with equal digits are found with
-//      __match_any_sync, their leader claims a block of slots with one
-//      returning atomic, and each lane adds its rank among the peers; key,
+//      the totals over digits -> each digit's first slot in the tile; per
+//      digit, global base minus tile start
+//   C  stable slot = digit's first tile slot + warp prefix + rank; key,
 //      source and edge id are staged in three arrays
 //   D  the tile leaves in digit order, consecutive threads writing
 //      consecutive positions of each digit's run
@@ -203,6 +205,19 @@ constexpr int kDsItems = kTile / kDsThreads;   // 8 per lane
 size_t downsweep_smem(int radix) {
     return sizeof(uint32_t) * 3 * kTile + sizeof(int32_t) * kDsWarps * radix +
            sizeof(int32_t) * 2 * radix + sizeof(int32_t) * 32;
+}
+
+// Lanes of the warp whose value of dig equals this lane's, for dig below
+// 2^(width + 1): one ballot per bit (measured faster here than
+// __match_any_sync).
+__device__ __forceinline__ unsigned same_digit_lanes(uint32_t dig, int width) {
+    unsigned peers = kFull;
+    for (int b = 0; b <= width; ++b) {
+        const bool set = (dig >> b) & 1u;
+        const unsigned bal = __ballot_sync(kFull, set);
+        peers &= set ? bal : ~bal;
+    }
+    return peers;
 }
 
 template <bool FIRST>
@@ -253,10 +268,28 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     }
     __syncwarp();
 
-    // A: per-warp digit counts.
+    const unsigned lower = (1u << lane) - 1u;
+    // A: per-warp digit counts, and each element's rank among the warp's
+    // earlier elements of its digit (one leader per digit group bumps the
+    // warp's private counter)
+    uint32_t rank_lo = 0, rank_hi = 0;   // 8 ranks < 256, one byte each
 #pragma unroll
-    for (int r = 0; r < kDsItems; ++r)
-        if (wbase + r * 32 + lane < e) atomicAdd(&mine[(keys[r] >> shift) & (radix - 1)], 1);
+    for (int r = 0; r < kDsItems; ++r) {
+        const bool ok = wbase + r * 32 + lane < e;
+        const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
+        const unsigned peers = same_digit_lanes(dig, width);
+        const int leader = __ffs(peers) - 1;
+        int32_t base = 0;
+        if (ok && lane == leader) {
+            base = mine[dig];
+            mine[dig] = base + __popc(peers);
+        }
+        base = __shfl_sync(kFull, base, leader);
+        const uint32_t rk = static_cast<uint32_t>(base + __popc(peers & lower));
+        if (r < 4) rank_lo |= rk << (8 * r);
+        else rank_hi |= rk << (8 * (r - 4));
+        __syncwarp();
+    }
     __syncthreads();
 
     // B: warp-major prefix per digit, tile totals, then a block scan over digits.
@@ -300,25 +333,19 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     __syncthreads();
     for (int d = threadIdx.x; d < radix; d += kDsThreads) {
         const int32_t ts = s_tstart[d] + s_chunk[d >> 5];
+        s_tstart[d] = ts;   // first tile slot of digit d
         s_delta[d] -= ts;   // global position of tile slot i of digit d = delta[d] + i
-#pragma unroll
-        for (int w = 0; w < kDsWarps; ++w) s_cnt[w * radix + d] += ts;
     }
     __syncthreads();
 
     // C: stable slot of every element; stage (key, source, edge id).
-    const unsigned lower = (1u << lane) - 1u;
 #pragma unroll
     for (int r = 0; r < kDsItems; ++r) {
         const bool ok = wbase + r * 32 + lane < e;
         const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
-        const unsigned peers = __match_any_sync(kFull, dig);
-        const int leader = __ffs(peers) - 1;
-        int32_t base = 0;
-        if (ok && lane == leader) base = atomicAdd(&mine[dig], __popc(peers));
-        base = __shfl_sync(kFull, base, leader);
         if (ok) {
-            const int slot = base + __popc(peers & lower);
+            const uint32_t rk = (r < 4 ? rank_lo >> (8 * r) : rank_hi >> (8 * (r - 4))) & 0xffu;
+            const int slot = mine[dig] + s_tstart[dig] + static_cast<int>(rk);
             s_key[slot] = keys[r];
             s_src[slot] = srcs[r];
             s_eid[slot] = eids[r];
