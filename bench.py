@@ -186,7 +186,8 @@ def oracle_sample(wl, n_nodes: int):
     return {"edge_index": sub, "n": n_nodes, "x_bf16": wl.x_bf16[:n_nodes],
             "x": wl.x[:n_nodes], "batch": wl.batch[:n_nodes],
             "g": int(wl.batch[n_nodes - 1]) + 1, "a_src": wl.a_src, "a_dst": wl.a_dst,
-            "heads": wl.heads, "channels": wl.channels}
+            "heads": wl.heads, "channels": wl.channels,
+            "cut": bool(n_nodes < wl.num_nodes and wl.batch[n_nodes] == wl.batch[n_nodes - 1])}
 
 
 def oracle_step(s) -> int:
@@ -232,8 +233,10 @@ def time_oracle(wl, budget_s: float, steps: int = 1):
 
 
 def cpu_desc(s) -> str:
+    comm = (f"{s['g'] - 1} whole communities and part of the next" if s["cut"]
+            else f"{s['g']} whole communities")
     return (f"oracle (fp64, single thread) on the node-induced subgraph of the first {s['n']} nodes "
-            f"({s['g']} whole communities, {s['edge_index'].shape[1]} edges) of the same workload")
+            f"({comm}, {s['edge_index'].shape[1]} edges) of the same workload")
 
 
 # ---------------------------------------------------------------------------

@@ -25,6 +25,8 @@
 //    head (NCH chunks of 32), the logit finished by a full-warp butterfly.
 #include <math_constants.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 
 namespace tfg {
@@ -38,7 +40,9 @@ constexpr int kDotThreads = 256;
 #ifndef TFG_DOT_MINB
 #define TFG_DOT_MINB 2     // resident CTAs per SM asked of the compiler, 16-byte bf16 path
 #endif
-constexpr int kDotUnroll = TFG_DOT_UNROLL;
+// (the fp32 path, with half the features per load, keeps 4 in flight: 8 spill there)
+template <int VEC>
+__host__ __device__ constexpr int dot_unroll() { return VEC >= 8 ? TFG_DOT_UNROLL : 4; }
 constexpr int64_t kDotMinWork = 2048;      // edges + rows per CTA, at least
 constexpr int kDotMaxChannels = 256;
 
@@ -116,6 +120,7 @@ template <typename XT, int VEC, int LPR>
 __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh, int64_t t, int lane) {
     using V = VecLoad<XT, VEC>;
     constexpr int G = 32 / LPR;
+    constexpr int kDotUnroll = dot_unroll<VEC>();
     const int g = lane / LPR, sub = lane % LPR;
     const int64_t f = static_cast<int64_t>(a.heads) * a.channels;
     const XT *qp = static_cast<const XT *>(a.q);
@@ -135,20 +140,22 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh, int64_t t
         float m = -CUDART_INF_F, den = 0.f, acc[VEC];
 #pragma unroll
         for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
-        for (int64_t base = beg; base < end; base += 32) {
-            const int cnt = static_cast<int>(min64(32, end - base));
-            const int c = lane < cnt ? __ldg(a.col + base + lane) : 0;
+        // one 32-edge chunk; FULL chunks (all 32 slots used) skip every slot test
+        auto chunk = [&](auto full_tag, int64_t base, int cnt) {
+            constexpr bool FULL = decltype(full_tag)::value;
+            const int c = (FULL || lane < cnt) ? __ldg(a.col + base + lane) : 0;
             float den_part = 0.f, part[VEC];
 #pragma unroll
             for (int q = 0; q < VEC; ++q) part[q] = 0.f;
-            for (int j = 0; j < cnt; j += G * kDotUnroll) {
+#pragma unroll
+            for (int j = 0; j < (FULL ? 32 : cnt); j += G * kDotUnroll) {
                 typename V::Raw rk[kDotUnroll], rv[kDotUnroll];
                 bool ok[kDotUnroll];
 #pragma unroll
                 for (int u = 0; u < kDotUnroll; ++u) {
                     const int k = j + u * G + g;
                     const int64_t src = __shfl_sync(kFull, c, k & 31);
-                    ok[u] = k < cnt;
+                    ok[u] = FULL || k < cnt;
                     rk[u] = ok[u] ? V::raw(kp + src * f + fl) : V::zero();
                     rv[u] = ok[u] ? V::raw(vp + src * f + fl) : V::zero();
                 }
@@ -186,6 +193,11 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh, int64_t t
             den += den_part;
 #pragma unroll
             for (int q = 0; q < VEC; ++q) acc[q] += part[q];
+        };
+        for (int64_t base = beg; base < end; base += 32) {
+            const int cnt = static_cast<int>(min64(32, end - base));
+            if (cnt == 32) chunk(std::true_type{}, base, 32);
+            else chunk(std::false_type{}, base, cnt);
         }
         // merge the G groups' states in a fixed butterfly order
 #pragma unroll

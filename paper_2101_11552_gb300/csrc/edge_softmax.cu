@@ -21,6 +21,7 @@
 #include <math_constants.h>
 
 #include <mutex>
+#include <type_traits>
 
 #include "common.cuh"
 
@@ -32,6 +33,10 @@ constexpr int kSmThreads = 256;
 #define TFG_SM_UNROLL 8   // gathers in flight per lane (tuning knob)
 #endif
 constexpr int kSmUnroll = TFG_SM_UNROLL;   // fast kernel
+#ifndef TFG_SM_FULL_CHUNKS
+#define TFG_SM_FULL_CHUNKS 1   // separate code for full 32-edge chunks (no slot tests)
+#endif
+constexpr bool kSmFullChunks = TFG_SM_FULL_CHUNKS != 0;
 constexpr int kGenUnroll = 4;               // generic kernel
 
 // Compensated dot product (the "Dot2" scheme of Ogita, Rump and Oishi,
@@ -223,9 +228,10 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
     float m = -CUDART_INF_F, den = 0.f, acc[VEC];
 #pragma unroll
     for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
-    for (int64_t base = beg; base < end; base += 32) {
-        const int cnt = static_cast<int>(min64(32, end - base));
-        const int c = lane < cnt ? __ldg(col + base + lane) : 0;
+    // one 32-edge chunk; FULL chunks (all 32 slots used) skip every slot test
+    auto chunk = [&](auto full_tag, int64_t base, int cnt) {
+        constexpr bool FULL = decltype(full_tag)::value;
+        const int c = (FULL || lane < cnt) ? __ldg(col + base + lane) : 0;
         // the first step's row gathers need only the column ids: issue them
         // before the scores so that their latency overlaps the score work
         typename V::Raw raw0[kSmUnroll];
@@ -240,8 +246,9 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
         for (int r = 0; r < R; ++r) {
             const int k = r * ES + se;
             const int src = __shfl_sync(kFull, c, k);
-            p[r] = k < cnt ? leaky(__ldg(s_src + static_cast<int64_t>(src) * H + sh) + sd, slope)
-                           : -CUDART_INF_F;
+            p[r] = (FULL || k < cnt)
+                       ? leaky(__ldg(s_src + static_cast<int64_t>(src) * H + sh) + sd, slope)
+                       : -CUDART_INF_F;
             cm = fmaxf(cm, p[r]);
         }
 #pragma unroll
@@ -259,7 +266,7 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
 #pragma unroll
         for (int r = 0; r < R; ++r) {
             const int k = r * ES + se;
-            p[r] = k < cnt ? __expf(p[r] - m) : 0.f;
+            p[r] = (FULL || k < cnt) ? __expf(p[r] - m) : 0.f;
             den_part += p[r];
         }
         den += den_part;
@@ -268,7 +275,7 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
         for (int q = 0; q < VEC; ++q) part[q] = 0.f;
 #pragma unroll
         for (int e = 0; e < 32; e += G * kSmUnroll) {
-            if (e >= cnt) break;   // warp-uniform
+            if (!FULL && e >= cnt) break;   // warp-uniform
             typename V::Raw raw[kSmUnroll];
             float pw[kSmUnroll];
 #pragma unroll
@@ -305,6 +312,11 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
         }
 #pragma unroll
         for (int q = 0; q < VEC; ++q) acc[q] += part[q];
+    };
+    for (int64_t base = beg; base < end; base += 32) {
+        const int cnt = static_cast<int>(min64(32, end - base));
+        if (kSmFullChunks && cnt == 32) chunk(std::true_type{}, base, 32);
+        else chunk(std::false_type{}, base, cnt);
     }
 #pragma unroll
     for (int o = H; o < 32; o <<= 1) den += __shfl_xor_sync(kFull, den, o);
