@@ -17,6 +17,8 @@
 // the int64 edge_index directly and checks every id; the last pass writes
 // col (source) and perm (original edge id) in final order, plus the sorted
 // keys from which rowptr is found by binary search.
+#include <type_traits>
+
 #include "common.cuh"
 
 namespace tfg {
@@ -198,6 +200,10 @@ cudaError_t exclusive_scan(int32_t *data, int64_t m, int32_t *sums, cudaStream_t
 //      source and edge id are staged in three arrays
 //   D  the tile leaves in digit order, consecutive threads writing
 //      consecutive positions of each digit's run
+#ifndef TFG_DS_FULL_TILES
+#define TFG_DS_FULL_TILES 1   // separate code for full tiles (no bounds tests)
+#endif
+constexpr bool kDsFullTiles = TFG_DS_FULL_TILES != 0;
 constexpr int kDsWarps = 16;
 constexpr int kDsThreads = kDsWarps * 32;
 constexpr int kDsItems = kTile / kDsThreads;   // 8 per lane
@@ -239,133 +245,139 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t tile0 = static_cast<int64_t>(blockIdx.x) * kTile;
     const int count = static_cast<int>(min64(kTile, e - tile0));
-    int32_t *mine = s_cnt + warp * radix;
-    for (int d = lane; d < radix; d += 32) mine[d] = 0;
-    for (int d = threadIdx.x; d < radix; d += kDsThreads)
-        s_delta[d] = offs[static_cast<int64_t>(d) * num_tiles + blockIdx.x];   // global base for now
+    // every tile but the last is full: its copy of the code has no bounds tests
+    auto run = [&](auto full_tag) {
+        constexpr bool FULL = decltype(full_tag)::value;
+        int32_t *mine = s_cnt + warp * radix;
+        for (int d = lane; d < radix; d += 32) mine[d] = 0;
+        for (int d = threadIdx.x; d < radix; d += kDsThreads)
+            s_delta[d] = offs[static_cast<int64_t>(d) * num_tiles + blockIdx.x];   // global base for now
 
-    // All loads of this warp's sub-tile, issued together.
-    const int64_t wbase = tile0 + static_cast<int64_t>(warp) * 32 * kDsItems;
-    uint32_t keys[kDsItems];
-    int32_t srcs[kDsItems], eids[kDsItems];
-#pragma unroll
-    for (int r = 0; r < kDsItems; ++r) {
-        const int64_t idx = wbase + r * 32 + lane;
-        keys[r] = 0;
-        srcs[r] = 0;
-        eids[r] = 0;
-        if (idx < e) {
-            if (FIRST) {
-                keys[r] = checked_id(__ldg(dst64 + idx), n, nullptr);
-                srcs[r] = static_cast<int32_t>(checked_id(__ldg(src64 + idx), n, status));
-                eids[r] = static_cast<int32_t>(idx);
-            } else {
-                keys[r] = __ldg(key_in + idx);
-                srcs[r] = __ldg(src_in + idx);
-                eids[r] = __ldg(eid_in + idx);
+        // All loads of this warp's sub-tile, issued together.
+        const int64_t wbase = tile0 + static_cast<int64_t>(warp) * 32 * kDsItems;
+        uint32_t keys[kDsItems];
+        int32_t srcs[kDsItems], eids[kDsItems];
+    #pragma unroll
+        for (int r = 0; r < kDsItems; ++r) {
+            const int64_t idx = wbase + r * 32 + lane;
+            keys[r] = 0;
+            srcs[r] = 0;
+            eids[r] = 0;
+            if (FULL || idx < e) {
+                if (FIRST) {
+                    keys[r] = checked_id(__ldg(dst64 + idx), n, nullptr);
+                    srcs[r] = static_cast<int32_t>(checked_id(__ldg(src64 + idx), n, status));
+                    eids[r] = static_cast<int32_t>(idx);
+                } else {
+                    keys[r] = __ldg(key_in + idx);
+                    srcs[r] = __ldg(src_in + idx);
+                    eids[r] = __ldg(eid_in + idx);
+                }
             }
         }
-    }
-    __syncwarp();
-
-    const unsigned lower = (1u << lane) - 1u;
-    // A: per-warp digit counts, and each element's rank among the warp's
-    // earlier elements of its digit (one leader per digit group bumps the
-    // warp's private counter)
-    uint32_t rank_lo = 0, rank_hi = 0;   // 8 ranks < 256, one byte each
-#pragma unroll
-    for (int r = 0; r < kDsItems; ++r) {
-        const bool ok = wbase + r * 32 + lane < e;
-        const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
-        const unsigned peers = same_digit_lanes(dig, width);
-        const int leader = __ffs(peers) - 1;
-        int32_t base = 0;
-        if (ok && lane == leader) {
-            base = mine[dig];
-            mine[dig] = base + __popc(peers);
-        }
-        base = __shfl_sync(kFull, base, leader);
-        const uint32_t rk = static_cast<uint32_t>(base + __popc(peers & lower));
-        if (r < 4) rank_lo |= rk << (8 * r);
-        else rank_hi |= rk << (8 * (r - 4));
         __syncwarp();
-    }
-    __syncthreads();
 
-    // B: warp-major prefix per digit, tile totals, then a block scan over digits.
-    for (int d = threadIdx.x; d < radix; d += kDsThreads) {
-        int32_t c[kDsWarps];
-#pragma unroll
-        for (int w = 0; w < kDsWarps; ++w) c[w] = s_cnt[w * radix + d];
-        int32_t run = 0;
-#pragma unroll
-        for (int w = 0; w < kDsWarps; ++w) {
-            s_cnt[w * radix + d] = run;
-            run += c[w];
+        const unsigned lower = (1u << lane) - 1u;
+        // A: per-warp digit counts, and each element's rank among the warp's
+        // earlier elements of its digit (one leader per digit group bumps the
+        // warp's private counter)
+        uint32_t rank_lo = 0, rank_hi = 0;   // 8 ranks < 256, one byte each
+    #pragma unroll
+        for (int r = 0; r < kDsItems; ++r) {
+            const bool ok = FULL || wbase + r * 32 + lane < e;
+            const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
+            const unsigned peers = same_digit_lanes(dig, width);
+            const int leader = __ffs(peers) - 1;
+            int32_t base = 0;
+            if (ok && lane == leader) {
+                base = mine[dig];
+                mine[dig] = base + __popc(peers);
+            }
+            base = __shfl_sync(kFull, base, leader);
+            const uint32_t rk = static_cast<uint32_t>(base + __popc(peers & lower));
+            if (r < 4) rank_lo |= rk << (8 * r);
+            else rank_hi |= rk << (8 * (r - 4));
+            __syncwarp();
         }
-        s_tstart[d] = run;
-    }
-    __syncthreads();
-    const int chunks = (radix + 31) / 32;   // <= 32
-    for (int ch = warp; ch < chunks; ch += kDsWarps) {   // scan of each 32-digit chunk
-        const int d = ch * 32 + lane;
-        const int32_t v = d < radix ? s_tstart[d] : 0;
-        int32_t incl = v;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int32_t y = __shfl_up_sync(kFull, incl, o);
-            if (lane >= o) incl += y;
-        }
-        if (d < radix) s_tstart[d] = incl - v;
-        if (lane == 31) s_chunk[ch] = incl;
-    }
-    __syncthreads();
-    if (warp == 0) {   // exclusive scan of the chunk totals
-        const int32_t v = lane < chunks ? s_chunk[lane] : 0;
-        int32_t incl = v;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int32_t y = __shfl_up_sync(kFull, incl, o);
-            if (lane >= o) incl += y;
-        }
-        if (lane < chunks) s_chunk[lane] = incl - v;
-    }
-    __syncthreads();
-    for (int d = threadIdx.x; d < radix; d += kDsThreads) {
-        const int32_t ts = s_tstart[d] + s_chunk[d >> 5];
-        s_tstart[d] = ts;   // first tile slot of digit d
-        s_delta[d] -= ts;   // global position of tile slot i of digit d = delta[d] + i
-    }
-    __syncthreads();
+        __syncthreads();
 
-    // C: stable slot of every element; stage (key, source, edge id).
-#pragma unroll
-    for (int r = 0; r < kDsItems; ++r) {
-        const bool ok = wbase + r * 32 + lane < e;
-        const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
-        if (ok) {
-            const uint32_t rk = (r < 4 ? rank_lo >> (8 * r) : rank_hi >> (8 * (r - 4))) & 0xffu;
-            const int slot = mine[dig] + s_tstart[dig] + static_cast<int>(rk);
-            s_key[slot] = keys[r];
-            s_src[slot] = srcs[r];
-            s_eid[slot] = eids[r];
+        // B: warp-major prefix per digit, tile totals, then a block scan over digits.
+        for (int d = threadIdx.x; d < radix; d += kDsThreads) {
+            int32_t c[kDsWarps];
+    #pragma unroll
+            for (int w = 0; w < kDsWarps; ++w) c[w] = s_cnt[w * radix + d];
+            int32_t run = 0;
+    #pragma unroll
+            for (int w = 0; w < kDsWarps; ++w) {
+                s_cnt[w * radix + d] = run;
+                run += c[w];
+            }
+            s_tstart[d] = run;
         }
-    }
-    __syncthreads();
+        __syncthreads();
+        const int chunks = (radix + 31) / 32;   // <= 32
+        for (int ch = warp; ch < chunks; ch += kDsWarps) {   // scan of each 32-digit chunk
+            const int d = ch * 32 + lane;
+            const int32_t v = d < radix ? s_tstart[d] : 0;
+            int32_t incl = v;
+    #pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int32_t y = __shfl_up_sync(kFull, incl, o);
+                if (lane >= o) incl += y;
+            }
+            if (d < radix) s_tstart[d] = incl - v;
+            if (lane == 31) s_chunk[ch] = incl;
+        }
+        __syncthreads();
+        if (warp == 0) {   // exclusive scan of the chunk totals
+            const int32_t v = lane < chunks ? s_chunk[lane] : 0;
+            int32_t incl = v;
+    #pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int32_t y = __shfl_up_sync(kFull, incl, o);
+                if (lane >= o) incl += y;
+            }
+            if (lane < chunks) s_chunk[lane] = incl - v;
+        }
+        __syncthreads();
+        for (int d = threadIdx.x; d < radix; d += kDsThreads) {
+            const int32_t ts = s_tstart[d] + s_chunk[d >> 5];
+            s_tstart[d] = ts;   // first tile slot of digit d
+            s_delta[d] -= ts;   // global position of tile slot i of digit d = delta[d] + i
+        }
+        __syncthreads();
 
-    // D: write the tile out, one coalesced run per digit.
-#pragma unroll
-    for (int j = 0; j < kDsItems; ++j) {
-        const int i = threadIdx.x + j * kDsThreads;
-        if (i < count) {
-            const uint32_t k = s_key[i];
-            const int d = static_cast<int>((k >> shift) & (radix - 1));
-            const int64_t pos = static_cast<int64_t>(s_delta[d]) + i;
-            key_out[pos] = k;
-            src_out[pos] = s_src[i];
-            eid_out[pos] = s_eid[i];
+        // C: stable slot of every element; stage (key, source, edge id).
+    #pragma unroll
+        for (int r = 0; r < kDsItems; ++r) {
+            const bool ok = FULL || wbase + r * 32 + lane < e;
+            const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
+            if (ok) {
+                const uint32_t rk = (r < 4 ? rank_lo >> (8 * r) : rank_hi >> (8 * (r - 4))) & 0xffu;
+                const int slot = mine[dig] + s_tstart[dig] + static_cast<int>(rk);
+                s_key[slot] = keys[r];
+                s_src[slot] = srcs[r];
+                s_eid[slot] = eids[r];
+            }
         }
-    }
+        __syncthreads();
+
+        // D: write the tile out, one coalesced run per digit.
+    #pragma unroll
+        for (int j = 0; j < kDsItems; ++j) {
+            const int i = threadIdx.x + j * kDsThreads;
+            if (FULL || i < count) {
+                const uint32_t k = s_key[i];
+                const int d = static_cast<int>((k >> shift) & (radix - 1));
+                const int64_t pos = static_cast<int64_t>(s_delta[d]) + i;
+                key_out[pos] = k;
+                src_out[pos] = s_src[i];
+                eid_out[pos] = s_eid[i];
+            }
+        }
+    };
+    if (kDsFullTiles && count == kTile) run(std::true_type{});
+    else run(std::false_type{});
 }
 
 // rowptr[k] = first sorted position whose key is >= k, for k in [0, n].

@@ -314,6 +314,66 @@ def test_c4_batched_gcn_then_pool_full():
         np.testing.assert_allclose(h32[s0:s1], ref_g, rtol=1e-5, atol=1e-5)
 
 
+def test_c1_appnp_and_sgc_full():
+    """APPNP with the settings of its paper (K = 10, alpha = 0.1) and SGC with
+    K = 2 on the 2,708-node citation-sized graph (explicit self-loops)."""
+    wl = gg.make_c1()
+    n = wl.num_nodes
+    csr = gpu_csr(wl.edge_index, n)
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
+    got = np_(tfg.tfg_appnp_propagate(csr.rowptr, csr.col, dinv, dev(wl.x), 10, 0.1))
+    ref, scale = oracle.appnp(wl.edge_index, n, wl.x, 10, 0.1)
+    assert_scaled_close(got, ref, scale, TOL_F32, "c1 appnp")
+    got = np_(tfg.tfg_sgc_propagate(csr.rowptr, csr.col, dinv, dev(wl.x), 2))
+    ref, scale = oracle.sgc(wl.edge_index, n, wl.x, 2)
+    assert_scaled_close(got, ref, scale, TOL_F32, "c1 sgc")
+
+
+def test_c3_dot_softmax_full():
+    """Transformer-style attention on the GAT workload's graph (169,343 nodes,
+    1,166,243 edges, 8 heads x 16): q from the features, k and v seeded."""
+    wl = gg.make_c3()
+    n = wl.num_nodes
+    csr = gpu_csr(wl.edge_index, n)
+    rng = np.random.default_rng(1303)
+    k = rng.standard_normal(wl.x.shape, dtype=np.float32)
+    v = rng.standard_normal(wl.x.shape, dtype=np.float32)
+    out, alpha = tfg.tfg_dot_edge_softmax_aggregate(csr.rowptr, csr.col, dev(wl.x), dev(k), dev(v),
+                                                    wl.heads, wl.channels, want_alpha=True)
+    ref, ref_alpha, scale = oracle.dot_softmax(wl.edge_index, n, wl.x, k, v, wl.heads, wl.channels,
+                                               float(np.float32(1.0 / np.sqrt(wl.channels))))
+    assert_scaled_close(np_(out), ref, scale, TOL_F32, "c3 dot out")
+    perm = np_(csr.perm)
+    assert_scaled_close(np_(alpha), ref_alpha[perm], alpha_scale(ref_alpha[perm]), TOL_F32, "c3 dot alpha")
+
+
+def test_c4_device_batching_and_meanmax_full():
+    """The 1,024 molecule graphs batched on the device equal the generator's
+    BatchGraph; the Mean-Max readout of the GCN output equals the oracle."""
+    wl = gg.make_c4()
+    sizes = np.asarray(wl.graph_sizes, np.int64)
+    offs = np.concatenate([[0], np.cumsum(sizes)[:-1]])
+    src_graph = wl.batch[wl.edge_index[0]]
+    local = np.ascontiguousarray(wl.edge_index - offs[src_graph][None, :])
+    ecount = np.bincount(src_graph, minlength=len(sizes)).astype(np.int64)
+    bg = tfg.tfg_batch_graphs(dev(sizes), dev(ecount), dev(local), wl.num_nodes)
+    tfg.check_status(bg.status)
+    ei, batch, node_offsets = oracle.batch_graphs(sizes, ecount, local)
+    assert np.array_equal(np_(bg.edge_index), ei) and np.array_equal(ei, wl.edge_index)
+    assert np.array_equal(np_(bg.batch), batch) and np.array_equal(batch, wl.batch)
+    assert np.array_equal(np_(bg.node_offsets), node_offsets)
+    n = wl.num_nodes
+    csr = gpu_csr(wl.edge_index, n)
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
+    h = tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, dev(wl.x))
+    out, status = tfg.tfg_segment_pool_meanmax(h, bg.batch, wl.num_graphs)
+    tfg.check_status(status)
+    ref, scale = oracle.segment_pool_meanmax(np_(h), wl.batch, wl.num_graphs)
+    f = wl.x.shape[1]
+    assert_scaled_close(np_(out)[:, :f], ref[:, :f], scale[:, :f], TOL_F32, "c4 mean")
+    assert_exact_f32(np_(out)[:, f:], ref[:, f:], "c4 max")
+
+
 def test_deterministic_bitwise():
     wl = gg.random_edge_case_graph(20000, 400000, 128, 5, hub=3, isolated=100)
     n = wl.num_nodes
