@@ -607,6 +607,18 @@ def main():
     e2e_t, e2e_units = combine_ranks(e0.elapsed_time(e1) / 1e3,
                                      units_per_step(n, e, f) * args.e2e_steps, world, pg)
     assert np.isfinite(ho_pm.numpy()).all()
+    # host link rates seen by the copies above (one 1.83 GB edge-list copy in
+    # each direction, alone on the device)
+    link = {}
+    for name, dst_t, src_t in (("h2d_gbs", other_io["edge"], hp_edge), ("d2h_gbs", hp_edge, other_io["edge"])):
+        c0 = torch.cuda.Event(enable_timing=True)
+        c1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        c0.record(stream)
+        dst_t.copy_(src_t, non_blocking=True)
+        c1.record(stream)
+        torch.cuda.synchronize()
+        link[name] = round(hp_edge.numel() * hp_edge.element_size() / (c0.elapsed_time(c1) * 1e-3) / 1e9, 1)
 
     if rank != 0:
         if pg:
@@ -651,7 +663,7 @@ def main():
         "kernels": kernels,
         "gpu_launches": launches_per_step(n, e) * args.steps,
         "e2e": {"value": e2e_units / e2e_t, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "steps": args.e2e_steps},
+                "d2h_bytes_per_step": d2h, "steps": args.e2e_steps, **link},
         "clocks": clocks.summary(),
     }
     line["kernels_cold_l2_ms"] = cold_l2_ms({
