@@ -649,7 +649,7 @@ def main():
                        "pool_mean": "pool_kernel", "pool_max": "pool_kernel"}[dom],
             "call": dom, "bound": "hbm", "achieved": kernels[dom]["gbs"], "peak": hbm_peak,
             "unit": "GB/s", "frac": round(kernels[dom]["gbs"] / hbm_peak, 4), "traffic": traffic,
-            "peak_source": peak_src}
+            "peak_source": peak_src, "frac_of_nominal_8tbs": round(kernels[dom]["gbs"] / 8000.0, 4)}
     value = units_all / t_max
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
