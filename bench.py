@@ -39,7 +39,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "aggregated edge-features/sec (E*F/s) and achieved HBM GB/s vs peak, 1 GB300"
 UNIT = "edge-features/s"
-WORKLOAD = "c5-dcsbm-232965n-114.6Me-41blocks-F128-bf16: csr+gcn_norm+gcn+edge_softmax(8x16)+pool(mean,max)"
+WORKLOAD = "dcsbm-232965n-114.6Me-41blocks-F128-bf16: csr+gcn_norm+gcn+edge_softmax(8x16)+pool(mean,max)"
 
 
 # ---------------------------------------------------------------------------
@@ -345,7 +345,7 @@ def next_rows(L, wl, bufs, stream, hbm_peak):
                             "frac": round(abytes / (ms * 1e-3) / 1e9 / hbm_peak, 4),
                             "algorithmic_bytes": abytes}
 
-    mol = gg.make_c4()
+    mol = gg.make_molecules_1024()
     sizes = np.asarray(mol.graph_sizes, np.int64)
     offs = np.concatenate([[0], np.cumsum(sizes)[:-1]])
     src_graph = mol.batch[mol.edge_index[0]]
@@ -388,7 +388,7 @@ def run_reference(args, rank, world):
     if rank != 0:
         return
     from paper_2101_11552_gb300 import graphgen as gg
-    wl = gg.make_c5(num_pairs=args.pairs)
+    wl = gg.make_dcsbm_232965(num_pairs=args.pairs)
     total_steps = args.steps + args.warmup
     budget = min(150.0, 0.35 * total_steps)
     import oracle
@@ -435,7 +435,7 @@ def main():
     tfg_build.build_library()
     L = tfg.lib()
 
-    wl = gg.make_c5(num_pairs=args.pairs)
+    wl = gg.make_dcsbm_232965(num_pairs=args.pairs)
     n, e, f, heads, ch, g = (wl.num_nodes, wl.num_edges, wl.num_features, wl.heads, wl.channels,
                              wl.num_graphs)
     dev = torch.device("cuda", local)

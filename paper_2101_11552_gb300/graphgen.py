@@ -16,8 +16,11 @@ Pubmed-sized citation graphs, a large citation graph, mini-batched molecule
 graphs and a large dense-community graph, Section 4).  None of those datasets
 is available, so each is replaced by a random graph of the same shape.
 
-Seeds: the graph of workload ``c`` uses ``numpy.random.default_rng(1000 + c)``,
-its features ``default_rng(1100 + c)``.
+Seeds (``numpy.random.default_rng``), graph / features: Erdos-Renyi 2,708
+nodes 1001 / 1101; Barabasi-Albert 19,717 nodes 1002 / 1102; Barabasi-Albert
+169,343 nodes with attention vectors 1003 / 1103; 1,024 molecule graphs
+1004 / 1104; dense-community 232,965 nodes 1005 / 1105 (attention vectors
+1205).
 """
 from __future__ import annotations
 
@@ -29,17 +32,9 @@ import numpy as np
 __all__ = [
     "Workload", "er_pairs", "ba_pairs", "symmetrise", "with_self_loops",
     "batch_graphs", "dcsbm_pairs", "bf16_bits_rne", "bf16_bits_to_f32",
-    "make_c1", "make_c2", "make_c3", "make_c4", "make_c5", "make_workload",
-    "random_edge_case_graph", "CONFIG_NAMES",
+    "make_er_2708", "make_ba_19717", "make_gat_169343", "make_molecules_1024", "make_dcsbm_232965", "make_workload",
+    "random_edge_case_graph", "WORKLOADS",
 ]
-
-CONFIG_NAMES = {
-    1: "c1-er-gcn-2708",
-    2: "c2-ba-19717-sum-mean-max",
-    3: "c3-gat-edge-softmax-169343",
-    4: "c4-batched-1024-graphs-pool",
-    5: "c5-dcsbm-232965-bf16-gcn",
-}
 
 
 @dataclasses.dataclass
@@ -291,25 +286,25 @@ def dcsbm_pairs(n: int, blocks: int, m: int, rng: np.random.Generator,
 # --------------------------------------------------------------------------
 # The five workloads
 # --------------------------------------------------------------------------
-def make_c1() -> Workload:
+def make_er_2708() -> Workload:
     """GCN on G(2708, 5278) symmetrised + 2708 explicit self-loops, F=64 fp32."""
     n = 2708
     rng = np.random.default_rng(1001)
     ei = with_self_loops(symmetrise(er_pairs(n, 5278, rng)), n)
     x = np.random.default_rng(1101).standard_normal((n, 64), dtype=np.float32)
-    return Workload(CONFIG_NAMES[1], n, ei, x, add_self_loops=0)
+    return Workload("er-gcn-2708", n, ei, x, add_self_loops=0)
 
 
-def make_c2() -> Workload:
+def make_ba_19717() -> Workload:
     """BA(19717, m=2) symmetrised + self-loops, F=256 fp32, unweighted reducers."""
     n = 19717
     rng = np.random.default_rng(1002)
     ei = with_self_loops(symmetrise(ba_pairs(n, 2, rng)), n)
     x = np.random.default_rng(1102).standard_normal((n, 256), dtype=np.float32)
-    return Workload(CONFIG_NAMES[2], n, ei, x)
+    return Workload("ba-19717-sum-mean-max", n, ei, x)
 
 
-def make_c3() -> Workload:
+def make_gat_169343() -> Workload:
     """BA(169343, m=7), subsampled to 1,166,243 edges, each oriented by a coin.
 
     No self-loops.  8 heads x 16 channels fp32, a_src/a_dst ~ N(0, 1), slope 0.2.
@@ -327,11 +322,11 @@ def make_c3() -> Workload:
     x = frng.standard_normal((n, 128), dtype=np.float32)
     a_src = frng.standard_normal(128, dtype=np.float32)
     a_dst = frng.standard_normal(128, dtype=np.float32)
-    return Workload(CONFIG_NAMES[3], n, ei, x, heads=8, channels=16,
+    return Workload("gat-edge-softmax-169343", n, ei, x, heads=8, channels=16,
                     a_src=a_src, a_dst=a_dst, negative_slope=0.2)
 
 
-def make_c4() -> Workload:
+def make_molecules_1024() -> Workload:
     """1,024 graphs of U{20..200} nodes, each G(n_g, 2 n_g) symmetrised + self-loops.
 
     Graphs are combined by the reindexing trick; batch is the sorted graph id.
@@ -346,11 +341,11 @@ def make_c4() -> Workload:
     ei, batch, _ = batch_graphs(parts, [int(s) for s in sizes])
     n = int(sizes.sum())
     x = np.random.default_rng(1104).standard_normal((n, 128), dtype=np.float32)
-    return Workload(CONFIG_NAMES[4], n, ei, x, batch=batch, num_graphs=g,
+    return Workload("batched-1024-graphs-pool", n, ei, x, batch=batch, num_graphs=g,
                     graph_sizes=sizes.astype(np.int64))
 
 
-def make_c5(num_pairs: int = 57_300_000, n: int = 232_965) -> Workload:
+def make_dcsbm_232965(num_pairs: int = 57_300_000, n: int = 232_965) -> Workload:
     """Degree-corrected SBM: 41 blocks, ~114.6M directed edges, bf16 F=128.
 
     GCN with implicit self-loops (fill 1).  ``batch`` is the block id of each
@@ -364,14 +359,23 @@ def make_c5(num_pairs: int = 57_300_000, n: int = 232_965) -> Workload:
     frng = np.random.default_rng(1205)
     a_src = frng.standard_normal(128, dtype=np.float32)
     a_dst = frng.standard_normal(128, dtype=np.float32)
-    return Workload(CONFIG_NAMES[5], n, ei, x, x_bf16=bf16_bits_rne(x),
+    return Workload("dcsbm-232965-bf16-gcn", n, ei, x, x_bf16=bf16_bits_rne(x),
                     add_self_loops=1, self_loop_fill=1.0,
                     heads=8, channels=16, a_src=a_src, a_dst=a_dst,
                     batch=block_of, num_graphs=41, graph_sizes=sizes)
 
 
-def make_workload(cfg: int, **kw) -> Workload:
-    return {1: make_c1, 2: make_c2, 3: make_c3, 4: make_c4, 5: make_c5}[cfg](**kw)
+WORKLOADS = {
+    "er-gcn-2708": make_er_2708,
+    "ba-19717-sum-mean-max": make_ba_19717,
+    "gat-edge-softmax-169343": make_gat_169343,
+    "batched-1024-graphs-pool": make_molecules_1024,
+    "dcsbm-232965-bf16-gcn": make_dcsbm_232965,
+}
+
+
+def make_workload(name: str, **kw) -> Workload:
+    return WORKLOADS[name](**kw)
 
 
 def random_edge_case_graph(n: int, e: int, f: int, seed: int, *, hub: int = -1,

@@ -20,12 +20,12 @@ pytestmark = [pytest.mark.gpu, pytest.mark.slow]
 
 
 @pytest.fixture(scope="module")
-def c5():
+def dcsbm():
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     from paper_2101_11552_gb300 import build
     build.build_library()
-    wl = gg.make_c5()
+    wl = gg.make_dcsbm_232965()
     ocsr = oracle.build_csr(wl.edge_index, wl.num_nodes)
     ei = dev(wl.edge_index)
     csr = tfg.tfg_build_csr(ei, wl.num_nodes)
@@ -40,14 +40,14 @@ def c5():
     return wl, ocsr, csr, rows
 
 
-def test_c5_csr_bit_exact(c5):
-    wl, ocsr, csr, _ = c5
+def test_dcsbm_csr_bit_exact(dcsbm):
+    wl, ocsr, csr, _ = dcsbm
     for name, g, w in zip(("rowptr", "col", "perm", "in_degree"), csr[:4], ocsr):
         assert np.array_equal(g.cpu().numpy(), w), name
 
 
-def test_c5_gcn_bf16_sampled_rows(c5):
-    wl, ocsr, csr, rows = c5
+def test_dcsbm_gcn_bf16_sampled_rows(dcsbm):
+    wl, ocsr, csr, rows = dcsbm
     n = wl.num_nodes
     dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 1, 1.0, want_w_csr=False)
     ref_norm = oracle.gcn_norm(wl.edge_index, n, None, 1, 1.0)
@@ -58,13 +58,13 @@ def test_c5_gcn_bf16_sampled_rows(c5):
     w_norm = ref_norm["w_norm"]
     ref, scale = oracle.aggregate_rows(ocsr, n, wl.x_bf16, "sum", rows, w=w_norm,
                                        self_w=ref_norm["self_w"])
-    assert_scaled_close(got, ref, scale, TOL_BF16, "c5 gcn bf16")
+    assert_scaled_close(got, ref, scale, TOL_BF16, "dcsbm gcn bf16")
     # the bf16 bound is loose by design; the fp32 accumulation is far tighter
     assert max_scaled_error(got, ref, scale) < 1e-5
 
 
-def test_c5_edge_softmax_sampled_rows(c5):
-    wl, ocsr, csr, rows = c5
+def test_dcsbm_edge_softmax_sampled_rows(dcsbm):
+    wl, ocsr, csr, rows = dcsbm
     n = wl.num_nodes
     x = dev(wl.x_bf16.view(np.int16)).view(torch.bfloat16)
     out, alpha = tfg.tfg_edge_softmax_aggregate(csr.rowptr, csr.col, x, wl.heads,
@@ -74,44 +74,44 @@ def test_c5_edge_softmax_sampled_rows(c5):
     ref, ref_alpha, scale = oracle.edge_softmax_rows(ocsr, n, wl.x_bf16, wl.heads, wl.channels,
                                                      wl.a_src, wl.a_dst, wl.negative_slope, sub)
     got = out[dev(sub)].cpu().numpy()
-    assert_scaled_close(got, ref, scale, TOL_BF16, "c5 softmax")
+    assert_scaled_close(got, ref, scale, TOL_BF16, "dcsbm softmax")
     assert max_scaled_error(got, ref, scale) < 1e-5
     rp = ocsr[0]
     got_alpha = np.concatenate([alpha[int(rp[r]):int(rp[r + 1])].cpu().numpy() for r in sub])
-    assert_scaled_close(got_alpha, ref_alpha, alpha_scale(ref_alpha), TOL_F32, "c5 alpha")
+    assert_scaled_close(got_alpha, ref_alpha, alpha_scale(ref_alpha), TOL_F32, "dcsbm alpha")
 
 
-def test_c5_max_and_mean_sampled_rows(c5):
-    wl, ocsr, csr, rows = c5
+def test_dcsbm_max_and_mean_sampled_rows(dcsbm):
+    wl, ocsr, csr, rows = dcsbm
     n = wl.num_nodes
     x = dev(wl.x_bf16.view(np.int16)).view(torch.bfloat16)
     for reduce, fn in (("max", tfg.tfg_aggregate_max), ("mean", tfg.tfg_aggregate_mean)):
         got = fn(csr.rowptr, csr.col, x)[dev(rows)].cpu().numpy()
         ref, scale = oracle.aggregate_rows(ocsr, n, wl.x_bf16, reduce, rows)
         if reduce == "max":
-            assert_exact_f32(got, ref, "c5 max")
+            assert_exact_f32(got, ref, "dcsbm max")
         else:
-            assert_scaled_close(got, ref, scale, TOL_BF16, "c5 mean")
+            assert_scaled_close(got, ref, scale, TOL_BF16, "dcsbm mean")
 
 
-def test_c5_community_pool(c5):
-    wl, _, csr, _ = c5
+def test_dcsbm_community_pool(dcsbm):
+    wl, _, csr, _ = dcsbm
     x = dev(wl.x)
     for reduce in ("sum", "mean", "max"):
         out, status = tfg.tfg_segment_pool(x, dev(wl.batch), wl.num_graphs, reduce)
         tfg.check_status(status)
         ref, scale = oracle.segment_pool(wl.x, wl.batch, wl.num_graphs, reduce)
         if reduce == "max":
-            assert_exact_f32(out.cpu().numpy(), ref, "c5 pool max")
+            assert_exact_f32(out.cpu().numpy(), ref, "dcsbm pool max")
         else:
-            assert_scaled_close(out.cpu().numpy(), ref, scale, TOL_F32, f"c5 pool {reduce}")
+            assert_scaled_close(out.cpu().numpy(), ref, scale, TOL_F32, f"dcsbm pool {reduce}")
 
 
-def test_c5_appnp_sqrt_degree_fixed_point(c5):
+def test_dcsbm_appnp_sqrt_degree_fixed_point(dcsbm):
     """On a symmetric graph with self-loops Ahat sqrt(d) = sqrt(d), so
     x0 = sqrt(d) v^T is a fixed point of every APPNP step; the error scale
     |Ahat|^k |x0| is |x0| itself."""
-    wl, ocsr, csr, _ = c5
+    wl, ocsr, csr, _ = dcsbm
     n = wl.num_nodes
     dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 1, 1.0, want_w_csr=False)
     d = ocsr[3].astype(np.float64) + 1.0
@@ -120,11 +120,11 @@ def test_c5_appnp_sqrt_degree_fixed_point(c5):
     out = tfg.tfg_appnp_propagate(csr.rowptr, csr.col, dinv, dev(x0), 10, 0.1, add_self_loops=1)
     got = out.cpu().numpy()
     assert_scaled_close(got, x0.astype(np.float64), np.abs(x0).astype(np.float64), TOL_F32,
-                        "c5 appnp fixed point")
+                        "dcsbm appnp fixed point")
 
 
-def test_c5_appnp_one_hop_sampled_rows_and_sgc_chain(c5):
-    wl, ocsr, csr, rows = c5
+def test_dcsbm_appnp_one_hop_sampled_rows_and_sgc_chain(dcsbm):
+    wl, ocsr, csr, rows = dcsbm
     n = wl.num_nodes
     dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 1, 1.0, want_w_csr=False)
     x = dev(wl.x_bf16.view(np.int16)).view(torch.bfloat16)
@@ -136,16 +136,16 @@ def test_c5_appnp_one_hop_sampled_rows_and_sgc_chain(c5):
     x0 = oracle.widen(wl.x_bf16)[rows]
     ref = (1 - alpha) * agg + alpha * x0
     sc = (1 - alpha) * scale + alpha * np.abs(x0)
-    assert_scaled_close(out[dev(rows)].cpu().numpy(), ref, sc, TOL_F32, "c5 appnp 1 hop")
+    assert_scaled_close(out[dev(rows)].cpu().numpy(), ref, sc, TOL_F32, "dcsbm appnp 1 hop")
     sgc = tfg.tfg_sgc_propagate(csr.rowptr, csr.col, dinv, x, 2, add_self_loops=1)
     h = tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, x, None, 1, 1.0)
     h = tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, h, None, 1, 1.0)
     assert torch.equal(sgc, h)
 
 
-def test_c5_dot_softmax_sampled_rows(c5):
+def test_dcsbm_dot_softmax_sampled_rows(dcsbm):
     """Transformer-style attention at full size: q, k, v bf16 [N, 8 x 16]."""
-    wl, ocsr, csr, rows = c5
+    wl, ocsr, csr, rows = dcsbm
     n = wl.num_nodes
     rng = np.random.default_rng(1305)
     bits = [gg.bf16_bits_rne(rng.standard_normal((n, 128), dtype=np.float32)) for _ in range(3)]
@@ -155,7 +155,7 @@ def test_c5_dot_softmax_sampled_rows(c5):
     sub = rows[:400]
     ref, ref_alpha, scale = oracle.dot_softmax_rows(ocsr, n, *bits, 8, 16, 0.25, sub)
     got = out[dev(sub)].cpu().numpy()
-    assert_scaled_close(got, ref, scale, TOL_F32, "c5 dot softmax")
+    assert_scaled_close(got, ref, scale, TOL_F32, "dcsbm dot softmax")
     rp = ocsr[0]
     got_alpha = np.concatenate([alpha[int(rp[r]):int(rp[r + 1])].cpu().numpy() for r in sub])
-    assert_scaled_close(got_alpha, ref_alpha, alpha_scale(ref_alpha), TOL_F32, "c5 dot alpha")
+    assert_scaled_close(got_alpha, ref_alpha, alpha_scale(ref_alpha), TOL_F32, "dcsbm dot alpha")

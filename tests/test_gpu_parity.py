@@ -241,8 +241,8 @@ def test_segment_pool_bad_batch_sets_status():
 # ---------------------------------------------------------------------------
 # The four smaller workloads at full size
 # ---------------------------------------------------------------------------
-def test_c1_gcn_full():
-    wl = gg.make_c1()
+def test_er2708_gcn_full():
+    wl = gg.make_er_2708()
     n = wl.num_nodes
     csr = gpu_csr(wl.edge_index, n)
     want = oracle.build_csr(wl.edge_index, n)
@@ -250,13 +250,13 @@ def test_c1_gcn_full():
     dinv, w_csr = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0)
     got = np_(tfg.tfg_aggregate_sum(csr.rowptr, csr.col, dev(wl.x), w_csr))
     ref, scale = oracle.gcn_aggregate(wl.edge_index, n, wl.x, None, 0)
-    assert_scaled_close(got, ref, scale, TOL_F32, "c1")
+    assert_scaled_close(got, ref, scale, TOL_F32, "er2708")
     got2 = np_(tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, dev(wl.x)))
-    assert_scaled_close(got2, ref, scale, TOL_F32, "c1 on the fly")
+    assert_scaled_close(got2, ref, scale, TOL_F32, "er2708 on the fly")
 
 
-def test_c2_sum_mean_max_full():
-    wl = gg.make_c2()
+def test_ba19717_sum_mean_max_full():
+    wl = gg.make_ba_19717()
     n = wl.num_nodes
     csr = gpu_csr(wl.edge_index, n)
     x = dev(wl.x)
@@ -265,13 +265,13 @@ def test_c2_sum_mean_max_full():
         got = np_(fn(csr.rowptr, csr.col, x))
         ref, scale = oracle.aggregate(wl.edge_index, n, wl.x, reduce)
         if reduce == "max":
-            assert_exact_f32(got, ref, "c2 max")
+            assert_exact_f32(got, ref, "ba19717 max")
         else:
-            assert_scaled_close(got, ref, scale, TOL_F32, f"c2 {reduce}")
+            assert_scaled_close(got, ref, scale, TOL_F32, f"ba19717 {reduce}")
 
 
-def test_c3_edge_softmax_full():
-    wl = gg.make_c3()
+def test_gat169343_edge_softmax_full():
+    wl = gg.make_gat_169343()
     n = wl.num_nodes
     csr = gpu_csr(wl.edge_index, n)
     out, alpha = tfg.tfg_edge_softmax_aggregate(csr.rowptr, csr.col, dev(wl.x), wl.heads,
@@ -279,21 +279,21 @@ def test_c3_edge_softmax_full():
                                                 wl.negative_slope, want_alpha=True)
     ref, ref_alpha, scale = oracle.edge_softmax(wl.edge_index, n, wl.x, wl.heads, wl.channels,
                                                 wl.a_src, wl.a_dst, wl.negative_slope)
-    assert_scaled_close(np_(out), ref, scale, TOL_F32, "c3 out")
+    assert_scaled_close(np_(out), ref, scale, TOL_F32, "gat169343 out")
     perm = np_(csr.perm)
-    assert_scaled_close(np_(alpha), ref_alpha[perm], alpha_scale(ref_alpha[perm]), TOL_F32, "c3 alpha")
+    assert_scaled_close(np_(alpha), ref_alpha[perm], alpha_scale(ref_alpha[perm]), TOL_F32, "gat169343 alpha")
     deg = np.bincount(wl.edge_index[1], minlength=n)
     assert np.all(np_(out)[deg == 0] == 0.0)
 
 
-def test_c4_batched_gcn_then_pool_full():
-    wl = gg.make_c4()
+def test_molecules_batched_gcn_then_pool_full():
+    wl = gg.make_molecules_1024()
     n = wl.num_nodes
     csr = gpu_csr(wl.edge_index, n)
     dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
     h = tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, dev(wl.x))
     ref_h, scale = oracle.gcn_aggregate(wl.edge_index, n, wl.x, None, 0)
-    assert_scaled_close(np_(h), ref_h, scale, TOL_F32, "c4 gcn")
+    assert_scaled_close(np_(h), ref_h, scale, TOL_F32, "molecules gcn")
     batch = dev(wl.batch)
     h32 = np_(h)                      # the pooling oracle reads what the GPU pooled
     for reduce in ("sum", "mean", "max"):
@@ -301,9 +301,9 @@ def test_c4_batched_gcn_then_pool_full():
         tfg.check_status(status)
         ref, pscale = oracle.segment_pool(h32, wl.batch, wl.num_graphs, reduce)
         if reduce == "max":
-            assert_exact_f32(np_(out), ref, "c4 pool max")
+            assert_exact_f32(np_(out), ref, "molecules pool max")
         else:
-            assert_scaled_close(np_(out), ref, pscale, TOL_F32, f"c4 pool {reduce}")
+            assert_scaled_close(np_(out), ref, pscale, TOL_F32, f"molecules pool {reduce}")
     # batched == per graph (Section 2.1.1): graph g's rows only see graph g
     offs = np.concatenate([[0], np.cumsum(wl.graph_sizes)])
     for g in (0, 511, 1023):
@@ -314,25 +314,25 @@ def test_c4_batched_gcn_then_pool_full():
         np.testing.assert_allclose(h32[s0:s1], ref_g, rtol=1e-5, atol=1e-5)
 
 
-def test_c1_appnp_and_sgc_full():
+def test_er2708_appnp_and_sgc_full():
     """APPNP with the settings of its paper (K = 10, alpha = 0.1) and SGC with
     K = 2 on the 2,708-node citation-sized graph (explicit self-loops)."""
-    wl = gg.make_c1()
+    wl = gg.make_er_2708()
     n = wl.num_nodes
     csr = gpu_csr(wl.edge_index, n)
     dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
     got = np_(tfg.tfg_appnp_propagate(csr.rowptr, csr.col, dinv, dev(wl.x), 10, 0.1))
     ref, scale = oracle.appnp(wl.edge_index, n, wl.x, 10, 0.1)
-    assert_scaled_close(got, ref, scale, TOL_F32, "c1 appnp")
+    assert_scaled_close(got, ref, scale, TOL_F32, "er2708 appnp")
     got = np_(tfg.tfg_sgc_propagate(csr.rowptr, csr.col, dinv, dev(wl.x), 2))
     ref, scale = oracle.sgc(wl.edge_index, n, wl.x, 2)
-    assert_scaled_close(got, ref, scale, TOL_F32, "c1 sgc")
+    assert_scaled_close(got, ref, scale, TOL_F32, "er2708 sgc")
 
 
-def test_c3_dot_softmax_full():
+def test_gat169343_dot_softmax_full():
     """Transformer-style attention on the GAT workload's graph (169,343 nodes,
     1,166,243 edges, 8 heads x 16): q from the features, k and v seeded."""
-    wl = gg.make_c3()
+    wl = gg.make_gat_169343()
     n = wl.num_nodes
     csr = gpu_csr(wl.edge_index, n)
     rng = np.random.default_rng(1303)
@@ -342,15 +342,15 @@ def test_c3_dot_softmax_full():
                                                     wl.heads, wl.channels, want_alpha=True)
     ref, ref_alpha, scale = oracle.dot_softmax(wl.edge_index, n, wl.x, k, v, wl.heads, wl.channels,
                                                float(np.float32(1.0 / np.sqrt(wl.channels))))
-    assert_scaled_close(np_(out), ref, scale, TOL_F32, "c3 dot out")
+    assert_scaled_close(np_(out), ref, scale, TOL_F32, "gat169343 dot out")
     perm = np_(csr.perm)
-    assert_scaled_close(np_(alpha), ref_alpha[perm], alpha_scale(ref_alpha[perm]), TOL_F32, "c3 dot alpha")
+    assert_scaled_close(np_(alpha), ref_alpha[perm], alpha_scale(ref_alpha[perm]), TOL_F32, "gat169343 dot alpha")
 
 
-def test_c4_device_batching_and_meanmax_full():
+def test_molecules_device_batching_and_meanmax_full():
     """The 1,024 molecule graphs batched on the device equal the generator's
     BatchGraph; the Mean-Max readout of the GCN output equals the oracle."""
-    wl = gg.make_c4()
+    wl = gg.make_molecules_1024()
     sizes = np.asarray(wl.graph_sizes, np.int64)
     offs = np.concatenate([[0], np.cumsum(sizes)[:-1]])
     src_graph = wl.batch[wl.edge_index[0]]
@@ -370,8 +370,8 @@ def test_c4_device_batching_and_meanmax_full():
     tfg.check_status(status)
     ref, scale = oracle.segment_pool_meanmax(np_(h), wl.batch, wl.num_graphs)
     f = wl.x.shape[1]
-    assert_scaled_close(np_(out)[:, :f], ref[:, :f], scale[:, :f], TOL_F32, "c4 mean")
-    assert_exact_f32(np_(out)[:, f:], ref[:, f:], "c4 max")
+    assert_scaled_close(np_(out)[:, :f], ref[:, :f], scale[:, :f], TOL_F32, "molecules mean")
+    assert_exact_f32(np_(out)[:, f:], ref[:, f:], "molecules max")
 
 
 def test_deterministic_bitwise():

@@ -5,8 +5,8 @@ import pytest
 from paper_2101_11552_gb300 import graphgen as gg
 
 
-def test_c1_shape():
-    w = gg.make_c1()
+def test_er2708_shape():
+    w = gg.make_er_2708()
     assert (w.num_nodes, w.num_edges, w.num_features) == (2708, 10556 + 2708, 64)
     ei = w.edge_index
     # symmetric: every (i, j) has its (j, i); explicit self-loops at the end
@@ -15,20 +15,20 @@ def test_c1_shape():
     assert np.array_equal(ei[0, 10556:], np.arange(2708)) and np.array_equal(ei[1, 10556:], np.arange(2708))
 
 
-def test_c2_shape():
-    w = gg.make_c2()
+def test_ba19717_shape():
+    w = gg.make_ba_19717()
     assert (w.num_nodes, w.num_edges, w.num_features) == (19717, 78860 + 19717, 256)
 
 
-def test_c3_shape():
-    w = gg.make_c3()
+def test_gat169343_shape():
+    w = gg.make_gat_169343()
     assert (w.num_nodes, w.num_edges, w.heads, w.channels) == (169343, 1166243, 8, 16)
     assert w.num_features == 128
     assert not np.any(w.edge_index[0] == w.edge_index[1])
 
 
-def test_c4_shape_and_batch():
-    w = gg.make_c4()
+def test_molecules_shape_and_batch():
+    w = gg.make_molecules_1024()
     assert w.num_graphs == 1024
     assert 20 <= w.graph_sizes.min() and w.graph_sizes.max() <= 200
     assert w.num_nodes == int(w.graph_sizes.sum())
@@ -40,7 +40,7 @@ def test_c4_shape_and_batch():
 
 
 def test_generators_are_deterministic():
-    a, b = gg.make_c1(), gg.make_c1()
+    a, b = gg.make_er_2708(), gg.make_er_2708()
     assert np.array_equal(a.edge_index, b.edge_index) and np.array_equal(a.x, b.x)
 
 
