@@ -283,6 +283,7 @@ def cold_l2_ms(fns: dict, stream, reps: int = 5) -> dict:
 def next_rows(L, wl, bufs, stream, hbm_peak):
     """The rows built beyond the timed step, each measured on its own (not part
     of the headline value): APPNP K = 10 on the same graph and bf16 features,
+    the backward of the GCN aggregation,
     Transformer-style (dot-product) attention with bf16 q, k, v of the same
     8 x 16 layout, the fused Mean-Max pool on the GCN output, and device
     BatchGraph construction on 1,024 molecule-sized graphs."""
@@ -317,6 +318,30 @@ def next_rows(L, wl, bufs, stream, hbm_peak):
                          "gbs": round(abytes / (ms * 1e-3) / 1e9, 1),
                          "frac": round(abytes / (ms * 1e-3) / 1e9 / hbm_peak, 4),
                          "algorithmic_bytes": abytes}
+
+    # backward of the GCN aggregation: source-grouped CSR (built once per graph,
+    # like the forward CSR) and the gradient with respect to the features
+    e_dev = torch.from_numpy(wl.edge_index).to(dev)
+    csr_src = tfg.tfg_build_csr_by_source(e_dev, n)
+    ws_src = torch.empty(tfg.tfg_build_csr_workspace_size(n, e), dtype=torch.uint8, device=dev)
+    st_src = torch.zeros(1, dtype=torch.int32, device=dev)
+    ms_build = _event_ms(lambda: check(L.tfg_build_csr_by_source(
+        P(e_dev), e, n, P(csr_src.rowptr), P(csr_src.col), P(csr_src.perm), P(csr_src.in_degree),
+        P(ws_src), ws_src.numel(), P(st_src), sp)), stream, 5)
+    del ws_src, e_dev
+    grad_x = torch.empty(n, f, dtype=torch.float32, device=dev)
+    ms = _event_ms(lambda: check(L.tfg_gcn_aggregate_backward(
+        P(csr_src.rowptr), P(csr_src.col), P(bufs["dinv"]), P(bufs["h"]), n, f, 1, 1.0, P(grad_x),
+        sp)), stream, 10)
+    # gathered fp32 gradient rows once + col + rowptr + dinv + grad_x written
+    abytes = 4 * e + 4 * (n + 1) + 4 * n + 4 * n * f + 4 * n * f
+    rows["gcn_backward"] = {"ms": round(ms, 4), "csr_by_source_ms": round(ms_build, 4),
+                            "edge_features_per_s": (e + n) * f / (ms * 1e-3),
+                            "gbs": round(abytes / (ms * 1e-3) / 1e9, 1),
+                            "frac": round(abytes / (ms * 1e-3) / 1e9 / hbm_peak, 4),
+                            "algorithmic_bytes": abytes,
+                            "note": "grad_out = the GCN output (fp32); CSR by source built once"}
+    del csr_src, grad_x
 
     heads, ch = wl.heads, wl.channels
     gen = torch.Generator(device=dev)

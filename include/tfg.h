@@ -96,6 +96,14 @@ int tfg_build_csr(const int64_t *edge_index, int64_t num_edges, int64_t num_node
                   int32_t *rowptr, int32_t *col, int32_t *perm, int32_t *in_degree,
                   void *workspace, size_t workspace_bytes, int32_t *status,
                   tfg_stream_t stream);
+/* The same grouping by SOURCE (the CSR of the transposed graph, used by the
+ * backward calls): rows are sources, col_src holds the targets, perm_src the
+ * original edge ids (stable: original order within a row), out_degree the
+ * number of edges leaving each node.  Same workspace size and errors. */
+int tfg_build_csr_by_source(const int64_t *edge_index, int64_t num_edges, int64_t num_nodes,
+                            int32_t *rowptr_src, int32_t *col_src, int32_t *perm_src,
+                            int32_t *out_degree, void *workspace, size_t workspace_bytes,
+                            int32_t *status, tfg_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * GCN symmetric normalisation of A + I (the propagation rule of the GCN
@@ -164,6 +172,55 @@ int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float
                           const float *w_csr, const void *x, int x_dtype, int64_t num_nodes,
                           int64_t num_features, int add_self_loops, float self_loop_fill,
                           float *out, tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Backward of the aggregation (the gradient with respect to x; the paper
+ * keeps every aggregation differentiable, Sections 2.1.2 and 3).  For
+ *   out[t] = sum over edges e = (s -> t) of w_e x[s]
+ * the gradient is the same sum over the transposed graph:
+ *   grad_x[s] = sum over edges e = (s -> t) of w_e grad_out[t].
+ * All backward calls take the CSR grouped by SOURCE (tfg_build_csr_by_source):
+ * rowptr_src indexes sources, col_src holds targets, perm_src the original
+ * edge ids.
+ *
+ * tfg_aggregate_backward: reduce TFG_SUM (w_e = edge_weight[e], or 1) or
+ *   TFG_MEAN (w_e / in_degree[t], in_degree the forward CSR's, as written by
+ *   tfg_build_csr).  edge_weight is in ORIGINAL edge order, or NULL.  A
+ *   workspace of tfg_aggregate_backward_workspace_size() bytes holds the
+ *   weights in source-grouped order when there are any (NULL allowed for an
+ *   unweighted sum).
+ * tfg_gcn_aggregate_backward: the backward of tfg_gcn_aggregate_sum with
+ *   weights formed from dinv.  The symmetric normalisation is its own
+ *   transpose, so this is the GCN propagation on the source-grouped CSR with
+ *   the forward's dinv (add_self_loops / self_loop_fill as in the forward).
+ * tfg_aggregate_max_argmax: tfg_aggregate_max plus, per (t, f), the ORIGINAL
+ *   id of the first edge (in original order) whose product w_k * x attains the
+ *   maximum, -1 for a row without edges; perm is the forward CSR's.
+ *   argmax int32 [num_nodes, num_features].
+ * tfg_aggregate_max_backward: grad_x[s, f] = sum over edges e = (s -> t)
+ *   with argmax[t, f] == e of grad_out[t, f] (the weight of a weighted max is
+ *   not applied: scale grad_out beforehand if the forward used w_csr).
+ * grad_out, grad_x: fp32 [num_nodes, num_features]; grad_x is written.
+ * Every sum runs in a fixed order: results are bitwise reproducible.
+ * ---------------------------------------------------------------------- */
+int tfg_aggregate_backward_workspace_size(int reduce, int64_t num_edges, size_t *bytes);
+int tfg_aggregate_backward(int reduce, const int32_t *rowptr_src, const int32_t *col_src,
+                           const int32_t *perm_src, const float *edge_weight,
+                           const int32_t *in_degree, const float *grad_out, int64_t num_nodes,
+                           int64_t num_edges, int64_t num_features, float *grad_x,
+                           void *workspace, size_t workspace_bytes, tfg_stream_t stream);
+int tfg_gcn_aggregate_backward(const int32_t *rowptr_src, const int32_t *col_src,
+                               const float *dinv, const float *grad_out, int64_t num_nodes,
+                               int64_t num_features, int add_self_loops, float self_loop_fill,
+                               float *grad_x, tfg_stream_t stream);
+int tfg_aggregate_max_argmax(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
+                             const float *w_csr, const void *x, int x_dtype, int64_t num_nodes,
+                             int64_t num_features, float *out, int32_t *argmax,
+                             tfg_stream_t stream);
+int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src,
+                               const int32_t *perm_src, const int32_t *argmax,
+                               const float *grad_out, int64_t num_nodes, int64_t num_features,
+                               float *grad_x, tfg_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * Multi-hop propagation: APPNP and SGC, node-level models the paper lists

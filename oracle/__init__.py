@@ -74,6 +74,9 @@ def _load(plant: Optional[str] = None) -> ctypes.CDLL:
                 "oracle_segment_pool": [I, I64, I64, I64, P, P, P, P],
                 "oracle_appnp": [I64, I64, P, P, P, P, I64, I64, D, P, P],
                 "oracle_dot_softmax": [I64, I64, P, P, P, P, I, I, D, P, P, P],
+                "oracle_aggregate_backward": [I, I64, I64, P, P, P, P, I64, P, P],
+                "oracle_max_argmax": [I64, I64, P, P, P, I64, P, P],
+                "oracle_max_backward": [I64, I64, P, P, P, I64, P, P],
                 "oracle_dot_softmax_rows": [I64, P, P, P, P, P, I, I, D, P, I64, P, P, P],
             }
             for fn, args in sigs.items():
@@ -196,6 +199,56 @@ class _Oracle:
             self._p(a_s), self._p(a_d), float(slope), self._p(rows), len(rows), self._p(out),
             self._p(alpha), self._p(ab)))
         return out[:len(rows)], alpha[:total], ab[:len(rows)]
+
+    # -- backward of the aggregation ------------------------------------
+    def aggregate_backward(self, edge_index, n, grad_out, reduce, w=None, self_w=None):
+        """dL/dx of aggregate(edge_index, n, x, reduce, w, self_w) for a given
+        dL/dout (sum or mean; GCN = sum with w_norm and self_w).  Returns
+        (grad_x, error scale), both [N, F]."""
+        ei = np.ascontiguousarray(edge_index, dtype=np.int64)
+        e = ei.shape[1]
+        g = widen(grad_out)
+        f = g.shape[1]
+        w = None if w is None else np.ascontiguousarray(w, np.float64)
+        sw = None if self_w is None else np.ascontiguousarray(self_w, np.float64)
+        out = np.zeros((max(n, 1), f))
+        ab = np.zeros((max(n, 1), f))
+        self._check(self.lib.oracle_aggregate_backward(REDUCE[reduce], n, e, self._p(ei), self._p(w),
+                                                       self._p(sw), self._p(g), f, self._p(out),
+                                                       self._p(ab)))
+        return out[:n], ab[:n]
+
+    def gcn_aggregate_backward(self, edge_index, n, grad_out, edge_weight=None, add_self_loops=0,
+                               fill=1.0):
+        nrm = self.gcn_norm(edge_index, n, edge_weight, add_self_loops, fill)
+        return self.aggregate_backward(edge_index, n, grad_out, "sum", w=nrm["w_norm"],
+                                       self_w=nrm["self_w"])
+
+    def max_argmax(self, edge_index, n, x, w=None):
+        """(out [N, F], argmax int32 [N, F]): first edge (original order) with
+        the largest fp32 product per (target, feature), -1 without edges."""
+        ei = np.ascontiguousarray(edge_index, dtype=np.int64)
+        e = ei.shape[1]
+        x = widen(x)
+        f = x.shape[1]
+        w32 = None if w is None else np.ascontiguousarray(w, np.float32)
+        out = np.zeros((max(n, 1), f))
+        arg = np.zeros((max(n, 1), f), np.int32)
+        self._check(self.lib.oracle_max_argmax(n, e, self._p(ei), self._p(w32), self._p(x), f,
+                                               self._p(out), self._p(arg)))
+        return out[:n], arg[:n]
+
+    def max_backward(self, edge_index, n, argmax, grad_out):
+        ei = np.ascontiguousarray(edge_index, dtype=np.int64)
+        e = ei.shape[1]
+        g = widen(grad_out)
+        f = g.shape[1]
+        arg = np.ascontiguousarray(argmax, np.int32)
+        out = np.zeros((max(n, 1), f))
+        ab = np.zeros((max(n, 1), f))
+        self._check(self.lib.oracle_max_backward(n, e, self._p(ei), self._p(arg), self._p(g), f,
+                                                 self._p(out), self._p(ab)))
+        return out[:n], ab[:n]
 
     # -- dot-product (Transformer-style) attention ----------------------
     def dot_softmax(self, edge_index, n, q, k, v, heads, channels, scale=None):
@@ -341,6 +394,10 @@ edge_softmax_rows = default.edge_softmax_rows
 segment_pool = default.segment_pool
 appnp = default.appnp
 dot_softmax = default.dot_softmax
+aggregate_backward = default.aggregate_backward
+gcn_aggregate_backward = default.gcn_aggregate_backward
+max_argmax = default.max_argmax
+max_backward = default.max_backward
 dot_softmax_rows = default.dot_softmax_rows
 sgc = default.sgc
 

@@ -579,3 +579,102 @@ int oracle_dot_softmax_rows(int64_t n, const int32_t *rowptr, const int32_t *col
     }
     return OK;
 }
+
+/* ---------------------------------------------------------------------------
+ * Backward of the aggregation: the gradient with respect to x of the
+ * aggregation out[t] = sum over edges e = (s -> t) of w_e x[s] (sum), the
+ * same divided by the number of edges into t (mean), or with the GCN weights
+ * w_e = w_norm[e] plus the implicit self-loop term self_w[t] x[t].  With
+ * grad_out = dL/dout, dL/dx[s] = sum over edges e = (s -> t) of
+ * w_e grad_out[t] (/ count[t] for the mean) (+ self_w[s] grad_out[s]).
+ * Loops over the edges in original order, fp64.  absout = same with |terms|.
+ * ------------------------------------------------------------------------- */
+int oracle_aggregate_backward(int reduce, int64_t n, int64_t e, const int64_t *edge_index,
+                              const double *w, const double *self_w, const double *grad_out,
+                              int64_t f, double *grad_x, double *absout)
+{
+    if (n < 0 || e < 0 || f < 0) return E_ARG;
+    if (reduce != R_SUM && reduce != R_MEAN) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+    for (int64_t i = 0; i < e; ++i)
+        if (src[i] < 0 || src[i] >= n || dst[i] < 0 || dst[i] >= n) return E_RANGE;
+    int64_t *count = (int64_t *)calloc((size_t)(n > 0 ? n : 1), sizeof(int64_t));
+    if (!count) return E_ARG;
+    for (int64_t i = 0; i < e; ++i) count[dst[i]] += 1;
+    for (int64_t k = 0; k < n * f; ++k) { grad_x[k] = 0.0; absout[k] = 0.0; }
+    for (int64_t i = 0; i < e; ++i) {
+#ifdef ORACLE_PLANT_BACKWARD_NO_TRANSPOSE
+        int64_t s = dst[i], t = src[i];            /* planted: gradient sent along the edge */
+#else
+        int64_t s = src[i], t = dst[i];
+#endif
+        double we = w ? w[i] : 1.0;
+        if (reduce == R_MEAN) we /= (double)count[dst[i]];
+        for (int64_t c = 0; c < f; ++c) {
+            double m = we * grad_out[t * f + c];
+            grad_x[s * f + c] += m;
+            absout[s * f + c] += fabs(m);
+        }
+    }
+    if (self_w && reduce == R_SUM)
+        for (int64_t s = 0; s < n; ++s)
+            for (int64_t c = 0; c < f; ++c) {
+                double m = self_w[s] * grad_out[s * f + c];
+                grad_x[s * f + c] += m;
+                absout[s * f + c] += fabs(m);
+            }
+    free(count);
+    return OK;
+}
+
+/* Max with argmax: per (t, c) the original id of the FIRST edge into t (in
+ * original order) whose product w_e x[s, c] is the largest, -1 without
+ * edges.  The product is compared after rounding to fp32 (the precision in
+ * which the CUDA kernel forms and compares it), so both sides make the same
+ * choice; out holds the exact fp64 value of the chosen product. */
+int oracle_max_argmax(int64_t n, int64_t e, const int64_t *edge_index, const float *w,
+                      const double *x, int64_t f, double *out, int32_t *argmax)
+{
+    if (n < 0 || e < 0 || f < 0) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+    for (int64_t i = 0; i < e; ++i)
+        if (src[i] < 0 || src[i] >= n || dst[i] < 0 || dst[i] >= n) return E_RANGE;
+    float *best = (float *)malloc(sizeof(float) * (size_t)(n * f > 0 ? n * f : 1));
+    if (!best) return E_ARG;
+    for (int64_t k = 0; k < n * f; ++k) { out[k] = 0.0; argmax[k] = -1; }
+    for (int64_t i = 0; i < e; ++i) {
+        int64_t s = src[i], t = dst[i];
+        double we = w ? (double)w[i] : 1.0;
+        for (int64_t c = 0; c < f; ++c) {
+            double m = we * x[s * f + c];
+            float m32 = (float)m;
+            if (argmax[t * f + c] < 0 || m32 > best[t * f + c]) {
+                best[t * f + c] = m32;
+                out[t * f + c] = m;
+                argmax[t * f + c] = (int32_t)i;
+            }
+        }
+    }
+    free(best);
+    return OK;
+}
+
+/* grad_x[s, c] = sum over edges e = (s -> t), in original order, with
+ * argmax[t, c] == e of grad_out[t, c]. */
+int oracle_max_backward(int64_t n, int64_t e, const int64_t *edge_index, const int32_t *argmax,
+                        const double *grad_out, int64_t f, double *grad_x, double *absout)
+{
+    if (n < 0 || e < 0 || f < 0) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+    for (int64_t k = 0; k < n * f; ++k) { grad_x[k] = 0.0; absout[k] = 0.0; }
+    for (int64_t i = 0; i < e; ++i) {
+        int64_t s = src[i], t = dst[i];
+        if (s < 0 || s >= n || t < 0 || t >= n) return E_RANGE;
+        for (int64_t c = 0; c < f; ++c)
+            if (argmax[t * f + c] == (int32_t)i) {
+                grad_x[s * f + c] += grad_out[t * f + c];
+                absout[s * f + c] += fabs(grad_out[t * f + c]);
+            }
+    }
+    return OK;
+}

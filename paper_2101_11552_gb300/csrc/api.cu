@@ -146,11 +146,11 @@ int tfg_build_csr_workspace_size(int64_t num_nodes, int64_t num_edges, size_t *b
     return ok();
 }
 
-int tfg_build_csr(const int64_t *edge_index, int64_t num_edges, int64_t num_nodes,
-                  int32_t *rowptr, int32_t *col, int32_t *perm, int32_t *in_degree,
-                  void *workspace, size_t workspace_bytes, int32_t *status,
-                  tfg_stream_t stream) {
-    const char *fn = "tfg_build_csr";
+namespace {
+int build_csr_common(const char *fn, bool by_source, const int64_t *edge_index, int64_t num_edges,
+                     int64_t num_nodes, int32_t *rowptr, int32_t *col, int32_t *perm,
+                     int32_t *in_degree, void *workspace, size_t workspace_bytes, int32_t *status,
+                     tfg_stream_t stream) {
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     TFG_NEED(edge_index, num_edges > 0, fn, "edge_index");
     TFG_NEED(rowptr, true, fn, "rowptr");
@@ -168,8 +168,26 @@ int tfg_build_csr(const int64_t *edge_index, int64_t num_edges, int64_t num_node
     }
     return cuda_result(tfg::launch_build_csr(edge_index, num_edges, num_nodes, rowptr, col, perm,
                                              in_degree, workspace, status,
-                                             reinterpret_cast<cudaStream_t>(stream)),
+                                             reinterpret_cast<cudaStream_t>(stream), by_source),
                        fn);
+}
+}  // namespace
+
+int tfg_build_csr(const int64_t *edge_index, int64_t num_edges, int64_t num_nodes,
+                  int32_t *rowptr, int32_t *col, int32_t *perm, int32_t *in_degree,
+                  void *workspace, size_t workspace_bytes, int32_t *status,
+                  tfg_stream_t stream) {
+    return build_csr_common("tfg_build_csr", false, edge_index, num_edges, num_nodes, rowptr, col,
+                            perm, in_degree, workspace, workspace_bytes, status, stream);
+}
+
+int tfg_build_csr_by_source(const int64_t *edge_index, int64_t num_edges, int64_t num_nodes,
+                            int32_t *rowptr_src, int32_t *col_src, int32_t *perm_src,
+                            int32_t *out_degree, void *workspace, size_t workspace_bytes,
+                            int32_t *status, tfg_stream_t stream) {
+    return build_csr_common("tfg_build_csr_by_source", true, edge_index, num_edges, num_nodes,
+                            rowptr_src, col_src, perm_src, out_degree, workspace, workspace_bytes,
+                            status, stream);
 }
 
 int tfg_gcn_norm(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
@@ -215,6 +233,91 @@ int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float
                           float *out, tfg_stream_t stream) {
     return aggregate_common("tfg_gcn_aggregate_sum", 3, rowptr, col, w_csr, dinv, x, x_dtype,
                             num_nodes, num_features, add_self_loops, self_loop_fill, out, stream);
+}
+
+int tfg_aggregate_backward_workspace_size(int reduce, int64_t num_edges, size_t *bytes) {
+    const char *fn = "tfg_aggregate_backward_workspace_size";
+    TFG_TRY(check_counts(fn, 1, num_edges));
+    if (reduce != TFG_SUM && reduce != TFG_MEAN)
+        return fail(TFG_ERR_INVALID_ARG, "%s: reduce must be TFG_SUM or TFG_MEAN", fn);
+    TFG_NEED(bytes, true, fn, "bytes");
+    *bytes = tfg::backward_workspace_bytes(reduce, num_edges);
+    return ok();
+}
+
+int tfg_aggregate_backward(int reduce, const int32_t *rowptr_src, const int32_t *col_src,
+                           const int32_t *perm_src, const float *edge_weight,
+                           const int32_t *in_degree, const float *grad_out, int64_t num_nodes,
+                           int64_t num_edges, int64_t num_features, float *grad_x,
+                           void *workspace, size_t workspace_bytes, tfg_stream_t stream) {
+    const char *fn = "tfg_aggregate_backward";
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    TFG_TRY(check_features(fn, num_nodes, num_features));
+    if (reduce != TFG_SUM && reduce != TFG_MEAN)
+        return fail(TFG_ERR_INVALID_ARG, "%s: reduce must be TFG_SUM or TFG_MEAN", fn);
+    TFG_NEED(rowptr_src, true, fn, "rowptr_src");
+    TFG_NEED(col_src, num_edges > 0, fn, "col_src");
+    TFG_NEED(perm_src, num_edges > 0 && (edge_weight != nullptr || reduce == TFG_MEAN), fn,
+             "perm_src");
+    TFG_NEED(in_degree, reduce == TFG_MEAN && num_edges > 0, fn, "in_degree");
+    TFG_NEED(grad_out, num_nodes > 0, fn, "grad_out");
+    TFG_NEED(grad_x, num_nodes > 0, fn, "grad_x");
+    const bool weighted = num_edges > 0 && (edge_weight != nullptr || reduce == TFG_MEAN);
+    const size_t need = weighted ? tfg::backward_workspace_bytes(reduce, num_edges) : 0;
+    if (need > 0 && (workspace == nullptr || workspace_bytes < need))
+        return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
+                    workspace ? workspace_bytes : size_t(0));
+    return cuda_result(tfg::launch_aggregate_backward(reduce, rowptr_src, col_src, perm_src,
+                                                      edge_weight, in_degree, grad_out, num_nodes,
+                                                      num_edges, num_features, grad_x, workspace,
+                                                      reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+int tfg_gcn_aggregate_backward(const int32_t *rowptr_src, const int32_t *col_src,
+                               const float *dinv, const float *grad_out, int64_t num_nodes,
+                               int64_t num_features, int add_self_loops, float self_loop_fill,
+                               float *grad_x, tfg_stream_t stream) {
+    return aggregate_common("tfg_gcn_aggregate_backward", 3, rowptr_src, col_src, nullptr, dinv,
+                            grad_out, TFG_F32, num_nodes, num_features, add_self_loops,
+                            self_loop_fill, grad_x, stream);
+}
+
+int tfg_aggregate_max_argmax(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
+                             const float *w_csr, const void *x, int x_dtype, int64_t num_nodes,
+                             int64_t num_features, float *out, int32_t *argmax,
+                             tfg_stream_t stream) {
+    const char *fn = "tfg_aggregate_max_argmax";
+    TFG_TRY(check_counts(fn, num_nodes, 0));
+    TFG_TRY(check_features(fn, num_nodes, num_features));
+    TFG_TRY(check_dtype(fn, x_dtype));
+    TFG_NEED(rowptr, true, fn, "rowptr");
+    TFG_NEED(perm, col != nullptr, fn, "perm");
+    TFG_NEED(x, num_nodes > 0, fn, "x");
+    TFG_NEED(out, num_nodes > 0, fn, "out");
+    TFG_NEED(argmax, num_nodes > 0, fn, "argmax");
+    return cuda_result(tfg::launch_max_argmax(rowptr, col, perm, w_csr, x, x_dtype, num_nodes,
+                                              num_features, out, argmax,
+                                              reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src,
+                               const int32_t *perm_src, const int32_t *argmax,
+                               const float *grad_out, int64_t num_nodes, int64_t num_features,
+                               float *grad_x, tfg_stream_t stream) {
+    const char *fn = "tfg_aggregate_max_backward";
+    TFG_TRY(check_counts(fn, num_nodes, 0));
+    TFG_TRY(check_features(fn, num_nodes, num_features));
+    TFG_NEED(rowptr_src, true, fn, "rowptr_src");
+    TFG_NEED(perm_src, col_src != nullptr, fn, "perm_src");
+    TFG_NEED(argmax, num_nodes > 0, fn, "argmax");
+    TFG_NEED(grad_out, num_nodes > 0, fn, "grad_out");
+    TFG_NEED(grad_x, num_nodes > 0, fn, "grad_x");
+    return cuda_result(tfg::launch_max_backward(rowptr_src, col_src, perm_src, argmax, grad_out,
+                                                num_nodes, num_features, grad_x,
+                                                reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
 }
 
 int tfg_propagate_workspace_size(int64_t num_nodes, int64_t num_features, int64_t num_hops,

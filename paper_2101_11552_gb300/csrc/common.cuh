@@ -134,7 +134,7 @@ namespace tfg {
 size_t csr_workspace_bytes(int64_t n, int64_t e);
 cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
                              int32_t *col, int32_t *perm, int32_t *in_degree, void *ws,
-                             int32_t *status, cudaStream_t s);
+                             int32_t *status, cudaStream_t s, bool by_source = false);
 cudaError_t launch_gcn_norm(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
                             const float *ew, int64_t n, int add_self, float fill, float *dinv,
                             float *w_csr, cudaStream_t s);
@@ -142,6 +142,19 @@ cudaError_t launch_gcn_norm(const int32_t *rowptr, const int32_t *col, const int
 cudaError_t launch_aggregate(int mode, const int32_t *rowptr, const int32_t *col, const float *w,
                              const float *dinv, const void *x, int x_dtype, int64_t n, int64_t f,
                              int add_self, float fill, float *out, cudaStream_t s);
+size_t backward_workspace_bytes(int mode, int64_t e);
+cudaError_t launch_aggregate_backward(int mode, const int32_t *rowptr_src, const int32_t *col_src,
+                                      const int32_t *perm_src, const float *edge_weight,
+                                      const int32_t *in_degree, const float *grad_out, int64_t n,
+                                      int64_t e, int64_t f, float *grad_x, void *ws,
+                                      cudaStream_t s);
+cudaError_t launch_max_argmax(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
+                              const float *w, const void *x, int x_dtype, int64_t n, int64_t f,
+                              float *out, int32_t *argmax, cudaStream_t s);
+cudaError_t launch_max_backward(const int32_t *rowptr_src, const int32_t *col_src,
+                                const int32_t *perm_src, const int32_t *argmax,
+                                const float *grad_out, int64_t n, int64_t f, float *grad_x,
+                                cudaStream_t s);
 size_t propagate_workspace_bytes(int64_t n, int64_t f, int64_t hops);
 cudaError_t launch_propagate(const int32_t *rowptr, const int32_t *col, const float *w,
                              const float *dinv, const void *x0, int x_dtype, int64_t n, int64_t f,

@@ -416,7 +416,7 @@ size_t csr_workspace_bytes(int64_t n, int64_t e) {
 
 cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
                              int32_t *col, int32_t *perm, int32_t *in_degree, void *ws,
-                             int32_t *status, cudaStream_t s) {
+                             int32_t *status, cudaStream_t s, bool by_source) {
     cudaError_t err = cudaMemsetAsync(status, 0, sizeof(int32_t), s);
     if (err != cudaSuccess) return err;
     const uint32_t *sorted_keys = nullptr;
@@ -438,7 +438,9 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
         w += align256(sizeof(int32_t) * size_t(int64_t(radix) * tiles));
         int32_t *sums = reinterpret_cast<int32_t *>(w);
 
-        const int64_t *src64 = edge_index, *dst64 = edge_index + e;
+        // the key row is row 1 (targets), or row 0 (sources) for the transposed CSR
+        const int64_t *src64 = by_source ? edge_index + e : edge_index;
+        const int64_t *dst64 = by_source ? edge_index : edge_index + e;
         const int smem_max = static_cast<int>(downsweep_smem(1 << kMaxDigitBits));
         err = cudaFuncSetAttribute(radix_downsweep<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
         if (err == cudaSuccess)

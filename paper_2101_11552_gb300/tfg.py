@@ -59,6 +59,12 @@ def lib() -> ctypes.CDLL:
                 "tfg_version": [],
                 "tfg_build_csr_workspace_size": [I64, I64, ctypes.POINTER(SZ)],
                 "tfg_build_csr": [P, I64, I64, P, P, P, P, P, SZ, P, P],
+                "tfg_build_csr_by_source": [P, I64, I64, P, P, P, P, P, SZ, P, P],
+                "tfg_aggregate_backward_workspace_size": [I, I64, ctypes.POINTER(SZ)],
+                "tfg_aggregate_backward": [I, P, P, P, P, P, P, I64, I64, I64, P, P, SZ, P],
+                "tfg_gcn_aggregate_backward": [P, P, P, P, I64, I64, I, F, P, P],
+                "tfg_aggregate_max_argmax": [P, P, P, P, P, I, I64, I64, P, P, P],
+                "tfg_aggregate_max_backward": [P, P, P, P, P, I64, I64, P, P],
                 "tfg_gcn_norm": [P, P, P, P, I64, I64, I, F, P, P, P],
                 "tfg_aggregate_sum": [P, P, P, P, I, I64, I64, P, P],
                 "tfg_aggregate_mean": [P, P, P, P, I, I64, I64, P, P],
@@ -168,6 +174,89 @@ def tfg_build_csr(edge_index: torch.Tensor, num_nodes: int,
                                _ptr(deg), _ptr(workspace), workspace.numel(), _ptr(status),
                                _stream(dev)))
     return CSR(rowptr, col, perm, deg, status)
+
+
+def tfg_build_csr_by_source(edge_index: torch.Tensor, num_nodes: int,
+                            workspace: Optional[torch.Tensor] = None) -> CSR:
+    """Group the edges by SOURCE (the transposed graph's CSR).  Returns the CSR
+    tuple with rowptr over sources, col = targets, perm = original edge ids,
+    in_degree = out-degrees."""
+    _need_cuda("edge_index", edge_index, torch.int64)
+    if edge_index.dim() != 2 or edge_index.shape[0] != 2:
+        raise ValueError("edge_index must have shape [2, E]")
+    dev = edge_index.device
+    e = edge_index.shape[1]
+    rowptr = torch.empty(num_nodes + 1, dtype=torch.int32, device=dev)
+    col = torch.empty(e, dtype=torch.int32, device=dev)
+    perm = torch.empty(e, dtype=torch.int32, device=dev)
+    deg = torch.empty(num_nodes, dtype=torch.int32, device=dev)
+    status = torch.empty(1, dtype=torch.int32, device=dev)
+    need = tfg_build_csr_workspace_size(num_nodes, e)
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+    _check(lib().tfg_build_csr_by_source(_ptr(edge_index), e, num_nodes, _ptr(rowptr), _ptr(col),
+                                         _ptr(perm), _ptr(deg), _ptr(workspace), workspace.numel(),
+                                         _ptr(status), _stream(dev)))
+    return CSR(rowptr, col, perm, deg, status)
+
+
+def tfg_aggregate_backward(reduce: str, csr_src: CSR, grad_out, edge_weight=None, in_degree=None,
+                           out=None):
+    """grad_x of tfg_aggregate_sum / _mean: the sum over the transposed graph
+    (csr_src from tfg_build_csr_by_source; edge_weight in original order; the
+    forward CSR's in_degree for the mean)."""
+    _need_cuda("grad_out", grad_out, torch.float32)
+    dev = grad_out.device
+    n, f = grad_out.shape
+    e = csr_src.col.numel()
+    code = REDUCERS[reduce]
+    nb = ctypes.c_size_t(0)
+    _check(lib().tfg_aggregate_backward_workspace_size(code, e, ctypes.byref(nb)))
+    ws = torch.empty(max(nb.value, 1), dtype=torch.uint8, device=dev)
+    if out is None:
+        out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    _check(lib().tfg_aggregate_backward(code, _ptr(csr_src.rowptr), _ptr(csr_src.col), _ptr(csr_src.perm),
+                                        _ptr(edge_weight), _ptr(in_degree), _ptr(grad_out), n, e, f,
+                                        _ptr(out), _ptr(ws), ws.numel(), _stream(dev)))
+    return out
+
+
+def tfg_gcn_aggregate_backward(csr_src: CSR, dinv, grad_out, add_self_loops: int = 0,
+                               self_loop_fill: float = 1.0, out=None):
+    """grad_x of tfg_gcn_aggregate_sum (on-the-fly weights), with the forward's dinv."""
+    _need_cuda("grad_out", grad_out, torch.float32)
+    dev = grad_out.device
+    n, f = grad_out.shape
+    if out is None:
+        out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    _check(lib().tfg_gcn_aggregate_backward(_ptr(csr_src.rowptr), _ptr(csr_src.col), _ptr(dinv),
+                                            _ptr(grad_out), n, f, int(add_self_loops),
+                                            float(self_loop_fill), _ptr(out), _stream(dev)))
+    return out
+
+
+def tfg_aggregate_max_argmax(csr: CSR, x, w_csr=None):
+    """(out, argmax): the max aggregation and, per (t, f), the original id of
+    the first edge attaining it (-1 for a row without edges)."""
+    _need_cuda("x", x)
+    dev = x.device
+    n, f = x.shape
+    out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    arg = torch.empty(n, f, dtype=torch.int32, device=dev)
+    _check(lib().tfg_aggregate_max_argmax(_ptr(csr.rowptr), _ptr(csr.col), _ptr(csr.perm), _ptr(w_csr),
+                                          _ptr(x), _x_dtype(x), n, f, _ptr(out), _ptr(arg), _stream(dev)))
+    return out, arg
+
+
+def tfg_aggregate_max_backward(csr_src: CSR, argmax, grad_out, out=None):
+    _need_cuda("grad_out", grad_out, torch.float32)
+    dev = grad_out.device
+    n, f = grad_out.shape
+    if out is None:
+        out = torch.empty(n, f, dtype=torch.float32, device=dev)
+    _check(lib().tfg_aggregate_max_backward(_ptr(csr_src.rowptr), _ptr(csr_src.col), _ptr(csr_src.perm),
+                                            _ptr(argmax), _ptr(grad_out), n, f, _ptr(out), _stream(dev)))
+    return out
 
 
 def tfg_gcn_norm(rowptr: torch.Tensor, col: torch.Tensor, perm: torch.Tensor, num_nodes: int,

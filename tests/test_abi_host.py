@@ -177,3 +177,30 @@ def test_dot_softmax_rejects(lib):
     assert call(col=None) == -1
     assert call(out=None) == -1
     assert call(e=-1) == -1
+
+
+def test_backward_rejects(lib):
+    n = ctypes.c_size_t(0)
+    assert lib.tfg_aggregate_backward_workspace_size(0, 100, ctypes.byref(n)) == 0 and n.value >= 400
+    assert lib.tfg_aggregate_backward_workspace_size(2, 100, ctypes.byref(n)) == -1     # max
+    f = lib.tfg_aggregate_backward
+    ok = dict(r=0, rp=FAKE, col=FAKE, perm=FAKE, w=None, deg=None, g=FAKE, n=10, e=20, f=4,
+              gx=FAKE, ws=FAKE, wsb=1 << 12, st=None)
+    call = lambda **kw: f(*[kw.get(key, val) for key, val in ok.items()])  # noqa: E731
+    assert call(r=2) == -1
+    assert call(r=1) == -1               # the mean needs in_degree
+    assert call(r=1, deg=FAKE, perm=None) == -1
+    assert call(w=FAKE, perm=None) == -1
+    assert call(w=FAKE, ws=None) == -3
+    assert call(g=None) == -1
+    assert call(gx=None) == -1
+    assert call(f=0) == -1
+    assert lib.tfg_gcn_aggregate_backward(FAKE, FAKE, None, FAKE, 10, 4, 1, 1.0, FAKE, None) == -1
+    am = lib.tfg_aggregate_max_argmax
+    assert am(FAKE, FAKE, None, None, FAKE, 0, 10, 4, FAKE, FAKE, None) == -1           # perm
+    assert am(FAKE, FAKE, FAKE, None, FAKE, 0, 10, 4, FAKE, None, None) == -1           # argmax
+    assert am(FAKE, FAKE, FAKE, None, FAKE, 3, 10, 4, FAKE, FAKE, None) == -1           # dtype
+    mb = lib.tfg_aggregate_max_backward
+    assert mb(FAKE, FAKE, None, FAKE, FAKE, 10, 4, FAKE, None) == -1                    # perm_src
+    assert mb(FAKE, FAKE, FAKE, None, FAKE, 10, 4, FAKE, None) == -1                    # argmax
+    assert lib.tfg_build_csr_by_source(None, 10, 5, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20, FAKE, None) == -1

@@ -1,0 +1,106 @@
+"""Backward of the aggregation against the oracle.
+
+CSR by source and argmax indices are compared bit for bit; gradients within
+TOL_F32 of the oracle's sum of absolute terms (the gradient sums are plain
+fp32 sums of grad_out rows, in a fixed order).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2101_11552_gb300 import graphgen as gg
+from paper_2101_11552_gb300 import tfg
+from _helpers import TOL_F32, assert_exact_f32, assert_scaled_close, dev, features, host_features
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2101_11552_gb300 import build
+    build.build_library()
+
+
+def _graphs(n, e, seed, f=1):
+    wl = gg.random_edge_case_graph(n, e, f, seed, hub=3, isolated=30)
+    csr = tfg.tfg_build_csr(dev(wl.edge_index), n)
+    csr_src = tfg.tfg_build_csr_by_source(dev(wl.edge_index), n)
+    tfg.check_status(csr.status)
+    tfg.check_status(csr_src.status)
+    return wl, csr, csr_src
+
+
+@pytest.mark.parametrize("n,e,seed", [(1, 0, 1), (500, 0, 2), (3000, 40000, 3), (20000, 300000, 4)])
+def test_csr_by_source_bit_exact(n, e, seed):
+    wl = gg.random_edge_case_graph(n, e, 1, seed, hub=3 if n > 4 else -1, isolated=min(30, n - 1))
+    got = tfg.tfg_build_csr_by_source(dev(wl.edge_index), n)
+    tfg.check_status(got.status)
+    want = oracle.build_csr(wl.edge_index[::-1].copy(), n)
+    for a, b, name in zip(got[:4], want, ("rowptr", "col", "perm", "out_degree")):
+        assert np.array_equal(a.cpu().numpy(), b), name
+
+
+@pytest.mark.parametrize("reduce", ["sum", "mean"])
+@pytest.mark.parametrize("weighted", [False, True])
+@pytest.mark.parametrize("f", [1, 7, 64, 128])
+def test_aggregate_backward(reduce, weighted, f):
+    n, e = 3000, 40000
+    wl, csr, csr_src = _graphs(n, e, 30 + f)
+    rng = np.random.default_rng(f)
+    g = rng.standard_normal((n, f)).astype(np.float32)
+    ew = rng.uniform(0.1, 3.0, size=e).astype(np.float32) if weighted else None
+    got = tfg.tfg_aggregate_backward(reduce, csr_src, dev(g), None if ew is None else dev(ew),
+                                     csr.in_degree)
+    ref, scale = oracle.aggregate_backward(wl.edge_index, n, g, reduce,
+                                           w=None if ew is None else ew.astype(np.float64))
+    assert_scaled_close(got.cpu().numpy(), ref, scale, TOL_F32, f"{reduce} backward")
+
+
+@pytest.mark.parametrize("add_self", [0, 1])
+@pytest.mark.parametrize("f", [5, 128])
+def test_gcn_aggregate_backward(add_self, f):
+    n, e = 4000, 60000
+    wl, csr, csr_src = _graphs(n, e, 50 + f)
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, add_self, 1.0,
+                               want_w_csr=False)
+    g = np.random.default_rng(f).standard_normal((n, f)).astype(np.float32)
+    got = tfg.tfg_gcn_aggregate_backward(csr_src, dinv, dev(g), add_self, 1.0)
+    ref, scale = oracle.gcn_aggregate_backward(wl.edge_index, n, g, None, add_self, 1.0)
+    assert_scaled_close(got.cpu().numpy(), ref, scale, TOL_F32, "gcn backward")
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("weighted", [False, True])
+@pytest.mark.parametrize("f", [1, 33, 128])
+def test_max_argmax_and_backward(dtype, weighted, f):
+    n, e = 3000, 40000
+    wl, csr, csr_src = _graphs(n, e, 70 + f, f)
+    rng = np.random.default_rng(f)
+    ew = rng.uniform(0.1, 3.0, size=e).astype(np.float32) if weighted else None
+    w_csr = None if ew is None else dev(ew[csr.perm.cpu().numpy()])
+    out, arg = tfg.tfg_aggregate_max_argmax(csr, features(wl, dtype), w_csr)
+    ref, ref_arg = oracle.max_argmax(wl.edge_index, n, host_features(wl, dtype), ew)
+    assert np.array_equal(arg.cpu().numpy(), ref_arg), "argmax"
+    assert_exact_f32(out.cpu().numpy(), ref, "max with argmax")
+    plain = tfg.tfg_aggregate_max(csr.rowptr, csr.col, features(wl, dtype), w_csr)
+    assert torch.equal(out, plain)                   # the same values as the forward max
+    g = rng.standard_normal((n, f)).astype(np.float32)
+    got = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g))
+    refg, scale = oracle.max_backward(wl.edge_index, n, ref_arg, g)
+    assert_scaled_close(got.cpu().numpy(), refg, scale, TOL_F32, "max backward")
+
+
+def test_backward_is_deterministic_and_validates():
+    n, e, f = 20000, 400000, 64
+    wl, csr, csr_src = _graphs(n, e, 99, f)
+    g = dev(np.random.default_rng(9).standard_normal((n, f)).astype(np.float32))
+    a = tfg.tfg_aggregate_backward("mean", csr_src, g, None, csr.in_degree)
+    b = tfg.tfg_aggregate_backward("mean", csr_src, g, None, csr.in_degree)
+    assert torch.equal(a, b)
+    with pytest.raises(tfg.TfgError):
+        tfg.tfg_aggregate_backward("max", csr_src, g)
+    with pytest.raises(tfg.TfgError):                # the mean needs the forward in-degrees
+        tfg.tfg_aggregate_backward("mean", csr_src, g, None, None)

@@ -159,3 +159,24 @@ def test_dcsbm_dot_softmax_sampled_rows(dcsbm):
     rp = ocsr[0]
     got_alpha = np.concatenate([alpha[int(rp[r]):int(rp[r + 1])].cpu().numpy() for r in sub])
     assert_scaled_close(got_alpha, ref_alpha, alpha_scale(ref_alpha), TOL_F32, "dcsbm dot alpha")
+
+
+def test_dcsbm_gcn_backward_sampled_rows(dcsbm):
+    """Backward of the GCN aggregation at full size: the CSR grouped by
+    source, then the GCN kernel on it with the forward's dinv."""
+    wl, ocsr, csr, rows = dcsbm
+    n = wl.num_nodes
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 1, 1.0, want_w_csr=False)
+    ei = dev(wl.edge_index)
+    csr_src = tfg.tfg_build_csr_by_source(ei, n)
+    tfg.check_status(csr_src.status)
+    del ei
+    g = np.random.default_rng(31).standard_normal((n, 128)).astype(np.float32)
+    got = tfg.tfg_gcn_aggregate_backward(csr_src, dinv, dev(g), 1, 1.0)[dev(rows)].cpu().numpy()
+    ocsr_src = oracle.build_csr(np.ascontiguousarray(wl.edge_index[::-1]), n)
+    assert np.array_equal(csr_src.rowptr.cpu().numpy(), ocsr_src[0])
+    nrm = oracle.gcn_norm(wl.edge_index, n, None, 1, 1.0)
+    # row s of the source-grouped CSR sums w_norm[e] * g[target]: the backward
+    ref, scale = oracle.aggregate_rows(ocsr_src, n, g, "sum", rows, w=nrm["w_norm"],
+                                       self_w=nrm["self_w"])
+    assert_scaled_close(got, ref, scale, TOL_F32, "dcsbm gcn backward")

@@ -389,6 +389,90 @@ def test_bf16_widening_is_exact():
 
 
 # ---------------------------------------------------------------------------
+# Backward of the aggregation
+# ---------------------------------------------------------------------------
+def _fd_directional(forward, x, g, u, h):
+    """(L(x + h u) - L(x - h u)) / 2h for L(x) = <g, forward(x)>."""
+    return (np.sum(g * forward(x + h * u)) - np.sum(g * forward(x - h * u))) / (2 * h)
+
+
+def pin_backward_finite_differences(o):
+    """<grad_x, u> equals the central difference of <grad_out, forward(x)>
+    along u: exact (to rounding) for the linear sum, mean and GCN
+    aggregations, and for max away from ties (distinct random values)."""
+    for seed in range(3):
+        n, e, f = 40, 260, 3
+        wl = gg.random_edge_case_graph(n, e, f, 80 + seed, hub=1, isolated=4)
+        ei = wl.edge_index
+        rng = np.random.default_rng(80 + seed)
+        x = rng.standard_normal((n, f))
+        g = rng.standard_normal((n, f))
+        u = rng.standard_normal((n, f))
+        ew = rng.uniform(0.2, 2.0, size=e)
+        for reduce, w in (("sum", None), ("sum", ew), ("mean", None), ("mean", ew)):
+            gx, _ = o.aggregate_backward(ei, n, g, reduce, w=w)
+            fd = _fd_directional(lambda z: o.aggregate(ei, n, z, reduce, w=w)[0], x, g, u, 1e-3)
+            assert abs(np.sum(gx * u) - fd) <= 1e-9 * (1 + abs(fd)), (reduce, w is None)
+        for selfl in (0, 1):
+            gx, _ = o.gcn_aggregate_backward(ei, n, g, ew, selfl, 1.5)
+            fd = _fd_directional(lambda z: o.gcn_aggregate(ei, n, z, ew, selfl, 1.5)[0], x, g, u, 1e-3)
+            assert abs(np.sum(gx * u) - fd) <= 1e-9 * (1 + abs(fd)), ("gcn", selfl)
+        _, arg = o.max_argmax(ei, n, x.astype(np.float32))
+        gx, _ = o.max_backward(ei, n, arg, g)
+        xm = x.astype(np.float32).astype(np.float64)
+        fd = _fd_directional(lambda z: o.max_argmax(ei, n, z)[0], xm, g, u, 1e-7)
+        assert abs(np.sum(gx * u) - fd) <= 1e-5 * (1 + abs(fd)), "max"
+
+
+def test_backward_finite_differences():
+    pin_backward_finite_differences(oracle.default)
+
+
+def pin_backward_dense_transpose(o):
+    """grad_x = M^T grad_out with M the numpy dense aggregation matrix."""
+    for seed in range(4):
+        n = [1, 7, 25, 60][seed]
+        e = [3, 20, 150, 400][seed]
+        wl = gg.random_edge_case_graph(n, e, 4, 90 + seed, hub=0 if n > 2 else -1,
+                                       isolated=min(2, n - 1))
+        ei = wl.edge_index
+        g = np.random.default_rng(seed).standard_normal((n, 4))
+        ew = np.random.default_rng(seed + 1).uniform(0.1, 3.0, size=e)
+        m = oracle.dense_adjacency(ei, n, ew)
+        gx, _ = o.aggregate_backward(ei, n, g, "sum", w=ew)
+        np.testing.assert_allclose(gx, m.T @ g, rtol=1e-12, atol=1e-12)
+        cnt = oracle.dense_adjacency(ei, n, None).sum(axis=1)
+        mm = m / np.maximum(cnt, 1)[:, None]
+        gx, _ = o.aggregate_backward(ei, n, g, "mean", w=ew)
+        np.testing.assert_allclose(gx, mm.T @ g, rtol=1e-12, atol=1e-12)
+        a_hat = oracle.dense_gcn_matrix(ei, n, ew, 1, 1.0)
+        gx, _ = o.gcn_aggregate_backward(ei, n, g, ew, 1, 1.0)
+        np.testing.assert_allclose(gx, a_hat.T @ g, rtol=1e-12, atol=1e-12)
+
+
+def test_backward_dense_transpose():
+    pin_backward_dense_transpose(oracle.default)
+
+
+def pin_max_argmax_first_of_ties(o):
+    """Ties keep the first edge in original order; the argmax points at an
+    edge into the row whose product equals the maximum; empty rows give -1."""
+    ei = np.array([[1, 2, 3, 0], [0, 0, 0, 4]])
+    x = np.array([[9.0], [2.0], [5.0], [5.0], [0.0]])
+    out, arg = o.max_argmax(ei, 5, x)
+    assert arg[0, 0] == 1 and out[0, 0] == 5.0           # edges 1 and 2 tie at 5: the first wins
+    assert arg[4, 0] == 3 and out[4, 0] == 9.0
+    assert np.all(arg[1:4] == -1) and np.all(out[1:4] == 0.0)
+    g = np.array([[1.0], [0.0], [0.0], [0.0], [2.0]])
+    gx, _ = o.max_backward(ei, 5, arg, g)
+    np.testing.assert_array_equal(gx[:, 0], [2.0, 0.0, 1.0, 0.0, 0.0])
+
+
+def test_max_argmax_first_of_ties():
+    pin_max_argmax_first_of_ties(oracle.default)
+
+
+# ---------------------------------------------------------------------------
 # Dot-product (Transformer-style) attention
 # ---------------------------------------------------------------------------
 def pin_dot_star(o):
@@ -554,6 +638,7 @@ PLANTS = {
     "POOL_SKIP_LAST": [pin_pool_counts],
     "APPNP_TELEPORT_FROM_H": [pin_appnp_hand_example, pin_appnp_dense_closed_form],
     "DOT_KEY_AT_TARGET": [pin_dot_star],
+    "BACKWARD_NO_TRANSPOSE": [pin_backward_finite_differences, pin_backward_dense_transpose],
 }
 
 
