@@ -283,7 +283,7 @@ def cold_l2_ms(fns: dict, stream, reps: int = 5) -> dict:
 def next_rows(L, wl, bufs, stream, hbm_peak):
     """The rows built beyond the timed step, each measured on its own (not part
     of the headline value): APPNP K = 10 on the same graph and bf16 features,
-    the backward of the GCN aggregation,
+    the backward of the GCN aggregation, max with argmax and its backward,
     Transformer-style (dot-product) attention with bf16 q, k, v of the same
     8 x 16 layout, the fused Mean-Max pool on the GCN output, and device
     BatchGraph construction on 1,024 molecule-sized graphs."""
@@ -341,7 +341,22 @@ def next_rows(L, wl, bufs, stream, hbm_peak):
                             "frac": round(abytes / (ms * 1e-3) / 1e9 / hbm_peak, 4),
                             "algorithmic_bytes": abytes,
                             "note": "grad_out = the GCN output (fp32); CSR by source built once"}
-    del csr_src, grad_x
+    # max with argmax (bf16 features) and its backward
+    out_max = torch.empty(n, f, dtype=torch.float32, device=dev)
+    argmax = torch.empty(n, f, dtype=torch.int32, device=dev)
+    perm_fwd = bufs["perm"]
+    ms_fwd = _event_ms(lambda: check(L.tfg_aggregate_max_argmax(
+        P(bufs["rowptr"]), P(bufs["col"]), P(perm_fwd), None, P(bufs["xb"]), tfg.TFG_BF16, n, f,
+        P(out_max), P(argmax), sp)), stream, 5)
+    ms_bwd = _event_ms(lambda: check(L.tfg_aggregate_max_backward(
+        P(csr_src.rowptr), P(csr_src.col), P(csr_src.perm), P(argmax), None, P(bufs["h"]), n, f,
+        P(grad_x), sp)), stream, 5)
+    rows["max_argmax_and_backward"] = {
+        "forward_ms": round(ms_fwd, 4), "backward_ms": round(ms_bwd, 4),
+        "forward_edge_features_per_s": e * f / (ms_fwd * 1e-3),
+        "backward_edge_features_per_s": e * f / (ms_bwd * 1e-3),
+        "note": "bf16 features, argmax int32 [N, F]; backward reads argmax and gradient rows per out-edge"}
+    del csr_src, grad_x, out_max, argmax
 
     heads, ch = wl.heads, wl.channels
     gen = torch.Generator(device=dev)
@@ -700,8 +715,8 @@ def main():
         "pool_mean": lambda: check(L.tfg_segment_pool(
             P(h), tfg.TFG_F32, P(batch), n, g, f, tfg.REDUCERS["mean"], P(pool_mean), st1, sp)),
     }, stream)
-    line["next_rows"] = next_rows(L, wl, dict(rowptr=rowptr, col=col, dinv=dinv, xb=xb, h=h,
-                                              batch=batch), stream, hbm_peak)
+    line["next_rows"] = next_rows(L, wl, dict(rowptr=rowptr, col=col, perm=perm, dinv=dinv, xb=xb,
+                                              h=h, batch=batch), stream, hbm_peak)
     if world == 1 and not args.no_cpu_baseline:
         cu, ct, s = time_oracle(wl, args.cpu_budget)
         line["cpu_baseline"] = {"value": cu / ct, "unit": UNIT, "cores": 1, "kind": "oracle",

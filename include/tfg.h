@@ -198,8 +198,9 @@ int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float
  *   maximum, -1 for a row without edges; perm is the forward CSR's.
  *   argmax int32 [num_nodes, num_features].
  * tfg_aggregate_max_backward: grad_x[s, f] = sum over edges e = (s -> t)
- *   with argmax[t, f] == e of grad_out[t, f] (the weight of a weighted max is
- *   not applied: scale grad_out beforehand if the forward used w_csr).
+ *   with argmax[t, f] == e of w_e grad_out[t, f], w_e = edge_weight[e] in
+ *   ORIGINAL edge order (the weights of the forward, w_csr[k] =
+ *   edge_weight[perm[k]]), or 1 when edge_weight is NULL.
  * grad_out, grad_x: fp32 [num_nodes, num_features]; grad_x is written.
  * Every sum runs in a fixed order: results are bitwise reproducible.
  * ---------------------------------------------------------------------- */
@@ -219,8 +220,9 @@ int tfg_aggregate_max_argmax(const int32_t *rowptr, const int32_t *col, const in
                              tfg_stream_t stream);
 int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src,
                                const int32_t *perm_src, const int32_t *argmax,
-                               const float *grad_out, int64_t num_nodes, int64_t num_features,
-                               float *grad_x, tfg_stream_t stream);
+                               const float *edge_weight, const float *grad_out,
+                               int64_t num_nodes, int64_t num_features, float *grad_x,
+                               tfg_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * Multi-hop propagation: APPNP and SGC, node-level models the paper lists

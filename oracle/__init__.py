@@ -76,7 +76,7 @@ def _load(plant: Optional[str] = None) -> ctypes.CDLL:
                 "oracle_dot_softmax": [I64, I64, P, P, P, P, I, I, D, P, P, P],
                 "oracle_aggregate_backward": [I, I64, I64, P, P, P, P, I64, P, P],
                 "oracle_max_argmax": [I64, I64, P, P, P, I64, P, P],
-                "oracle_max_backward": [I64, I64, P, P, P, I64, P, P],
+                "oracle_max_backward": [I64, I64, P, P, P, P, I64, P, P],
                 "oracle_dot_softmax_rows": [I64, P, P, P, P, P, I, I, D, P, I64, P, P, P],
             }
             for fn, args in sigs.items():
@@ -238,16 +238,18 @@ class _Oracle:
                                                self._p(out), self._p(arg)))
         return out[:n], arg[:n]
 
-    def max_backward(self, edge_index, n, argmax, grad_out):
+    def max_backward(self, edge_index, n, argmax, grad_out, w=None):
+        """dL/dx of the max: w_e grad_out[t, c] to the source of edge argmax[t, c]."""
         ei = np.ascontiguousarray(edge_index, dtype=np.int64)
+        w = None if w is None else np.ascontiguousarray(w, np.float64)
         e = ei.shape[1]
         g = widen(grad_out)
         f = g.shape[1]
         arg = np.ascontiguousarray(argmax, np.int32)
         out = np.zeros((max(n, 1), f))
         ab = np.zeros((max(n, 1), f))
-        self._check(self.lib.oracle_max_backward(n, e, self._p(ei), self._p(arg), self._p(g), f,
-                                                 self._p(out), self._p(ab)))
+        self._check(self.lib.oracle_max_backward(n, e, self._p(ei), self._p(arg), self._p(w),
+                                                 self._p(g), f, self._p(out), self._p(ab)))
         return out[:n], ab[:n]
 
     # -- dot-product (Transformer-style) attention ----------------------

@@ -660,9 +660,10 @@ int oracle_max_argmax(int64_t n, int64_t e, const int64_t *edge_index, const flo
 }
 
 /* grad_x[s, c] = sum over edges e = (s -> t), in original order, with
- * argmax[t, c] == e of grad_out[t, c]. */
+ * argmax[t, c] == e of w_e grad_out[t, c] (w NULL: 1). */
 int oracle_max_backward(int64_t n, int64_t e, const int64_t *edge_index, const int32_t *argmax,
-                        const double *grad_out, int64_t f, double *grad_x, double *absout)
+                        const double *w, const double *grad_out, int64_t f, double *grad_x,
+                        double *absout)
 {
     if (n < 0 || e < 0 || f < 0) return E_ARG;
     const int64_t *src = edge_index, *dst = edge_index + e;
@@ -672,8 +673,9 @@ int oracle_max_backward(int64_t n, int64_t e, const int64_t *edge_index, const i
         if (s < 0 || s >= n || t < 0 || t >= n) return E_RANGE;
         for (int64_t c = 0; c < f; ++c)
             if (argmax[t * f + c] == (int32_t)i) {
-                grad_x[s * f + c] += grad_out[t * f + c];
-                absout[s * f + c] += fabs(grad_out[t * f + c]);
+                double m = (w ? w[i] : 1.0) * grad_out[t * f + c];
+                grad_x[s * f + c] += m;
+                absout[s * f + c] += fabs(m);
             }
     }
     return OK;

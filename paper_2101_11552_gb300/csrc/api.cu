@@ -304,8 +304,9 @@ int tfg_aggregate_max_argmax(const int32_t *rowptr, const int32_t *col, const in
 
 int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src,
                                const int32_t *perm_src, const int32_t *argmax,
-                               const float *grad_out, int64_t num_nodes, int64_t num_features,
-                               float *grad_x, tfg_stream_t stream) {
+                               const float *edge_weight, const float *grad_out,
+                               int64_t num_nodes, int64_t num_features, float *grad_x,
+                               tfg_stream_t stream) {
     const char *fn = "tfg_aggregate_max_backward";
     TFG_TRY(check_counts(fn, num_nodes, 0));
     TFG_TRY(check_features(fn, num_nodes, num_features));
@@ -314,8 +315,9 @@ int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src
     TFG_NEED(argmax, num_nodes > 0, fn, "argmax");
     TFG_NEED(grad_out, num_nodes > 0, fn, "grad_out");
     TFG_NEED(grad_x, num_nodes > 0, fn, "grad_x");
-    return cuda_result(tfg::launch_max_backward(rowptr_src, col_src, perm_src, argmax, grad_out,
-                                                num_nodes, num_features, grad_x,
+    return cuda_result(tfg::launch_max_backward(rowptr_src, col_src, perm_src, argmax,
+                                                edge_weight, grad_out, num_nodes, num_features,
+                                                grad_x,
                                                 reinterpret_cast<cudaStream_t>(stream)),
                        fn);
 }

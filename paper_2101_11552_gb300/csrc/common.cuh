@@ -153,8 +153,8 @@ cudaError_t launch_max_argmax(const int32_t *rowptr, const int32_t *col, const i
                               float *out, int32_t *argmax, cudaStream_t s);
 cudaError_t launch_max_backward(const int32_t *rowptr_src, const int32_t *col_src,
                                 const int32_t *perm_src, const int32_t *argmax,
-                                const float *grad_out, int64_t n, int64_t f, float *grad_x,
-                                cudaStream_t s);
+                                const float *edge_weight, const float *grad_out, int64_t n,
+                                int64_t f, float *grad_x, cudaStream_t s);
 size_t propagate_workspace_bytes(int64_t n, int64_t f, int64_t hops);
 cudaError_t launch_propagate(const int32_t *rowptr, const int32_t *col, const float *w,
                              const float *dinv, const void *x0, int x_dtype, int64_t n, int64_t f,

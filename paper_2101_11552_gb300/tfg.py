@@ -64,7 +64,7 @@ def lib() -> ctypes.CDLL:
                 "tfg_aggregate_backward": [I, P, P, P, P, P, P, I64, I64, I64, P, P, SZ, P],
                 "tfg_gcn_aggregate_backward": [P, P, P, P, I64, I64, I, F, P, P],
                 "tfg_aggregate_max_argmax": [P, P, P, P, P, I, I64, I64, P, P, P],
-                "tfg_aggregate_max_backward": [P, P, P, P, P, I64, I64, P, P],
+                "tfg_aggregate_max_backward": [P, P, P, P, P, P, I64, I64, P, P],
                 "tfg_gcn_norm": [P, P, P, P, I64, I64, I, F, P, P, P],
                 "tfg_aggregate_sum": [P, P, P, P, I, I64, I64, P, P],
                 "tfg_aggregate_mean": [P, P, P, P, I, I64, I64, P, P],
@@ -248,14 +248,17 @@ def tfg_aggregate_max_argmax(csr: CSR, x, w_csr=None):
     return out, arg
 
 
-def tfg_aggregate_max_backward(csr_src: CSR, argmax, grad_out, out=None):
+def tfg_aggregate_max_backward(csr_src: CSR, argmax, grad_out, edge_weight=None, out=None):
+    """grad_x of the max: w_e grad_out[t, f] to the source of the edge argmax[t, f]
+    (edge_weight in original edge order, or None)."""
     _need_cuda("grad_out", grad_out, torch.float32)
     dev = grad_out.device
     n, f = grad_out.shape
     if out is None:
         out = torch.empty(n, f, dtype=torch.float32, device=dev)
     _check(lib().tfg_aggregate_max_backward(_ptr(csr_src.rowptr), _ptr(csr_src.col), _ptr(csr_src.perm),
-                                            _ptr(argmax), _ptr(grad_out), n, f, _ptr(out), _stream(dev)))
+                                            _ptr(argmax), _ptr(edge_weight), _ptr(grad_out), n, f,
+                                            _ptr(out), _stream(dev)))
     return out
 
 

@@ -201,6 +201,6 @@ def test_backward_rejects(lib):
     assert am(FAKE, FAKE, FAKE, None, FAKE, 0, 10, 4, FAKE, None, None) == -1           # argmax
     assert am(FAKE, FAKE, FAKE, None, FAKE, 3, 10, 4, FAKE, FAKE, None) == -1           # dtype
     mb = lib.tfg_aggregate_max_backward
-    assert mb(FAKE, FAKE, None, FAKE, FAKE, 10, 4, FAKE, None) == -1                    # perm_src
-    assert mb(FAKE, FAKE, FAKE, None, FAKE, 10, 4, FAKE, None) == -1                    # argmax
+    assert mb(FAKE, FAKE, None, FAKE, None, FAKE, 10, 4, FAKE, None) == -1              # perm_src
+    assert mb(FAKE, FAKE, FAKE, None, None, FAKE, 10, 4, FAKE, None) == -1              # argmax
     assert lib.tfg_build_csr_by_source(None, 10, 5, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20, FAKE, None) == -1

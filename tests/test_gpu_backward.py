@@ -88,8 +88,9 @@ def test_max_argmax_and_backward(dtype, weighted, f):
     plain = tfg.tfg_aggregate_max(csr.rowptr, csr.col, features(wl, dtype), w_csr)
     assert torch.equal(out, plain)                   # the same values as the forward max
     g = rng.standard_normal((n, f)).astype(np.float32)
-    got = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g))
-    refg, scale = oracle.max_backward(wl.edge_index, n, ref_arg, g)
+    got = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g), None if ew is None else dev(ew))
+    refg, scale = oracle.max_backward(wl.edge_index, n, ref_arg, g,
+                                      None if ew is None else ew.astype(np.float64))
     assert_scaled_close(got.cpu().numpy(), refg, scale, TOL_F32, "max backward")
 
 

@@ -417,11 +417,12 @@ def pin_backward_finite_differences(o):
             gx, _ = o.gcn_aggregate_backward(ei, n, g, ew, selfl, 1.5)
             fd = _fd_directional(lambda z: o.gcn_aggregate(ei, n, z, ew, selfl, 1.5)[0], x, g, u, 1e-3)
             assert abs(np.sum(gx * u) - fd) <= 1e-9 * (1 + abs(fd)), ("gcn", selfl)
-        _, arg = o.max_argmax(ei, n, x.astype(np.float32))
-        gx, _ = o.max_backward(ei, n, arg, g)
         xm = x.astype(np.float32).astype(np.float64)
-        fd = _fd_directional(lambda z: o.max_argmax(ei, n, z)[0], xm, g, u, 1e-7)
-        assert abs(np.sum(gx * u) - fd) <= 1e-5 * (1 + abs(fd)), "max"
+        for w in (None, ew.astype(np.float32)):
+            _, arg = o.max_argmax(ei, n, xm, w)
+            gx, _ = o.max_backward(ei, n, arg, g, None if w is None else w.astype(np.float64))
+            fd = _fd_directional(lambda z: o.max_argmax(ei, n, z, w)[0], xm, g, u, 1e-7)
+            assert abs(np.sum(gx * u) - fd) <= 1e-5 * (1 + abs(fd)), ("max", w is None)
 
 
 def test_backward_finite_differences():
