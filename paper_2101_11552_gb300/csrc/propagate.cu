@@ -69,7 +69,7 @@ cudaError_t launch_propagate(const int32_t *rowptr, const int32_t *col, const fl
     if (n <= 0) return cudaSuccess;
     if (hops == 0) {
         const int64_t count = n * f;
-        const int grid = static_cast<int>(min64(ceil_div(count, 256), int64_t(152) * 32));
+        const int grid = static_cast<int>(min64((count + 255) / 256, int64_t(152) * 32));
         if (x_dtype == TFG_BF16)
             widen_kernel<uint16_t><<<grid, 256, 0, s>>>(static_cast<const uint16_t *>(x0), count, out);
         else
