@@ -4,8 +4,10 @@
  * The library implements the data-parallel core of the graph map-reduce
  * framework of tf_geometric (arXiv:2101.11552): gathering source-node
  * features along the edges of a COO edge list, weighting them, and reducing
- * them per target node; plus the per-graph segment reduction used for graph
- * pooling over a BatchGraph.
+ * them per target node (sum / mean / max, GCN normalisation, additive and
+ * dot-product attention, multi-hop APPNP / SGC propagation, and the
+ * gradients of the aggregations); plus BatchGraph construction and the
+ * per-graph segment reductions used for graph pooling.
  *
  * Conventions shared by every entry point
  * ---------------------------------------

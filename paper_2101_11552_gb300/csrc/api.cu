@@ -134,7 +134,7 @@ int balanced_grid(int64_t n, int64_t e, int64_t min_work) {
 
 extern "C" {
 
-int tfg_version(void) { return 100; }
+int tfg_version(void) { return 200; }
 
 const char *tfg_last_error(void) { return g_err; }
 

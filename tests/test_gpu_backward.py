@@ -105,3 +105,25 @@ def test_backward_is_deterministic_and_validates():
         tfg.tfg_aggregate_backward("max", csr_src, g)
     with pytest.raises(tfg.TfgError):                # the mean needs the forward in-degrees
         tfg.tfg_aggregate_backward("mean", csr_src, g, None, None)
+
+
+@pytest.mark.parametrize("n", [1, 500])
+def test_backward_without_edges(n):
+    """No edges: every gradient is 0 (plus the self-loop term for GCN), the
+    argmax is -1 everywhere."""
+    f = 8
+    ei = np.zeros((2, 0), np.int64)
+    csr = tfg.tfg_build_csr(dev(ei), n)
+    csr_src = tfg.tfg_build_csr_by_source(dev(ei), n)
+    g = np.random.default_rng(n).standard_normal((n, f)).astype(np.float32)
+    for reduce in ("sum", "mean"):
+        got = tfg.tfg_aggregate_backward(reduce, csr_src, dev(g), None, csr.in_degree)
+        assert torch.count_nonzero(got).item() == 0
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 1, 1.0, want_w_csr=False)
+    got = tfg.tfg_gcn_aggregate_backward(csr_src, dinv, dev(g), 1, 1.0)
+    ref, scale = oracle.gcn_aggregate_backward(ei, n, g, None, 1, 1.0)
+    assert_scaled_close(got.cpu().numpy(), ref, scale, TOL_F32, "gcn backward without edges")
+    out, arg = tfg.tfg_aggregate_max_argmax(csr, dev(g))
+    assert torch.count_nonzero(out).item() == 0 and bool((arg == -1).all())
+    got = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g))
+    assert torch.count_nonzero(got).item() == 0

@@ -68,6 +68,14 @@ def test_batch_graphs_paper_example_on_device():
     assert got.edge_index.cpu().numpy().tolist() == [[0, 3, 5, 8], [1, 2, 4, 7]]
 
 
+def test_batch_graphs_zero_graphs():
+    empty = torch.zeros(0, dtype=torch.int64, device="cuda")
+    bg = tfg.tfg_batch_graphs(empty, empty, torch.zeros(2, 0, dtype=torch.int64, device="cuda"), 0)
+    tfg.check_status(bg.status)
+    assert bg.node_offsets.cpu().tolist() == [0]
+    assert bg.edge_index.shape == (2, 0) and bg.batch.numel() == 0
+
+
 def test_batch_graphs_bad_input_sets_status():
     sizes = np.array([2, 2], np.int64)
     stacked = np.array([[0, 5], [1, 0]], np.int64)   # 5 is outside graph 1
