@@ -214,26 +214,40 @@ size_t downsweep_smem(int radix) {
 }
 
 // Lanes of the warp whose value of dig equals this lane's, for dig below
-// 2^(width + 1): one ballot per bit (measured faster here than
-// __match_any_sync).
-__device__ __forceinline__ unsigned same_digit_lanes(uint32_t dig, int width) {
+// 2^bits: one ballot per bit (measured faster here than __match_any_sync).
+__device__ __forceinline__ unsigned peers_from_bit(unsigned peers, uint32_t dig, int b) {
+    const bool set = (dig >> b) & 1u;
+    const unsigned bal = __ballot_sync(kFull, set);
+    return peers & (set ? bal : ~bal);
+}
+
+template <int BITS>   // bit count known at compile time: the loop unrolls
+__device__ __forceinline__ unsigned same_digit_lanes(uint32_t dig) {
     unsigned peers = kFull;
-    for (int b = 0; b <= width; ++b) {
-        const bool set = (dig >> b) & 1u;
-        const unsigned bal = __ballot_sync(kFull, set);
-        peers &= set ? bal : ~bal;
-    }
+#pragma unroll
+    for (int b = 0; b < BITS; ++b) peers = peers_from_bit(peers, dig, b);
     return peers;
 }
 
-template <bool FIRST>
+__device__ __forceinline__ unsigned same_digit_lanes(uint32_t dig, int bits) {
+    unsigned peers = kFull;
+#pragma unroll 1
+    for (int b = 0; b < bits; ++b) peers = peers_from_bit(peers, dig, b);
+    return peers;
+}
+
+// W > 0 fixes the digit width at compile time (the ballot loop unrolls and
+// the per-digit loops get constant bounds); W = 0 takes it from width_arg.
+template <bool FIRST, int W>
 __global__ void __launch_bounds__(kDsThreads, 2)
 radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ dst64,
                 const uint32_t *__restrict__ key_in, const int32_t *__restrict__ src_in,
-                const int32_t *__restrict__ eid_in, int64_t e, int64_t n, int shift, int width,
-                int num_tiles, const int32_t *__restrict__ offs, uint32_t *__restrict__ key_out,
-                int32_t *__restrict__ src_out, int32_t *__restrict__ eid_out, int32_t *status) {
+                const int32_t *__restrict__ eid_in, int64_t e, int64_t n, int shift,
+                int width_arg, int num_tiles, const int32_t *__restrict__ offs,
+                uint32_t *__restrict__ key_out, int32_t *__restrict__ src_out,
+                int32_t *__restrict__ eid_out, int32_t *status) {
     extern __shared__ __align__(16) unsigned char smem[];
+    const int width = W > 0 ? W : width_arg;
     const int radix = 1 << width;
     uint32_t *s_key = reinterpret_cast<uint32_t *>(smem);                 // [tile]
     int32_t *s_src = reinterpret_cast<int32_t *>(s_key + kTile);           // [tile]
@@ -286,7 +300,10 @@ radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ d
         for (int r = 0; r < kDsItems; ++r) {
             const bool ok = FULL || wbase + r * 32 + lane < e;
             const uint32_t dig = ok ? ((keys[r] >> shift) & (radix - 1)) : uint32_t(radix);
-            const unsigned peers = same_digit_lanes(dig, width);
+            // a partial tile marks its missing elements with digit radix: one bit more
+            unsigned peers;
+            if constexpr (W > 0) peers = same_digit_lanes<FULL ? W : W + 1>(dig);
+            else peers = same_digit_lanes(dig, FULL ? width : width + 1);
             const int leader = __ffs(peers) - 1;
             int32_t base = 0;
             if (ok && lane == leader) {
@@ -400,6 +417,28 @@ __global__ void degree_from_rowptr(const int32_t *__restrict__ rowptr, int64_t n
     if (t < n) deg[t] = rowptr[t + 1] - rowptr[t];
 }
 
+#ifndef TFG_DS_STATIC_WIDTH
+#define TFG_DS_STATIC_WIDTH 1   // downsweeps with compile-time digit widths 6..10
+#endif
+
+using DownsweepFn = void (*)(const int64_t *, const int64_t *, const uint32_t *, const int32_t *,
+                             const int32_t *, int64_t, int64_t, int, int, int, const int32_t *,
+                             uint32_t *, int32_t *, int32_t *, int32_t *);
+
+// Every multi-pass plan has digits of 6..10 bits (plan_for), so those widths
+// get their own code; single-pass sorts of small graphs take the generic one.
+template <bool FIRST>
+DownsweepFn downsweep_for(int width) {
+    switch (TFG_DS_STATIC_WIDTH ? width : 0) {
+        case 6: return radix_downsweep<FIRST, 6>;
+        case 7: return radix_downsweep<FIRST, 7>;
+        case 8: return radix_downsweep<FIRST, 8>;
+        case 9: return radix_downsweep<FIRST, 9>;
+        case 10: return radix_downsweep<FIRST, 10>;
+        default: return radix_downsweep<FIRST, 0>;
+    }
+}
+
 }  // namespace
 
 size_t csr_workspace_bytes(int64_t n, int64_t e) {
@@ -441,10 +480,14 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
         // the key row is row 1 (targets), or row 0 (sources) for the transposed CSR
         const int64_t *src64 = by_source ? edge_index + e : edge_index;
         const int64_t *dst64 = by_source ? edge_index : edge_index + e;
+        const DownsweepFn down_first = downsweep_for<true>(p.width);
+        const DownsweepFn down_later = downsweep_for<false>(p.width);
+        // the limit is set to the largest tile any width needs, so concurrent
+        // builds of different sizes never lower it under one another's launch
         const int smem_max = static_cast<int>(downsweep_smem(1 << kMaxDigitBits));
-        err = cudaFuncSetAttribute(radix_downsweep<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
+        err = cudaFuncSetAttribute(down_first, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
         if (err == cudaSuccess)
-            err = cudaFuncSetAttribute(radix_downsweep<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
+            err = cudaFuncSetAttribute(down_later, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_max);
         if (err != cudaSuccess) return err;
         for (int pass = 0; pass < p.passes; ++pass) {
             const int shift = pass * p.width;
@@ -462,11 +505,11 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
             if (err != cudaSuccess) return err;
             const size_t smem = downsweep_smem(radix);
             if (first)
-                radix_downsweep<true><<<tiles, kDsThreads, smem, s>>>(
+                down_first<<<tiles, kDsThreads, smem, s>>>(
                     src64, dst64, nullptr, nullptr, nullptr, e, n, shift, p.width, tiles, cnt,
                     out.key, out.src, out.eid, status);
             else
-                radix_downsweep<false><<<tiles, kDsThreads, smem, s>>>(
+                down_later<<<tiles, kDsThreads, smem, s>>>(
                     nullptr, nullptr, in.key, in.src, in.eid, e, n, shift, p.width, tiles, cnt,
                     out.key, out.src, out.eid, status);
             err = cudaGetLastError();
