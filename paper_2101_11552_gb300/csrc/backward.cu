@@ -29,8 +29,6 @@
 namespace tfg {
 namespace {
 
-constexpr int kBwThreads = 256;
-constexpr int kBwEdges = 4;   // edges whose rows the max-with-argmax kernel requests together
 
 // w_src[k] = (edge_weight ? edge_weight[perm_src[k]] : 1) / (mean ? max(deg[col_src[k]], 1) : 1)
 __global__ void transposed_weights(const int32_t *__restrict__ perm_src,
@@ -45,114 +43,270 @@ __global__ void transposed_weights(const int32_t *__restrict__ perm_src,
     w_src[k] = w;
 }
 
-// Forward max with argmax: one warp per target row, each lane VEC adjacent
-// features (VEC = 4 when the layout allows 8- or 16-byte loads, else 1),
-// lanes striding over the row, edges in CSR (= original) order; a strictly
-// larger value replaces the running maximum, so ties keep the first edge.
+// ---- max with argmax, and its backward ------------------------------------
+// Both kernels walk CSR rows in 32-edge chunks: one coalesced load brings the
+// chunk's indices (and weights) and lanes pass them on by shuffle; the
+// forward has kMxUnroll row gathers in flight before any is used.  Each CTA owns a work-balanced
+// range of rows (balanced_rows); its warps take rows from a shared counter.
+// A row longer than kMxHeavyDeg is set aside and then split over all the
+// CTA's warps in contiguous edge segments, whose states are merged in segment
+// order, so the result is what one warp walking the row in order would give.
+constexpr int kMxWarps = 8;
+constexpr int kMxThreads = kMxWarps * 32;
+#ifndef TFG_MXF_UNROLL
+#define TFG_MXF_UNROLL 8   // forward: feature-row gathers in flight per warp
+#endif
+constexpr int kMxUnroll = TFG_MXF_UNROLL;
+constexpr int64_t kMxHeavyDeg = 1024;
+constexpr int kMxMaxHeavy = 64;
+
+struct MaxArgs {
+    const int32_t *rowptr, *col, *perm;
+    const float *w;   // forward: w_csr (CSR order); backward: edge_weight (original order)
+    const void *x;    // forward: features; backward: grad_out
+    const int32_t *argmax_in;   // backward only
+    int64_t n, f;
+    float *out;
+    int32_t *argmax_out;        // forward only
+};
+
+// Forward state of VEC features over an edge range, in order: a value
+// strictly above the running maximum replaces it, so ties keep the first
+// edge; the row's first edge is taken whatever its value (NaN included).
 template <typename XT, int VEC>
-__global__ void __launch_bounds__(kBwThreads)
-max_argmax(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,
-           const int32_t *__restrict__ perm, const float *__restrict__ w, const XT *__restrict__ x,
-           int64_t n, int64_t f, float *__restrict__ out, int32_t *__restrict__ argmax) {
-    const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-    const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    for (int64_t t = warp; t < n; t += nwarps) {
-        const int64_t beg = rowptr[t], end = col ? rowptr[t + 1] : rowptr[t];
-        for (int64_t f0 = static_cast<int64_t>(lane) * VEC; f0 < f; f0 += 32 * VEC) {
-            float best[VEC];
-            int32_t arg[VEC];
+struct MaxFwd {
+    float best[VEC];
+    int32_t arg[VEC];
+
+    __device__ void init() {
 #pragma unroll
-            for (int q = 0; q < VEC; ++q) {
-                best[q] = -CUDART_INF_F;
-                arg[q] = -1;
-            }
-            // kBwEdges rows requested at once, then compared in edge order
-            for (int64_t k0 = beg; k0 < end; k0 += kBwEdges) {
-                float v[kBwEdges][VEC];
-                int32_t e[kBwEdges];
-                float wk[kBwEdges];
+        for (int q = 0; q < VEC; ++q) {
+            best[q] = -CUDART_INF_F;
+            arg[q] = -1;
+        }
+    }
+
+    // edges [k0, k1) of the row; first = k0 is the row's first edge
+    __device__ void scan(const MaxArgs &a, int64_t k0, int64_t k1, int64_t fl, bool first,
+                         int lane) {
+        using V = VecLoad<XT, VEC>;
+        const XT *x = static_cast<const XT *>(a.x);
+        for (int64_t base = k0; base < k1; base += 32) {
+            const int cnt = static_cast<int>(min64(32, k1 - base));
+            const bool mine = lane < cnt;
+            const int c = mine ? __ldg(a.col + base + lane) : 0;
+            const int32_t ec = mine ? __ldg(a.perm + base + lane) : 0;
+            const float wc = a.w ? (mine ? __ldg(a.w + base + lane) : 0.f) : 1.f;
+            for (int j = 0; j < cnt; j += kMxUnroll) {
+                typename V::Raw raw[kMxUnroll];
 #pragma unroll
-                for (int u = 0; u < kBwEdges; ++u) {
-                    const int64_t k = k0 + u < end ? k0 + u : end - 1;   // tail repeats the last edge
-                    const int64_t s = __ldg(col + k);
-                    e[u] = __ldg(perm + k);
-                    wk[u] = w ? __ldg(w + k) : 1.f;
-                    VecLoad<XT, VEC>::load(x + s * f + f0, v[u]);
+                for (int u = 0; u < kMxUnroll; ++u) {
+                    const int k = j + u;
+                    const int64_t src = __shfl_sync(kFull, c, k & 31);
+                    raw[u] = k < cnt ? V::raw(x + src * a.f + fl) : V::zero();
                 }
 #pragma unroll
-                for (int u = 0; u < kBwEdges; ++u) {
-                    if (k0 + u >= end) break;
+                for (int u = 0; u < kMxUnroll; ++u) {
+                    const int k = j + u;
+                    const int32_t e = __shfl_sync(kFull, ec, k & 31);
+                    const float wk = __shfl_sync(kFull, wc, k & 31);
+                    if (k < cnt) {
+                        float v[VEC];
+                        V::widen(raw[u], v);
+                        const bool take_any = first && base == k0 && k == 0;
 #pragma unroll
-                    for (int q = 0; q < VEC; ++q) {
-                        const float m = w ? wk[u] * v[u][q] : v[u][q];
-                        if (m > best[q] || arg[q] < 0) {
-                            best[q] = m;
-                            arg[q] = e[u];
+                        for (int q = 0; q < VEC; ++q) {
+                            const float m = a.w ? wk * v[q] : v[q];
+                            if (m > best[q] || take_any) {
+                                best[q] = m;
+                                arg[q] = e;
+                            }
                         }
                     }
                 }
             }
-#pragma unroll
-            for (int q = 0; q < VEC; ++q) {
-                out[t * f + f0 + q] = arg[q] < 0 ? 0.f : best[q];
-                argmax[t * f + f0 + q] = arg[q];
-            }
         }
     }
-}
 
-// grad_x[s, f] = sum over the out-edges e = (s -> t) of s, in original order,
-// of w_e grad_out[t, f] where argmax[t, f] == e (w_e = 1 without weights).
-// VEC adjacent features per lane.
-template <int VEC>
-__global__ void __launch_bounds__(kBwThreads)
-max_backward(const int32_t *__restrict__ rowptr_src, const int32_t *__restrict__ col_src,
-             const int32_t *__restrict__ perm_src, const int32_t *__restrict__ argmax,
-             const float *__restrict__ edge_weight, const float *__restrict__ grad_out, int64_t n,
-             int64_t f, float *__restrict__ grad_x) {
-    const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-    const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    for (int64_t s = warp; s < n; s += nwarps) {
-        const int64_t beg = rowptr_src[s], end = col_src ? rowptr_src[s + 1] : rowptr_src[s];
-        for (int64_t f0 = static_cast<int64_t>(lane) * VEC; f0 < f; f0 += 32 * VEC) {
-            float acc[VEC];
+    // the state of the segment after this one (edges later in the row)
+    __device__ void merge_later(const float (&b)[VEC], const int32_t (&g)[VEC]) {
 #pragma unroll
-            for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
-            for (int64_t k = beg; k < end; ++k) {
-                const int64_t t = __ldg(col_src + k);
-                const int32_t e = __ldg(perm_src + k);
-                const float we = edge_weight ? __ldg(edge_weight + e) : 1.f;
-                int32_t a[VEC];
-                float g[VEC];
+        for (int q = 0; q < VEC; ++q)
+            if (b[q] > best[q]) {
+                best[q] = b[q];
+                arg[q] = g[q];
+            }
+    }
+
+    __device__ void store(const MaxArgs &a, int64_t t, int64_t f0) const {
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) {
+            a.out[t * a.f + f0 + q] = arg[q] < 0 ? 0.f : best[q];
+            a.argmax_out[t * a.f + f0 + q] = arg[q];
+        }
+    }
+};
+
+// Backward state: grad_x[s, f] = sum over the out-edges e = (s -> t) of s,
+// in CSR (= original) order, of w_e grad_out[t, f] where argmax[t, f] == e.
+// Per edge a lane requests its slice of the argmax row and of the gradient
+// row of t together, one round trip; this was measured faster than waiting
+// for the argmax row to skip gradient reads, and faster than more edges in
+// flight per warp, which cost registers and so resident warps.
+template <int VEC>
+struct MaxBwd {
+    float acc[VEC];
+
+    __device__ void init() {
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
+    }
+
+    __device__ void scan(const MaxArgs &a, int64_t k0, int64_t k1, int64_t fl, bool, int lane) {
+        const float *g = static_cast<const float *>(a.x);
+        for (int64_t base = k0; base < k1; base += 32) {
+            const int cnt = static_cast<int>(min64(32, k1 - base));
+            const bool mine = lane < cnt;
+            const int c = mine ? __ldg(a.col + base + lane) : 0;
+            const int32_t ec = mine ? __ldg(a.perm + base + lane) : 0;
+            const float wc = a.w ? (mine ? __ldg(a.w + ec) : 0.f) : 1.f;
+            for (int k = 0; k < cnt; ++k) {
+                const int64_t t = __shfl_sync(kFull, c, k);
+                const int32_t e = __shfl_sync(kFull, ec, k);
+                const float we = __shfl_sync(kFull, wc, k);
+                int32_t am[VEC];
+                float gv[VEC];
                 if constexpr (VEC == 4) {
-                    const int4 a4 = __ldg(reinterpret_cast<const int4 *>(argmax + t * f + f0));
-                    const float4 g4 = __ldg(reinterpret_cast<const float4 *>(grad_out + t * f + f0));
-                    a[0] = a4.x; a[1] = a4.y; a[2] = a4.z; a[3] = a4.w;
-                    g[0] = g4.x; g[1] = g4.y; g[2] = g4.z; g[3] = g4.w;
+                    const int4 v = __ldg(reinterpret_cast<const int4 *>(a.argmax_in + t * a.f + fl));
+                    const float4 w4 = __ldg(reinterpret_cast<const float4 *>(g + t * a.f + fl));
+                    am[0] = v.x; am[1] = v.y; am[2] = v.z; am[3] = v.w;
+                    gv[0] = w4.x; gv[1] = w4.y; gv[2] = w4.z; gv[3] = w4.w;
                 } else {
-                    a[0] = __ldg(argmax + t * f + f0);
-                    g[0] = __ldg(grad_out + t * f + f0);
+                    am[0] = __ldg(a.argmax_in + t * a.f + fl);
+                    gv[0] = __ldg(g + t * a.f + fl);
                 }
 #pragma unroll
                 for (int q = 0; q < VEC; ++q)
-                    if (a[q] == e) acc[q] = fmaf(we, g[q], acc[q]);
+                    if (am[q] == e) acc[q] = fmaf(we, gv[q], acc[q]);
             }
-#pragma unroll
-            for (int q = 0; q < VEC; ++q) grad_x[s * f + f0 + q] = acc[q];
         }
+    }
+
+    __device__ void merge_later(const float (&b)[VEC], const int32_t (&)[VEC]) {
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) acc[q] += b[q];
+    }
+
+    __device__ void store(const MaxArgs &a, int64_t s, int64_t f0) const {
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) a.out[s * a.f + f0 + q] = acc[q];
+    }
+};
+
+// Accessors that let one merge routine serve both states.
+template <typename XT, int VEC>
+__device__ __forceinline__ float *state_values(MaxFwd<XT, VEC> &st) { return st.best; }
+template <typename XT, int VEC>
+__device__ __forceinline__ int32_t *state_args(MaxFwd<XT, VEC> &st) { return st.arg; }
+template <int VEC>
+__device__ __forceinline__ float *state_values(MaxBwd<VEC> &st) { return st.acc; }
+template <int VEC>
+__device__ __forceinline__ int32_t *state_args(MaxBwd<VEC> &) { return nullptr; }
+
+// One row by one warp, feature tiles of 32 * VEC.
+template <typename State, int VEC>
+__device__ void max_warp_row(const MaxArgs &a, int64_t t, int lane) {
+    const int64_t beg = a.rowptr[t], end = a.col ? a.rowptr[t + 1] : a.rowptr[t];
+    for (int64_t ft = 0; ft < a.f; ft += 32 * VEC) {
+        const int64_t f0 = ft + static_cast<int64_t>(lane) * VEC;
+        const bool fok = f0 < a.f;
+        State st;
+        st.init();
+        st.scan(a, beg, end, fok ? f0 : 0, true, lane);
+        if (fok) st.store(a, t, f0);
     }
 }
 
+// One long row by all warps of the CTA: warp w takes the w-th of kMxWarps
+// contiguous edge segments; warp 0 folds the later segments into its own in
+// order.  Every thread of the CTA calls this.
+template <typename State, int VEC>
+__device__ void max_cta_row(const MaxArgs &a, int64_t t, float *s_val, int32_t *s_arg) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t beg = a.rowptr[t], end = a.rowptr[t + 1], d = end - beg;
+    const int64_t k0 = beg + d * warp / kMxWarps, k1 = beg + d * (warp + 1) / kMxWarps;
+    for (int64_t ft = 0; ft < a.f; ft += 32 * VEC) {
+        const int64_t f0 = ft + static_cast<int64_t>(lane) * VEC;
+        const bool fok = f0 < a.f;
+        State st;
+        st.init();
+        st.scan(a, k0, k1, fok ? f0 : 0, warp == 0, lane);
+        if (warp > 0) {
+            const int32_t *ar = state_args(st);
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) {
+                s_val[(warp * 32 + lane) * VEC + q] = state_values(st)[q];
+                if (ar) s_arg[(warp * 32 + lane) * VEC + q] = ar[q];
+            }
+        }
+        __syncthreads();
+        if (warp == 0) {
+            for (int w = 1; w < kMxWarps; ++w) {
+                float b[VEC];
+                int32_t g[VEC];
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) {
+                    b[q] = s_val[(w * 32 + lane) * VEC + q];
+                    g[q] = state_args(st) ? s_arg[(w * 32 + lane) * VEC + q] : 0;
+                }
+                st.merge_later(b, g);
+            }
+            if (fok) st.store(a, t, f0);
+        }
+        __syncthreads();
+    }
+}
+
+template <typename State, int VEC>
+__global__ void __launch_bounds__(kMxThreads) max_rows_kernel(MaxArgs a) {
+    __shared__ int s_next, s_nheavy;
+    __shared__ int64_t s_heavy[kMxMaxHeavy];
+    __shared__ float s_val[kMxWarps * 32 * VEC];
+    __shared__ int32_t s_arg[kMxWarps * 32 * VEC];
+    int64_t r0, r1;
+    balanced_rows(a.rowptr, a.n, gridDim.x, blockIdx.x, r0, r1);
+    const int64_t nrows = r1 - r0;
+    if (threadIdx.x == 0) {
+        s_next = 0;
+        s_nheavy = 0;
+    }
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    for (;;) {
+        int i = 0;
+        if (lane == 0) i = atomicAdd(&s_next, 1);
+        i = __shfl_sync(kFull, i, 0);
+        if (i >= nrows) break;
+        const int64_t t = r0 + i;
+        if (a.col != nullptr && a.rowptr[t + 1] - a.rowptr[t] > kMxHeavyDeg) {
+            int slot = 0;
+            if (lane == 0) slot = atomicAdd(&s_nheavy, 1);
+            slot = __shfl_sync(kFull, slot, 0);
+            if (slot < kMxMaxHeavy) {
+                if (lane == 0) s_heavy[slot] = t;
+                continue;
+            }
+        }
+        max_warp_row<State, VEC>(a, t, lane);
+    }
+    __syncthreads();
+    const int nh = min(s_nheavy, kMxMaxHeavy);
+    for (int h = 0; h < nh; ++h) max_cta_row<State, VEC>(a, s_heavy[h], s_val, s_arg);
+}
+
+
 bool aligned(const void *p, uintptr_t b) { return reinterpret_cast<uintptr_t>(p) % b == 0; }
 
-int rows_grid(int64_t n) {
-    const int64_t warps_per_block = kBwThreads / 32;
-    const int64_t want = (n + warps_per_block - 1) / warps_per_block;
-    const int64_t cap = int64_t(152) * 64;
-    return static_cast<int>(want < 1 ? 1 : (want < cap ? want : cap));
-}
 
 }  // namespace
 
@@ -183,17 +337,17 @@ cudaError_t launch_max_argmax(const int32_t *rowptr, const int32_t *col, const i
                               const float *w, const void *x, int x_dtype, int64_t n, int64_t f,
                               float *out, int32_t *argmax, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
-    const int grid = rows_grid(n);
+    const MaxArgs a{rowptr, col, perm, w, x, nullptr, n, f, out, argmax};
+    // E is not known on the host; the kernel reads rowptr[N] for the split
+    const int grid = balanced_grid(n, 0, 1);
     const bool v4 = f % 4 == 0 && aligned(out, 16) && aligned(argmax, 16) &&
                     aligned(x, x_dtype == TFG_BF16 ? 8 : 16);
     if (x_dtype == TFG_BF16) {
-        const uint16_t *xp = static_cast<const uint16_t *>(x);
-        if (v4) max_argmax<uint16_t, 4><<<grid, kBwThreads, 0, s>>>(rowptr, col, perm, w, xp, n, f, out, argmax);
-        else max_argmax<uint16_t, 1><<<grid, kBwThreads, 0, s>>>(rowptr, col, perm, w, xp, n, f, out, argmax);
+        if (v4) max_rows_kernel<MaxFwd<uint16_t, 4>, 4><<<grid, kMxThreads, 0, s>>>(a);
+        else max_rows_kernel<MaxFwd<uint16_t, 1>, 1><<<grid, kMxThreads, 0, s>>>(a);
     } else {
-        const float *xp = static_cast<const float *>(x);
-        if (v4) max_argmax<float, 4><<<grid, kBwThreads, 0, s>>>(rowptr, col, perm, w, xp, n, f, out, argmax);
-        else max_argmax<float, 1><<<grid, kBwThreads, 0, s>>>(rowptr, col, perm, w, xp, n, f, out, argmax);
+        if (v4) max_rows_kernel<MaxFwd<float, 4>, 4><<<grid, kMxThreads, 0, s>>>(a);
+        else max_rows_kernel<MaxFwd<float, 1>, 1><<<grid, kMxThreads, 0, s>>>(a);
     }
     return cudaGetLastError();
 }
@@ -203,13 +357,12 @@ cudaError_t launch_max_backward(const int32_t *rowptr_src, const int32_t *col_sr
                                 const float *edge_weight, const float *grad_out, int64_t n,
                                 int64_t f, float *grad_x, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
+    const MaxArgs a{rowptr_src, col_src, perm_src, edge_weight, grad_out, argmax, n, f, grad_x,
+                    nullptr};
+    const int grid = balanced_grid(n, 0, 1);
     const bool v4 = f % 4 == 0 && aligned(argmax, 16) && aligned(grad_out, 16) && aligned(grad_x, 16);
-    if (v4)
-        max_backward<4><<<rows_grid(n), kBwThreads, 0, s>>>(rowptr_src, col_src, perm_src, argmax,
-                                                            edge_weight, grad_out, n, f, grad_x);
-    else
-        max_backward<1><<<rows_grid(n), kBwThreads, 0, s>>>(rowptr_src, col_src, perm_src, argmax,
-                                                            edge_weight, grad_out, n, f, grad_x);
+    if (v4) max_rows_kernel<MaxBwd<4>, 4><<<grid, kMxThreads, 0, s>>>(a);
+    else max_rows_kernel<MaxBwd<1>, 1><<<grid, kMxThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -116,8 +116,11 @@ __device__ __forceinline__ void axpy_vec(float (&part)[VEC], float p, const floa
     }
 }
 
-template <typename XT, int VEC, int LPR>
-__device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh, int64_t t, int lane) {
+// LH > 0: lanes per head fixed at compile time (the butterfly unrolls);
+// LH = 0 takes lh_arg.
+template <typename XT, int VEC, int LPR, int LH>
+__device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh_arg, int64_t t, int lane) {
+    const int lh = LH > 0 ? LH : lh_arg;
     using V = VecLoad<XT, VEC>;
     constexpr int G = 32 / LPR;
     constexpr int kDotUnroll = dot_unroll<VEC>();
@@ -166,6 +169,7 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh, int64_t t
                     float kv[VEC];
                     V::widen(rk[u], kv);
                     float d = lane_dot(qv, kv);
+#pragma unroll
                     for (int o = 1; o < lh; o <<= 1) d += __shfl_xor_sync(kFull, d, o);
                     l[u] = ok[u] ? d * a.scale : -CUDART_INF_F;
                     mc = fmaxf(mc, l[u]);
@@ -332,9 +336,9 @@ __device__ __forceinline__ void dot_general_row(const DotArgs &a, int64_t t, int
 
 // 16-byte bf16 rows hold twice the features per gather: two resident CTAs
 // per SM leave the registers for kDotUnroll key + value gathers in flight.
-template <typename XT, int VEC, int LPR>
+template <typename XT, int VEC, int LPR, int LH>
 __global__ void __launch_bounds__(kDotThreads, VEC >= 8 ? TFG_DOT_MINB : 3) dot_fast(DotArgs a, int lh) {
-    dot_rows(a.rowptr, a.n, [&](int64_t t, int lane) { dot_fast_row<XT, VEC, LPR>(a, lh, t, lane); });
+    dot_rows(a.rowptr, a.n, [&](int64_t t, int lane) { dot_fast_row<XT, VEC, LPR, LH>(a, lh, t, lane); });
 }
 
 template <typename XT, int NCH>
@@ -342,12 +346,40 @@ __global__ void __launch_bounds__(kDotThreads, 3) dot_general(DotArgs a) {
     dot_rows(a.rowptr, a.n, [&](int64_t t, int lane) { dot_general_row<XT, NCH>(a, t, lane); });
 }
 
+#ifndef TFG_DOT_STATIC_LH
+#define TFG_DOT_STATIC_LH 1   // one kernel per lanes-per-head count
+#endif
+
+// lh (a power of two <= LPR) picks the kernel with that many lanes per head.
+template <typename XT, int VEC, int LPR>
+void launch_fast_lpr(const DotArgs &a, int lh, int grid, cudaStream_t s) {
+    if (!TFG_DOT_STATIC_LH) {
+        dot_fast<XT, VEC, LPR, 0><<<grid, kDotThreads, 0, s>>>(a, lh);
+        return;
+    }
+    switch (lh) {
+        case 1: dot_fast<XT, VEC, LPR, 1><<<grid, kDotThreads, 0, s>>>(a, lh); break;
+        case 2: dot_fast<XT, VEC, LPR, 2><<<grid, kDotThreads, 0, s>>>(a, lh); break;
+        case 4: dot_fast<XT, VEC, LPR, 4><<<grid, kDotThreads, 0, s>>>(a, lh); break;
+        case 8: dot_fast<XT, VEC, LPR, 8><<<grid, kDotThreads, 0, s>>>(a, lh); break;
+        default:
+            if constexpr (LPR >= 16) {
+                if (lh == 16) {
+                    dot_fast<XT, VEC, LPR, 16><<<grid, kDotThreads, 0, s>>>(a, lh);
+                    break;
+                }
+            }
+            if constexpr (LPR >= 32) dot_fast<XT, VEC, LPR, 32><<<grid, kDotThreads, 0, s>>>(a, lh);
+            break;
+    }
+}
+
 template <typename XT, int VEC>
 void launch_fast_vec(const DotArgs &a, int lh, int grid, cudaStream_t s) {
     const int64_t chunks = static_cast<int64_t>(a.heads) * a.channels / VEC;
-    if (chunks >= 32 || lh > 16) dot_fast<XT, VEC, 32><<<grid, kDotThreads, 0, s>>>(a, lh);
-    else if (chunks > 8 || lh > 8) dot_fast<XT, VEC, 16><<<grid, kDotThreads, 0, s>>>(a, lh);
-    else dot_fast<XT, VEC, 8><<<grid, kDotThreads, 0, s>>>(a, lh);
+    if (chunks >= 32 || lh > 16) launch_fast_lpr<XT, VEC, 32>(a, lh, grid, s);
+    else if (chunks > 8 || lh > 8) launch_fast_lpr<XT, VEC, 16>(a, lh, grid, s);
+    else launch_fast_lpr<XT, VEC, 8>(a, lh, grid, s);
 }
 
 template <typename XT>

@@ -24,8 +24,10 @@ def _built():
     build.build_library()
 
 
-def _graphs(n, e, seed, f=1):
+def _graphs(n, e, seed, f=1, reverse=False):
     wl = gg.random_edge_case_graph(n, e, f, seed, hub=3, isolated=30)
+    if reverse:
+        wl.edge_index = np.ascontiguousarray(wl.edge_index[::-1])
     csr = tfg.tfg_build_csr(dev(wl.edge_index), n)
     csr_src = tfg.tfg_build_csr_by_source(dev(wl.edge_index), n)
     tfg.check_status(csr.status)
@@ -72,12 +74,15 @@ def test_gcn_aggregate_backward(add_self, f):
     assert_scaled_close(got.cpu().numpy(), ref, scale, TOL_F32, "gcn backward")
 
 
+@pytest.mark.parametrize("reverse", [False, True])
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("weighted", [False, True])
 @pytest.mark.parametrize("f", [1, 33, 128])
-def test_max_argmax_and_backward(dtype, weighted, f):
+def test_max_argmax_and_backward(dtype, weighted, f, reverse):
+    """The hub (about 20,000 edges) is a target row, split over a CTA in the
+    forward; reversed, it is a source row, split in the backward."""
     n, e = 3000, 40000
-    wl, csr, csr_src = _graphs(n, e, 70 + f, f)
+    wl, csr, csr_src = _graphs(n, e, 70 + f, f, reverse)
     rng = np.random.default_rng(f)
     ew = rng.uniform(0.1, 3.0, size=e).astype(np.float32) if weighted else None
     w_csr = None if ew is None else dev(ew[csr.perm.cpu().numpy()])
@@ -127,3 +132,27 @@ def test_backward_without_edges(n):
     assert torch.count_nonzero(out).item() == 0 and bool((arg == -1).all())
     got = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g))
     assert torch.count_nonzero(got).item() == 0
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_max_argmax_ties_across_hub_segments(dtype):
+    """Equal values everywhere: every argmax is the row's first edge in input
+    order, also in hub rows that the kernel splits into segments, and the
+    backward hands each gradient to that edge's source."""
+    n, e, f = 3000, 40000, 64
+    wl, csr, csr_src = _graphs(n, e, 5, f)
+    x = np.ones((n, f), np.float32)
+    xd = dev(x) if dtype == "f32" else dev(x).to(torch.bfloat16)
+    out, arg = tfg.tfg_aggregate_max_argmax(csr, xd)
+    rowptr, perm = csr.rowptr.cpu().numpy(), csr.perm.cpu().numpy()
+    deg = np.diff(rowptr)
+    assert deg.max() > 4096                          # the hub is split
+    first = np.where(deg > 0, perm[np.minimum(rowptr[:-1], e - 1)], -1)
+    assert np.array_equal(arg.cpu().numpy(), np.repeat(first[:, None], f, axis=1))
+    ref, ref_arg = oracle.max_argmax(wl.edge_index, n, x, None)
+    assert np.array_equal(arg.cpu().numpy(), ref_arg)
+    assert_exact_f32(out.cpu().numpy(), ref, "max of ones")
+    g = np.random.default_rng(6).standard_normal((n, f)).astype(np.float32)
+    got = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g))
+    refg, scale = oracle.max_backward(wl.edge_index, n, ref_arg, g, None)
+    assert_scaled_close(got.cpu().numpy(), refg, scale, TOL_F32, "max backward, ties")
