@@ -54,7 +54,10 @@ __global__ void transposed_weights(const int32_t *__restrict__ perm_src,
 constexpr int kMxWarps = 8;
 constexpr int kMxThreads = kMxWarps * 32;
 #ifndef TFG_MXF_UNROLL
-#define TFG_MXF_UNROLL 8   // forward: feature-row gathers in flight per warp
+#define TFG_MXF_UNROLL 4   // forward: feature-row gathers in flight per lane group
+#endif
+#ifndef TFG_MXF_VEC8
+#define TFG_MXF_VEC8 1     // forward, bf16: 8 features per lane and lane groups
 #endif
 constexpr int kMxUnroll = TFG_MXF_UNROLL;
 constexpr int64_t kMxHeavyDeg = 1024;
@@ -73,16 +76,44 @@ struct MaxArgs {
 // Forward state of VEC features over an edge range, in order: a value
 // strictly above the running maximum replaces it, so ties keep the first
 // edge; the row's first edge is taken whatever its value (NaN included).
-template <typename XT, int VEC>
+// Forward state of VEC features over an edge range, in CSR order (= original
+// order for a CSR from tfg_build_csr).  The running maximum keeps the CSR
+// POSITION of its edge; the original id is looked up once per row (perm) when
+// the result is stored.  The row's first edge is taken whatever its value
+// (NaN included); after that only a strictly larger value replaces the
+// maximum, so ties keep the earliest edge and a NaN is only ever held from
+// the first edge.  The G = 32 / LPR lane groups of a warp take every G-th
+// edge of a chunk; their states, like those of the segments of a split hub
+// row, combine by max_combine, which depends only on values and positions:
+// the larger value wins, equal values go to the smaller position, and a NaN
+// held from the row's first edge wins over everything.  That is exactly what
+// one pass over the row in order gives.
+__device__ __forceinline__ void max_combine(float &b, int32_t &p, float ob, int32_t op,
+                                            int32_t row_beg) {
+    if (op < 0) return;
+    const bool mine_first_nan = p == row_beg && isnan(b);
+    const bool other_first_nan = op == row_beg && isnan(ob);
+    bool take;
+    if (p < 0 || other_first_nan) take = true;
+    else if (mine_first_nan) take = false;
+    else take = ob > b || (ob == b && op < p);
+    if (take) {
+        b = ob;
+        p = op;
+    }
+}
+
+template <typename XT, int VEC, int LPR>
 struct MaxFwd {
+    static constexpr int kVec = VEC, kLpr = LPR, kGroups = 32 / LPR;
     float best[VEC];
-    int32_t arg[VEC];
+    int32_t pos[VEC];
 
     __device__ void init() {
 #pragma unroll
         for (int q = 0; q < VEC; ++q) {
             best[q] = -CUDART_INF_F;
-            arg[q] = -1;
+            pos[q] = -1;
         }
     }
 
@@ -90,36 +121,37 @@ struct MaxFwd {
     __device__ void scan(const MaxArgs &a, int64_t k0, int64_t k1, int64_t fl, bool first,
                          int lane) {
         using V = VecLoad<XT, VEC>;
+        constexpr int G = kGroups;
+        const int g = lane / LPR;
         const XT *x = static_cast<const XT *>(a.x);
         for (int64_t base = k0; base < k1; base += 32) {
             const int cnt = static_cast<int>(min64(32, k1 - base));
             const bool mine = lane < cnt;
             const int c = mine ? __ldg(a.col + base + lane) : 0;
-            const int32_t ec = mine ? __ldg(a.perm + base + lane) : 0;
             const float wc = a.w ? (mine ? __ldg(a.w + base + lane) : 0.f) : 1.f;
-            for (int j = 0; j < cnt; j += kMxUnroll) {
+            for (int j = 0; j < cnt; j += G * kMxUnroll) {
                 typename V::Raw raw[kMxUnroll];
 #pragma unroll
                 for (int u = 0; u < kMxUnroll; ++u) {
-                    const int k = j + u;
+                    const int k = j + u * G + g;
                     const int64_t src = __shfl_sync(kFull, c, k & 31);
                     raw[u] = k < cnt ? V::raw(x + src * a.f + fl) : V::zero();
                 }
 #pragma unroll
                 for (int u = 0; u < kMxUnroll; ++u) {
-                    const int k = j + u;
-                    const int32_t e = __shfl_sync(kFull, ec, k & 31);
+                    const int k = j + u * G + g;
                     const float wk = __shfl_sync(kFull, wc, k & 31);
                     if (k < cnt) {
                         float v[VEC];
                         V::widen(raw[u], v);
                         const bool take_any = first && base == k0 && k == 0;
+                        const int32_t kp = static_cast<int32_t>(base + k);
 #pragma unroll
                         for (int q = 0; q < VEC; ++q) {
                             const float m = a.w ? wk * v[q] : v[q];
                             if (m > best[q] || take_any) {
                                 best[q] = m;
-                                arg[q] = e;
+                                pos[q] = kp;
                             }
                         }
                     }
@@ -128,21 +160,33 @@ struct MaxFwd {
         }
     }
 
-    // the state of the segment after this one (edges later in the row)
-    __device__ void merge_later(const float (&b)[VEC], const int32_t (&g)[VEC]) {
+    // fold the lane groups together (every lane ends with the row's state)
+    __device__ void finish(int32_t row_beg) {
 #pragma unroll
-        for (int q = 0; q < VEC; ++q)
-            if (b[q] > best[q]) {
-                best[q] = b[q];
-                arg[q] = g[q];
+        for (int sh = LPR; sh < 32; sh <<= 1) {
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) {
+                const float ob = __shfl_xor_sync(kFull, best[q], sh);
+                const int32_t op = __shfl_xor_sync(kFull, pos[q], sh);
+                max_combine(best[q], pos[q], ob, op, row_beg);
             }
+        }
     }
+
+    // the state of another segment of the same row
+    __device__ void merge(const float (&b)[VEC], const int32_t (&p)[VEC], int32_t row_beg) {
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) max_combine(best[q], pos[q], b[q], p[q], row_beg);
+    }
+
+    __device__ float *values() { return best; }
+    __device__ int32_t *positions() { return pos; }
 
     __device__ void store(const MaxArgs &a, int64_t t, int64_t f0) const {
 #pragma unroll
         for (int q = 0; q < VEC; ++q) {
-            a.out[t * a.f + f0 + q] = arg[q] < 0 ? 0.f : best[q];
-            a.argmax_out[t * a.f + f0 + q] = arg[q];
+            a.out[t * a.f + f0 + q] = pos[q] < 0 ? 0.f : best[q];
+            a.argmax_out[t * a.f + f0 + q] = pos[q] < 0 ? -1 : __ldg(a.perm + pos[q]);
         }
     }
 };
@@ -155,6 +199,7 @@ struct MaxFwd {
 // flight per warp, which cost registers and so resident warps.
 template <int VEC>
 struct MaxBwd {
+    static constexpr int kVec = VEC, kLpr = 32, kGroups = 1;
     float acc[VEC];
 
     __device__ void init() {
@@ -192,10 +237,16 @@ struct MaxBwd {
         }
     }
 
-    __device__ void merge_later(const float (&b)[VEC], const int32_t (&)[VEC]) {
+    __device__ void finish(int32_t) {}
+
+    // the sum over a later segment of the same row
+    __device__ void merge(const float (&b)[VEC], const int32_t (&)[VEC], int32_t) {
 #pragma unroll
         for (int q = 0; q < VEC; ++q) acc[q] += b[q];
     }
+
+    __device__ float *values() { return acc; }
+    __device__ int32_t *positions() { return nullptr; }
 
     __device__ void store(const MaxArgs &a, int64_t s, int64_t f0) const {
 #pragma unroll
@@ -203,63 +254,58 @@ struct MaxBwd {
     }
 };
 
-// Accessors that let one merge routine serve both states.
-template <typename XT, int VEC>
-__device__ __forceinline__ float *state_values(MaxFwd<XT, VEC> &st) { return st.best; }
-template <typename XT, int VEC>
-__device__ __forceinline__ int32_t *state_args(MaxFwd<XT, VEC> &st) { return st.arg; }
-template <int VEC>
-__device__ __forceinline__ float *state_values(MaxBwd<VEC> &st) { return st.acc; }
-template <int VEC>
-__device__ __forceinline__ int32_t *state_args(MaxBwd<VEC> &) { return nullptr; }
-
-// One row by one warp, feature tiles of 32 * VEC.
-template <typename State, int VEC>
+// One row by one warp, feature tiles of LPR * VEC.
+template <typename State>
 __device__ void max_warp_row(const MaxArgs &a, int64_t t, int lane) {
+    constexpr int VEC = State::kVec, LPR = State::kLpr;
     const int64_t beg = a.rowptr[t], end = a.col ? a.rowptr[t + 1] : a.rowptr[t];
-    for (int64_t ft = 0; ft < a.f; ft += 32 * VEC) {
-        const int64_t f0 = ft + static_cast<int64_t>(lane) * VEC;
+    for (int64_t ft = 0; ft < a.f; ft += LPR * VEC) {
+        const int64_t f0 = ft + static_cast<int64_t>(lane % LPR) * VEC;
         const bool fok = f0 < a.f;
         State st;
         st.init();
         st.scan(a, beg, end, fok ? f0 : 0, true, lane);
-        if (fok) st.store(a, t, f0);
+        st.finish(static_cast<int32_t>(beg));
+        if (fok && lane < LPR) st.store(a, t, f0);
     }
 }
 
 // One long row by all warps of the CTA: warp w takes the w-th of kMxWarps
-// contiguous edge segments; warp 0 folds the later segments into its own in
-// order.  Every thread of the CTA calls this.
-template <typename State, int VEC>
-__device__ void max_cta_row(const MaxArgs &a, int64_t t, float *s_val, int32_t *s_arg) {
+// contiguous edge segments; warp 0 folds the other segments into its own,
+// in segment order.  Every thread of the CTA calls this.
+template <typename State>
+__device__ void max_cta_row(const MaxArgs &a, int64_t t, float *s_val, int32_t *s_pos) {
+    constexpr int VEC = State::kVec, LPR = State::kLpr;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t beg = a.rowptr[t], end = a.rowptr[t + 1], d = end - beg;
     const int64_t k0 = beg + d * warp / kMxWarps, k1 = beg + d * (warp + 1) / kMxWarps;
-    for (int64_t ft = 0; ft < a.f; ft += 32 * VEC) {
-        const int64_t f0 = ft + static_cast<int64_t>(lane) * VEC;
+    const int32_t rb = static_cast<int32_t>(beg);
+    for (int64_t ft = 0; ft < a.f; ft += LPR * VEC) {
+        const int64_t f0 = ft + static_cast<int64_t>(lane % LPR) * VEC;
         const bool fok = f0 < a.f;
         State st;
         st.init();
         st.scan(a, k0, k1, fok ? f0 : 0, warp == 0, lane);
-        if (warp > 0) {
-            const int32_t *ar = state_args(st);
+        st.finish(rb);
+        if (warp > 0 && lane < LPR) {
+            const int32_t *ps = st.positions();
 #pragma unroll
             for (int q = 0; q < VEC; ++q) {
-                s_val[(warp * 32 + lane) * VEC + q] = state_values(st)[q];
-                if (ar) s_arg[(warp * 32 + lane) * VEC + q] = ar[q];
+                s_val[(warp * LPR + lane) * VEC + q] = st.values()[q];
+                if (ps) s_pos[(warp * LPR + lane) * VEC + q] = ps[q];
             }
         }
         __syncthreads();
-        if (warp == 0) {
+        if (warp == 0 && lane < LPR) {
             for (int w = 1; w < kMxWarps; ++w) {
                 float b[VEC];
-                int32_t g[VEC];
+                int32_t p[VEC];
 #pragma unroll
                 for (int q = 0; q < VEC; ++q) {
-                    b[q] = s_val[(w * 32 + lane) * VEC + q];
-                    g[q] = state_args(st) ? s_arg[(w * 32 + lane) * VEC + q] : 0;
+                    b[q] = s_val[(w * LPR + lane) * VEC + q];
+                    p[q] = st.positions() ? s_pos[(w * LPR + lane) * VEC + q] : 0;
                 }
-                st.merge_later(b, g);
+                st.merge(b, p, rb);
             }
             if (fok) st.store(a, t, f0);
         }
@@ -267,12 +313,12 @@ __device__ void max_cta_row(const MaxArgs &a, int64_t t, float *s_val, int32_t *
     }
 }
 
-template <typename State, int VEC>
+template <typename State>
 __global__ void __launch_bounds__(kMxThreads) max_rows_kernel(MaxArgs a) {
     __shared__ int s_next, s_nheavy;
     __shared__ int64_t s_heavy[kMxMaxHeavy];
-    __shared__ float s_val[kMxWarps * 32 * VEC];
-    __shared__ int32_t s_arg[kMxWarps * 32 * VEC];
+    __shared__ float s_val[kMxWarps * State::kLpr * State::kVec];
+    __shared__ int32_t s_pos[kMxWarps * State::kLpr * State::kVec];
     int64_t r0, r1;
     balanced_rows(a.rowptr, a.n, gridDim.x, blockIdx.x, r0, r1);
     const int64_t nrows = r1 - r0;
@@ -297,13 +343,12 @@ __global__ void __launch_bounds__(kMxThreads) max_rows_kernel(MaxArgs a) {
                 continue;
             }
         }
-        max_warp_row<State, VEC>(a, t, lane);
+        max_warp_row<State>(a, t, lane);
     }
     __syncthreads();
     const int nh = min(s_nheavy, kMxMaxHeavy);
-    for (int h = 0; h < nh; ++h) max_cta_row<State, VEC>(a, s_heavy[h], s_val, s_arg);
+    for (int h = 0; h < nh; ++h) max_cta_row<State>(a, s_heavy[h], s_val, s_pos);
 }
-
 
 bool aligned(const void *p, uintptr_t b) { return reinterpret_cast<uintptr_t>(p) % b == 0; }
 
@@ -340,14 +385,20 @@ cudaError_t launch_max_argmax(const int32_t *rowptr, const int32_t *col, const i
     const MaxArgs a{rowptr, col, perm, w, x, nullptr, n, f, out, argmax};
     // E is not known on the host; the kernel reads rowptr[N] for the split
     const int grid = balanced_grid(n, 0, 1);
-    const bool v4 = f % 4 == 0 && aligned(out, 16) && aligned(argmax, 16) &&
-                    aligned(x, x_dtype == TFG_BF16 ? 8 : 16);
     if (x_dtype == TFG_BF16) {
-        if (v4) max_rows_kernel<MaxFwd<uint16_t, 4>, 4><<<grid, kMxThreads, 0, s>>>(a);
-        else max_rows_kernel<MaxFwd<uint16_t, 1>, 1><<<grid, kMxThreads, 0, s>>>(a);
+        if (TFG_MXF_VEC8 && f % 8 == 0 && aligned(x, 16)) {   // 16-byte row slices: 8 features per lane
+            const int64_t lanes = f / 8;
+            if (lanes >= 32) max_rows_kernel<MaxFwd<uint16_t, 8, 32>><<<grid, kMxThreads, 0, s>>>(a);
+            else if (lanes > 8) max_rows_kernel<MaxFwd<uint16_t, 8, 16>><<<grid, kMxThreads, 0, s>>>(a);
+            else max_rows_kernel<MaxFwd<uint16_t, 8, 8>><<<grid, kMxThreads, 0, s>>>(a);
+        } else if (f % 4 == 0 && aligned(x, 8)) {
+            max_rows_kernel<MaxFwd<uint16_t, 4, 32>><<<grid, kMxThreads, 0, s>>>(a);
+        } else {
+            max_rows_kernel<MaxFwd<uint16_t, 1, 32>><<<grid, kMxThreads, 0, s>>>(a);
+        }
     } else {
-        if (v4) max_rows_kernel<MaxFwd<float, 4>, 4><<<grid, kMxThreads, 0, s>>>(a);
-        else max_rows_kernel<MaxFwd<float, 1>, 1><<<grid, kMxThreads, 0, s>>>(a);
+        if (f % 4 == 0 && aligned(x, 16)) max_rows_kernel<MaxFwd<float, 4, 32>><<<grid, kMxThreads, 0, s>>>(a);
+        else max_rows_kernel<MaxFwd<float, 1, 32>><<<grid, kMxThreads, 0, s>>>(a);
     }
     return cudaGetLastError();
 }
@@ -361,8 +412,8 @@ cudaError_t launch_max_backward(const int32_t *rowptr_src, const int32_t *col_sr
                     nullptr};
     const int grid = balanced_grid(n, 0, 1);
     const bool v4 = f % 4 == 0 && aligned(argmax, 16) && aligned(grad_out, 16) && aligned(grad_x, 16);
-    if (v4) max_rows_kernel<MaxBwd<4>, 4><<<grid, kMxThreads, 0, s>>>(a);
-    else max_rows_kernel<MaxBwd<1>, 1><<<grid, kMxThreads, 0, s>>>(a);
+    if (v4) max_rows_kernel<MaxBwd<4>><<<grid, kMxThreads, 0, s>>>(a);
+    else max_rows_kernel<MaxBwd<1>><<<grid, kMxThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 
