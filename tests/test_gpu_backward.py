@@ -156,3 +156,36 @@ def test_max_argmax_ties_across_hub_segments(dtype):
     got = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g))
     refg, scale = oracle.max_backward(wl.edge_index, n, ref_arg, g, None)
     assert_scaled_close(got.cpu().numpy(), refg, scale, TOL_F32, "max backward, ties")
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("weighted", [False, True])
+def test_max_argmax_with_nan_and_inf(dtype, weighted):
+    """NaN, +inf and -inf features (and 0 * inf = NaN products with zero
+    weights): the first edge of a row is taken whatever its value, later
+    edges only when strictly larger, as in one ordered pass -- also across
+    the lane groups and the segments of the split hub row."""
+    n, e, f = 3000, 40000, 16
+    wl, csr, csr_src = _graphs(n, e, 11, f)
+    rng = np.random.default_rng(12)
+    x = rng.standard_normal((n, f)).astype(np.float32)
+    for val, frac in ((np.nan, 0.02), (np.inf, 0.01), (-np.inf, 0.02)):
+        x[rng.random((n, f)) < frac] = val
+    xt = torch.from_numpy(x)
+    if dtype == "bf16":
+        xt = xt.to(torch.bfloat16)
+        x = xt.float().numpy()                       # the values the kernel reads
+    ew = None
+    if weighted:
+        ew = rng.uniform(0.5, 2.0, size=e).astype(np.float32)
+        ew[rng.random(e) < 0.05] = 0.0
+    w_csr = None if ew is None else dev(ew[csr.perm.cpu().numpy()])
+    out, arg = tfg.tfg_aggregate_max_argmax(csr, xt.cuda(), w_csr)
+    ref, ref_arg = oracle.max_argmax(wl.edge_index, n, x, ew)
+    assert np.array_equal(arg.cpu().numpy(), ref_arg), "argmax"
+    np.testing.assert_array_equal(out.cpu().numpy(), ref.astype(np.float32))   # NaN == NaN here
+    g = rng.standard_normal((n, f)).astype(np.float32)
+    got = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g), None if ew is None else dev(ew))
+    refg, scale = oracle.max_backward(wl.edge_index, n, ref_arg, g,
+                                      None if ew is None else ew.astype(np.float64))
+    assert_scaled_close(got.cpu().numpy(), refg, scale, TOL_F32, "max backward, NaN and inf")
