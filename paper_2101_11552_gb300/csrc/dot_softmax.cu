@@ -353,7 +353,7 @@ __global__ void __launch_bounds__(kDotThreads, 3) dot_general(DotArgs a) {
 // lh (a power of two <= LPR) picks the kernel with that many lanes per head.
 template <typename XT, int VEC, int LPR>
 void launch_fast_lpr(const DotArgs &a, int lh, int grid, cudaStream_t s) {
-    if (!TFG_DOT_STATIC_LH) {
+    if constexpr (!TFG_DOT_STATIC_LH) {
         dot_fast<XT, VEC, LPR, 0><<<grid, kDotThreads, 0, s>>>(a, lh);
         return;
     }
