@@ -46,11 +46,12 @@ __global__ void transposed_weights(const int32_t *__restrict__ perm_src,
 // ---- max with argmax, and its backward ------------------------------------
 // Both kernels walk CSR rows in 32-edge chunks: one coalesced load brings the
 // chunk's indices (and weights) and lanes pass them on by shuffle; the
-// forward has kMxUnroll row gathers in flight before any is used.  Each CTA owns a work-balanced
-// range of rows (balanced_rows); its warps take rows from a shared counter.
-// A row longer than kMxHeavyDeg is set aside and then split over all the
-// CTA's warps in contiguous edge segments, whose states are merged in segment
-// order, so the result is what one warp walking the row in order would give.
+// forward has kMxUnroll row gathers per lane group in flight before any is
+// used.  Each CTA owns a work-balanced range of rows (balanced_rows); its
+// warps take rows from a shared counter.  A row longer than kMxHeavyDeg is
+// set aside and then split over all the CTA's warps in contiguous edge
+// segments, whose states are merged, so the result is what one warp walking
+// the row in order would give.
 constexpr int kMxWarps = 8;
 constexpr int kMxThreads = kMxWarps * 32;
 #ifndef TFG_MXF_UNROLL
@@ -73,9 +74,6 @@ struct MaxArgs {
     int32_t *argmax_out;        // forward only
 };
 
-// Forward state of VEC features over an edge range, in order: a value
-// strictly above the running maximum replaces it, so ties keep the first
-// edge; the row's first edge is taken whatever its value (NaN included).
 // Forward state of VEC features over an edge range, in CSR order (= original
 // order for a CSR from tfg_build_csr).  The running maximum keeps the CSR
 // POSITION of its edge; the original id is looked up once per row (perm) when
