@@ -197,7 +197,7 @@ struct MaxFwd {
 // flight per warp, which cost registers and so resident warps.
 template <int VEC>
 struct MaxBwd {
-    static constexpr int kVec = VEC, kLpr = 32, kGroups = 1;
+    static constexpr int kVec = VEC, kLpr = 32;
     float acc[VEC];
 
     __device__ void init() {
