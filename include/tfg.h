@@ -177,7 +177,8 @@ int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float
 
 /* ------------------------------------------------------------------------
  * Backward of the aggregation (the gradient with respect to x; the paper
- * keeps every aggregation differentiable, Sections 2.1.2 and 3).  For
+ * keeps graph construction and mini-batching differentiable, Sections 2.1.1
+ * and 2.1.3, so gradients flow through the aggregation).  For
  *   out[t] = sum over edges e = (s -> t) of w_e x[s]
  * the gradient is the same sum over the transposed graph:
  *   grad_x[s] = sum over edges e = (s -> t) of w_e grad_out[t].
@@ -228,7 +229,7 @@ int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src
 
 /* ------------------------------------------------------------------------
  * Multi-hop propagation: APPNP and SGC, node-level models the paper lists
- * beside GCN and GAT (Section 3) and evaluates in Table 1.  With Ahat the
+ * beside GCN and GAT (Section 2.2) and evaluates in Table 1.  With Ahat the
  * GCN-normalised adjacency of tfg_gcn_aggregate_sum:
  *   h_0 = x0,   h_{k+1} = (1 - alpha) * Ahat h_k + alpha * x0,   out = h_K
  * (K = num_hops).  APPNP (Klicpera et al.) is the power iteration for
@@ -294,7 +295,7 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
 
 /* ------------------------------------------------------------------------
  * Dot-product (Transformer-style) edge-softmax aggregation: the attention
- * form of tf_geometric's own GAT (Section 3 calls it Transformer-based), on
+ * form of tf_geometric's own GAT (Section 4.2 calls it Transformer-based), on
  * the map-reduce workflow of Fig. 5a:
  *   map:    l[k, h] = scale * <q[t, h, :], k[col[k], h, :]>  (position k of row t)
  *   reduce: alpha[k, h] = exp(l[k, h]) / sum over row t of exp(l[., h])
@@ -341,7 +342,11 @@ int tfg_dot_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, co
  * without the workspace.  Nothing is allocated or freed by any call.
  * The first call on each device looks up the array's device address (which
  * may load the library's GPU code), so make that first call outside any
- * stream capture.  All calls on a device share the one array, and each call
+ * stream capture.  The address is then cached per device for the life of
+ * the process: a cudaDeviceReset (or anything else that destroys the
+ * device's primary context) unloads the array and makes the cached address
+ * stale, so after such a reset this entry point must not be called again in
+ * that process.  All calls on a device share the one array, and each call
  * overwrites it: calls that may overlap on the GPU (different streams,
  * different host threads) race with each other and must be serialised by the
  * caller.

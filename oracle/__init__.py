@@ -290,7 +290,7 @@ class _Oracle:
     def appnp(self, edge_index, n, x0, num_hops, alpha, edge_weight=None, add_self_loops=0,
               fill=1.0):
         """K steps of h <- (1 - alpha) Ahat h + alpha x0 from h = x0 (APPNP, the
-        propagation model of Section 3 / Table 1; alpha = 0 is SGC).  Ahat is the
+        propagation model of Section 2.2 / Table 1; alpha = 0 is SGC).  Ahat is the
         GCN normalisation of gcn_norm.  Returns (h_K, error scale), both [N, F]."""
         ei = np.ascontiguousarray(edge_index, dtype=np.int64)
         e = ei.shape[1]

@@ -39,6 +39,15 @@
 #define R_MEAN 1
 #define R_MAX 2
 
+/* The magnitude one term m adds to an error scale (absout): |m|.  The tests
+ * multiply the fp32 tolerance by that scale, so a slip here would loosen or
+ * tighten every comparison; the planted variant doubles it. */
+#ifdef ORACLE_PLANT_SCALE_DOUBLED
+#define SCALE_TERM(m) (2.0 * fabs(m))                    /* planted: inflated scale */
+#else
+#define SCALE_TERM(m) fabs(m)
+#endif
+
 /* ---------------------------------------------------------------------------
  * CSR grouped by target: a stable counting sort of the edges by edge_index[1].
  * The "reduce key" of Section 2.1.2 is the target node; grouping by it makes
@@ -155,7 +164,7 @@ int oracle_aggregate(int reduce, int64_t n, int64_t e, const int64_t *edge_index
             } else {
                 out[t * f + c] += m;
             }
-            absout[t * f + c] += fabs(m);
+            absout[t * f + c] += SCALE_TERM(m);
         }
         count[t] += 1;
     }
@@ -175,7 +184,7 @@ int oracle_aggregate(int reduce, int64_t n, int64_t e, const int64_t *edge_index
             for (int64_t c = 0; c < f; ++c) {
                 double m = self_w[t] * x[t * f + c];
                 out[t * f + c] += m;
-                absout[t * f + c] += fabs(m);
+                absout[t * f + c] += SCALE_TERM(m);
             }
     }
     free(count);
@@ -209,7 +218,7 @@ int oracle_aggregate_rows(int reduce, int64_t n, const int32_t *rowptr, const in
                 } else {
                     o[c] += m;
                 }
-                a[c] += fabs(m);
+                a[c] += SCALE_TERM(m);
             }
             cnt += 1;
         }
@@ -219,7 +228,7 @@ int oracle_aggregate_rows(int reduce, int64_t n, const int32_t *rowptr, const in
             for (int64_t c = 0; c < f; ++c) {
                 double m = self_w[t] * x[t * f + c];
                 o[c] += m;
-                a[c] += fabs(m);
+                a[c] += SCALE_TERM(m);
             }
     }
     return OK;
@@ -301,7 +310,7 @@ int oracle_edge_softmax(int64_t n, int64_t e, const int64_t *edge_index, const d
             for (int cc = 0; cc < c; ++cc) {
                 double m = al * x[src[i] * f + hh * c + cc];
                 out[dst[i] * f + hh * c + cc] += m;
-                absout[dst[i] * f + hh * c + cc] += fabs(m);
+                absout[dst[i] * f + hh * c + cc] += SCALE_TERM(m);
             }
         }
     free(s_src); free(s_dst); free(mx); free(den); free(seen); free(logit);
@@ -349,7 +358,7 @@ int oracle_edge_softmax_rows(int64_t n, const int32_t *rowptr, const int32_t *co
                 for (int cc = 0; cc < c; ++cc) {
                     double m = al * x[s * f + hh * c + cc];
                     o[hh * c + cc] += m;
-                    ab[hh * c + cc] += fabs(m);
+                    ab[hh * c + cc] += SCALE_TERM(m);
                 }
             }
         }
@@ -390,7 +399,7 @@ int oracle_segment_pool(int reduce, int64_t n, int64_t f, int64_t g, const int64
             } else {
                 out[b * f + c] += m;
             }
-            absout[b * f + c] += fabs(m);
+            absout[b * f + c] += SCALE_TERM(m);
         }
         count[b] += 1;
     }
@@ -408,7 +417,7 @@ int oracle_segment_pool(int reduce, int64_t n, int64_t f, int64_t g, const int64
 
 /* ---------------------------------------------------------------------------
  * Multi-hop propagation: APPNP and SGC, two of the node-level models the
- * paper lists (Section 3) and evaluates (Table 1).  APPNP (Klicpera et al.)
+ * paper lists (Section 2.2) and evaluates (Table 1).  APPNP (Klicpera et al.)
  * runs K steps of
  *     h_0 = x0,   h_{k+1}[t] = (1 - alpha) * (sum over edges e into t of
  *                   w_e * h_k[src_e]  +  self_w[t] * h_k[t])  +  alpha * x0[t]
@@ -463,7 +472,7 @@ int oracle_appnp(int64_t n, int64_t e, const int64_t *edge_index, const double *
 
 /* ---------------------------------------------------------------------------
  * Dot-product (Transformer-style) attention, the GAT form the paper says
- * tf_geometric uses (Section 3), on the workflow of Fig. 5a:
+ * tf_geometric uses (Section 4.2), on the workflow of Fig. 5a:
  *   map        l[e,h] = scale * sum_c q[dst_e,h,c] k[src_e,h,c]
  *   reduce     m[t,h] = max over edges into t of l[e,h]          (stability)
  *              den[t,h] = sum over edges into t of exp(l[e,h] - m[t,h])
@@ -529,7 +538,7 @@ int oracle_dot_softmax(int64_t n, int64_t e, const int64_t *edge_index, const do
             for (int cc = 0; cc < c; ++cc) {
                 double m = al * v[src[i] * f + hh * c + cc];
                 out[dst[i] * f + hh * c + cc] += m;
-                absout[dst[i] * f + hh * c + cc] += fabs(m);
+                absout[dst[i] * f + hh * c + cc] += SCALE_TERM(m);
             }
         }
     free(mx); free(den); free(seen); free(logit);
@@ -570,7 +579,7 @@ int oracle_dot_softmax_rows(int64_t n, const int32_t *rowptr, const int32_t *col
                 for (int cc = 0; cc < c; ++cc) {
                     double m = al * v[s * f + hh * c + cc];
                     o[hh * c + cc] += m;
-                    ab[hh * c + cc] += fabs(m);
+                    ab[hh * c + cc] += SCALE_TERM(m);
                 }
             }
         }
@@ -613,7 +622,7 @@ int oracle_aggregate_backward(int reduce, int64_t n, int64_t e, const int64_t *e
         for (int64_t c = 0; c < f; ++c) {
             double m = we * grad_out[t * f + c];
             grad_x[s * f + c] += m;
-            absout[s * f + c] += fabs(m);
+            absout[s * f + c] += SCALE_TERM(m);
         }
     }
     if (self_w && reduce == R_SUM)
@@ -621,7 +630,7 @@ int oracle_aggregate_backward(int reduce, int64_t n, int64_t e, const int64_t *e
             for (int64_t c = 0; c < f; ++c) {
                 double m = self_w[s] * grad_out[s * f + c];
                 grad_x[s * f + c] += m;
-                absout[s * f + c] += fabs(m);
+                absout[s * f + c] += SCALE_TERM(m);
             }
     free(count);
     return OK;
@@ -675,7 +684,7 @@ int oracle_max_backward(int64_t n, int64_t e, const int64_t *edge_index, const i
             if (argmax[t * f + c] == (int32_t)i) {
                 double m = (w ? w[i] : 1.0) * grad_out[t * f + c];
                 grad_x[s * f + c] += m;
-                absout[s * f + c] += fabs(m);
+                absout[s * f + c] += SCALE_TERM(m);
             }
     }
     return OK;

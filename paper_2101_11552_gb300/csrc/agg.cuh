@@ -24,7 +24,7 @@
 //    weight array is read.  With w_csr it adds fill * dinv[t]^2 * x[t] to the
 //    weighted sum.
 //  * APPNP mode (one propagation step, Klicpera et al., the APPNP model the
-//    paper lists in Section 3 and Table 1) is GCN mode with an epilogue:
+//    paper lists in Section 2.2 and Table 1) is GCN mode with an epilogue:
 //    out[t] = (1 - alpha) * gcn(h)[t] + alpha * x0[t], x0 read in its own
 //    storage type X0T.  alpha = 0 is one SGC step.
 //
@@ -82,6 +82,9 @@ struct Agg {
     static constexpr bool kIsMax = KIND == kMax;
     static constexpr bool kGcnLike = KIND == kGcn || KIND == kAppnp;
     static constexpr int kUnroll = unroll_for<VEC, kIsMax>();
+    // a step's slots j + u * G + g must stay inside one 32-edge chunk: full
+    // chunks take no slot test, so a wider step would add edges twice
+    static_assert(G * kUnroll <= 32, "G * kUnroll must not exceed the 32-edge chunk");
 
     static __device__ __forceinline__ float identity() { return kIsMax ? -CUDART_INF_F : 0.f; }
 

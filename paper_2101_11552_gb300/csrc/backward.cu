@@ -1,7 +1,8 @@
 // Backward of the message aggregation: the gradient with respect to the node
-// features x of out = aggregate(x) (the paper stresses that every
-// aggregation stays differentiable, Sections 2.1.2 and 3).  For a sum with
-// edge weights w, out[t] = sum over edges e = (s -> t) of w_e x[s], so
+// features x of out = aggregate(x) (the paper keeps graph construction and
+// mini-batching differentiable, Sections 2.1.1 and 2.1.3, so gradients flow
+// through the aggregation to the features).  For a sum with edge weights w,
+// out[t] = sum over edges e = (s -> t) of w_e x[s], so
 //
 //   grad_x[s] = sum over edges e = (s -> t) of w_e grad_out[t]
 //

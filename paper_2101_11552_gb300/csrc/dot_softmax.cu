@@ -1,5 +1,5 @@
 // Dot-product (Transformer-style) edge-softmax aggregation: the attention
-// form of the GAT that tf_geometric ships (Section 3 names it a
+// form of the GAT that tf_geometric ships (Section 4.2 names it a
 // Transformer-based GAT), on the same map-reduce workflow as Fig. 5a:
 //
 //   map      l[k, h] = scale * <q[t, h, :], k[src, h, :]>   for position k of row t
@@ -46,9 +46,16 @@ __host__ __device__ constexpr int dot_unroll() { return VEC >= 8 ? TFG_DOT_UNROL
 constexpr int64_t kDotMinWork = 2048;      // edges + rows per CTA, at least
 constexpr int kDotMaxChannels = 256;
 
-// exp(m_old - m_new), with exp(-inf - anything) = 0 (an empty state has m = -inf).
+// Logits are kept in base-2 units: the launcher folds log2(e) into the
+// scale once, so every logit, maximum and difference is log2(e) times its
+// natural-log value and exp(l - m) = exp2f(l2 - m2) -- the CUDA math
+// library's base-2 exponential (documented maximum error 2 ulp over its
+// whole range), so the weights' error is set by the fp32 logits alone.
+constexpr float kDotLog2e = 1.4426950408889634f;
+
+// 2^(m_old - m_new), with 2^(-inf - anything) = 0 (an empty state has m = -inf).
 __device__ __forceinline__ float dot_rescale(float m_old, float m_new) {
-    return m_old == -CUDART_INF_F ? 0.f : __expf(m_old - m_new);
+    return m_old == -CUDART_INF_F ? 0.f : exp2f(m_old - m_new);
 }
 
 struct DotArgs {
@@ -124,6 +131,9 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh_arg, int64
     using V = VecLoad<XT, VEC>;
     constexpr int G = 32 / LPR;
     constexpr int kDotUnroll = dot_unroll<VEC>();
+    // a step's slots j + u * G + g must stay inside one 32-edge chunk: full
+    // chunks take no slot test, so a wider step would add edges twice
+    static_assert(G * kDotUnroll <= 32, "G * kDotUnroll must not exceed the 32-edge chunk");
     const int g = lane / LPR, sub = lane % LPR;
     const int64_t f = static_cast<int64_t>(a.heads) * a.channels;
     const XT *qp = static_cast<const XT *>(a.q);
@@ -187,7 +197,7 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh_arg, int64
                 }
 #pragma unroll
                 for (int u = 0; u < kDotUnroll; ++u) {
-                    const float p = ok[u] ? __expf(l[u] - m) : 0.f;
+                    const float p = ok[u] ? exp2f(l[u] - m) : 0.f;
                     den_part += p;
                     float vv[VEC];
                     V::widen(rv[u], vv);
@@ -235,7 +245,7 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh_arg, int64
                 float d = lane_dot(qv, kv);
                 for (int o = 1; o < lh; o <<= 1) d += __shfl_xor_sync(kFull, d, o);
                 if (ok && fok && sub % lh == 0)
-                    a.alpha[k * a.heads + h] = __expf(d * a.scale - m) / den;
+                    a.alpha[k * a.heads + h] = exp2f(d * a.scale - m) / den;
             }
         }
     }
@@ -301,7 +311,7 @@ __device__ __forceinline__ void dot_general_row(const DotArgs &a, int64_t t, int
                     }
                     m = l;
                 }
-                const float p = __expf(l - m);
+                const float p = exp2f(l - m);
                 den_part += p;
 #pragma unroll
                 for (int j = 0; j < NCH; ++j) part[j] = fmaf(p, vv[j], part[j]);
@@ -328,7 +338,7 @@ __device__ __forceinline__ void dot_general_row(const DotArgs &a, int64_t t, int
                 }
 #pragma unroll
                 for (int o = 1; o < 32; o <<= 1) d += __shfl_xor_sync(kFull, d, o);
-                if (lane == 0) a.alpha[k * a.heads + h] = __expf(d * a.scale - m) / den;
+                if (lane == 0) a.alpha[k * a.heads + h] = exp2f(d * a.scale - m) / den;
             }
         }
     }
@@ -402,7 +412,7 @@ cudaError_t launch_dot_softmax(const int32_t *rowptr, const int32_t *col, const 
                                int heads, int channels, float scale, float *out, float *alpha,
                                cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
-    const DotArgs a{rowptr, col, q, k, v, n, heads, channels, scale, out, alpha};
+    const DotArgs a{rowptr, col, q, k, v, n, heads, channels, scale * kDotLog2e, out, alpha};
     const int grid = balanced_grid(n, e, kDotMinWork);
     auto a16 = [](const void *p) { return reinterpret_cast<uintptr_t>(p) % 16 == 0; };
     const bool aligned = a16(q) && a16(k) && a16(v) && a16(out);

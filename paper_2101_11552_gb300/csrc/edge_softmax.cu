@@ -18,6 +18,14 @@
 // keep fp32 chains short.  Every lane of a head evaluates the same logits in
 // the same order, so the lanes agree and results are deterministic.  With
 // alpha requested, a second pass over the row writes the normalised weights.
+//
+// Logits are kept in base-2 units: the node scores are multiplied by log2(e)
+// once, and since LeakyReLU(c v) = c LeakyReLU(v) for c > 0 every logit,
+// maximum and difference is log2(e) times its natural-log value, so
+// exp(l - m) = exp2f(l2 - m2).  exp2f is the CUDA math library's base-2
+// exponential (documented maximum error 2 ulp over its whole range), so the
+// relative error of each weight is set by the fp32 rounding of the logits,
+// not by an approximate exponential.
 #include <math_constants.h>
 
 #include <mutex>
@@ -38,6 +46,7 @@ constexpr int kSmUnroll = TFG_SM_UNROLL;   // fast kernel
 #endif
 constexpr bool kSmFullChunks = TFG_SM_FULL_CHUNKS != 0;
 constexpr int kGenUnroll = 4;               // generic kernel
+constexpr float kLog2e = 1.4426950408889634f;   // log2(e): natural-log units -> base-2 units
 
 // Compensated dot product (the "Dot2" scheme of Ogita, Rump and Oishi,
 // "Accurate sum and dot product", SIAM J. Sci. Comput. 2005): each product
@@ -77,15 +86,16 @@ __global__ void node_scores(const XT *__restrict__ x, int64_t n, int heads, int 
         a.add(xv[0], __ldg(as + c));
         b.add(xv[0], __ldg(ad + c));
     }
-    s_src[i] = a.value();
-    s_dst[i] = b.value();
+    s_src[i] = a.value() * kLog2e;
+    s_dst[i] = b.value() * kLog2e;
 }
 
 __device__ __forceinline__ float leaky(float v, float slope) { return v > 0.f ? v : slope * v; }
 
-// exp(m_old - m_new), with exp(-inf - anything) = 0 (an empty group has m = -inf).
+// 2^(m_old - m_new) for base-2 maxima, with 2^(-inf - anything) = 0 (an
+// empty group has m = -inf).
 __device__ __forceinline__ float rescale(float m_old, float m_new) {
-    return m_old == -CUDART_INF_F ? 0.f : __expf(m_old - m_new);
+    return m_old == -CUDART_INF_F ? 0.f : exp2f(m_old - m_new);
 }
 
 template <typename XT, int VEC, int LPR>
@@ -143,7 +153,7 @@ __device__ __forceinline__ void generic_row(const int32_t *__restrict__ rowptr,
                         }
                         m = l[u];
                     }
-                    const float p = __expf(l[u] - m);
+                    const float p = exp2f(l[u] - m);
                     den_part += p;
                     float v[VEC];
                     V::widen(raw[u], v);
@@ -180,7 +190,7 @@ __device__ __forceinline__ void generic_row(const int32_t *__restrict__ rowptr,
             for (int64_t k = beg; k < end; ++k) {
                 const int src = __ldg(col + k);
                 const float l = leaky(__ldg(s_src + static_cast<int64_t>(src) * heads + h) + sd, slope);
-                alpha[k * heads + h] = __expf(l - m) / den;
+                alpha[k * heads + h] = exp2f(l - m) / den;
             }
         }
     }
@@ -210,6 +220,9 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
     constexpr int ES = 32 / H;      // edges per score step
     constexpr int R = 32 / ES;      // score steps per 32-edge chunk (= H)
     static_assert(ES % G == 0, "score step must hold whole feature steps");
+    // a step's slots e + u * G + g must stay inside one 32-edge chunk (full
+    // chunks take no slot test, and p[k0 / ES] must stay inside p[R])
+    static_assert(G * kSmUnroll <= 32, "G * kSmUnroll must not exceed the 32-edge chunk");
     const int se = lane / H, sh = lane % H;
     const int g = lane / LPR, sub = lane % LPR;
     const int f = H * channels;
@@ -255,7 +268,7 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
         for (int o = H; o < 32; o <<= 1) cm = fmaxf(cm, __shfl_xor_sync(kFull, cm, o));
         const bool rises = cm > m;
         if (__any_sync(kFull, rises)) {   // warp-uniform; rare after the first chunks
-            const float sc = rises ? (m == -CUDART_INF_F ? 0.f : __expf(m - cm)) : 1.f;
+            const float sc = rises ? (m == -CUDART_INF_F ? 0.f : exp2f(m - cm)) : 1.f;
             den *= sc;
             const float fsc = __shfl_sync(kFull, sc, fh);   // lane fh scores head fh
 #pragma unroll
@@ -266,7 +279,7 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
 #pragma unroll
         for (int r = 0; r < R; ++r) {
             const int k = r * ES + se;
-            p[r] = (FULL || k < cnt) ? __expf(p[r] - m) : 0.f;
+            p[r] = (FULL || k < cnt) ? exp2f(p[r] - m) : 0.f;
             den_part += p[r];
         }
         den += den_part;
@@ -340,7 +353,7 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
                 const int src = __shfl_sync(kFull, c, k);
                 if (k < cnt) {
                     const float l = leaky(__ldg(s_src + static_cast<int64_t>(src) * H + sh) + sd, slope);
-                    alpha[(base + k) * H + sh] = __expf(l - m) / den;
+                    alpha[(base + k) * H + sh] = exp2f(l - m) / den;
                 }
             }
         }

@@ -1,6 +1,6 @@
 // Multi-hop propagation with the GCN-normalised adjacency: the APPNP model
 // (Klicpera et al.) and its alpha = 0 special case SGC (Wu et al.), two of the
-// node-level models tf_geometric provides (Section 3, Table 1):
+// node-level models tf_geometric provides (Section 2.2, Table 1):
 //
 //   h_0 = x0,   h_{k+1} = (1 - alpha) * Ahat h_k + alpha * x0,   out = h_K
 //

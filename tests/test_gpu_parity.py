@@ -13,7 +13,8 @@ import torch
 import oracle
 from paper_2101_11552_gb300 import graphgen as gg
 from paper_2101_11552_gb300 import tfg
-from _helpers import (TOL_BF16, TOL_F32, alpha_scale, assert_exact_f32, assert_scaled_close, dev,
+from _helpers import (KAPPA_GAT, TOL_F32, assert_alpha_close, assert_exact_f32, assert_scaled_close,
+                      csr_rows, dev, dot_logit_mag, gat_logit_mag, kappa_dot,
                       features, host_features)
 
 pytestmark = pytest.mark.gpu
@@ -126,7 +127,7 @@ def test_aggregate(reduce, dtype, weighted, f):
         if reduce == "max":
             assert_exact_f32(got, ref, what)
         else:
-            assert_scaled_close(got, ref, scale, TOL_F32 if dtype == "f32" else TOL_BF16, what)
+            assert_scaled_close(got, ref, scale, TOL_F32, what)
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
@@ -141,8 +142,7 @@ def test_gcn_aggregate_on_the_fly(dtype, add_self, f):
     got = np_(tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, features(wl, dtype), None,
                                         add_self, 1.0))
     ref, scale = oracle.gcn_aggregate(wl.edge_index, n, host_features(wl, dtype), None, add_self, 1.0)
-    assert_scaled_close(got, ref, scale, TOL_F32 if dtype == "f32" else TOL_BF16,
-                        f"gcn {dtype} self={add_self} F={f}")
+    assert_scaled_close(got, ref, scale, TOL_F32, f"gcn {dtype} self={add_self} F={f}")
 
 
 @pytest.mark.parametrize("add_self", [0, 1])
@@ -181,9 +181,11 @@ def test_edge_softmax(heads, channels, dtype):
                                                 channels, a_s, a_d, 0.2)
     # the oracle reads the same bf16 values, so fp32 arithmetic is the only error
     assert_scaled_close(np_(out), ref, scale, TOL_F32, f"softmax {dtype} H={heads} C={channels}")
-    perm = oracle.build_csr(wl.edge_index, n)[2]
-    want = ref_alpha[perm]
-    assert_scaled_close(np_(alpha), want, alpha_scale(want), TOL_F32, "alpha")
+    rowptr, col, perm, _ = oracle.build_csr(wl.edge_index, n)
+    row = csr_rows(rowptr)
+    lam = gat_logit_mag(oracle.widen(host_features(wl, dtype)), col, row, heads, channels, a_s, a_d)
+    assert_alpha_close(np_(alpha), ref_alpha[perm], lam, row, KAPPA_GAT,
+                       f"alpha {dtype} H={heads} C={channels}")
 
 
 # ---------------------------------------------------------------------------
@@ -281,7 +283,9 @@ def test_gat169343_edge_softmax_full():
                                                 wl.a_src, wl.a_dst, wl.negative_slope)
     assert_scaled_close(np_(out), ref, scale, TOL_F32, "gat169343 out")
     perm = np_(csr.perm)
-    assert_scaled_close(np_(alpha), ref_alpha[perm], alpha_scale(ref_alpha[perm]), TOL_F32, "gat169343 alpha")
+    row = csr_rows(np_(csr.rowptr))
+    lam = gat_logit_mag(wl.x, np_(csr.col), row, wl.heads, wl.channels, wl.a_src, wl.a_dst)
+    assert_alpha_close(np_(alpha), ref_alpha[perm], lam, row, KAPPA_GAT, "gat169343 alpha")
     deg = np.bincount(wl.edge_index[1], minlength=n)
     assert np.all(np_(out)[deg == 0] == 0.0)
 
@@ -344,7 +348,11 @@ def test_gat169343_dot_softmax_full():
                                                float(np.float32(1.0 / np.sqrt(wl.channels))))
     assert_scaled_close(np_(out), ref, scale, TOL_F32, "gat169343 dot out")
     perm = np_(csr.perm)
-    assert_scaled_close(np_(alpha), ref_alpha[perm], alpha_scale(ref_alpha[perm]), TOL_F32, "gat169343 dot alpha")
+    row = csr_rows(np_(csr.rowptr))
+    lam = dot_logit_mag(wl.x, k, np_(csr.col), row, wl.heads, wl.channels,
+                        float(np.float32(1.0 / np.sqrt(wl.channels))))
+    assert_alpha_close(np_(alpha), ref_alpha[perm], lam, row, kappa_dot(wl.channels),
+                       "gat169343 dot alpha")
 
 
 def test_molecules_device_batching_and_meanmax_full():

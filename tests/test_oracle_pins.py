@@ -626,6 +626,113 @@ def test_appnp_limits():
 
 
 # ---------------------------------------------------------------------------
+# Error scales: every tolerance is a multiple of the oracle's absout, so it is
+# pinned to an independent numpy form -- |M| |X| with dense matrices, and for
+# attention the weights re-derived densely from their definition
+# ---------------------------------------------------------------------------
+def _np_softmax_weights(logit, dst, n, heads):
+    """alpha[e, h] = exp(l[e, h]) / sum over the edges into dst_e of exp(l[., h])."""
+    alpha = np.zeros_like(logit)
+    for t in range(n):
+        m = dst == t
+        if m.any():
+            ex = np.exp(logit[m] - logit[m].max(axis=0))
+            alpha[m] = ex / ex.sum(axis=0)
+    return alpha
+
+
+def _np_attention_scale(alpha, ei, n, vals, heads, channels):
+    """sum over the edges into t of alpha[e, h] |vals[src_e, h, :]|."""
+    ab = np.zeros((n, heads * channels))
+    for e in range(ei.shape[1]):
+        s, t = ei[0, e], ei[1, e]
+        ab[t] += np.repeat(alpha[e], channels) * np.abs(vals[s])
+    return ab
+
+
+def pin_error_scales(o):
+    for seed in range(3):
+        n, e, h, c = [(30, 200, 2, 3), (45, 380, 1, 4), (12, 60, 3, 2)][seed]
+        f = h * c
+        wl = gg.random_edge_case_graph(n, e, f, 140 + seed, hub=1, isolated=3)
+        ei = wl.edge_index
+        rng = np.random.default_rng(140 + seed)
+        x = rng.standard_normal((n, f))
+        w = rng.uniform(-2.0, 2.0, e)
+        wpos = np.abs(w) + 0.1
+        ax = np.abs(x)
+        mabs = oracle.dense_adjacency(ei, n, np.abs(w))
+        cnt = oracle.dense_adjacency(ei, n, None).sum(axis=1)
+        for reduce in ("sum", "mean", "max"):
+            _, ab = o.aggregate(ei, n, x, reduce, w=w)
+            want = mabs @ ax
+            if reduce == "mean":
+                want = want / np.maximum(cnt, 1)[:, None]
+            np.testing.assert_allclose(ab, want, rtol=1e-12, atol=1e-12)
+        csr = o.build_csr(ei, n)
+        rows = np.array([0, n - 1, 5, 2], np.int64)
+        _, ab = o.aggregate_rows(csr, n, x, "mean", rows, w=w)
+        np.testing.assert_allclose(ab, (mabs @ ax / np.maximum(cnt, 1)[:, None])[rows],
+                                   rtol=1e-12, atol=1e-12)
+        for selfl in (0, 1):
+            _, ab = o.gcn_aggregate(ei, n, x, wpos, selfl, 1.5)
+            want = oracle.dense_gcn_matrix(ei, n, wpos, selfl, 1.5) @ ax
+            np.testing.assert_allclose(ab, want, rtol=1e-12, atol=1e-12)
+        # additive attention: weights from the definition, then sum alpha |x|
+        a_s, a_d = rng.standard_normal(f), rng.standard_normal(f)
+        xs = x.reshape(n, h, c)
+        s_src = np.einsum("nhc,hc->nh", xs, a_s.reshape(h, c))
+        s_dst = np.einsum("nhc,hc->nh", xs, a_d.reshape(h, c))
+        z = s_src[ei[0]] + s_dst[ei[1]]
+        alpha = _np_softmax_weights(np.where(z > 0, z, 0.2 * z), ei[1], n, h)
+        want = _np_attention_scale(alpha, ei, n, x, h, c)
+        _, _, ab = o.edge_softmax(ei, n, x, h, c, a_s, a_d, 0.2)
+        np.testing.assert_allclose(ab, want, rtol=1e-11, atol=1e-12)
+        _, _, ab = o.edge_softmax_rows(csr, n, x, h, c, a_s, a_d, 0.2, rows)
+        np.testing.assert_allclose(ab, want[rows], rtol=1e-11, atol=1e-12)
+        # dot-product attention
+        q, k, v = (rng.standard_normal((n, f)) for _ in range(3))
+        lg = 0.3 * np.einsum("ehc,ehc->eh", q[ei[1]].reshape(-1, h, c), k[ei[0]].reshape(-1, h, c))
+        alpha = _np_softmax_weights(lg, ei[1], n, h)
+        want = _np_attention_scale(alpha, ei, n, v, h, c)
+        _, _, ab = o.dot_softmax(ei, n, q, k, v, h, c, 0.3)
+        np.testing.assert_allclose(ab, want, rtol=1e-11, atol=1e-12)
+        _, _, ab = o.dot_softmax_rows(csr, n, q, k, v, h, c, 0.3, rows)
+        np.testing.assert_allclose(ab, want[rows], rtol=1e-11, atol=1e-12)
+        # pooling: sum of |x| per graph (divided by the count for mean)
+        batch = np.sort(rng.integers(0, 4, n))
+        pool_abs = np.zeros((5, f))
+        np.add.at(pool_abs, batch, ax)
+        counts = np.bincount(batch, minlength=5)
+        for reduce in ("sum", "mean", "max"):
+            _, ab = o.segment_pool(x, batch, 5, reduce)
+            want = pool_abs / np.maximum(counts, 1)[:, None] if reduce == "mean" else pool_abs
+            np.testing.assert_allclose(ab, want, rtol=1e-12, atol=1e-12)
+        # backward: |M|^T |grad_out|
+        g = rng.standard_normal((n, f))
+        _, ab = o.aggregate_backward(ei, n, g, "sum", w=w)
+        np.testing.assert_allclose(ab, mabs.T @ np.abs(g), rtol=1e-12, atol=1e-12)
+        _, ab = o.aggregate_backward(ei, n, g, "mean", w=w)
+        np.testing.assert_allclose(ab, (mabs / np.maximum(cnt, 1)[:, None]).T @ np.abs(g),
+                                   rtol=1e-12, atol=1e-12)
+        _, ab = o.gcn_aggregate_backward(ei, n, g, wpos, 1, 1.5)
+        np.testing.assert_allclose(ab, oracle.dense_gcn_matrix(ei, n, wpos, 1, 1.5).T @ np.abs(g),
+                                   rtol=1e-12, atol=1e-12)
+        _, arg = o.max_argmax(ei, n, x.astype(np.float32), w.astype(np.float32))
+        want = np.zeros((n, f))
+        for t in range(n):
+            for j in range(f):
+                if arg[t, j] >= 0:
+                    want[ei[0, arg[t, j]], j] += abs(w[arg[t, j]] * g[t, j])
+        _, ab = o.max_backward(ei, n, arg, g, w)
+        np.testing.assert_allclose(ab, want, rtol=1e-12, atol=1e-12)
+
+
+def test_error_scales():
+    pin_error_scales(oracle.default)
+
+
+# ---------------------------------------------------------------------------
 # Planted mistakes: each one must trip at least one pin
 # ---------------------------------------------------------------------------
 PLANTS = {
@@ -640,6 +747,7 @@ PLANTS = {
     "APPNP_TELEPORT_FROM_H": [pin_appnp_hand_example, pin_appnp_dense_closed_form],
     "DOT_KEY_AT_TARGET": [pin_dot_star],
     "BACKWARD_NO_TRANSPOSE": [pin_backward_finite_differences, pin_backward_dense_transpose],
+    "SCALE_DOUBLED": [pin_error_scales],
 }
 
 
