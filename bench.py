@@ -176,6 +176,18 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # the fp64 oracle on a bounded sample (CPU baseline / reference arm)
 # ---------------------------------------------------------------------------
+SAMPLE_EDGES = 6_000_000   # edges of the CPU baselines' sample (both legs use the same one)
+
+
+def sample_nodes(wl, target_edges: int = SAMPLE_EDGES) -> int:
+    """Smallest k whose node-induced subgraph on nodes [0, k) holds at least
+    target_edges edges (all nodes if the graph is smaller)."""
+    ei = wl.edge_index
+    counts = np.bincount(np.maximum(ei[0], ei[1]), minlength=wl.num_nodes).cumsum()
+    k = int(np.searchsorted(counts, target_edges)) + 1
+    return min(max(k, 2), wl.num_nodes)
+
+
 def oracle_sample(wl, n_nodes: int):
     """Node-induced subgraph on the first n_nodes nodes.  Nodes are numbered
     community by community, so this keeps whole communities (the last one
@@ -202,41 +214,72 @@ def oracle_step(s) -> int:
     return units_per_step(n, ei.shape[1], s["x"].shape[1])
 
 
-def time_oracle(wl, budget_s: float, steps: int = 1):
-    """Size a sample so that `steps` oracle steps take about budget_s, run them.
-
-    The oracle's cost grows with the sample's nodes and edges; a probe on the
-    first 1,500 nodes fixes the scale."""
+def oracle_step_all_cores(s) -> int:
+    """The same step with the row-parallel parts (GCN aggregation, edge
+    softmax) on every host core: the oracle's own row functions on blocks
+    of target rows (OpenMP), over the oracle's own CSR.  CSR, normalisation
+    and pooling stay single-threaded, as the oracle writes them."""
     import oracle
-    oracle.build()
-    n0 = min(wl.num_nodes, 1500)
-    probe = oracle_sample(wl, n0)
-    t0 = time.perf_counter()
-    oracle_step(probe)
-    t_probe = time.perf_counter() - t0
-    per_step = budget_s / max(steps, 1)
-    n1 = n0
-    for _ in range(2):   # cost is not exactly linear in nodes: refine once
-        n1 = int(min(wl.num_nodes, max(200, n1 * per_step / max(t_probe, 1e-6))))
-        s = oracle_sample(wl, n1)
-        t0 = time.perf_counter()
-        oracle_step(s)
-        t_probe = time.perf_counter() - t0
-        if 0.6 * per_step < t_probe < 1.6 * per_step:
-            break
+    n, ei = s["n"], s["edge_index"]
+    csr = oracle.build_csr(ei, n)
+    nrm = oracle.gcn_norm(ei, n, None, 1, 1.0)
+    h, _ = oracle.omp_rows.aggregate_all(csr, n, s["x_bf16"], "sum", w=nrm["w_norm"],
+                                         self_w=nrm["self_w"])
+    oracle.omp_rows.edge_softmax_all(csr, n, s["x_bf16"], s["heads"], s["channels"], s["a_src"],
+                                     s["a_dst"], 0.2)
+    oracle.segment_pool(h, s["batch"], s["g"], "mean")
+    oracle.segment_pool(h, s["batch"], s["g"], "max")
+    return units_per_step(n, ei.shape[1], s["x"].shape[1])
+
+
+def time_steps(step_fn, s, steps: int):
     units, t = 0, 0.0
     for _ in range(steps):
         t0 = time.perf_counter()
-        units += oracle_step(s)
+        units += step_fn(s)
         t += time.perf_counter() - t0
-    return units, t, s
+    return units, t
+
+
+def host_cpu() -> dict:
+    """Core count and model of the host the baselines run on (read at run time)."""
+    model = ""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() in ("Model name", "Model"):
+                model = line.split(":", 1)[1].strip()
+                if line.startswith("Model name"):
+                    break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return {"cpu_count": os.cpu_count(), "model": model}
 
 
 def cpu_desc(s) -> str:
     comm = (f"{s['g'] - 1} whole communities and part of the next" if s["cut"]
             else f"{s['g']} whole communities")
-    return (f"oracle (fp64, single thread) on the node-induced subgraph of the first {s['n']} nodes "
+    return (f"oracle (fp64) on the node-induced subgraph of the first {s['n']} nodes "
             f"({comm}, {s['edge_index'].shape[1]} edges) of the same workload")
+
+
+def cpu_baselines(wl) -> dict:
+    """The oracle single-threaded (as it stands) and on all host cores, one
+    step each after one untimed step, on the same fixed sample."""
+    import oracle
+    oracle.build()
+    s = oracle_sample(wl, sample_nodes(wl))
+    oracle_step(s)
+    u1, t1 = time_steps(oracle_step, s, 1)
+    oracle_step_all_cores(s)
+    ua, ta = time_steps(oracle_step_all_cores, s, 1)
+    return {"value": u1 / t1, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": cpu_desc(s),
+            "seconds": round(t1, 2), "host": host_cpu(),
+            "all_cores": {"value": ua / ta, "unit": UNIT, "cores": oracle.omp_rows.threads(),
+                          "seconds": round(ta, 2),
+                          "how": "GCN aggregation and edge softmax on blocks of target rows in "
+                                 "parallel (OpenMP, the oracle's row functions); CSR, "
+                                 "normalisation and pooling single-threaded"}}
 
 
 # ---------------------------------------------------------------------------
@@ -257,12 +300,20 @@ def _event_ms(fn, stream, reps: int) -> float:
     return t0.elapsed_time(t1) / reps
 
 
+def l2_flush_bytes() -> int:
+    """Twice the device's L2 (read from the device), at least 256 MB."""
+    import torch
+    l2 = int(getattr(torch.cuda.get_device_properties(torch.cuda.current_device()),
+                     "L2_cache_size", 0) or 0)
+    return max(2 * l2, 256 << 20)
+
+
 def cold_l2_ms(fns: dict, stream, reps: int = 5) -> dict:
-    """Each call timed alone right after a write of 256 MB (twice the L2), so
+    """Each call timed alone right after a write of twice the L2 size, so
     that its node features and edge arrays come from HBM: the cold-L2
     counterpart of the per-call times inside the step."""
     import torch
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=torch.cuda.current_device())
+    flush = torch.empty(l2_flush_bytes(), dtype=torch.uint8, device=torch.cuda.current_device())
     out = {}
     for name, fn in fns.items():
         fn()
@@ -278,6 +329,129 @@ def cold_l2_ms(fns: dict, stream, reps: int = 5) -> dict:
             ts.append(a.elapsed_time(b))
         out[name] = round(statistics.median(ts), 4)
     return out
+
+
+def small_configs(L, stream, hbm_peak):
+    """The four smaller workloads, each call timed hot (mean of repeated calls,
+    inputs left in L2 by the previous call) and cold (after an L2 flush):
+    edge-features/s, algorithmic GB/s and its fraction of the measured HBM
+    peak (hot).  The 2,708-node and 19,717-node graphs fit in L2 and are
+    launch- or latency-bound; they are reported, not roofline targets."""
+    import torch
+    from paper_2101_11552_gb300 import graphgen as gg
+    from paper_2101_11552_gb300 import tfg
+    P = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
+    sp = ctypes.c_void_p(stream.cuda_stream)
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    def check(rc):
+        if rc != 0:
+            raise RuntimeError(f"libtfg error {rc}: {tfg.tfg_last_error()}")
+
+    def measure(fn, units, abytes, reps):
+        hot = _event_ms(fn, stream, reps)
+        cold = cold_l2_ms({"c": fn}, stream)["c"]
+        gbs = abytes / (hot * 1e-3) / 1e9
+        return {"ms": round(hot, 5), "cold_l2_ms": round(cold, 5),
+                "edge_features_per_s": units / (hot * 1e-3), "gbs": round(gbs, 1),
+                "frac": round(gbs / hbm_peak, 4), "algorithmic_bytes": abytes}
+
+    def csr_of(wl):
+        csr = tfg.tfg_build_csr(torch.from_numpy(wl.edge_index).to(dev), wl.num_nodes)
+        tfg.check_status(csr.status)
+        return csr
+
+    out = {}
+    # GCN propagation on the 2,708-node graph (explicit self-loops), fp32 F = 64
+    wl = gg.make_er_2708()
+    n, e, f = wl.num_nodes, wl.num_edges, wl.num_features
+    csr = csr_of(wl)
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
+    x = torch.from_numpy(wl.x).to(dev)
+    y = torch.empty(n, f, dtype=torch.float32, device=dev)
+    out["er_2708_gcn"] = {"workload": "G(2708, 5278) + self-loops, F = 64 fp32, GCN sum",
+                          "nodes": n, "edges": e, "calls": {"gcn_aggregate": measure(
+        lambda: check(L.tfg_gcn_aggregate_sum(P(csr.rowptr), P(csr.col), P(dinv), None, P(x),
+                                              tfg.TFG_F32, n, f, 0, 1.0, P(y), sp)),
+        e * f, 4 * e + 4 * (n + 1) + 4 * n + 8 * n * f, 200)}}
+    # unweighted sum / mean / max on the 19,717-node power-law graph, fp32 F = 256
+    wl = gg.make_ba_19717()
+    n, e, f = wl.num_nodes, wl.num_edges, wl.num_features
+    csr = csr_of(wl)
+    x = torch.from_numpy(wl.x).to(dev)
+    y = torch.empty(n, f, dtype=torch.float32, device=dev)
+    calls = {}
+    for red, fn in (("sum", L.tfg_aggregate_sum), ("mean", L.tfg_aggregate_mean),
+                    ("max", L.tfg_aggregate_max)):
+        calls[red] = measure(
+            lambda fn=fn: check(fn(P(csr.rowptr), P(csr.col), None, P(x), tfg.TFG_F32, n, f,
+                                   P(y), sp)),
+            e * f, 4 * e + 4 * (n + 1) + 8 * n * f, 100)
+    out["ba_19717_sum_mean_max"] = {"workload": "BA(19717, m=2) + self-loops, F = 256 fp32",
+                                    "nodes": n, "edges": e, "calls": calls}
+    # GAT edge softmax on the 169,343-node oriented power-law graph, fp32 8 x 16
+    wl = gg.make_gat_169343()
+    n, e, f, heads, ch = wl.num_nodes, wl.num_edges, wl.num_features, wl.heads, wl.channels
+    csr = csr_of(wl)
+    x = torch.from_numpy(wl.x).to(dev)
+    y = torch.empty(n, f, dtype=torch.float32, device=dev)
+    a_s, a_d = torch.from_numpy(wl.a_src).to(dev), torch.from_numpy(wl.a_dst).to(dev)
+    ws = torch.empty(tfg.tfg_edge_softmax_workspace_size(n, heads), dtype=torch.uint8, device=dev)
+    out["gat_169343_edge_softmax"] = {
+        "workload": "BA(169343, m=7) subsampled to 1,166,243 edges, oriented; F = 8 x 16 fp32",
+        "nodes": n, "edges": e, "calls": {"edge_softmax": measure(
+            lambda: check(L.tfg_edge_softmax_aggregate(P(csr.rowptr), P(csr.col), P(x), tfg.TFG_F32,
+                                                       n, e, heads, ch, P(a_s), P(a_d), 0.2, P(y),
+                                                       None, P(ws), ws.numel(), sp)),
+            e * f, 4 * e + 4 * (n + 1) + 8 * n * f + 16 * n * heads, 50)}}
+    # 1,024 batched molecule-sized graphs: GCN, then sum / mean / max pooling
+    wl = gg.make_molecules_1024()
+    n, e, f, g = wl.num_nodes, wl.num_edges, wl.num_features, wl.num_graphs
+    csr = csr_of(wl)
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
+    x = torch.from_numpy(wl.x).to(dev)
+    hh = torch.empty(n, f, dtype=torch.float32, device=dev)
+    batch = torch.from_numpy(wl.batch).to(dev)
+    pooled = torch.empty(g, f, dtype=torch.float32, device=dev)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    calls = {"gcn_aggregate": measure(
+        lambda: check(L.tfg_gcn_aggregate_sum(P(csr.rowptr), P(csr.col), P(dinv), None, P(x),
+                                              tfg.TFG_F32, n, f, 0, 1.0, P(hh), sp)),
+        e * f, 4 * e + 4 * (n + 1) + 4 * n + 8 * n * f, 100)}
+    for red in ("sum", "mean", "max"):
+        calls[f"pool_{red}"] = measure(
+            lambda red=red: check(L.tfg_segment_pool(P(hh), tfg.TFG_F32, P(batch), n, g, f,
+                                                     tfg.REDUCERS[red], P(pooled), P(st), sp)),
+            n * f, 4 * n * f + 8 * n + 4 * g * f, 100)
+    torch.cuda.synchronize()
+    if int(st.item()) != 0:
+        raise RuntimeError("pooling status word set on the molecule batch")
+    out["molecules_1024_gcn_pool"] = {"workload": "1,024 graphs of 20-200 nodes (avg degree 4 + "
+                                      "self-loops), F = 128 fp32", "nodes": n, "edges": e,
+                                      "graphs": g, "calls": calls}
+    return out
+
+
+def gather_floor(L, col, x, e, n, stream) -> dict:
+    """Gather-only floor on the step's own column array and bf16 rows: every
+    row x[col[k]] read once (tfg_gather_xor), inputs hot in L2 as in the
+    step."""
+    import torch
+    from paper_2101_11552_gb300 import tfg
+    P = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
+    sp = ctypes.c_void_p(stream.cuda_stream)
+    row_bytes = x.shape[1] * x.element_size()
+    out = torch.empty(row_bytes // 4, dtype=torch.int32, device=x.device)
+
+    def call():
+        rc = L.tfg_gather_xor(P(col), e, P(x), n, row_bytes, P(out), sp)
+        if rc != 0:
+            raise RuntimeError(f"libtfg error {rc}: {tfg.tfg_last_error()}")
+
+    ms = _event_ms(call, stream, 20)
+    return {"kernel": "gather_xor_kernel", "floor_ms": round(ms, 5), "row_bytes": row_bytes,
+            "gathered_bytes": e * row_bytes,
+            "gather_tbs": round(e * row_bytes / (ms * 1e-3) / 1e12, 2)}
 
 
 def next_rows(L, wl, bufs, stream, hbm_peak):
@@ -418,8 +592,13 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["tfg", "reference"], default="tfg")
     ap.add_argument("--e2e-steps", type=int, default=20)
-    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--ref-edges", type=int, default=SAMPLE_EDGES,
+                    help="edges of the oracle's sample (both CPU baselines)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the four smaller workloads")
+    ap.add_argument("--configs-only", action="store_true",
+                    help="measure only the four smaller workloads")
     ap.add_argument("--pairs", type=int, default=57_300_000, help=argparse.SUPPRESS)
     return ap.parse_args()
 
@@ -429,23 +608,22 @@ def run_reference(args, rank, world):
         return
     from paper_2101_11552_gb300 import graphgen as gg
     wl = gg.make_dcsbm_232965(num_pairs=args.pairs)
-    total_steps = args.steps + args.warmup
-    budget = min(150.0, 0.35 * total_steps)
     import oracle
     oracle.build()
-    units, t, s = time_oracle(wl, budget * args.warmup / total_steps, args.warmup)  # warm-up
-    units, t, s = 0, 0.0, s
-    for _ in range(args.steps):
-        t0 = time.perf_counter()
-        units += oracle_step(s)
-        t += time.perf_counter() - t0
+    # the same fixed sample as the cpu_baseline leg of the GPU arm, unless
+    # K + W steps of it would run past ~3 minutes (about 0.65 us per edge and
+    # step on one core): then a smaller prefix of the same graph
+    budget_edges = int(180.0 / max(args.steps + args.warmup, 1) / 0.65e-6)
+    s = oracle_sample(wl, sample_nodes(wl, min(args.ref_edges, budget_edges)))
+    time_steps(oracle_step, s, args.warmup)
+    units, t = time_steps(oracle_step, s, args.steps)
     value = units / t
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": {"workload": WORKLOAD, "sample": cpu_desc(s)},
             "cpu_baseline": {"kind": "oracle", "cores": 1, "sample": cpu_desc(s), "value": value,
-                             "unit": UNIT},
+                             "unit": UNIT, "host": host_cpu()},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -474,6 +652,12 @@ def main():
         pg = dist
     tfg_build.build_library()
     L = tfg.lib()
+
+    if args.configs_only:   # the four smaller workloads alone (profiling their kernels)
+        peaks = os.path.join(ROOT, "MEASURED_PEAKS.json")
+        hbm = float(json.load(open(peaks)).get("hbm_gbs", 6800.0)) if os.path.exists(peaks) else 6800.0
+        print(json.dumps({"configs": small_configs(L, torch.cuda.current_stream(), hbm)}), flush=True)
+        return
 
     wl = gg.make_dcsbm_232965(num_pairs=args.pairs)
     n, e, f, heads, ch, g = (wl.num_nodes, wl.num_edges, wl.num_features, wl.heads, wl.channels,
@@ -690,6 +874,11 @@ def main():
             "call": dom, "bound": "hbm", "achieved": kernels[dom]["gbs"], "peak": hbm_peak,
             "unit": "GB/s", "frac": round(kernels[dom]["gbs"] / hbm_peak, 4), "traffic": traffic,
             "peak_source": peak_src, "frac_of_nominal_8tbs": round(kernels[dom]["gbs"] / 8000.0, 4)}
+    # the binding roof of the row aggregations: the L2 -> SM row gather
+    floor = gather_floor(L, col, xb, e, n, stream)
+    floor["achieved_frac"] = round(floor["floor_ms"] / kernels[dom]["ms"], 4)
+    floor["gcn_aggregate_frac"] = round(floor["floor_ms"] / kernels["gcn_aggregate"]["ms"], 4)
+    roof["l2_gather"] = floor
     value = units_all / t_max
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -717,10 +906,10 @@ def main():
     }, stream)
     line["next_rows"] = next_rows(L, wl, dict(rowptr=rowptr, col=col, perm=perm, dinv=dinv, xb=xb,
                                               h=h, batch=batch), stream, hbm_peak)
+    if not args.no_configs:
+        line["configs"] = small_configs(L, stream, hbm_peak)
     if world == 1 and not args.no_cpu_baseline:
-        cu, ct, s = time_oracle(wl, args.cpu_budget)
-        line["cpu_baseline"] = {"value": cu / ct, "unit": UNIT, "cores": 1, "kind": "oracle",
-                                "sample": cpu_desc(s), "seconds": round(ct, 2)}
+        line["cpu_baseline"] = cpu_baselines(wl)
     print(json.dumps(line), flush=True)
     if pg:
         dist.destroy_process_group()

@@ -358,6 +358,44 @@ int tfg_edge_softmax_aggregate_noalloc(const int32_t *rowptr, const int32_t *col
                                        float *alpha, tfg_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Backward of the GAT edge-softmax aggregation (tfg_edge_softmax_aggregate):
+ * the gradients of the Fig. 5a workflow with respect to x, a_src and a_dst,
+ * given grad_out = dL/dout (the paper keeps graph construction and
+ * mini-batching differentiable, Sections 2.1.1 and 2.1.3).  With alpha the
+ * forward's weights, e = (s -> t), z = s_src[s,h] + s_dst[t,h]:
+ *   dalpha[e,h] = <grad_out[t,h,:], x[s,h,:]>
+ *   beta[t,h]   = <grad_out[t,h,:], out[t,h,:]>  (= sum over e into t of alpha dalpha)
+ *   dz[e,h]     = alpha (dalpha - beta[t,h]) (z > 0 ? 1 : negative_slope)
+ *   grad_x[s,h,:]  = sum over e out of s of alpha grad_out[t,h,:]
+ *                    + ds_src[s,h] a_src[h,:] + ds_dst[s,h] a_dst[h,:]
+ *   ds_src[s,h] = sum over e out of s of dz;  ds_dst[t,h] = sum over e into t of dz
+ *   grad_a_src[h,c] = sum_v ds_src[v,h] x[v,h,c];  grad_a_dst likewise.
+ *
+ *   rowptr, col: the CSR by target of the forward (tfg_build_csr).
+ *   rowptr_src, col_src: the CSR by source (tfg_build_csr_by_source).
+ *   x, x_dtype, num_nodes, num_edges, heads, channels, a_src, a_dst,
+ *          negative_slope: the forward's arguments.
+ *   out (device) fp32 [num_nodes, H*C]: the forward's output.
+ *   grad_out (device) fp32 [num_nodes, H*C].
+ *   grad_x (device) fp32 [num_nodes, H*C]; grad_a_src, grad_a_dst (device)
+ *          fp32 [H*C]: written.
+ *   workspace >= tfg_edge_softmax_backward_workspace_size() bytes.
+ * Layouts: channels a power of two up to 32, or a multiple of 32; H*C <= 256.
+ * Others return TFG_ERR_INVALID_ARG.  Deterministic (no atomics).
+ * ---------------------------------------------------------------------- */
+int tfg_edge_softmax_backward_workspace_size(int64_t num_nodes, int heads, int channels,
+                                             size_t *bytes);
+int tfg_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t *col,
+                                        const int32_t *rowptr_src, const int32_t *col_src,
+                                        const void *x, int x_dtype, int64_t num_nodes,
+                                        int64_t num_edges, int heads, int channels,
+                                        const float *a_src, const float *a_dst,
+                                        float negative_slope, const float *out,
+                                        const float *grad_out, float *grad_x, float *grad_a_src,
+                                        float *grad_a_dst, void *workspace,
+                                        size_t workspace_bytes, tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * Graph pooling keyed by node_graph_index (Section 2.1.1 BatchGraph; Fig. 2a
  * common graph pooling):
  *   out[g, :] = REDUCE over nodes v with batch[v] == g of x[v, :]
@@ -412,6 +450,27 @@ int tfg_batch_graphs(int64_t num_graphs, const int64_t *node_counts, const int64
                      int64_t *out_edge_index, int64_t *batch, int64_t *node_offsets,
                      void *workspace, size_t workspace_bytes, int32_t *status,
                      tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Gather-only floor (a measurement call; the paper has no counterpart).
+ * The aggregations above read, for every CSR edge, the whole feature row of
+ * its source node (Fig. 1 message aggregation: gather, weight, reduce).  This
+ * call performs only the gather, on the same column array and rows, with
+ * nothing else to compute: every row x[col[k]] for k < num_edges is read
+ * once as 16-byte vectors and the rows are folded with bitwise XOR,
+ *   out[j] = XOR over k of the j-th 32-bit word of x[col[k]].
+ * Its duration is the time the SMs need to pull the gathered rows out of
+ * the memory system, the floor the aggregation kernels are measured
+ * against.  The result is exact and independent of order.
+ *
+ *   col (device) int32 [num_edges], values in [0, num_nodes) (not checked:
+ *        pass a column array from tfg_build_csr).
+ *   x (device) [num_nodes, row_bytes] of any element type, 16-byte aligned.
+ *   row_bytes: 16, 32, 64, 128, 256 or 512 (bytes per row).
+ *   out (device) uint32 [row_bytes / 4], written (zeroed first on stream).
+ * ---------------------------------------------------------------------- */
+int tfg_gather_xor(const int32_t *col, int64_t num_edges, const void *x, int64_t num_nodes,
+                   int64_t row_bytes, uint32_t *out, tfg_stream_t stream);
 
 #ifdef __cplusplus
 }

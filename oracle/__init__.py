@@ -56,6 +56,24 @@ def build(plant: Optional[str] = None, out_dir: Optional[str] = None) -> str:
     return path
 
 
+_SRC_OMP = os.path.join(_HERE, "tfg_oracle_omp.c")
+
+
+def build_omp(out_dir: Optional[str] = None) -> str:
+    """Compile tfg_oracle.c with tfg_oracle_omp.c and -fopenmp (the all-cores
+    CPU baseline: the oracle's row functions on blocks of rows in parallel)."""
+    out_dir = out_dir or _BUILD
+    os.makedirs(out_dir, exist_ok=True)
+    path = os.path.join(out_dir, "liboracle_omp.so")
+    newest = max(os.path.getmtime(_SRC), os.path.getmtime(_SRC_OMP))
+    if (not os.path.exists(path)) or os.path.getmtime(path) < newest:
+        cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-shared", "-fPIC", "-o", path + ".tmp",
+               _SRC, _SRC_OMP, "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(path + ".tmp", path)
+    return path
+
+
 def _load(plant: Optional[str] = None) -> ctypes.CDLL:
     with _lock:
         if plant not in _libs:
@@ -78,6 +96,8 @@ def _load(plant: Optional[str] = None) -> ctypes.CDLL:
                 "oracle_max_argmax": [I64, I64, P, P, P, I64, P, P],
                 "oracle_max_backward": [I64, I64, P, P, P, P, I64, P, P],
                 "oracle_dot_softmax_rows": [I64, P, P, P, P, P, I, I, D, P, I64, P, P, P],
+                "oracle_edge_softmax_backward": [I64, I64, P, P, I, I, P, P, D, P, P, P, P, P,
+                                                 P, P],
             }
             for fn, args in sigs.items():
                 getattr(lib, fn).argtypes = args
@@ -199,6 +219,27 @@ class _Oracle:
             self._p(a_s), self._p(a_d), float(slope), self._p(rows), len(rows), self._p(out),
             self._p(alpha), self._p(ab)))
         return out[:len(rows)], alpha[:total], ab[:len(rows)]
+
+    def edge_softmax_backward(self, edge_index, n, x, heads, channels, a_src, a_dst, slope,
+                              grad_out):
+        """Gradients of edge_softmax's output with respect to x, a_src and a_dst
+        for a given dL/dout.  Returns (grad_x [N, F], grad_a_src [F],
+        grad_a_dst [F], (scale_x, scale_a_src, scale_a_dst))."""
+        ei = np.ascontiguousarray(edge_index, dtype=np.int64)
+        e = ei.shape[1]
+        x = widen(x)
+        g = widen(grad_out)
+        f = x.shape[1]
+        assert f == heads * channels and g.shape == x.shape
+        a_s = np.ascontiguousarray(a_src, np.float64)
+        a_d = np.ascontiguousarray(a_dst, np.float64)
+        gx, ax = np.zeros((max(n, 1), f)), np.zeros((max(n, 1), f))
+        gs, gd, as_, ad = (np.zeros(f) for _ in range(4))
+        self._check(self.lib.oracle_edge_softmax_backward(
+            n, e, self._p(ei), self._p(x), heads, channels, self._p(a_s), self._p(a_d),
+            float(slope), self._p(g), self._p(gx), self._p(gs), self._p(gd), self._p(ax),
+            self._p(as_), self._p(ad)))
+        return gx[:n], gs, gd, (ax[:n], as_, ad)
 
     # -- backward of the aggregation ------------------------------------
     def aggregate_backward(self, edge_index, n, grad_out, reduce, w=None, self_w=None):
@@ -322,6 +363,64 @@ class _Oracle:
         return out[:num_graphs], ab[:num_graphs]
 
 
+class _OmpRows:
+    """The oracle's row functions over all rows, blocks of rows in parallel on
+    every host core (OpenMP).  A CPU baseline for the benchmark; the values
+    equal those of the single-threaded row functions."""
+
+    def __init__(self):
+        self._lib = None
+
+    @property
+    def lib(self) -> ctypes.CDLL:
+        with _lock:
+            if self._lib is None:
+                lib = ctypes.CDLL(build_omp())
+                P, I64, I, D = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_double
+                lib.oracle_omp_threads.argtypes = []
+                lib.oracle_omp_aggregate_all.argtypes = [I, I64, P, P, P, P, P, I64, P, P, P]
+                lib.oracle_omp_edge_softmax_all.argtypes = [I64, P, P, P, I, I, P, P, D, P, P]
+                for fn in ("oracle_omp_threads", "oracle_omp_aggregate_all",
+                           "oracle_omp_edge_softmax_all"):
+                    getattr(lib, fn).restype = ctypes.c_int
+                self._lib = lib
+            return self._lib
+
+    def threads(self) -> int:
+        return int(self.lib.oracle_omp_threads())
+
+    def aggregate_all(self, csr, n, x, reduce, w=None, self_w=None):
+        rowptr, col, perm, _ = csr
+        x = widen(x)
+        f = x.shape[1]
+        w = None if w is None else np.ascontiguousarray(w, np.float64)
+        sw = None if self_w is None else np.ascontiguousarray(self_w, np.float64)
+        out = np.zeros((max(n, 1), f))
+        ab = np.zeros((max(n, 1), f))
+        p = _Oracle._p
+        _Oracle._check(self.lib.oracle_omp_aggregate_all(
+            REDUCE[reduce], n, p(rowptr), p(np.ascontiguousarray(col)),
+            p(np.ascontiguousarray(perm)), p(w), p(x), f, p(sw), p(out), p(ab)))
+        return out[:n], ab[:n]
+
+    def edge_softmax_all(self, csr, n, x, heads, channels, a_src, a_dst, slope=0.2):
+        rowptr, col, _, _ = csr
+        x = widen(x)
+        f = x.shape[1]
+        a_s = np.ascontiguousarray(a_src, np.float64)
+        a_d = np.ascontiguousarray(a_dst, np.float64)
+        out = np.zeros((max(n, 1), f))
+        ab = np.zeros((max(n, 1), f))
+        p = _Oracle._p
+        _Oracle._check(self.lib.oracle_omp_edge_softmax_all(
+            n, p(rowptr), p(np.ascontiguousarray(col)), p(x), heads, channels, p(a_s), p(a_d),
+            float(slope), p(out), p(ab)))
+        return out[:n], ab[:n]
+
+
+omp_rows = _OmpRows()
+
+
 def batch_graphs(node_counts, edge_counts, edge_index):
     """BatchGraph by the reindexing trick (Section 2.1.1, Fig. 4), one graph
     at a time: node j of graph g becomes offset_g + j with offset_g the number
@@ -400,6 +499,7 @@ aggregate_backward = default.aggregate_backward
 gcn_aggregate_backward = default.gcn_aggregate_backward
 max_argmax = default.max_argmax
 max_backward = default.max_backward
+edge_softmax_backward = default.edge_softmax_backward
 dot_softmax_rows = default.dot_softmax_rows
 sgc = default.sgc
 

@@ -590,6 +590,152 @@ int oracle_dot_softmax_rows(int64_t n, const int32_t *rowptr, const int32_t *col
 }
 
 /* ---------------------------------------------------------------------------
+ * Backward of the GAT edge-softmax aggregation: gradients of the Fig. 5a
+ * workflow with respect to x, a_src and a_dst, given grad_out = dL/dout.
+ * The forward quantities (node scores, z = s_src[s] + s_dst[t], logits
+ * l = LeakyReLU(z), per-target maximum and denominator, alpha) are
+ * recomputed exactly as oracle_edge_softmax forms them.  Then, per edge
+ * e = (s -> t) and head h:
+ *   dalpha[e,h] = sum_c grad_out[t,h,c] x[s,h,c]
+ *   beta[t,h]   = sum over edges e' into t of alpha[e',h] dalpha[e',h]
+ *   dl[e,h]     = alpha[e,h] (dalpha[e,h] - beta[t,h])      (softmax Jacobian)
+ *   dz[e,h]     = dl[e,h] * (z > 0 ? 1 : slope)             (LeakyReLU)
+ *   grad_x[s,h,:]   += alpha[e,h] grad_out[t,h,:]           (weighted sum)
+ *   ds_src[s,h] += dz[e,h];   ds_dst[t,h] += dz[e,h]
+ * and per node v:  grad_x[v,h,c] += ds_src[v,h] a_src[h,c] + ds_dst[v,h] a_dst[h,c],
+ * grad_a_src[h,c] = sum_v ds_src[v,h] x[v,h,c], grad_a_dst likewise.
+ * absout_* run the same recursion on absolute values (|dalpha| = sum |g||x|,
+ * |beta| = sum alpha |dalpha|, |dl| = alpha (|dalpha| + |beta|), ...): the
+ * scale that a tolerance on each gradient is measured against.
+ * ------------------------------------------------------------------------- */
+int oracle_edge_softmax_backward(int64_t n, int64_t e, const int64_t *edge_index, const double *x,
+                                 int h, int c, const double *a_src, const double *a_dst,
+                                 double slope, const double *grad_out, double *grad_x,
+                                 double *grad_a_src, double *grad_a_dst, double *abs_x,
+                                 double *abs_a_src, double *abs_a_dst)
+{
+    if (n < 0 || e < 0 || h <= 0 || c <= 0) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+    for (int64_t i = 0; i < e; ++i)
+        if (src[i] < 0 || src[i] >= n || dst[i] < 0 || dst[i] >= n) return E_RANGE;
+    int64_t f = (int64_t)h * c;
+    size_t nh = (size_t)(n > 0 ? n : 1) * (size_t)h, eh = (size_t)(e > 0 ? e : 1) * (size_t)h;
+    double *s_src = (double *)calloc(nh, sizeof(double));
+    double *s_dst = (double *)calloc(nh, sizeof(double));
+    double *mx = (double *)calloc(nh, sizeof(double));
+    double *den = (double *)calloc(nh, sizeof(double));
+    double *beta = (double *)calloc(nh, sizeof(double));
+    double *abeta = (double *)calloc(nh, sizeof(double));
+    double *ds_src = (double *)calloc(nh, sizeof(double));
+    double *ds_dst = (double *)calloc(nh, sizeof(double));
+    double *as_src = (double *)calloc(nh, sizeof(double));
+    double *as_dst = (double *)calloc(nh, sizeof(double));
+    char *seen = (char *)calloc(nh, 1);
+    double *z = (double *)calloc(eh, sizeof(double));
+    double *alpha = (double *)calloc(eh, sizeof(double));
+    double *dal = (double *)calloc(eh, sizeof(double));
+    double *adal = (double *)calloc(eh, sizeof(double));
+    int rc = OK;
+    if (!s_src || !s_dst || !mx || !den || !beta || !abeta || !ds_src || !ds_dst || !as_src ||
+        !as_dst || !seen || !z || !alpha || !dal || !adal) { rc = E_ARG; goto done; }
+    /* forward: node scores, logits, per-target maximum and denominator, alpha */
+    for (int64_t v = 0; v < n; ++v)
+        for (int hh = 0; hh < h; ++hh) {
+            double a = 0.0, b = 0.0;
+            for (int cc = 0; cc < c; ++cc) {
+                a += x[v * f + hh * c + cc] * a_src[hh * c + cc];
+                b += x[v * f + hh * c + cc] * a_dst[hh * c + cc];
+            }
+            s_src[v * h + hh] = a;
+            s_dst[v * h + hh] = b;
+        }
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            double zz = s_src[src[i] * h + hh] + s_dst[dst[i] * h + hh];
+            z[i * h + hh] = zz;
+            double l = leaky(zz, slope);
+            size_t k = (size_t)dst[i] * h + hh;
+            if (!seen[k] || l > mx[k]) mx[k] = l;
+            seen[k] = 1;
+        }
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            size_t k = (size_t)dst[i] * h + hh;
+            den[k] += exp(leaky(z[i * h + hh], slope) - mx[k]);
+        }
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            size_t k = (size_t)dst[i] * h + hh;
+            alpha[i * h + hh] = exp(leaky(z[i * h + hh], slope) - mx[k]) / den[k];
+        }
+    /* dalpha and beta */
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            double d = 0.0, ad = 0.0;
+            for (int cc = 0; cc < c; ++cc) {
+                double p = grad_out[dst[i] * f + hh * c + cc] * x[src[i] * f + hh * c + cc];
+                d += p;
+                ad += fabs(p);
+            }
+            dal[i * h + hh] = d;
+            adal[i * h + hh] = ad;
+            size_t k = (size_t)dst[i] * h + hh;
+            beta[k] += alpha[i * h + hh] * d;
+            abeta[k] += alpha[i * h + hh] * ad;
+        }
+    for (int64_t k = 0; k < n * f; ++k) { grad_x[k] = 0.0; abs_x[k] = 0.0; }
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            size_t kt = (size_t)dst[i] * h + hh;
+            double al = alpha[i * h + hh];
+#ifdef ORACLE_PLANT_BWD_NO_SOFTMAX_JACOBIAN
+            double dl = al * dal[i * h + hh];                       /* planted: beta dropped */
+#else
+            double dl = al * (dal[i * h + hh] - beta[kt]);
+#endif
+            double adl = al * (adal[i * h + hh] + abeta[kt]);
+            double lk = z[i * h + hh] > 0.0 ? 1.0 : slope;
+            ds_src[src[i] * h + hh] += dl * lk;
+            ds_dst[kt] += dl * lk;
+            as_src[src[i] * h + hh] += adl * fabs(lk);
+            as_dst[kt] += adl * fabs(lk);
+            for (int cc = 0; cc < c; ++cc) {
+                double m = al * grad_out[dst[i] * f + hh * c + cc];
+                grad_x[src[i] * f + hh * c + cc] += m;
+                abs_x[src[i] * f + hh * c + cc] += SCALE_TERM(m);
+            }
+        }
+    for (int64_t v = 0; v < n; ++v)
+        for (int hh = 0; hh < h; ++hh)
+            for (int cc = 0; cc < c; ++cc) {
+                size_t k = (size_t)v * h + hh;
+                double m1 = ds_src[k] * a_src[hh * c + cc], m2 = ds_dst[k] * a_dst[hh * c + cc];
+                grad_x[v * f + hh * c + cc] += m1 + m2;
+                abs_x[v * f + hh * c + cc] += as_src[k] * fabs(a_src[hh * c + cc]) +
+                                              as_dst[k] * fabs(a_dst[hh * c + cc]);
+            }
+    for (int64_t k = 0; k < f; ++k) {
+        grad_a_src[k] = grad_a_dst[k] = 0.0;
+        abs_a_src[k] = abs_a_dst[k] = 0.0;
+    }
+    for (int64_t v = 0; v < n; ++v)
+        for (int hh = 0; hh < h; ++hh)
+            for (int cc = 0; cc < c; ++cc) {
+                size_t k = (size_t)v * h + hh;
+                double xv = x[v * f + hh * c + cc];
+                grad_a_src[hh * c + cc] += ds_src[k] * xv;
+                grad_a_dst[hh * c + cc] += ds_dst[k] * xv;
+                abs_a_src[hh * c + cc] += as_src[k] * fabs(xv);
+                abs_a_dst[hh * c + cc] += as_dst[k] * fabs(xv);
+            }
+done:
+    free(s_src); free(s_dst); free(mx); free(den); free(beta); free(abeta); free(ds_src);
+    free(ds_dst); free(as_src); free(as_dst); free(seen); free(z); free(alpha); free(dal);
+    free(adal);
+    return rc;
+}
+
+/* ---------------------------------------------------------------------------
  * Backward of the aggregation: the gradient with respect to x of the
  * aggregation out[t] = sum over edges e = (s -> t) of w_e x[s] (sum), the
  * same divided by the number of edges into t (mean), or with the GCN weights

@@ -162,8 +162,8 @@ struct Agg {
             int c = 0;
             float ww = 1.f;
             if (lane < cnt) {
-                c = __ldg(a.col + base + lane);
-                if (a.w) ww = __ldg(a.w + base + lane);
+                c = ld_stream(a.col + base + lane);
+                if (a.w) ww = ld_stream(a.w + base + lane);
                 else if (kGcnLike) ww = __ldg(a.dinv + c);
             }
             if constexpr (kIsMax) {
@@ -335,9 +335,275 @@ __global__ void __launch_bounds__(kAggThreads, VEC >= 8 ? TFG_AGG_MINB : 4) aggr
     for (int h = 0; h < nh; ++h) A::cta_row(a, s_heavy[h], s_part);
 }
 
+// ---------------------------------------------------------------------------
+// Merge-path kernel for rows that fit one feature tile (F <= LPR * VEC).
+//
+//  * A persistent grid of mp_blocks CTAs per SM.  CTA b owns whole rows, an
+//    equal share of rows + edges (balanced_rows).  Inside the CTA the same
+//    split is made again at the granularity of edges: warp w takes the
+//    items [qa, qb) of the CTA's merge coordinates Q(t) = rowptr[t] + t, so
+//    each warp gets an equal number of edges + row ends whatever the degree
+//    distribution, and a hub row is shared by as many warps as it needs.
+//  * A warp walks its range row by row in chunks of up to 32 edges; the next
+//    chunk's column ids are loaded before this chunk's rows are gathered,
+//    kMpDepth 16-byte gathers are in flight per lane.
+//  * A row that a warp finishes is written at once, unless earlier warps hold
+//    parts of it: then its owner (the warp holding its last edge) parks its
+//    own part in shared memory, and after the CTA's one barrier adds the
+//    earlier warps' parts and its own in warp order and writes the row.  No
+//    global scratch, one barrier per CTA, a fixed summation order.
+// ---------------------------------------------------------------------------
+#ifndef TFG_AGG_MP
+#define TFG_AGG_MP 1       // 0: every layout takes aggregate_kernel (for side-by-side timing)
+#endif
+// Measured on the 114.6M-edge graph (bf16, F = 128, ids and weights staged in
+// shared memory): GCN 1.82 ms at 4 CTAs per SM and 4 gathers in flight per
+// lane (3 CTAs and 8 in flight: 1.84 ms; 2 CTAs and 16: 2.06 ms; the
+// row-per-warp aggregate_kernel: 1.95 ms); max 2.84 ms (aggregate_kernel
+// 3.34 ms).  fp32 rows (512 bytes, one row per warp load) stay on
+// aggregate_kernel: 2.99 ms there against 3.10-3.50 ms here.
+#ifndef TFG_MP_BLOCKS
+#define TFG_MP_BLOCKS 4    // resident CTAs per SM for sums (64 registers per thread)
+#endif
+#ifndef TFG_MP_DEPTH
+#define TFG_MP_DEPTH 4     // 16-byte gathers in flight per lane for sums
+#endif
+template <bool IS_MAX>
+constexpr int mp_blocks() { return IS_MAX ? 4 : TFG_MP_BLOCKS; }
+template <int VEC, bool IS_MAX>
+constexpr int mp_depth() { return IS_MAX ? 4 : TFG_MP_DEPTH; }
+
+
+template <typename XT, int VEC, int LPR, int KIND, typename X0T>
+struct MpAgg {
+    using A = Agg<XT, VEC, LPR, KIND, X0T>;
+    using V = VecLoad<XT, VEC>;
+    static constexpr int G = 32 / LPR;
+    static constexpr int kSlots = 32 / G;                       // edges of a group per chunk
+    static constexpr int kDepth = kSlots < mp_depth<VEC, A::kIsMax>() ? kSlots
+                                                                      : mp_depth<VEC, A::kIsMax>();
+    static constexpr int kF = LPR * VEC;
+    static_assert(G * kDepth <= 32, "a batch must stay inside one 32-edge chunk");
+
+    // Write the finished row t from the lane groups' reduced accumulator.
+    static __device__ __forceinline__ void store_row(const AggArgs &a, int64_t t,
+                                                     const float (&acc)[VEC], int64_t f0,
+                                                     bool fok, int lane) {
+        if (lane >= LPR || !fok) return;
+        const int64_t deg = static_cast<int64_t>(a.rowptr[t + 1]) - a.rowptr[t];
+        const float dt = A::kGcnLike ? __ldg(a.dinv + t) : 1.f;
+        float xt[VEC], x0t[VEC];
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) xt[q] = x0t[q] = 0.f;
+        if (A::kGcnLike && a.add_self)
+            V::load(static_cast<const XT *>(a.x) + t * a.f + f0, xt);
+        if (KIND == kAppnp)
+            VecLoad<X0T, VEC>::load(static_cast<const X0T *>(a.x0) + t * a.f + f0, x0t);
+        float *o = a.out + t * a.f + f0;
+        float r[VEC];
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) r[q] = A::finish(a, t, deg, acc[q], xt[q], dt, x0t[q]);
+        if constexpr (VEC % 4 == 0) {
+#pragma unroll
+            for (int q = 0; q < VEC; q += 4)
+                *reinterpret_cast<float4 *>(o + q) = make_float4(r[q], r[q + 1], r[q + 2], r[q + 3]);
+        } else {
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) o[q] = r[q];
+        }
+    }
+
+    // Row slice of node src: byte offsets (one wide multiply-add per gather).
+    static __device__ __forceinline__ typename V::Raw gather(const char *xb, uint32_t row_bytes,
+                                                            uint32_t src) {
+        return V::raw(reinterpret_cast<const XT *>(xb + static_cast<uint64_t>(src) * row_bytes));
+    }
+
+    // Slot of edge k of a chunk in the warp's staging buffer: each lane group's
+    // edges k = i * G + g sit at g * kSlots + i, so a group reads the
+    // (id, weight) pairs of two consecutive edges with one 16-byte load.
+    static __device__ __forceinline__ int stage_slot(int k) { return (k % G) * kSlots + k / G; }
+
+    // One chunk of a sum: edges [k, k + cnt) of one row.  Lane j stages the id
+    // and weight of edge k + j (weight 0 past cnt, so those slots add an exact
+    // zero from a valid row); each group then reads its edges' pairs two at a
+    // time from shared memory instead of two shuffles per edge.
+    static __device__ __forceinline__ void chunk_sum(const char *xb, uint32_t row_bytes,
+                                                     float2 *stage, int c, float ww, int cnt,
+                                                     int lane, int g, float (&part)[VEC]) {
+        __syncwarp();                                      // the previous chunk's reads are done
+        stage[stage_slot(lane)] = make_float2(__int_as_float(c), lane < cnt ? ww : 0.f);
+        __syncwarp();
+        const float4 *mine = reinterpret_cast<const float4 *>(stage + g * kSlots);
+#pragma unroll
+        for (int j = 0; j < kSlots; j += kDepth) {
+            if (j * G >= cnt) break;                       // warp-uniform
+            typename V::Raw raw[kDepth];
+            float wt[kDepth];
+#pragma unroll
+            for (int u = 0; u < kDepth; u += 2) {
+                const float4 cw = mine[(j + u) / 2];       // (id, w) of slots j + u, j + u + 1
+                raw[u] = gather(xb, row_bytes, static_cast<uint32_t>(__float_as_int(cw.x)));
+                raw[u + 1] = gather(xb, row_bytes, static_cast<uint32_t>(__float_as_int(cw.z)));
+                wt[u] = cw.y;
+                wt[u + 1] = cw.w;
+            }
+#pragma unroll
+            for (int u = 0; u < kDepth; ++u) A::axpy(part, wt[u], raw[u]);
+        }
+    }
+
+    // One chunk of a max: edges [k, k + cnt) of one row, column ids in c
+    // (lane j holds the id of edge k + j), per-edge weights in ww.
+    static __device__ __forceinline__ void chunk(const XT *xf, uint32_t fs, int c, float ww,
+                                                 int cnt, int g, bool fok, float (&part)[VEC]) {
+#pragma unroll
+        for (int j = 0; j < kSlots; j += kDepth) {
+            if (j * G >= cnt) break;                       // warp-uniform
+            typename V::Raw raw[kDepth];
+#pragma unroll
+            for (int u = 0; u < kDepth; ++u) {
+                const int k = (j + u) * G + g;
+                const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k));
+                raw[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
+            }
+#pragma unroll
+            for (int u = 0; u < kDepth; ++u) {
+                const int k = (j + u) * G + g;
+                float wt = __shfl_sync(kFull, ww, k);   // ww = 1 without weights
+                if constexpr (A::kIsMax) {
+                    if (k < cnt && fok) {
+                        float v[VEC];
+                        V::widen(raw[u], v);
+#pragma unroll
+                        for (int q = 0; q < VEC; ++q) part[q] = fmaxf(part[q], wt * v[q]);
+                    }
+                } else {
+                    if (k >= cnt) wt = 0.f;
+                    A::axpy(part, wt, raw[u]);
+                }
+            }
+        }
+    }
+};
+
+template <typename XT, int VEC, int LPR, int KIND, typename X0T>
+__global__ void __launch_bounds__(kAggThreads, mp_blocks<KIND == kMax>()) aggregate_mp_kernel(AggArgs a) {
+    using M = MpAgg<XT, VEC, LPR, KIND, X0T>;
+    using A = typename M::A;
+    constexpr int kF = M::kF;
+    __shared__ float s_tail[kAggWarps][kF];    // each warp's part of its last, unfinished row
+    __shared__ float s_head[kAggWarps][kF];    // an owner's own part of a row begun by others
+    __shared__ int32_t s_tail_row[kAggWarps], s_head_row[kAggWarps];
+    __shared__ __align__(16) float2 s_stage[kAggWarps][32];   // a chunk's (id, weight) pairs
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = lane / LPR, sub = lane % LPR;
+    const int64_t f0 = static_cast<int64_t>(sub) * VEC;
+    const bool fok = f0 < a.f;
+    const XT *xf = static_cast<const XT *>(a.x) + (fok ? f0 : 0);
+    const uint32_t fs = static_cast<uint32_t>(a.f);
+    const char *xb = reinterpret_cast<const char *>(xf);
+    const uint32_t row_bytes = fs * static_cast<uint32_t>(sizeof(XT));
+
+    // node ids and edge positions fit int32 (the ABI caps N and E below 2^31)
+    int64_t r0l, r1l;
+    balanced_rows(a.rowptr, a.n, gridDim.x, blockIdx.x, r0l, r1l);
+    const int32_t r0 = static_cast<int32_t>(r0l), r1 = static_cast<int32_t>(r1l);
+    const int64_t q0 = static_cast<int64_t>(__ldg(a.rowptr + r0)) + r0;
+    const int64_t q1 = static_cast<int64_t>(__ldg(a.rowptr + r1)) + r1;
+    const int64_t per = (q1 - q0 + kAggWarps - 1) / kAggWarps;
+    const int64_t qa = min64(q1, q0 + warp * per), qb = min64(q1, qa + per);
+    const int32_t ta = last_row_at(a.rowptr, r0, r1, qa);
+    const int32_t tb = last_row_at(a.rowptr, ta, r1, qb);
+    const int32_t ka = static_cast<int32_t>(qa - ta), kb = static_cast<int32_t>(qb - tb);
+    const bool head_split = ka > __ldg(a.rowptr + ta);   // row ta begun by an earlier warp
+    if (lane == 0) s_head_row[warp] = -1;
+
+    float acc[VEC];
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) acc[q] = A::identity();
+    int32_t t = ta, k = ka;                            // this warp's edges are [ka, kb)
+    int32_t rend = t < tb ? __ldg(a.rowptr + t + 1) : kb;
+    int cnext = (k + lane < kb) ? __ldg(a.col + k + lane) : 0;
+    for (;;) {
+        while (k >= rend) {                            // row t has no edges left here
+            if (t >= tb) break;
+            A::reduce_groups(acc);
+            if (t == ta && head_split) {               // parts of it sit with earlier warps
+                if (lane < LPR) {
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q) s_head[warp][sub * VEC + q] = acc[q];
+                }
+                if (lane == 0) s_head_row[warp] = t;
+            } else {
+                M::store_row(a, t, acc, f0, fok, lane);
+            }
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] = A::identity();
+            ++t;
+            rend = t < tb ? __ldg(a.rowptr + t + 1) : kb;
+        }
+        if (k >= rend) break;                          // t == tb and its edges are done
+        const int cnt = min(32, rend - k);
+        const int c = cnext;
+        float ww = 1.f;
+        if (lane < cnt) {
+            if (a.w) ww = __ldg(a.w + k + lane);
+            else if (A::kGcnLike) ww = __ldg(a.dinv + c);
+        }
+        const int32_t kn = k + cnt;                    // the next chunk starts here
+        cnext = (kn + lane < kb) ? __ldg(a.col + kn + lane) : 0;
+        float part[VEC];
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) part[q] = A::identity();
+        if constexpr (A::kIsMax) M::chunk(xf, fs, c, ww, cnt, g, fok, part);
+        else M::chunk_sum(xb, row_bytes, s_stage[warp], c, ww, cnt, lane, g, part);
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) acc[q] = A::combine(acc[q], part[q]);
+        k = kn;
+    }
+    // the part of row tb held here (empty when the range ends on a row end)
+    A::reduce_groups(acc);
+    if (lane < LPR) {
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) s_tail[warp][sub * VEC + q] = acc[q];
+    }
+    if (lane == 0) s_tail_row[warp] = tb;
+    __syncthreads();
+    const int32_t hr = s_head_row[warp];
+    if (hr >= 0) {                                     // earlier parts in warp order, then ours
+        float r[VEC];
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) r[q] = A::identity();
+        if (lane < LPR) {
+            for (int w = 0; w < warp; ++w) {
+                if (s_tail_row[w] != hr) continue;
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) r[q] = A::combine(r[q], s_tail[w][sub * VEC + q]);
+            }
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) r[q] = A::combine(r[q], s_head[warp][sub * VEC + q]);
+        }
+        M::store_row(a, hr, r, f0, fok, lane);
+    }
+}
+
 template <typename XT, int VEC, int KIND, typename X0T = XT>
 cudaError_t launch_lpr(const AggArgs &a, int lpr, cudaStream_t s) {
     // E is not known on the host; the kernel reads rowptr[N] for the split.
+    // 16-byte bf16 slices in one feature tile: the merge-path kernel
+    if constexpr (sizeof(XT) == 2 && VEC == 8) {
+        if (TFG_AGG_MP && static_cast<int64_t>(lpr) * VEC >= a.f) {
+            const int grid = static_cast<int>(
+                min64(a.n, static_cast<int64_t>(sm_count()) * mp_blocks<KIND == kMax>()));
+            switch (lpr) {
+                case 32: aggregate_mp_kernel<XT, VEC, 32, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
+                case 16: aggregate_mp_kernel<XT, VEC, 16, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
+                default: aggregate_mp_kernel<XT, VEC, 8, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
+            }
+            return cudaGetLastError();
+        }
+    }
     const int grid = balanced_grid(a.n, 0, 1);
     switch (lpr) {
         case 32: aggregate_kernel<XT, VEC, 32, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;

@@ -116,7 +116,7 @@ int propagate_common(const char *fn, const int32_t *rowptr, const int32_t *col, 
 }  // namespace
 
 namespace tfg {
-int balanced_grid(int64_t n, int64_t e, int64_t min_work) {
+int sm_count() {
     thread_local int sms = 0, sms_dev = -1;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) dev = 0;
@@ -125,6 +125,11 @@ int balanced_grid(int64_t n, int64_t e, int64_t min_work) {
             sms = 148;
         sms_dev = dev;
     }
+    return sms;
+}
+
+int balanced_grid(int64_t n, int64_t e, int64_t min_work) {
+    const int sms = sm_count();
     const int64_t by_work = (n + e + min_work - 1) / min_work;
     const int64_t cap = int64_t(sms) * 16;
     const int64_t g = by_work < cap ? by_work : cap;
@@ -392,6 +397,59 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
                        fn);
 }
 
+int tfg_edge_softmax_backward_workspace_size(int64_t num_nodes, int heads, int channels,
+                                             size_t *bytes) {
+    const char *fn = "tfg_edge_softmax_backward_workspace_size";
+    TFG_NEED(bytes, true, fn, "bytes");
+    TFG_TRY(check_counts(fn, num_nodes, 0));
+    if (!tfg::attention_backward_layout_ok(heads, channels))
+        return fail(TFG_ERR_INVALID_ARG,
+                    "%s: channels must be a power of two up to 32 or a multiple of 32, H*C <= 256",
+                    fn);
+    *bytes = tfg::attention_backward_workspace_bytes(num_nodes, heads, channels);
+    return ok();
+}
+
+int tfg_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t *col,
+                                        const int32_t *rowptr_src, const int32_t *col_src,
+                                        const void *x, int x_dtype, int64_t num_nodes,
+                                        int64_t num_edges, int heads, int channels,
+                                        const float *a_src, const float *a_dst,
+                                        float negative_slope, const float *out,
+                                        const float *grad_out, float *grad_x, float *grad_a_src,
+                                        float *grad_a_dst, void *workspace,
+                                        size_t workspace_bytes, tfg_stream_t stream) {
+    const char *fn = "tfg_edge_softmax_aggregate_backward";
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    if (!tfg::attention_backward_layout_ok(heads, channels))
+        return fail(TFG_ERR_INVALID_ARG,
+                    "%s: channels must be a power of two up to 32 or a multiple of 32, H*C <= 256",
+                    fn);
+    TFG_TRY(check_features(fn, num_nodes, int64_t(heads) * channels));
+    TFG_TRY(check_dtype(fn, x_dtype));
+    TFG_NEED(rowptr, true, fn, "rowptr");
+    TFG_NEED(rowptr_src, true, fn, "rowptr_src");
+    TFG_NEED(col, num_edges > 0, fn, "col");
+    TFG_NEED(col_src, num_edges > 0, fn, "col_src");
+    TFG_NEED(x, num_nodes > 0, fn, "x");
+    TFG_NEED(out, num_nodes > 0, fn, "out");
+    TFG_NEED(grad_out, num_nodes > 0, fn, "grad_out");
+    TFG_NEED(grad_x, num_nodes > 0, fn, "grad_x");
+    TFG_NEED(a_src, true, fn, "a_src");
+    TFG_NEED(a_dst, true, fn, "a_dst");
+    TFG_NEED(grad_a_src, true, fn, "grad_a_src");
+    TFG_NEED(grad_a_dst, true, fn, "grad_a_dst");
+    const size_t need = tfg::attention_backward_workspace_bytes(num_nodes, heads, channels);
+    if (workspace == nullptr || workspace_bytes < need)
+        return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
+                    workspace ? workspace_bytes : size_t(0));
+    return cuda_result(tfg::launch_edge_softmax_backward(
+                           rowptr, col, rowptr_src, col_src, x, x_dtype, num_nodes, heads,
+                           channels, a_src, a_dst, negative_slope, out, grad_out, grad_x,
+                           grad_a_src, grad_a_dst, workspace, reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
 int tfg_dot_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const void *q,
                                    const void *k, const void *v, int x_dtype, int64_t num_nodes,
                                    int64_t num_edges, int heads, int channels, float scale,
@@ -535,6 +593,23 @@ int tfg_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n
     return cuda_result(tfg::launch_segment_pool(x, x_dtype, batch, num_nodes, num_graphs,
                                                 num_features, reduce, out, status,
                                                 reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+int tfg_gather_xor(const int32_t *col, int64_t num_edges, const void *x, int64_t num_nodes,
+                   int64_t row_bytes, uint32_t *out, tfg_stream_t stream) {
+    const char *fn = "tfg_gather_xor";
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    if (row_bytes < 16 || row_bytes > 512 || (row_bytes & (row_bytes - 1)) != 0)
+        return fail(TFG_ERR_INVALID_ARG, "%s: row_bytes must be a power of two in [16, 512] (%lld)",
+                    fn, (long long)row_bytes);
+    TFG_NEED(col, num_edges > 0, fn, "col");
+    TFG_NEED(x, num_edges > 0, fn, "x");
+    TFG_NEED(out, true, fn, "out");
+    if (reinterpret_cast<uintptr_t>(x) % 16 != 0)
+        return fail(TFG_ERR_INVALID_ARG, "%s: x must be 16-byte aligned", fn);
+    return cuda_result(tfg::launch_gather_xor(col, num_edges, x, row_bytes, out,
+                                              reinterpret_cast<cudaStream_t>(stream)),
                        fn);
 }
 

@@ -126,8 +126,8 @@ struct MaxFwd {
         for (int64_t base = k0; base < k1; base += 32) {
             const int cnt = static_cast<int>(min64(32, k1 - base));
             const bool mine = lane < cnt;
-            const int c = mine ? __ldg(a.col + base + lane) : 0;
-            const float wc = a.w ? (mine ? __ldg(a.w + base + lane) : 0.f) : 1.f;
+            const int c = mine ? ld_stream(a.col + base + lane) : 0;
+            const float wc = a.w ? (mine ? ld_stream(a.w + base + lane) : 0.f) : 1.f;
             for (int j = 0; j < cnt; j += G * kMxUnroll) {
                 typename V::Raw raw[kMxUnroll];
 #pragma unroll
@@ -211,7 +211,7 @@ struct MaxBwd {
         for (int64_t base = k0; base < k1; base += 32) {
             const int cnt = static_cast<int>(min64(32, k1 - base));
             const bool mine = lane < cnt;
-            const int c = mine ? __ldg(a.col + base + lane) : 0;
+            const int c = mine ? ld_stream(a.col + base + lane) : 0;
             const int32_t ec = mine ? __ldg(a.perm + base + lane) : 0;
             const float wc = a.w ? (mine ? __ldg(a.w + ec) : 0.f) : 1.f;
             for (int k = 0; k < cnt; ++k) {

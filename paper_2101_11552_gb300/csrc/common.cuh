@@ -19,6 +19,52 @@ __device__ __forceinline__ void set_status(int32_t *status, int32_t code) {
 __device__ __forceinline__ float bf16_lo(uint32_t packed) { return __uint_as_float(packed << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t packed) { return __uint_as_float(packed & 0xffff0000u); }
 
+// L2 residency of the two kinds of data the aggregation kernels read: the
+// CSR column array is streamed once per call, the gathered feature rows are
+// reused by every edge that names them.  TFG_L2_HINTS=1 marks the stream
+// evict-first (and keeps it out of L1) and the rows evict-last; measured on
+// GB300 the policy loads slowed the row gather (1.16 -> 1.30 ms for the
+// 114.6M-edge gather) and the GCN kernel, so the default is plain loads.
+#ifndef TFG_L2_HINTS
+#define TFG_L2_HINTS 0
+#endif
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+    uint64_t p;
+    asm("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+    uint64_t p;
+    asm("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+// One element of a streamed index array (col, CSR-order weights).
+__device__ __forceinline__ int32_t ld_stream(const int32_t *p) {
+#if TFG_L2_HINTS
+    int32_t v;
+    asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.b32 %0, [%1], %2;"
+                 : "=r"(v) : "l"(p), "l"(l2_policy_evict_first()));
+    return v;
+#else
+    return __ldg(p);
+#endif
+}
+__device__ __forceinline__ float ld_stream(const float *p) {
+    return __int_as_float(ld_stream(reinterpret_cast<const int32_t *>(p)));
+}
+// A 16-byte slice of a gathered row.
+__device__ __forceinline__ uint4 ld_row16(const void *p) {
+#if TFG_L2_HINTS
+    uint4 v;
+    asm volatile("ld.global.nc.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p), "l"(l2_policy_evict_last()));
+    return v;
+#else
+    return __ldg(reinterpret_cast<const uint4 *>(p));
+#endif
+}
+
 // VEC consecutive features of one row: a raw load (kept packed in registers
 // while the load is in flight) and its widening to fp32.
 template <typename XT, int VEC> struct VecLoad;
@@ -26,7 +72,9 @@ template <typename XT, int VEC> struct VecLoad;
 template <> struct VecLoad<float, 4> {
     using Raw = float4;
     static __device__ __forceinline__ Raw raw(const float *p) {
-        return __ldg(reinterpret_cast<const float4 *>(p));
+        const uint4 v = ld_row16(p);
+        return make_float4(__uint_as_float(v.x), __uint_as_float(v.y), __uint_as_float(v.z),
+                           __uint_as_float(v.w));
     }
     static __device__ __forceinline__ Raw zero() { return make_float4(0.f, 0.f, 0.f, 0.f); }
     static __device__ __forceinline__ void widen(const Raw &q, float (&v)[4]) {
@@ -43,9 +91,7 @@ template <> struct VecLoad<float, 1> {
 };
 template <> struct VecLoad<uint16_t, 8> {
     using Raw = uint4;
-    static __device__ __forceinline__ Raw raw(const uint16_t *p) {
-        return __ldg(reinterpret_cast<const uint4 *>(p));
-    }
+    static __device__ __forceinline__ Raw raw(const uint16_t *p) { return ld_row16(p); }
     static __device__ __forceinline__ Raw zero() { return make_uint4(0u, 0u, 0u, 0u); }
     static __device__ __forceinline__ void widen(const Raw &q, float (&v)[8]) {
         v[0] = bf16_lo(q.x); v[1] = bf16_hi(q.x);
@@ -112,6 +158,18 @@ __device__ __forceinline__ int64_t first_row_at(const int32_t *rowptr, int64_t n
     return lo;
 }
 
+// Last t in [lo, hi] with rowptr[t] + t <= q (rowptr[lo] + lo <= q holds):
+// the row open at merge coordinate q; q - t is the CSR position reached.
+__device__ __forceinline__ int32_t last_row_at(const int32_t *rowptr, int32_t lo, int32_t hi,
+                                               int64_t q) {
+    while (lo < hi) {
+        const int32_t mid = lo + (hi - lo + 1) / 2;
+        if (static_cast<int64_t>(__ldg(rowptr + mid)) + mid <= q) lo = mid;
+        else hi = mid - 1;
+    }
+    return lo;
+}
+
 __device__ __forceinline__ void balanced_rows(const int32_t *rowptr, int64_t n, int64_t nb,
                                               int64_t b, int64_t &r0, int64_t &r1) {
     const int64_t total = static_cast<int64_t>(__ldg(rowptr + n)) + n;
@@ -126,6 +184,7 @@ __device__ __forceinline__ void balanced_rows(const int32_t *rowptr, int64_t n, 
 // several resident CTAs per SM, and at least min_work units of work each.
 namespace tfg {
 int balanced_grid(int64_t n, int64_t e, int64_t min_work);
+int sm_count();   // multiprocessors of the current device
 }
 
 // Host-side launchers implemented in the kernel files; api.cu validates
@@ -177,6 +236,17 @@ cudaError_t launch_batch_graphs(int64_t g, const int64_t *node_counts, const int
                                 void *ws, int32_t *status, cudaStream_t s);
 int64_t noalloc_softmax_max_node_heads();
 cudaError_t noalloc_softmax_scratch(void **ptr, size_t *bytes);
+bool attention_backward_layout_ok(int heads, int channels);
+size_t attention_backward_workspace_bytes(int64_t n, int heads, int channels);
+cudaError_t launch_edge_softmax_backward(const int32_t *rowptr, const int32_t *col,
+                                         const int32_t *rowptr_src, const int32_t *col_src,
+                                         const void *x, int x_dtype, int64_t n, int heads,
+                                         int channels, const float *a_src, const float *a_dst,
+                                         float slope, const float *out, const float *grad_out,
+                                         float *grad_x, float *grad_a_src, float *grad_a_dst,
+                                         void *ws, cudaStream_t s);
+cudaError_t launch_gather_xor(const int32_t *col, int64_t e, const void *x, int64_t row_bytes,
+                              uint32_t *out, cudaStream_t s);
 cudaError_t launch_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n,
                                 int64_t g, int64_t f, int reduce, float *out, int32_t *status,
                                 cudaStream_t s);

@@ -156,7 +156,7 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh_arg, int64
         // one 32-edge chunk; FULL chunks (all 32 slots used) skip every slot test
         auto chunk = [&](auto full_tag, int64_t base, int cnt) {
             constexpr bool FULL = decltype(full_tag)::value;
-            const int c = (FULL || lane < cnt) ? __ldg(a.col + base + lane) : 0;
+            const int c = (FULL || lane < cnt) ? ld_stream(a.col + base + lane) : 0;
             float den_part = 0.f, part[VEC];
 #pragma unroll
             for (int q = 0; q < VEC; ++q) part[q] = 0.f;
@@ -276,7 +276,7 @@ __device__ __forceinline__ void dot_general_row(const DotArgs &a, int64_t t, int
         for (int j = 0; j < NCH; ++j) acc[j] = 0.f;
         for (int64_t base = beg; base < end; base += 32) {
             const int cnt = static_cast<int>(min64(32, end - base));
-            const int c = lane < cnt ? __ldg(a.col + base + lane) : 0;
+            const int c = lane < cnt ? ld_stream(a.col + base + lane) : 0;
             float den_part = 0.f, part[NCH];
 #pragma unroll
             for (int j = 0; j < NCH; ++j) part[j] = 0.f;

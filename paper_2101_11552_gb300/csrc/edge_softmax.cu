@@ -38,7 +38,7 @@ namespace {
 
 constexpr int kSmThreads = 256;
 #ifndef TFG_SM_UNROLL
-#define TFG_SM_UNROLL 8   // gathers in flight per lane (tuning knob)
+#define TFG_SM_UNROLL 4   // gathers in flight per lane (tuning knob)
 #endif
 constexpr int kSmUnroll = TFG_SM_UNROLL;   // fast kernel
 #ifndef TFG_SM_FULL_CHUNKS
@@ -123,7 +123,7 @@ __device__ __forceinline__ void generic_row(const int32_t *__restrict__ rowptr,
         for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
         for (int64_t base = beg; base < end; base += 32) {
             const int cnt = static_cast<int>(min64(32, end - base));
-            const int c = lane < cnt ? __ldg(col + base + lane) : 0;
+            const int c = lane < cnt ? ld_stream(col + base + lane) : 0;
             float den_part = 0.f, part[VEC];
 #pragma unroll
             for (int q = 0; q < VEC; ++q) part[q] = 0.f;
@@ -229,8 +229,12 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
     const int f0 = sub * VEC;
     const bool fok = f0 < f;
     const int fh = fok ? f0 / channels : 0;
-    const XT *xf = x + (fok ? f0 : 0);
-    const uint32_t fs = static_cast<uint32_t>(f);
+    const char *xb = reinterpret_cast<const char *>(x + (fok ? f0 : 0));
+    const uint32_t row_bytes = static_cast<uint32_t>(f) * static_cast<uint32_t>(sizeof(XT));
+    // row slice of node src, addressed in bytes (one wide multiply-add per gather)
+    auto gather = [&](uint32_t src) {
+        return V::raw(reinterpret_cast<const XT *>(xb + static_cast<uint64_t>(src) * row_bytes));
+    };
     const int64_t beg = rowptr[t], end = col ? rowptr[t + 1] : rowptr[t];
     const float sd = __ldg(s_dst + t * H + sh);
 
@@ -244,15 +248,13 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
     // one 32-edge chunk; FULL chunks (all 32 slots used) skip every slot test
     auto chunk = [&](auto full_tag, int64_t base, int cnt) {
         constexpr bool FULL = decltype(full_tag)::value;
-        const int c = (FULL || lane < cnt) ? __ldg(col + base + lane) : 0;
+        const int c = (FULL || lane < cnt) ? ld_stream(col + base + lane) : 0;
         // the first step's row gathers need only the column ids: issue them
         // before the scores so that their latency overlaps the score work
         typename V::Raw raw0[kSmUnroll];
 #pragma unroll
-        for (int u = 0; u < kSmUnroll; ++u) {
-            const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, (u * G + g) & 31));
-            raw0[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
-        }
+        for (int u = 0; u < kSmUnroll; ++u)
+            raw0[u] = gather(static_cast<uint32_t>(__shfl_sync(kFull, c, (u * G + g) & 31)));
         float p[R];
         float cm = -CUDART_INF_F;
 #pragma unroll
@@ -297,12 +299,8 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
                 const int k = k0 + g;
                 // p of (edge k, head fh) sits in lane (k % ES) * H + fh, register k / ES
                 pw[u] = __shfl_sync(kFull, p[k0 / ES], ((k0 % ES) + g) * H + fh);
-                if (e == 0) {
-                    raw[u] = raw0[u];
-                } else {
-                    const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31));
-                    raw[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
-                }
+                if (e == 0) raw[u] = raw0[u];
+                else raw[u] = gather(static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31)));
             }
 #pragma unroll
             for (int u = 0; u < kSmUnroll; ++u) {
@@ -360,6 +358,293 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
     }
 }
 
+// ---------------------------------------------------------------------------
+// Merge-path form of the fast kernel (same layout conditions).  The work is
+// split as in aggregate_mp_kernel: whole rows per CTA, an equal number of
+// edges + row ends per warp inside it, so a hub row is shared by the warps it
+// spans; the next chunk's column ids are loaded before this chunk is
+// gathered.  A warp's part of a row is the running state (m, den, acc) of
+// fast_row; the owner of a row begun by earlier warps merges their parts and
+// its own in warp order after the CTA's one barrier:
+//   m = max(m1, m2),  den = den1 2^(m1 - m) + den2 2^(m2 - m),  acc likewise.
+// ---------------------------------------------------------------------------
+#ifndef TFG_SM_MP
+#define TFG_SM_MP 1          // 0: the fast layout takes softmax_fast (side-by-side timing)
+#endif
+#ifndef TFG_SMP_BLOCKS
+#define TFG_SMP_BLOCKS 3     // resident CTAs per SM
+#endif
+constexpr int kSmpBlocks = TFG_SMP_BLOCKS;
+// Measured: on the 169,343-node graph (mean in-degree 6.9) the merge-path form
+// takes 0.24 ms against 0.26 ms; on the 114.6M-edge graph (mean 492) 3.15 ms
+// against 2.62 ms for softmax_fast, whose per-row work is already balanced
+// by its long rows.  Graphs with a mean in-degree below this take it.
+constexpr int64_t kSmpMaxDegree = 32;
+constexpr int kSmWarps = kSmThreads / 32;
+
+// (M, D, A) absorbs another part (m2, d2, a2) of the same row and head.
+template <int VEC>
+__device__ __forceinline__ void merge_state(float &M, float &D, float (&A)[VEC], float m2,
+                                            float d2, const float *a2) {
+    const float mn = fmaxf(M, m2);
+    const float sa = M == -CUDART_INF_F ? 0.f : exp2f(M - mn);
+    const float sb = m2 == -CUDART_INF_F ? 0.f : exp2f(m2 - mn);
+    D = D * sa + d2 * sb;
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) A[q] = A[q] * sa + (a2 ? a2[q] * sb : 0.f);
+    M = mn;
+}
+
+template <typename XT, int VEC, int LPR, int H>
+struct SmMp {
+    using V = VecLoad<XT, VEC>;
+    static constexpr int G = 32 / LPR;     // edges per feature step
+    static constexpr int ES = 32 / H;      // edges per score step
+    static constexpr int R = 32 / ES;      // score steps per 32-edge chunk (= H)
+    static constexpr int kF = LPR * VEC;
+    static_assert(ES % G == 0, "score step must hold whole feature steps");
+    static_assert(G * kSmUnroll <= 32, "G * kSmUnroll must not exceed the 32-edge chunk");
+
+    // One chunk of up to 32 edges of one row (ids in c, lane j holds edge j):
+    // the logits of the chunk (score lanes), the running maximum, then the
+    // weighted rows (feature lanes), exactly as in fast_row.
+    static __device__ __forceinline__ void chunk(const XT *xf, uint32_t fs,
+                                                 const float *__restrict__ s_src, float sd,
+                                                 float slope, int c, int cnt, int lane, int fh,
+                                                 float &m, float &den, float (&acc)[VEC]) {
+        const int se = lane / H, sh = lane % H, g = lane / LPR;
+        typename V::Raw raw0[kSmUnroll];
+#pragma unroll
+        for (int u = 0; u < kSmUnroll; ++u) {
+            const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, u * G + g));
+            raw0[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
+        }
+        float p[R];
+        float cm = -CUDART_INF_F;
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const int k = r * ES + se;
+            const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k));
+            p[r] = k < cnt ? leaky(__ldg(s_src + static_cast<uint64_t>(src) * H + sh) + sd, slope)
+                           : -CUDART_INF_F;
+            cm = fmaxf(cm, p[r]);
+        }
+#pragma unroll
+        for (int o = H; o < 32; o <<= 1) cm = fmaxf(cm, __shfl_xor_sync(kFull, cm, o));
+        const bool rises = cm > m;
+        if (__any_sync(kFull, rises)) {   // warp-uniform; rare after the first chunks
+            const float sc = rises ? (m == -CUDART_INF_F ? 0.f : exp2f(m - cm)) : 1.f;
+            den *= sc;
+            const float fsc = __shfl_sync(kFull, sc, fh);   // lane fh scores head fh
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] *= fsc;
+            m = fmaxf(m, cm);
+        }
+        float den_part = 0.f;
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const int k = r * ES + se;
+            p[r] = k < cnt ? exp2f(p[r] - m) : 0.f;
+            den_part += p[r];
+        }
+        den += den_part;
+        float part[VEC];
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) part[q] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 32; e += G * kSmUnroll) {
+            if (e >= cnt) break;   // warp-uniform
+            typename V::Raw raw[kSmUnroll];
+            float pw[kSmUnroll];
+#pragma unroll
+            for (int u = 0; u < kSmUnroll; ++u) {
+                const int k0 = e + u * G;              // edge of group 0 in this step
+                // p of (edge k0 + g, head fh) sits in lane ((k0 + g) % ES) * H + fh, register k0 / ES
+                pw[u] = __shfl_sync(kFull, p[k0 / ES], ((k0 % ES) + g) * H + fh);
+                if (e == 0) {
+                    raw[u] = raw0[u];
+                } else {
+                    const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k0 + g));
+                    raw[u] = V::raw(xf + static_cast<uint64_t>(src) * fs);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kSmUnroll; ++u) {
+                float v[VEC];
+                V::widen(raw[u], v);
+                if constexpr (VEC % 2 == 0) {
+                    const float2 w2 = make_float2(pw[u], pw[u]);
+#pragma unroll
+                    for (int q = 0; q < VEC; q += 2) {
+                        const float2 r2 = fma2(make_float2(v[q], v[q + 1]), w2,
+                                               make_float2(part[q], part[q + 1]));
+                        part[q] = r2.x;
+                        part[q + 1] = r2.y;
+                    }
+                } else {
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q) part[q] = fmaf(pw[u], v[q], part[q]);
+                }
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) acc[q] += part[q];
+    }
+
+    // Normalised weights of every edge of row t, given the row's final
+    // maximum M and denominator D of this lane's score head.
+    static __device__ void write_alpha(const int32_t *__restrict__ rowptr,
+                                       const int32_t *__restrict__ col,
+                                       const float *__restrict__ s_src, float sd, float slope,
+                                       float M, float D, float *__restrict__ alpha, int32_t t,
+                                       int lane) {
+        const int se = lane / H, sh = lane % H;
+        const int32_t beg = __ldg(rowptr + t), end = __ldg(rowptr + t + 1);
+        for (int32_t base = beg; base < end; base += 32) {
+            const int cnt = min(32, end - base);
+            const int c = lane < cnt ? __ldg(col + base + lane) : 0;
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                const int k = r * ES + se;
+                const uint32_t src = static_cast<uint32_t>(__shfl_sync(kFull, c, k));
+                if (k < cnt) {
+                    const float l = leaky(__ldg(s_src + static_cast<uint64_t>(src) * H + sh) + sd, slope);
+                    alpha[(static_cast<int64_t>(base) + k) * H + sh] = exp2f(l - M) / D;
+                }
+            }
+        }
+    }
+};
+
+template <typename XT, int VEC, int LPR, int H>
+__global__ void __launch_bounds__(kSmThreads, kSmpBlocks)
+softmax_mp(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,
+           const XT *__restrict__ x, int64_t n, int channels, float slope,
+           const float *__restrict__ s_src, const float *__restrict__ s_dst,
+           float *__restrict__ out, float *__restrict__ alpha) {
+    using S = SmMp<XT, VEC, LPR, H>;
+    constexpr int kF = S::kF;
+    __shared__ float s_tacc[kSmWarps][kF], s_hacc[kSmWarps][kF];
+    __shared__ float s_tm[kSmWarps][H], s_tden[kSmWarps][H], s_hm[kSmWarps][H], s_hden[kSmWarps][H];
+    __shared__ int32_t s_tail_row[kSmWarps], s_head_row[kSmWarps];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int sh = lane % H, sub = lane % LPR;
+    const int f = H * channels;
+    const int f0 = sub * VEC;
+    const bool fok = f0 < f;
+    const int fh = fok ? f0 / channels : 0;
+    const XT *xf = x + (fok ? f0 : 0);
+    const uint32_t fs = static_cast<uint32_t>(f);
+
+    // node ids and edge positions fit int32 (the ABI caps N and E below 2^31)
+    int64_t r0l, r1l;
+    balanced_rows(rowptr, n, gridDim.x, blockIdx.x, r0l, r1l);
+    const int32_t r0 = static_cast<int32_t>(r0l), r1 = static_cast<int32_t>(r1l);
+    const int64_t q0 = static_cast<int64_t>(__ldg(rowptr + r0)) + r0;
+    const int64_t q1 = static_cast<int64_t>(__ldg(rowptr + r1)) + r1;
+    const int64_t per = (q1 - q0 + kSmWarps - 1) / kSmWarps;
+    const int64_t qa = min64(q1, q0 + warp * per), qb = min64(q1, qa + per);
+    const int32_t ta = last_row_at(rowptr, r0, r1, qa);
+    const int32_t tb = last_row_at(rowptr, ta, r1, qb);
+    const int32_t ka = static_cast<int32_t>(qa - ta), kb = static_cast<int32_t>(qb - tb);
+    const bool head_split = ka > __ldg(rowptr + ta);   // row ta begun by an earlier warp
+    if (lane == 0) s_head_row[warp] = -1;
+
+    float m = -CUDART_INF_F, den = 0.f, acc[VEC];
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
+    int32_t t = ta, k = ka;                            // this warp's edges are [ka, kb)
+    int32_t rend = t < tb ? __ldg(rowptr + t + 1) : kb;
+    float sd = t < n ? __ldg(s_dst + static_cast<int64_t>(t) * H + sh) : 0.f;
+    int cnext = (col && k + lane < kb) ? __ldg(col + k + lane) : 0;
+    for (;;) {
+        while (k >= rend) {                            // row t has no edges left here
+            if (t >= tb) break;
+#pragma unroll
+            for (int o = H; o < 32; o <<= 1) den += __shfl_xor_sync(kFull, den, o);
+#pragma unroll
+            for (int o = LPR; o < 32; o <<= 1)
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) acc[q] += __shfl_xor_sync(kFull, acc[q], o);
+            if (t == ta && head_split) {               // parts of it sit with earlier warps
+                if (lane < H) {
+                    s_hm[warp][lane] = m;
+                    s_hden[warp][lane] = den;
+                }
+                if (lane < LPR) {
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q) s_hacc[warp][f0 + q] = acc[q];
+                }
+                if (lane == 0) s_head_row[warp] = t;
+            } else {
+                const float dh = __shfl_sync(kFull, den, fh);   // lane fh: head fh's denominator
+                const bool any = __ldg(rowptr + t + 1) > __ldg(rowptr + t);
+                if (lane < LPR && fok) {
+                    float *o = out + static_cast<int64_t>(t) * f + f0;
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q) o[q] = any ? acc[q] / dh : 0.f;
+                }
+                if (alpha && any) S::write_alpha(rowptr, col, s_src, sd, slope, m, den, alpha, t, lane);
+            }
+            m = -CUDART_INF_F;
+            den = 0.f;
+#pragma unroll
+            for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
+            ++t;
+            rend = t < tb ? __ldg(rowptr + t + 1) : kb;
+            sd = t < n ? __ldg(s_dst + static_cast<int64_t>(t) * H + sh) : 0.f;
+        }
+        if (k >= rend) break;                          // t == tb and its edges are done
+        const int cnt = min(32, rend - k);
+        const int c = cnext;
+        const int32_t kn = k + cnt;                    // the next chunk starts here
+        cnext = (kn + lane < kb) ? __ldg(col + kn + lane) : 0;
+        S::chunk(xf, fs, s_src, sd, slope, c, cnt, lane, fh, m, den, acc);
+        k = kn;
+    }
+    // this warp's part of row tb (empty when the range ends on a row end)
+#pragma unroll
+    for (int o = H; o < 32; o <<= 1) den += __shfl_xor_sync(kFull, den, o);
+#pragma unroll
+    for (int o = LPR; o < 32; o <<= 1)
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) acc[q] += __shfl_xor_sync(kFull, acc[q], o);
+    if (lane < H) {
+        s_tm[warp][lane] = m;
+        s_tden[warp][lane] = den;
+    }
+    if (lane < LPR) {
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) s_tacc[warp][f0 + q] = acc[q];
+    }
+    if (lane == 0) s_tail_row[warp] = tb;
+    __syncthreads();
+    const int32_t hr = s_head_row[warp];
+    if (hr < 0) return;
+    // earlier warps' parts in warp order, then ours: (Ms, Ds) for the score
+    // head sh, (Mf, Df, A) for the feature head fh
+    float Ms = -CUDART_INF_F, Ds = 0.f, Mf = -CUDART_INF_F, Df = 0.f, A[VEC];
+    float none[1] = {0.f};
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) A[q] = 0.f;
+    for (int w = 0; w < warp; ++w) {
+        if (s_tail_row[w] != hr) continue;
+        merge_state<1>(Ms, Ds, none, s_tm[w][sh], s_tden[w][sh], nullptr);
+        merge_state<VEC>(Mf, Df, A, s_tm[w][fh], s_tden[w][fh], &s_tacc[w][fok ? f0 : 0]);
+    }
+    merge_state<1>(Ms, Ds, none, s_hm[warp][sh], s_hden[warp][sh], nullptr);
+    merge_state<VEC>(Mf, Df, A, s_hm[warp][fh], s_hden[warp][fh], &s_hacc[warp][fok ? f0 : 0]);
+    if (lane < LPR && fok) {
+        float *o = out + static_cast<int64_t>(hr) * f + f0;
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) o[q] = A[q] / Df;   // a split row has edges
+    }
+    if (alpha) {
+        const float sdr = __ldg(s_dst + static_cast<int64_t>(hr) * H + sh);
+        S::write_alpha(rowptr, col, s_src, sdr, slope, Ms, Ds, alpha, hr, lane);
+    }
+}
+
 // Each CTA owns a work-balanced range of rows (edges + rows split evenly
 // across CTAs); its warps take rows one at a time from a shared counter.
 template <typename RowFn>
@@ -391,8 +676,15 @@ softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict_
     });
 }
 
+// Measured on the 114.6M-edge graph (bf16, 8 heads x 16): 4 CTAs per SM with
+// 4 gathers in flight per lane 2.50 ms; 3 CTAs with 8 in flight 2.62 ms,
+// 3 with 4 2.57 ms, 4 with 8 2.75 ms, 2 with 8 3.48 ms.
+#ifndef TFG_SMF_BLOCKS
+#define TFG_SMF_BLOCKS 4     // resident CTAs per SM of softmax_fast
+#endif
+
 template <typename XT, int VEC, int LPR, int H>
-__global__ void __launch_bounds__(kSmThreads, 3)
+__global__ void __launch_bounds__(kSmThreads, TFG_SMF_BLOCKS)
 softmax_fast(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,
              const XT *__restrict__ x, int64_t n, int channels, float slope,
              const float *__restrict__ s_src, const float *__restrict__ s_dst,
@@ -415,11 +707,16 @@ bool launch_fast_lpr(const int32_t *rowptr, const int32_t *col, const void *x, i
     constexpr int G = 32 / LPR;
     const int grid = balanced_grid(n, e, kSmMinWork);
     const XT *xp = static_cast<const XT *>(x);
+    const int mp_grid = static_cast<int>(min64(n, static_cast<int64_t>(sm_count()) * kSmpBlocks));
 #define TFG_FAST(HH)                                                                              \
     if (heads == HH) {                                                                            \
         if constexpr ((32 / HH) % G == 0) {                                                       \
-            softmax_fast<XT, VEC, LPR, HH><<<grid, kSmThreads, 0, s>>>(rowptr, col, xp, n, channels, \
-                                                                       slope, s_src, s_dst, out, alpha); \
+            if (TFG_SM_MP && e < kSmpMaxDegree * n)                                              \
+                softmax_mp<XT, VEC, LPR, HH><<<mp_grid, kSmThreads, 0, s>>>(                      \
+                    rowptr, col, xp, n, channels, slope, s_src, s_dst, out, alpha);               \
+            else                                                                                  \
+                softmax_fast<XT, VEC, LPR, HH><<<grid, kSmThreads, 0, s>>>(                       \
+                    rowptr, col, xp, n, channels, slope, s_src, s_dst, out, alpha);               \
             return true;                                                                          \
         }                                                                                         \
         return false;                                                                             \
@@ -497,6 +794,19 @@ cudaError_t noalloc_softmax_scratch(void **ptr, size_t *bytes) {
     *ptr = addr[dev];
     *bytes = sizeof(g_noalloc_scores);
     return cudaSuccess;
+}
+
+cudaError_t launch_node_scores(const void *x, int x_dtype, int64_t n, int heads, int channels,
+                               const float *a_src, const float *a_dst, float *s_src, float *s_dst,
+                               cudaStream_t s) {
+    const int sgrid = ceil_div(n * heads, 256);
+    if (x_dtype == TFG_BF16)
+        node_scores<uint16_t><<<sgrid, 256, 0, s>>>(static_cast<const uint16_t *>(x), n, heads,
+                                                    channels, a_src, a_dst, s_src, s_dst);
+    else
+        node_scores<float><<<sgrid, 256, 0, s>>>(static_cast<const float *>(x), n, heads, channels,
+                                                 a_src, a_dst, s_src, s_dst);
+    return cudaGetLastError();
 }
 
 size_t softmax_workspace_bytes(int64_t n, int heads) {

@@ -81,6 +81,10 @@ def lib() -> ctypes.CDLL:
                 "tfg_segment_pool_meanmax": [P, I, P, I64, I64, I64, P, P, P],
                 "tfg_batch_graphs_workspace_size": [I64, ctypes.POINTER(SZ)],
                 "tfg_batch_graphs": [I64, P, P, P, I64, I64, P, P, P, P, SZ, P, P],
+                "tfg_gather_xor": [P, I64, P, I64, I64, P, P],
+                "tfg_edge_softmax_backward_workspace_size": [I64, I, I, ctypes.POINTER(SZ)],
+                "tfg_edge_softmax_aggregate_backward": [P, P, P, P, P, I, I64, I64, I, I, P, P, F,
+                                                        P, P, P, P, P, P, SZ, P],
             }
             for name, args in sigs.items():
                 fn = getattr(L, name)
@@ -525,3 +529,51 @@ def tfg_batch_graphs(node_counts: torch.Tensor, edge_counts: torch.Tensor,
                                   total_nodes, _ptr(out_ei), _ptr(batch), _ptr(offs), _ptr(ws),
                                   ws.numel(), _ptr(status), _stream(dev)))
     return BatchGraph(out_ei, batch, offs, status)
+
+
+def tfg_gather_xor(col: torch.Tensor, x: torch.Tensor, out=None) -> torch.Tensor:
+    """Gather-only floor: every row x[col[k]] read once and XOR-folded.
+    Returns uint32 words as an int32 tensor [row_bytes / 4]."""
+    _need_cuda("col", col, torch.int32)
+    _need_cuda("x", x)
+    dev = x.device
+    row_bytes = x[0].numel() * x.element_size() if x.shape[0] else 16
+    if out is None:
+        out = torch.empty(row_bytes // 4, dtype=torch.int32, device=dev)
+    _check(lib().tfg_gather_xor(_ptr(col), col.numel(), _ptr(x), x.shape[0], row_bytes, _ptr(out),
+                                _stream(dev)))
+    return out
+
+
+def tfg_edge_softmax_backward_workspace_size(num_nodes: int, heads: int, channels: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().tfg_edge_softmax_backward_workspace_size(num_nodes, heads, channels,
+                                                          ctypes.byref(n)))
+    return n.value
+
+
+def tfg_edge_softmax_aggregate_backward(rowptr, col, rowptr_src, col_src, x, heads: int,
+                                        channels: int, a_src, a_dst, negative_slope: float,
+                                        out, grad_out):
+    """Gradients of tfg_edge_softmax_aggregate with respect to x, a_src and
+    a_dst.  Returns (grad_x [N, H*C], grad_a_src [H*C], grad_a_dst [H*C])."""
+    _need_cuda("x", x)
+    dev = x.device
+    for name, t, dt in (("rowptr", rowptr, torch.int32), ("col", col, torch.int32),
+                        ("rowptr_src", rowptr_src, torch.int32), ("col_src", col_src, torch.int32),
+                        ("a_src", a_src, torch.float32), ("a_dst", a_dst, torch.float32),
+                        ("out", out, torch.float32), ("grad_out", grad_out, torch.float32)):
+        _need_cuda(name, t, dt, dev)
+    n = x.shape[0]
+    f = heads * channels
+    grad_x = torch.empty(n, f, dtype=torch.float32, device=dev)
+    ga_src = torch.empty(f, dtype=torch.float32, device=dev)
+    ga_dst = torch.empty(f, dtype=torch.float32, device=dev)
+    ws = torch.empty(max(tfg_edge_softmax_backward_workspace_size(n, heads, channels), 1),
+                     dtype=torch.uint8, device=dev)
+    _check(lib().tfg_edge_softmax_aggregate_backward(
+        _ptr(rowptr), _ptr(col), _ptr(rowptr_src), _ptr(col_src), _ptr(x), _x_dtype(x), n,
+        col.numel(), heads, channels, _ptr(a_src), _ptr(a_dst), negative_slope, _ptr(out),
+        _ptr(grad_out), _ptr(grad_x), _ptr(ga_src), _ptr(ga_dst), _ptr(ws), ws.numel(),
+        _stream(dev)))
+    return grad_x, ga_src, ga_dst

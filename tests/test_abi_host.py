@@ -204,3 +204,15 @@ def test_backward_rejects(lib):
     assert mb(FAKE, FAKE, None, FAKE, None, FAKE, 10, 4, FAKE, None) == -1              # perm_src
     assert mb(FAKE, FAKE, FAKE, None, None, FAKE, 10, 4, FAKE, None) == -1              # argmax
     assert lib.tfg_build_csr_by_source(None, 10, 5, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20, FAKE, None) == -1
+
+
+def test_gather_xor_rejects(lib):
+    g = lib.tfg_gather_xor
+    assert g(FAKE, 10, FAKE, 5, 48, FAKE, None) == -1            # not a power of two
+    assert "row_bytes" in lib.tfg_last_error().decode()
+    assert g(FAKE, 10, FAKE, 5, 1024, FAKE, None) == -1          # above 512
+    assert g(FAKE, 10, FAKE, 5, 8, FAKE, None) == -1             # below 16
+    assert g(None, 10, FAKE, 5, 256, FAKE, None) == -1
+    assert g(FAKE, 10, FAKE, 5, 256, None, None) == -1
+    assert g(FAKE, 10, ctypes.c_void_p(0x1004), 5, 256, FAKE, None) == -1   # unaligned x
+    assert g(FAKE, 10, FAKE, 1 << 31, 256, FAKE, None) == -2

@@ -3,6 +3,7 @@ reduction of replicas (two gloo ranks on the CPU)."""
 import os
 import socket
 
+import numpy as np
 import pytest
 import torch.distributed as dist
 import torch.multiprocessing as mp
@@ -59,3 +60,21 @@ def test_combine_ranks_two_gloo_ranks():
 
 def test_single_rank_passthrough():
     assert bench.combine_ranks(1.5, 7, 1, None) == (1.5, 7)
+
+
+def test_sample_nodes_is_the_smallest_prefix_with_enough_edges():
+    from paper_2101_11552_gb300 import graphgen as gg
+    wl = gg.make_ba_19717()
+    for target in (1000, 20_000, 90_000, 10 ** 9):
+        k = bench.sample_nodes(wl, target)
+        ei = wl.edge_index
+        inside = lambda m: int(((ei[0] < m) & (ei[1] < m)).sum())  # noqa: E731
+        if target <= wl.num_edges:
+            assert inside(k) >= target > inside(k - 1)
+        else:
+            assert k == wl.num_nodes
+        if k < wl.num_nodes:
+            wl.x_bf16 = np.zeros((wl.num_nodes, 1), np.uint16)
+            wl.batch = np.zeros(wl.num_nodes, np.int64)
+            s = bench.oracle_sample(wl, k)
+            assert s["edge_index"].shape[1] == inside(k) and s["n"] == k

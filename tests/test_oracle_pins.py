@@ -626,6 +626,72 @@ def test_appnp_limits():
 
 
 # ---------------------------------------------------------------------------
+# Backward of the GAT edge softmax
+# ---------------------------------------------------------------------------
+def pin_gat_backward_finite_differences(o):
+    """<grad, u> equals the central difference of <grad_out, forward> along u
+    for each of x, a_src and a_dst, the forward being the independent
+    forward oracle (edge_softmax)."""
+    for seed in range(3):
+        n, e, h, c = [(30, 220, 2, 3), (45, 400, 1, 5), (20, 90, 4, 2)][seed]
+        f = h * c
+        wl = gg.random_edge_case_graph(n, e, f, 150 + seed, hub=1, isolated=3)
+        ei = wl.edge_index
+        rng = np.random.default_rng(150 + seed)
+        x = rng.standard_normal((n, f))
+        a_s, a_d = rng.standard_normal(f), rng.standard_normal(f)
+        g = rng.standard_normal((n, f))
+        gx, gs, gd, _ = o.edge_softmax_backward(ei, n, x, h, c, a_s, a_d, 0.2, g)
+
+        def loss(xx, aa, bb):
+            out, _, _ = oracle.edge_softmax(ei, n, xx, h, c, aa, bb, 0.2)
+            return float(np.sum(out * g))
+        eps = 1e-6
+        ux, ua = rng.standard_normal((n, f)), rng.standard_normal(f)
+        fd = (loss(x + eps * ux, a_s, a_d) - loss(x - eps * ux, a_s, a_d)) / (2 * eps)
+        assert abs(np.sum(gx * ux) - fd) <= 1e-6 * (1 + abs(fd)), ("x", seed)
+        fd = (loss(x, a_s + eps * ua, a_d) - loss(x, a_s - eps * ua, a_d)) / (2 * eps)
+        assert abs(np.sum(gs * ua) - fd) <= 1e-6 * (1 + abs(fd)), ("a_src", seed)
+        fd = (loss(x, a_s, a_d + eps * ua) - loss(x, a_s, a_d - eps * ua)) / (2 * eps)
+        assert abs(np.sum(gd * ua) - fd) <= 1e-6 * (1 + abs(fd)), ("a_dst", seed)
+
+
+def test_gat_backward_finite_differences():
+    pin_gat_backward_finite_differences(oracle.default)
+
+
+def pin_gat_backward_limits(o):
+    """Zero attention vectors make every weight 1/in-degree, so the gradient
+    with respect to x is the mean aggregation's backward (and its scale the
+    mean backward's scale); a single in-edge per target has weight 1 whatever
+    the logits, so the softmax passes no gradient to a_src or a_dst and x's
+    gradient is grad_out routed back along the edge."""
+    n, e, h, c = 40, 300, 2, 4
+    wl = gg.random_edge_case_graph(n, e, h * c, 160, hub=2, isolated=4)
+    ei = wl.edge_index
+    rng = np.random.default_rng(160)
+    x, g = rng.standard_normal((n, h * c)), rng.standard_normal((n, h * c))
+    z = np.zeros(h * c)
+    gx, _, _, (ax, _, _) = o.edge_softmax_backward(ei, n, x, h, c, z, z, 0.2, g)
+    mb, mab = oracle.aggregate_backward(ei, n, g, "mean")
+    np.testing.assert_allclose(gx, mb, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(ax, mab, rtol=1e-12, atol=1e-12)
+    one = np.array([[3, 7, 1], [5, 9, 2]])        # 3 -> 5, 7 -> 9, 1 -> 2
+    a_s, a_d = rng.standard_normal(h * c), rng.standard_normal(h * c)
+    gx, gs, gd, _ = o.edge_softmax_backward(one, 10, x[:10], h, c, a_s, a_d, 0.2, g[:10])
+    np.testing.assert_allclose(gs, 0.0, atol=1e-13)
+    np.testing.assert_allclose(gd, 0.0, atol=1e-13)
+    want = np.zeros((10, h * c))
+    for s_, t_ in zip(one[0], one[1]):
+        want[s_] += g[t_]
+    np.testing.assert_allclose(gx, want, rtol=1e-13, atol=1e-13)
+
+
+def test_gat_backward_limits():
+    pin_gat_backward_limits(oracle.default)
+
+
+# ---------------------------------------------------------------------------
 # Error scales: every tolerance is a multiple of the oracle's absout, so it is
 # pinned to an independent numpy form -- |M| |X| with dense matrices, and for
 # attention the weights re-derived densely from their definition
@@ -747,7 +813,8 @@ PLANTS = {
     "APPNP_TELEPORT_FROM_H": [pin_appnp_hand_example, pin_appnp_dense_closed_form],
     "DOT_KEY_AT_TARGET": [pin_dot_star],
     "BACKWARD_NO_TRANSPOSE": [pin_backward_finite_differences, pin_backward_dense_transpose],
-    "SCALE_DOUBLED": [pin_error_scales],
+    "SCALE_DOUBLED": [pin_error_scales, pin_gat_backward_limits],
+    "BWD_NO_SOFTMAX_JACOBIAN": [pin_gat_backward_finite_differences],
 }
 
 
@@ -757,3 +824,26 @@ def test_planted_mistakes_are_caught(plant):
     for pin in PLANTS[plant]:
         with pytest.raises((AssertionError, oracle.OracleError)):
             pin(bad)
+
+
+def test_all_cores_rows_equal_single_thread():
+    """The OpenMP CPU baseline calls the same row functions on blocks of rows
+    in parallel: its results equal the single-threaded oracle's exactly."""
+    n = 2000
+    wl = gg.random_edge_case_graph(n, 40000, 16, 9, hub=2, isolated=30)
+    csr = oracle.build_csr(wl.edge_index, n)
+    rows = np.arange(n, dtype=np.int64)
+    nrm = oracle.gcn_norm(wl.edge_index, n, None, 1, 1.0)
+    a, ab = oracle.aggregate_rows(csr, n, wl.x_bf16, "sum", rows, w=nrm["w_norm"],
+                                  self_w=nrm["self_w"])
+    b, bb = oracle.omp_rows.aggregate_all(csr, n, wl.x_bf16, "sum", w=nrm["w_norm"],
+                                          self_w=nrm["self_w"])
+    np.testing.assert_array_equal(a, b)
+    np.testing.assert_array_equal(ab, bb)
+    rng = np.random.default_rng(9)
+    a_s, a_d = rng.standard_normal(16), rng.standard_normal(16)
+    a, _, ab = oracle.edge_softmax_rows(csr, n, wl.x_bf16, 2, 8, a_s, a_d, 0.2, rows)
+    b, bb = oracle.omp_rows.edge_softmax_all(csr, n, wl.x_bf16, 2, 8, a_s, a_d, 0.2)
+    np.testing.assert_array_equal(a, b)
+    np.testing.assert_array_equal(ab, bb)
+    assert oracle.omp_rows.threads() >= 1
