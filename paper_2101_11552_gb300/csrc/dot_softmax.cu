@@ -153,6 +153,11 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh_arg, int64
         float m = -CUDART_INF_F, den = 0.f, acc[VEC];
 #pragma unroll
         for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
+        // key and value row slices of node src, addressed in bytes (one wide
+        // multiply-add per gather)
+        const char *kb = reinterpret_cast<const char *>(kp + fl);
+        const char *vb = reinterpret_cast<const char *>(vp + fl);
+        const uint32_t row_bytes = static_cast<uint32_t>(f) * static_cast<uint32_t>(sizeof(XT));
         // one 32-edge chunk; FULL chunks (all 32 slots used) skip every slot test
         auto chunk = [&](auto full_tag, int64_t base, int cnt) {
             constexpr bool FULL = decltype(full_tag)::value;
@@ -167,10 +172,11 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh_arg, int64
 #pragma unroll
                 for (int u = 0; u < kDotUnroll; ++u) {
                     const int k = j + u * G + g;
-                    const int64_t src = __shfl_sync(kFull, c, k & 31);
+                    const uint64_t off = static_cast<uint64_t>(
+                        static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31))) * row_bytes;
                     ok[u] = FULL || k < cnt;
-                    rk[u] = ok[u] ? V::raw(kp + src * f + fl) : V::zero();
-                    rv[u] = ok[u] ? V::raw(vp + src * f + fl) : V::zero();
+                    rk[u] = ok[u] ? V::raw(reinterpret_cast<const XT *>(kb + off)) : V::zero();
+                    rv[u] = ok[u] ? V::raw(reinterpret_cast<const XT *>(vb + off)) : V::zero();
                 }
                 float l[kDotUnroll];
                 float mc = -CUDART_INF_F;
