@@ -432,6 +432,49 @@ def small_configs(L, stream, hbm_peak):
     return out
 
 
+def oracle_config_rates(with_oracle: bool = True) -> dict:
+    """The oracle as it stands, single-threaded and with its row functions on
+    all host cores, on each smaller workload's main call (edge-features/s;
+    one untimed call first).  CPU baselines beside the configs' GPU rates."""
+    if not with_oracle:
+        return {}
+    import oracle
+    from paper_2101_11552_gb300 import graphgen as gg
+    oracle.build()
+
+    def rate(fn, units):
+        fn()
+        t0 = time.perf_counter()
+        fn()
+        return units / (time.perf_counter() - t0)
+
+    res = {}
+    cases = (
+        ("er_2708_gcn", gg.make_er_2708(), "gcn"),
+        ("ba_19717_sum_mean_max", gg.make_ba_19717(), "sum"),
+        ("gat_169343_edge_softmax", gg.make_gat_169343(), "softmax"),
+        ("molecules_1024_gcn_pool", gg.make_molecules_1024(), "gcn"),
+    )
+    for name, wl, kind in cases:
+        n, ei, x, e, f = wl.num_nodes, wl.edge_index, wl.x, wl.num_edges, wl.num_features
+        csr = oracle.build_csr(ei, n)
+        if kind == "gcn":
+            nrm = oracle.gcn_norm(ei, n, None, 0, 1.0)
+            one = lambda: oracle.aggregate(ei, n, x, "sum", w=nrm["w_norm"])  # noqa: E731
+            allc = lambda: oracle.omp_rows.aggregate_all(csr, n, x, "sum", w=nrm["w_norm"])  # noqa: E731
+        elif kind == "sum":
+            one = lambda: oracle.aggregate(ei, n, x, "sum")  # noqa: E731
+            allc = lambda: oracle.omp_rows.aggregate_all(csr, n, x, "sum")  # noqa: E731
+        else:
+            args = (wl.heads, wl.channels, wl.a_src, wl.a_dst, wl.negative_slope)
+            one = lambda: oracle.edge_softmax(ei, n, x, *args)  # noqa: E731
+            allc = lambda: oracle.omp_rows.edge_softmax_all(csr, n, x, *args)  # noqa: E731
+        res[name] = {"oracle_1_thread": rate(one, e * f),
+                     "oracle_all_cores": rate(allc, e * f),
+                     "cores": oracle.omp_rows.threads(), "unit": UNIT}
+    return res
+
+
 def gather_floor(L, col, x, e, n, stream) -> dict:
     """Gather-only floor on the step's own column array and bf16 rows: every
     row x[col[k]] read once (tfg_gather_xor), inputs hot in L2 as in the
@@ -530,7 +573,29 @@ def next_rows(L, wl, bufs, stream, hbm_peak):
         "forward_edge_features_per_s": e * f / (ms_fwd * 1e-3),
         "backward_edge_features_per_s": e * f / (ms_bwd * 1e-3),
         "note": "bf16 features, argmax int32 [N, F]; backward reads argmax and gradient rows per out-edge"}
-    del csr_src, grad_x, out_max, argmax
+    # backward of the GAT edge softmax: grad_out = the softmax output of the
+    # step (fp32), the forward's output taken from a fresh forward call
+    heads, ch = wl.heads, wl.channels
+    a_s = torch.from_numpy(wl.a_src).to(dev)
+    a_d = torch.from_numpy(wl.a_dst).to(dev)
+    ws_f = torch.empty(tfg.tfg_edge_softmax_workspace_size(n, heads), dtype=torch.uint8, device=dev)
+    fwd = torch.empty(n, f, dtype=torch.float32, device=dev)
+    check(L.tfg_edge_softmax_aggregate(P(bufs["rowptr"]), P(bufs["col"]), P(bufs["xb"]), tfg.TFG_BF16,
+                                       n, e, heads, ch, P(a_s), P(a_d), 0.2, P(fwd), None, P(ws_f),
+                                       ws_f.numel(), sp))
+    ga_s = torch.empty(f, dtype=torch.float32, device=dev)
+    ga_d = torch.empty(f, dtype=torch.float32, device=dev)
+    ws_b = torch.empty(tfg.tfg_edge_softmax_backward_workspace_size(n, heads, ch), dtype=torch.uint8,
+                       device=dev)
+    ms = _event_ms(lambda: check(L.tfg_edge_softmax_aggregate_backward(
+        P(bufs["rowptr"]), P(bufs["col"]), P(csr_src.rowptr), P(csr_src.col), P(bufs["xb"]),
+        tfg.TFG_BF16, n, e, heads, ch, P(a_s), P(a_d), 0.2, P(fwd), P(fwd), P(grad_x), P(ga_s),
+        P(ga_d), P(ws_b), ws_b.numel(), sp)), stream, 3)
+    rows["gat_backward"] = {"ms": round(ms, 4), "heads": heads, "channels": ch,
+                            "edge_features_per_s": e * f / (ms * 1e-3),
+                            "note": "grad_x, grad_a_src, grad_a_dst of the bf16 8 x 16 edge softmax; "
+                                    "CSR by source built once; warp per row, lanes over features"}
+    del csr_src, grad_x, out_max, argmax, fwd, ws_b, ws_f
 
     heads, ch = wl.heads, wl.channels
     gen = torch.Generator(device=dev)
@@ -908,6 +973,9 @@ def main():
                                               h=h, batch=batch), stream, hbm_peak)
     if not args.no_configs:
         line["configs"] = small_configs(L, stream, hbm_peak)
+        if world == 1 and not args.no_cpu_baseline:
+            for name, rec in oracle_config_rates().items():
+                line["configs"][name]["cpu_baseline"] = rec
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baselines(wl)
     print(json.dumps(line), flush=True)

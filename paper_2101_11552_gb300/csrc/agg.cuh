@@ -356,15 +356,13 @@ __global__ void __launch_bounds__(kAggThreads, VEC >= 8 ? TFG_AGG_MINB : 4) aggr
 #ifndef TFG_AGG_MP
 #define TFG_AGG_MP 1       // 0: every layout takes aggregate_kernel (for side-by-side timing)
 #endif
-#ifndef TFG_MP_BF16_VEC4
-#define TFG_MP_BF16_VEC4 0 // 1: bf16 rows of <= 128 features as 8-byte slices (4 features per lane)
-#endif
 // Measured on the 114.6M-edge graph (bf16, F = 128, ids and weights staged in
 // shared memory): GCN 1.82 ms at 4 CTAs per SM and 4 gathers in flight per
 // lane (3 CTAs and 8 in flight: 1.84 ms; 2 CTAs and 16: 2.06 ms; the
 // row-per-warp aggregate_kernel: 1.95 ms); max 2.84 ms (aggregate_kernel
 // 3.34 ms).  fp32 rows (512 bytes, one row per warp load) stay on
-// aggregate_kernel: 2.99 ms there against 3.10-3.50 ms here.
+// aggregate_kernel: 2.99 ms there against 3.10-3.50 ms here; bf16 rows as
+// 8-byte slices (4 features per lane, up to 16 in flight) measured 1.90-3.04 ms.
 #ifndef TFG_MP_BLOCKS
 #define TFG_MP_BLOCKS 4    // resident CTAs per SM for sums (64 registers per thread)
 #endif
@@ -595,7 +593,7 @@ template <typename XT, int VEC, int KIND, typename X0T = XT>
 cudaError_t launch_lpr(const AggArgs &a, int lpr, cudaStream_t s) {
     // E is not known on the host; the kernel reads rowptr[N] for the split.
     // 16-byte bf16 slices in one feature tile: the merge-path kernel
-    if constexpr (sizeof(XT) == 2 && (VEC == 8 || (TFG_MP_BF16_VEC4 && VEC == 4))) {
+    if constexpr (sizeof(XT) == 2 && VEC == 8) {
         if (TFG_AGG_MP && static_cast<int64_t>(lpr) * VEC >= a.f) {
             const int grid = static_cast<int>(
                 min64(a.n, static_cast<int64_t>(sm_count()) * mp_blocks<KIND == kMax>()));

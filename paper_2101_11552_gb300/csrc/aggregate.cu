@@ -26,10 +26,6 @@ cudaError_t launch_aggregate(int mode, const int32_t *rowptr, const int32_t *col
     const bool aligned = (reinterpret_cast<uintptr_t>(x) % 16 == 0) &&
                          (reinterpret_cast<uintptr_t>(out) % 16 == 0);
     if (x_dtype == TFG_BF16) {
-#if TFG_MP_BF16_VEC4
-        if (aligned && f % 4 == 0 && f <= 128 && kind != kMax)
-            return launch_kind<uint16_t, 4>(a, kind, lanes_per_row(f / 4), s);
-#endif
         if (aligned && f % 8 == 0) return launch_kind<uint16_t, 8>(a, kind, lanes_per_row(f / 8), s);
         return launch_kind<uint16_t, 1>(a, kind, lanes_per_row(f), s);
     }

@@ -159,9 +159,9 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh_arg, int64
         const char *vb = reinterpret_cast<const char *>(vp + fl);
         const uint32_t row_bytes = static_cast<uint32_t>(f) * static_cast<uint32_t>(sizeof(XT));
         // one 32-edge chunk; FULL chunks (all 32 slots used) skip every slot test
-        auto chunk = [&](auto full_tag, int64_t base, int cnt) {
+        // c: the chunk's column ids (lane j: edge j; any valid id past cnt)
+        auto chunk = [&](auto full_tag, int c, int cnt) {
             constexpr bool FULL = decltype(full_tag)::value;
-            const int c = (FULL || lane < cnt) ? ld_stream(a.col + base + lane) : 0;
             float den_part = 0.f, part[VEC];
 #pragma unroll
             for (int q = 0; q < VEC; ++q) part[q] = 0.f;
@@ -214,10 +214,14 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh_arg, int64
 #pragma unroll
             for (int q = 0; q < VEC; ++q) acc[q] += part[q];
         };
+        // the next chunk's column ids are requested before this chunk's rows
+        int cnext = (a.col && beg + lane < end) ? ld_stream(a.col + beg + lane) : 0;
         for (int64_t base = beg; base < end; base += 32) {
             const int cnt = static_cast<int>(min64(32, end - base));
-            if (cnt == 32) chunk(std::true_type{}, base, 32);
-            else chunk(std::false_type{}, base, cnt);
+            const int c = cnext;
+            cnext = (base + 32 + lane < end) ? ld_stream(a.col + base + 32 + lane) : 0;
+            if (cnt == 32) chunk(std::true_type{}, c, 32);
+            else chunk(std::false_type{}, c, cnt);
         }
         // merge the G groups' states in a fixed butterfly order
 #pragma unroll

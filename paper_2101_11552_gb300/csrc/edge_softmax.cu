@@ -41,6 +41,12 @@ constexpr int kSmThreads = 256;
 #define TFG_SM_UNROLL 4   // gathers in flight per lane (tuning knob)
 #endif
 constexpr int kSmUnroll = TFG_SM_UNROLL;   // fast kernel
+// 1: the next chunk's column ids are requested one chunk ahead; 2: also its
+// node scores s_src, gathered while this chunk's rows are summed (measured on
+// the 114.6M-edge graph: 2.29 ms with 2, 2.40-2.50 ms with 1, 2.44-2.57 ms with 0)
+#ifndef TFG_SM_PREFETCH
+#define TFG_SM_PREFETCH 2
+#endif
 #ifndef TFG_SM_FULL_CHUNKS
 #define TFG_SM_FULL_CHUNKS 1   // separate code for full 32-edge chunks (no slot tests)
 #endif
@@ -245,10 +251,16 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
     float m = -CUDART_INF_F, den = 0.f, acc[VEC];
 #pragma unroll
     for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
-    // one 32-edge chunk; FULL chunks (all 32 slots used) skip every slot test
-    auto chunk = [&](auto full_tag, int64_t base, int cnt) {
+#if TFG_SM_PREFETCH
+    int cnext = 0;   // the next chunk's column ids (lane j: edge j of that chunk)
+#endif
+#if TFG_SM_PREFETCH >= 2
+    float sv[R];     // s_src of the chunk about to run, for (edge r * ES + se, head sh)
+#endif
+    // one 32-edge chunk with its column ids in c (lane j: edge base + j; any
+    // valid id past cnt); FULL chunks (all 32 slots used) skip every slot test
+    auto chunk = [&](auto full_tag, int c, int cnt) {
         constexpr bool FULL = decltype(full_tag)::value;
-        const int c = (FULL || lane < cnt) ? ld_stream(col + base + lane) : 0;
         // the first step's row gathers need only the column ids: issue them
         // before the scores so that their latency overlaps the score work
         typename V::Raw raw0[kSmUnroll];
@@ -260,10 +272,12 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
 #pragma unroll
         for (int r = 0; r < R; ++r) {
             const int k = r * ES + se;
-            const int src = __shfl_sync(kFull, c, k);
-            p[r] = (FULL || k < cnt)
-                       ? leaky(__ldg(s_src + static_cast<int64_t>(src) * H + sh) + sd, slope)
-                       : -CUDART_INF_F;
+#if TFG_SM_PREFETCH >= 2
+            const float ss = sv[r];                  // gathered during the previous chunk
+#else
+            const float ss = __ldg(s_src + static_cast<int64_t>(__shfl_sync(kFull, c, k)) * H + sh);
+#endif
+            p[r] = (FULL || k < cnt) ? leaky(ss + sd, slope) : -CUDART_INF_F;
             cm = fmaxf(cm, p[r]);
         }
 #pragma unroll
@@ -285,6 +299,12 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
             den_part += p[r];
         }
         den += den_part;
+#if TFG_SM_PREFETCH >= 2
+        // the next chunk's node scores, requested before this chunk's rows
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            sv[r] = __ldg(s_src + static_cast<int64_t>(__shfl_sync(kFull, cnext, r * ES + se)) * H + sh);
+#endif
         float part[VEC];
 #pragma unroll
         for (int q = 0; q < VEC; ++q) part[q] = 0.f;
@@ -324,10 +344,25 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
 #pragma unroll
         for (int q = 0; q < VEC; ++q) acc[q] += part[q];
     };
+#if TFG_SM_PREFETCH
+    // the next chunk's column ids are requested before this chunk's rows
+    cnext = (col && beg + lane < end) ? ld_stream(col + beg + lane) : 0;
+#endif
+#if TFG_SM_PREFETCH >= 2
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+        sv[r] = __ldg(s_src + static_cast<int64_t>(__shfl_sync(kFull, cnext, r * ES + se)) * H + sh);
+#endif
     for (int64_t base = beg; base < end; base += 32) {
         const int cnt = static_cast<int>(min64(32, end - base));
-        if (kSmFullChunks && cnt == 32) chunk(std::true_type{}, base, 32);
-        else chunk(std::false_type{}, base, cnt);
+#if TFG_SM_PREFETCH
+        const int c = cnext;
+        cnext = (base + 32 + lane < end) ? ld_stream(col + base + 32 + lane) : 0;
+#else
+        const int c = lane < cnt ? ld_stream(col + base + lane) : 0;
+#endif
+        if (kSmFullChunks && cnt == 32) chunk(std::true_type{}, c, 32);
+        else chunk(std::false_type{}, c, cnt);
     }
 #pragma unroll
     for (int o = H; o < 32; o <<= 1) den += __shfl_xor_sync(kFull, den, o);
@@ -676,11 +711,12 @@ softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict_
     });
 }
 
-// Measured on the 114.6M-edge graph (bf16, 8 heads x 16): 4 CTAs per SM with
-// 4 gathers in flight per lane 2.50 ms; 3 CTAs with 8 in flight 2.62 ms,
-// 3 with 4 2.57 ms, 4 with 8 2.75 ms, 2 with 8 3.48 ms.
+// Measured on the 114.6M-edge graph (bf16, 8 heads x 16), ids and scores
+// requested one chunk ahead: 3 CTAs per SM with 4 gathers in flight per lane
+// 2.29 ms; 4 CTAs 2.31 ms; 3 CTAs with 8 in flight 2.52 ms.  Without the
+// early requests: 4 CTAs / 4 in flight 2.44-2.50 ms, 3 / 8 2.62 ms, 2 / 8 3.48 ms.
 #ifndef TFG_SMF_BLOCKS
-#define TFG_SMF_BLOCKS 4     // resident CTAs per SM of softmax_fast
+#define TFG_SMF_BLOCKS 3     // resident CTAs per SM of softmax_fast
 #endif
 
 template <typename XT, int VEC, int LPR, int H>
