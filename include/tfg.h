@@ -396,6 +396,41 @@ int tfg_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t *co
                                         size_t workspace_bytes, tfg_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Backward of the dot-product attention aggregation
+ * (tfg_dot_edge_softmax_aggregate): the gradients with respect to q, k and v
+ * given grad_out = dL/dout, on the same Fig. 5a workflow.  With alpha the
+ * forward's weights and e = (s -> t):
+ *   dalpha[e,h] = <grad_out[t,h,:], v[s,h,:]>
+ *   beta[t,h]   = <grad_out[t,h,:], out[t,h,:]>  (= sum over e into t of alpha dalpha)
+ *   dl[e,h]     = alpha (dalpha - beta[t,h])
+ *   grad_q[t,h,:] = scale * sum over e into t of dl k[s,h,:]
+ *   grad_k[s,h,:] = scale * sum over e out of s of dl q[t,h,:]
+ *   grad_v[s,h,:] = sum over e out of s of alpha grad_out[t,h,:]
+ *
+ *   rowptr, col: the CSR by target of the forward (tfg_build_csr).
+ *   rowptr_src, col_src: the CSR by source (tfg_build_csr_by_source).
+ *   q, k, v, x_dtype, num_nodes, num_edges, heads, channels, scale: the
+ *          forward's arguments.
+ *   out (device) fp32 [num_nodes, H*C]: the forward's output.
+ *   grad_out (device) fp32 [num_nodes, H*C].
+ *   grad_q, grad_k, grad_v (device) fp32 [num_nodes, H*C]: written.
+ *   workspace >= tfg_dot_edge_softmax_backward_workspace_size() bytes.
+ * Layouts: channels a power of two up to 32, or a multiple of 32; H*C <= 256.
+ * Others return TFG_ERR_INVALID_ARG.  Deterministic (no atomics).
+ * ---------------------------------------------------------------------- */
+int tfg_dot_edge_softmax_backward_workspace_size(int64_t num_nodes, int heads, int channels,
+                                                 size_t *bytes);
+int tfg_dot_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t *col,
+                                            const int32_t *rowptr_src, const int32_t *col_src,
+                                            const void *q, const void *k, const void *v,
+                                            int x_dtype, int64_t num_nodes, int64_t num_edges,
+                                            int heads, int channels, float scale,
+                                            const float *out, const float *grad_out,
+                                            float *grad_q, float *grad_k, float *grad_v,
+                                            void *workspace, size_t workspace_bytes,
+                                            tfg_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * Graph pooling keyed by node_graph_index (Section 2.1.1 BatchGraph; Fig. 2a
  * common graph pooling):
  *   out[g, :] = REDUCE over nodes v with batch[v] == g of x[v, :]

@@ -98,6 +98,8 @@ def _load(plant: Optional[str] = None) -> ctypes.CDLL:
                 "oracle_dot_softmax_rows": [I64, P, P, P, P, P, I, I, D, P, I64, P, P, P],
                 "oracle_edge_softmax_backward": [I64, I64, P, P, I, I, P, P, D, P, P, P, P, P,
                                                  P, P],
+                "oracle_dot_softmax_backward": [I64, I64, P, P, P, P, I, I, D, P, P, P, P, P, P,
+                                                P],
             }
             for fn, args in sigs.items():
                 getattr(lib, fn).argtypes = args
@@ -240,6 +242,21 @@ class _Oracle:
             float(slope), self._p(g), self._p(gx), self._p(gs), self._p(gd), self._p(ax),
             self._p(as_), self._p(ad)))
         return gx[:n], gs, gd, (ax[:n], as_, ad)
+
+    def dot_softmax_backward(self, edge_index, n, q, k, v, heads, channels, scale, grad_out):
+        """Gradients of dot_softmax's output with respect to q, k and v for a
+        given dL/dout.  Returns (grad_q, grad_k, grad_v, (scale_q, scale_k, scale_v))."""
+        ei = np.ascontiguousarray(edge_index, dtype=np.int64)
+        e = ei.shape[1]
+        q, k, v, g = widen(q), widen(k), widen(v), widen(grad_out)
+        f = q.shape[1]
+        assert f == heads * channels and k.shape == q.shape and v.shape == q.shape
+        outs = [np.zeros((max(n, 1), f)) for _ in range(6)]
+        self._check(self.lib.oracle_dot_softmax_backward(
+            n, e, self._p(ei), self._p(q), self._p(k), self._p(v), heads, channels, float(scale),
+            self._p(g), *[self._p(o) for o in outs]))
+        gq, gk, gv, aq, ak, av = (o[:n] for o in outs)
+        return gq, gk, gv, (aq, ak, av)
 
     # -- backward of the aggregation ------------------------------------
     def aggregate_backward(self, edge_index, n, grad_out, reduce, w=None, self_w=None):
@@ -500,6 +517,7 @@ gcn_aggregate_backward = default.gcn_aggregate_backward
 max_argmax = default.max_argmax
 max_backward = default.max_backward
 edge_softmax_backward = default.edge_softmax_backward
+dot_softmax_backward = default.dot_softmax_backward
 dot_softmax_rows = default.dot_softmax_rows
 sgc = default.sgc
 

@@ -736,6 +736,102 @@ done:
 }
 
 /* ---------------------------------------------------------------------------
+ * Backward of the dot-product (Transformer-style) attention aggregation:
+ * gradients with respect to q, k and v given grad_out = dL/dout.  Forward
+ * quantities are recomputed as oracle_dot_softmax forms them; then per edge
+ * e = (s -> t) and head h:
+ *   dalpha[e,h] = sum_c grad_out[t,h,c] v[s,h,c]
+ *   beta[t,h]   = sum over edges e' into t of alpha[e',h] dalpha[e',h]
+ *   dl[e,h]     = alpha[e,h] (dalpha[e,h] - beta[t,h])          (softmax Jacobian)
+ *   grad_q[t,h,:] += scale dl[e,h] k[s,h,:]
+ *   grad_k[s,h,:] += scale dl[e,h] q[t,h,:]
+ *   grad_v[s,h,:] += alpha[e,h] grad_out[t,h,:]
+ * abs_* run the same recursion on absolute values.
+ * ------------------------------------------------------------------------- */
+int oracle_dot_softmax_backward(int64_t n, int64_t e, const int64_t *edge_index, const double *q,
+                                const double *k, const double *v, int h, int c, double scale,
+                                const double *grad_out, double *grad_q, double *grad_k,
+                                double *grad_v, double *abs_q, double *abs_k, double *abs_v)
+{
+    if (n < 0 || e < 0 || h <= 0 || c <= 0) return E_ARG;
+    const int64_t *src = edge_index, *dst = edge_index + e;
+    for (int64_t i = 0; i < e; ++i)
+        if (src[i] < 0 || src[i] >= n || dst[i] < 0 || dst[i] >= n) return E_RANGE;
+    int64_t f = (int64_t)h * c;
+    size_t nh = (size_t)(n > 0 ? n : 1) * (size_t)h, eh = (size_t)(e > 0 ? e : 1) * (size_t)h;
+    double *mx = (double *)calloc(nh, sizeof(double));
+    double *den = (double *)calloc(nh, sizeof(double));
+    double *beta = (double *)calloc(nh, sizeof(double));
+    double *abeta = (double *)calloc(nh, sizeof(double));
+    char *seen = (char *)calloc(nh, 1);
+    double *logit = (double *)calloc(eh, sizeof(double));
+    double *alpha = (double *)calloc(eh, sizeof(double));
+    double *dal = (double *)calloc(eh, sizeof(double));
+    double *adal = (double *)calloc(eh, sizeof(double));
+    int rc = OK;
+    if (!mx || !den || !beta || !abeta || !seen || !logit || !alpha || !dal || !adal) {
+        rc = E_ARG;
+        goto done;
+    }
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            double l = dot_logit(q, k, dst[i], src[i], f, hh, c, scale);
+            logit[i * h + hh] = l;
+            size_t kk = (size_t)dst[i] * h + hh;
+            if (!seen[kk] || l > mx[kk]) mx[kk] = l;
+            seen[kk] = 1;
+        }
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh)
+            den[(size_t)dst[i] * h + hh] += exp(logit[i * h + hh] - mx[(size_t)dst[i] * h + hh]);
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            size_t kk = (size_t)dst[i] * h + hh;
+            double al = exp(logit[i * h + hh] - mx[kk]) / den[kk];
+            double d = 0.0, ad = 0.0;
+            for (int cc = 0; cc < c; ++cc) {
+                double pr = grad_out[dst[i] * f + hh * c + cc] * v[src[i] * f + hh * c + cc];
+                d += pr;
+                ad += fabs(pr);
+            }
+            alpha[i * h + hh] = al;
+            dal[i * h + hh] = d;
+            adal[i * h + hh] = ad;
+            beta[kk] += al * d;
+            abeta[kk] += al * ad;
+        }
+    for (int64_t kk = 0; kk < n * f; ++kk) {
+        grad_q[kk] = grad_k[kk] = grad_v[kk] = 0.0;
+        abs_q[kk] = abs_k[kk] = abs_v[kk] = 0.0;
+    }
+    for (int64_t i = 0; i < e; ++i)
+        for (int hh = 0; hh < h; ++hh) {
+            size_t kt = (size_t)dst[i] * h + hh;
+            double al = alpha[i * h + hh];
+#ifdef ORACLE_PLANT_BWD_NO_SOFTMAX_JACOBIAN
+            double dl = al * dal[i * h + hh];                       /* planted: beta dropped */
+#else
+            double dl = al * (dal[i * h + hh] - beta[kt]);
+#endif
+            double adl = al * (adal[i * h + hh] + abeta[kt]);
+            for (int cc = 0; cc < c; ++cc) {
+                int64_t ot = dst[i] * f + hh * c + cc, os = src[i] * f + hh * c + cc;
+                double mq = scale * dl * k[os], mk = scale * dl * q[ot], mv = al * grad_out[ot];
+                grad_q[ot] += mq;
+                grad_k[os] += mk;
+                grad_v[os] += mv;
+                abs_q[ot] += fabs(scale) * adl * fabs(k[os]);
+                abs_k[os] += fabs(scale) * adl * fabs(q[ot]);
+                abs_v[os] += SCALE_TERM(mv);
+            }
+        }
+done:
+    free(mx); free(den); free(beta); free(abeta); free(seen); free(logit); free(alpha);
+    free(dal); free(adal);
+    return rc;
+}
+
+/* ---------------------------------------------------------------------------
  * Backward of the aggregation: the gradient with respect to x of the
  * aggregation out[t] = sum over edges e = (s -> t) of w_e x[s] (sum), the
  * same divided by the number of edges into t (mean), or with the GCN weights

@@ -444,9 +444,64 @@ int tfg_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t *co
         return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
                     workspace ? workspace_bytes : size_t(0));
     return cuda_result(tfg::launch_edge_softmax_backward(
-                           rowptr, col, rowptr_src, col_src, x, x_dtype, num_nodes, heads,
-                           channels, a_src, a_dst, negative_slope, out, grad_out, grad_x,
+                           rowptr, col, rowptr_src, col_src, x, x_dtype, num_nodes,
+                           num_edges, heads, channels, a_src, a_dst, negative_slope, out, grad_out, grad_x,
                            grad_a_src, grad_a_dst, workspace, reinterpret_cast<cudaStream_t>(stream)),
+                       fn);
+}
+
+int tfg_dot_edge_softmax_backward_workspace_size(int64_t num_nodes, int heads, int channels,
+                                                 size_t *bytes) {
+    const char *fn = "tfg_dot_edge_softmax_backward_workspace_size";
+    TFG_NEED(bytes, true, fn, "bytes");
+    TFG_TRY(check_counts(fn, num_nodes, 0));
+    if (!tfg::attention_backward_layout_ok(heads, channels))
+        return fail(TFG_ERR_INVALID_ARG,
+                    "%s: channels must be a power of two up to 32 or a multiple of 32, H*C <= 256",
+                    fn);
+    *bytes = tfg::dot_attention_backward_workspace_bytes(num_nodes, heads);
+    return TFG_OK;
+}
+
+int tfg_dot_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t *col,
+                                            const int32_t *rowptr_src, const int32_t *col_src,
+                                            const void *q, const void *k, const void *v,
+                                            int x_dtype, int64_t num_nodes, int64_t num_edges,
+                                            int heads, int channels, float scale,
+                                            const float *out, const float *grad_out,
+                                            float *grad_q, float *grad_k, float *grad_v,
+                                            void *workspace, size_t workspace_bytes,
+                                            tfg_stream_t stream) {
+    const char *fn = "tfg_dot_edge_softmax_aggregate_backward";
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    if (!tfg::attention_backward_layout_ok(heads, channels))
+        return fail(TFG_ERR_INVALID_ARG,
+                    "%s: channels must be a power of two up to 32 or a multiple of 32, H*C <= 256",
+                    fn);
+    TFG_TRY(check_features(fn, num_nodes, int64_t(heads) * channels));
+    TFG_TRY(check_dtype(fn, x_dtype));
+    if (!(scale == scale) || scale == INFINITY || scale == -INFINITY)
+        return fail(TFG_ERR_INVALID_ARG, "%s: scale must be finite", fn);
+    TFG_NEED(rowptr, true, fn, "rowptr");
+    TFG_NEED(rowptr_src, true, fn, "rowptr_src");
+    TFG_NEED(col, num_edges > 0, fn, "col");
+    TFG_NEED(col_src, num_edges > 0, fn, "col_src");
+    TFG_NEED(q, num_nodes > 0, fn, "q");
+    TFG_NEED(k, num_nodes > 0, fn, "k");
+    TFG_NEED(v, num_nodes > 0, fn, "v");
+    TFG_NEED(out, num_nodes > 0, fn, "out");
+    TFG_NEED(grad_out, num_nodes > 0, fn, "grad_out");
+    TFG_NEED(grad_q, num_nodes > 0, fn, "grad_q");
+    TFG_NEED(grad_k, num_nodes > 0, fn, "grad_k");
+    TFG_NEED(grad_v, num_nodes > 0, fn, "grad_v");
+    const size_t need = tfg::dot_attention_backward_workspace_bytes(num_nodes, heads);
+    if (workspace == nullptr || workspace_bytes < need)
+        return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
+                    workspace ? workspace_bytes : size_t(0));
+    return cuda_result(tfg::launch_dot_softmax_backward(
+                           rowptr, col, rowptr_src, col_src, q, k, v, x_dtype, num_nodes,
+                           num_edges, heads, channels, scale, out, grad_out, grad_q, grad_k,
+                           grad_v, workspace, reinterpret_cast<cudaStream_t>(stream)),
                        fn);
 }
 

@@ -178,6 +178,25 @@ __device__ __forceinline__ void balanced_rows(const int32_t *rowptr, int64_t n, 
     r1 = b + 1 == nb ? n : first_row_at(rowptr, n, (b + 1) * w);
 }
 
+// Each CTA owns a work-balanced range of rows (edges + rows split evenly
+// across CTAs); its warps take rows one at a time from a shared counter.
+template <typename RowFn>
+__device__ __forceinline__ void for_each_row(const int32_t *rowptr, int64_t n, RowFn fn) {
+    __shared__ int s_next;
+    int64_t r0, r1;
+    balanced_rows(rowptr, n, gridDim.x, blockIdx.x, r0, r1);
+    if (threadIdx.x == 0) s_next = 0;
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    for (;;) {
+        int i = 0;
+        if (lane == 0) i = atomicAdd(&s_next, 1);
+        i = __shfl_sync(kFull, i, 0);
+        if (i >= r1 - r0) break;
+        fn(r0 + i, lane);
+    }
+}
+
 }  // namespace tfg
 
 // Number of CTAs for a balanced launch over E edges and N rows: enough for
@@ -240,11 +259,19 @@ bool attention_backward_layout_ok(int heads, int channels);
 size_t attention_backward_workspace_bytes(int64_t n, int heads, int channels);
 cudaError_t launch_edge_softmax_backward(const int32_t *rowptr, const int32_t *col,
                                          const int32_t *rowptr_src, const int32_t *col_src,
-                                         const void *x, int x_dtype, int64_t n, int heads,
-                                         int channels, const float *a_src, const float *a_dst,
+                                         const void *x, int x_dtype, int64_t n, int64_t e,
+                                         int heads, int channels, const float *a_src,
+                                         const float *a_dst,
                                          float slope, const float *out, const float *grad_out,
                                          float *grad_x, float *grad_a_src, float *grad_a_dst,
                                          void *ws, cudaStream_t s);
+size_t dot_attention_backward_workspace_bytes(int64_t n, int heads);
+cudaError_t launch_dot_softmax_backward(const int32_t *rowptr, const int32_t *col,
+                                        const int32_t *rowptr_src, const int32_t *col_src,
+                                        const void *q, const void *k, const void *v, int x_dtype,
+                                        int64_t n, int64_t e, int heads, int channels, float scale,
+                                        const float *out, const float *grad_out, float *grad_q,
+                                        float *grad_k, float *grad_v, void *ws, cudaStream_t s);
 cudaError_t launch_gather_xor(const int32_t *col, int64_t e, const void *x, int64_t row_bytes,
                               uint32_t *out, cudaStream_t s);
 cudaError_t launch_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n,

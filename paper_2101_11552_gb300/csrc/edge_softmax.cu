@@ -680,25 +680,6 @@ softmax_mp(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,
     }
 }
 
-// Each CTA owns a work-balanced range of rows (edges + rows split evenly
-// across CTAs); its warps take rows one at a time from a shared counter.
-template <typename RowFn>
-__device__ __forceinline__ void for_each_row(const int32_t *rowptr, int64_t n, RowFn fn) {
-    __shared__ int s_next;
-    int64_t r0, r1;
-    balanced_rows(rowptr, n, gridDim.x, blockIdx.x, r0, r1);
-    if (threadIdx.x == 0) s_next = 0;
-    __syncthreads();
-    const int lane = threadIdx.x & 31;
-    for (;;) {
-        int i = 0;
-        if (lane == 0) i = atomicAdd(&s_next, 1);
-        i = __shfl_sync(kFull, i, 0);
-        if (i >= r1 - r0) break;
-        fn(r0 + i, lane);
-    }
-}
-
 template <typename XT, int VEC, int LPR>
 __global__ void __launch_bounds__(kSmThreads, 3)
 softmax_aggregate(const int32_t *__restrict__ rowptr, const int32_t *__restrict__ col,

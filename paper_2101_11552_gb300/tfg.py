@@ -85,6 +85,9 @@ def lib() -> ctypes.CDLL:
                 "tfg_edge_softmax_backward_workspace_size": [I64, I, I, ctypes.POINTER(SZ)],
                 "tfg_edge_softmax_aggregate_backward": [P, P, P, P, P, I, I64, I64, I, I, P, P, F,
                                                         P, P, P, P, P, P, SZ, P],
+                "tfg_dot_edge_softmax_backward_workspace_size": [I64, I, I, ctypes.POINTER(SZ)],
+                "tfg_dot_edge_softmax_aggregate_backward": [P, P, P, P, P, P, P, I, I64, I64, I, I,
+                                                            F, P, P, P, P, P, P, SZ, P],
             }
             for name, args in sigs.items():
                 fn = getattr(L, name)
@@ -577,3 +580,35 @@ def tfg_edge_softmax_aggregate_backward(rowptr, col, rowptr_src, col_src, x, hea
         _ptr(grad_out), _ptr(grad_x), _ptr(ga_src), _ptr(ga_dst), _ptr(ws), ws.numel(),
         _stream(dev)))
     return grad_x, ga_src, ga_dst
+
+
+def tfg_dot_edge_softmax_backward_workspace_size(num_nodes: int, heads: int, channels: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().tfg_dot_edge_softmax_backward_workspace_size(num_nodes, heads, channels,
+                                                              ctypes.byref(n)))
+    return n.value
+
+
+def tfg_dot_edge_softmax_aggregate_backward(rowptr, col, rowptr_src, col_src, q, k, v,
+                                            heads: int, channels: int, scale: float, out,
+                                            grad_out):
+    """Gradients of tfg_dot_edge_softmax_aggregate with respect to q, k and v.
+    Returns (grad_q, grad_k, grad_v), each [N, H*C] fp32."""
+    _need_cuda("q", q)
+    dev = q.device
+    _need_cuda("k", k, q.dtype, dev)
+    _need_cuda("v", v, q.dtype, dev)
+    for name, t, dt in (("rowptr", rowptr, torch.int32), ("col", col, torch.int32),
+                        ("rowptr_src", rowptr_src, torch.int32), ("col_src", col_src, torch.int32),
+                        ("out", out, torch.float32), ("grad_out", grad_out, torch.float32)):
+        _need_cuda(name, t, dt, dev)
+    n = q.shape[0]
+    f = heads * channels
+    grads = [torch.empty(n, f, dtype=torch.float32, device=dev) for _ in range(3)]
+    ws = torch.empty(max(tfg_dot_edge_softmax_backward_workspace_size(n, heads, channels), 1),
+                     dtype=torch.uint8, device=dev)
+    _check(lib().tfg_dot_edge_softmax_aggregate_backward(
+        _ptr(rowptr), _ptr(col), _ptr(rowptr_src), _ptr(col_src), _ptr(q), _ptr(k), _ptr(v),
+        _x_dtype(q), n, col.numel(), heads, channels, float(scale), _ptr(out), _ptr(grad_out),
+        _ptr(grads[0]), _ptr(grads[1]), _ptr(grads[2]), _ptr(ws), ws.numel(), _stream(dev)))
+    return tuple(grads)

@@ -112,6 +112,26 @@ def test_gat_backward_hub_rows_and_degenerate_graphs():
         assert_scaled_close(gd, rgd, sd, TOL_F32, f"grad_a_dst n={n}")
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_gat_backward_unaligned_rows_take_the_general_kernels(dtype):
+    """x shifted off 16-byte alignment runs the general kernels (the aligned
+    8 x 16 layout runs the fast ones); both meet the oracle's bound."""
+    heads, channels = 8, 16
+    n, f = 2000, heads * channels
+    wl, x, xh, a_s, a_d, g = _case(n, 25000, heads, channels, dtype, 41)
+    buf = torch.empty(n * f + 1, dtype=x.dtype, device=x.device)
+    buf[1:].copy_(x.reshape(-1))
+    xu = buf[1:].view(n, f)
+    rgx, rga, rgd, (sx, sa, sd) = oracle.edge_softmax_backward(wl.edge_index, n, xh, heads,
+                                                               channels, a_s, a_d, 0.2, g)
+    for xx, what in ((xu, "unaligned"), (x, "aligned")):
+        gx, ga, gd, csr = _run(wl, xx, heads, channels, a_s, a_d, g)
+        tol = _tol(wl, xh, heads, channels, a_s, a_d, csr)
+        assert_scaled_close(gx, rgx, sx, tol, f"grad_x {what} {dtype}")
+        assert_scaled_close(ga, rga, sa, tol, f"grad_a_src {what} {dtype}")
+        assert_scaled_close(gd, rgd, sd, tol, f"grad_a_dst {what} {dtype}")
+
+
 def test_gat_backward_is_deterministic_and_rejects_bad_layouts():
     heads, channels = 4, 16
     wl, x, _, a_s, a_d, g = _case(2000, 30000, heads, channels, "bf16", 9)

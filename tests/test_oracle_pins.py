@@ -691,6 +691,62 @@ def test_gat_backward_limits():
     pin_gat_backward_limits(oracle.default)
 
 
+def pin_dot_backward_finite_differences(o):
+    """<grad, u> equals the central difference of <grad_out, forward> along u
+    for each of q, k and v (the forward oracle dot_softmax)."""
+    for seed in range(3):
+        n, e, h, c = [(30, 220, 2, 3), (40, 350, 1, 4), (20, 90, 4, 2)][seed]
+        f = h * c
+        wl = gg.random_edge_case_graph(n, e, f, 170 + seed, hub=1, isolated=3)
+        ei = wl.edge_index
+        rng = np.random.default_rng(170 + seed)
+        q, k, v, g = (rng.standard_normal((n, f)) for _ in range(4))
+        gq, gk, gv, _ = o.dot_softmax_backward(ei, n, q, k, v, h, c, 0.4, g)
+
+        def loss(qq, kk, vv):
+            out, _, _ = oracle.dot_softmax(ei, n, qq, kk, vv, h, c, 0.4)
+            return float(np.sum(out * g))
+        eps = 1e-6
+        for name, grad, shift in (("q", gq, (1, 0, 0)), ("k", gk, (0, 1, 0)), ("v", gv, (0, 0, 1))):
+            u = rng.standard_normal((n, f))
+            plus = [t + eps * u * sh for t, sh in zip((q, k, v), shift)]
+            minus = [t - eps * u * sh for t, sh in zip((q, k, v), shift)]
+            fd = (loss(*plus) - loss(*minus)) / (2 * eps)
+            assert abs(np.sum(grad * u) - fd) <= 1e-6 * (1 + abs(fd)), (name, seed)
+
+
+def test_dot_backward_finite_differences():
+    pin_dot_backward_finite_differences(oracle.default)
+
+
+def pin_dot_backward_limits(o):
+    """q = 0 makes every weight 1/in-degree, so v's gradient is the mean
+    aggregation's backward; a single in-edge per target has weight 1, so q
+    and k receive no gradient and v's gradient is grad_out routed back."""
+    n, e, h, c = 40, 300, 2, 4
+    wl = gg.random_edge_case_graph(n, e, h * c, 180, hub=2, isolated=4)
+    ei = wl.edge_index
+    rng = np.random.default_rng(180)
+    k, v, g = (rng.standard_normal((n, h * c)) for _ in range(3))
+    _, _, gv, (_, _, av) = o.dot_softmax_backward(ei, n, np.zeros((n, h * c)), k, v, h, c, 0.5, g)
+    mb, mab = oracle.aggregate_backward(ei, n, g, "mean")
+    np.testing.assert_allclose(gv, mb, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(av, mab, rtol=1e-12, atol=1e-12)
+    one = np.array([[3, 7, 1], [5, 9, 2]])
+    q = rng.standard_normal((10, h * c))
+    gq, gk, gv, _ = o.dot_softmax_backward(one, 10, q, k[:10], v[:10], h, c, 0.5, g[:10])
+    np.testing.assert_allclose(gq, 0.0, atol=1e-13)
+    np.testing.assert_allclose(gk, 0.0, atol=1e-13)
+    want = np.zeros((10, h * c))
+    for s_, t_ in zip(one[0], one[1]):
+        want[s_] += g[t_]
+    np.testing.assert_allclose(gv, want, rtol=1e-13, atol=1e-13)
+
+
+def test_dot_backward_limits():
+    pin_dot_backward_limits(oracle.default)
+
+
 # ---------------------------------------------------------------------------
 # Error scales: every tolerance is a multiple of the oracle's absout, so it is
 # pinned to an independent numpy form -- |M| |X| with dense matrices, and for
@@ -813,8 +869,9 @@ PLANTS = {
     "APPNP_TELEPORT_FROM_H": [pin_appnp_hand_example, pin_appnp_dense_closed_form],
     "DOT_KEY_AT_TARGET": [pin_dot_star],
     "BACKWARD_NO_TRANSPOSE": [pin_backward_finite_differences, pin_backward_dense_transpose],
-    "SCALE_DOUBLED": [pin_error_scales, pin_gat_backward_limits],
-    "BWD_NO_SOFTMAX_JACOBIAN": [pin_gat_backward_finite_differences],
+    "SCALE_DOUBLED": [pin_error_scales, pin_gat_backward_limits, pin_dot_backward_limits],
+    "BWD_NO_SOFTMAX_JACOBIAN": [pin_gat_backward_finite_differences,
+                                pin_dot_backward_finite_differences],
 }
 
 
