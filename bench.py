@@ -502,7 +502,7 @@ def next_rows(L, wl, bufs, stream, hbm_peak):
     of the headline value): APPNP K = 10 on the same graph and bf16 features,
     the backward of the GCN aggregation, max with argmax and its backward,
     Transformer-style (dot-product) attention with bf16 q, k, v of the same
-    8 x 16 layout, the fused Mean-Max pool on the GCN output, and device
+    8 x 16 layout and its backward, the GAT backward, the fused Mean-Max pool on the GCN output, and device
     BatchGraph construction on 1,024 molecule-sized graphs."""
     import torch
     from paper_2101_11552_gb300 import graphgen as gg
@@ -594,8 +594,9 @@ def next_rows(L, wl, bufs, stream, hbm_peak):
     rows["gat_backward"] = {"ms": round(ms, 4), "heads": heads, "channels": ch,
                             "edge_features_per_s": e * f / (ms * 1e-3),
                             "note": "grad_x, grad_a_src, grad_a_dst of the bf16 8 x 16 edge softmax; "
-                                    "CSR by source built once; warp per row, lanes over features"}
-    del csr_src, grad_x, out_max, argmax, fwd, ws_b, ws_f
+                                    "CSR by source built once; one online pass per target row, "
+                                    "then one pass per source row gathering fp32 grad_out rows"}
+    del out_max, argmax, ws_b, ws_f
 
     heads, ch = wl.heads, wl.channels
     gen = torch.Generator(device=dev)
@@ -612,7 +613,18 @@ def next_rows(L, wl, bufs, stream, hbm_peak):
                            "gbs": round(abytes / (ms * 1e-3) / 1e9, 1),
                            "frac": round(abytes / (ms * 1e-3) / 1e9 / hbm_peak, 4),
                            "algorithmic_bytes": abytes}
-    del qkv, att
+    ws_d = torch.empty(tfg.tfg_dot_edge_softmax_backward_workspace_size(n, heads, ch),
+                       dtype=torch.uint8, device=dev)
+    gq, gk, gv = (torch.empty(n, f, dtype=torch.float32, device=dev) for _ in range(3))
+    ms = _event_ms(lambda: check(L.tfg_dot_edge_softmax_aggregate_backward(
+        P(bufs["rowptr"]), P(bufs["col"]), P(csr_src.rowptr), P(csr_src.col), *[P(t) for t in qkv],
+        tfg.TFG_BF16, n, e, heads, ch, 1.0 / ch ** 0.5, P(att), P(fwd), P(gq), P(gk), P(gv),
+        P(ws_d), ws_d.numel(), sp)), stream, 3)
+    rows["dot_backward"] = {"ms": round(ms, 4), "heads": heads, "channels": ch,
+                            "edge_features_per_s": e * f / (ms * 1e-3),
+                            "note": "grad_q, grad_k, grad_v of the bf16 8 x 16 dot-product "
+                                    "attention (grad_out = the GAT output, fp32)"}
+    del qkv, att, gq, gk, gv, ws_d, csr_src, grad_x, fwd
 
     pooled = torch.empty(g, 2 * f, dtype=torch.float32, device=dev)
     st = torch.zeros(1, dtype=torch.int32, device=dev)
