@@ -76,6 +76,16 @@ def test_csr_out_of_range_ids_set_status():
     assert rp[0] == 0 and rp[-1] == 4 and np.all(np.diff(rp) >= 0)
 
 
+def test_csr_many_tiles_bit_exact():
+    """2.5M edges over 200,000 nodes: 611 tiles in each of the two passes."""
+    n = 200_000
+    wl = gg.random_edge_case_graph(n, 2_500_000, 1, 78, hub=5, isolated=100)
+    want = oracle.build_csr(wl.edge_index, n)
+    got = gpu_csr(wl.edge_index, n)
+    for name, g, w in zip(("rowptr", "col", "perm", "in_degree"), got[:4], want):
+        assert np.array_equal(np_(g), w), name
+
+
 # ---------------------------------------------------------------------------
 # GCN normalisation
 # ---------------------------------------------------------------------------
