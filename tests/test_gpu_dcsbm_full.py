@@ -183,3 +183,87 @@ def test_dcsbm_gcn_backward_sampled_rows(dcsbm):
     ref, scale = oracle.aggregate_rows(ocsr_src, n, g, "sum", rows, w=nrm["w_norm"],
                                        self_w=nrm["self_w"])
     assert_scaled_close(got, ref, scale, TOL_F32, "dcsbm gcn backward")
+
+
+def _dependency_subgraph(wl, ocsr, sources):
+    """Original ids (ascending) of every edge the backward rows of `sources`
+    depend on: the in-edges of each source and of each target of its
+    out-edges (the softmax of a target runs over all of its in-edges)."""
+    ei = wl.edge_index
+    out_targets = np.unique(ei[1][np.isin(ei[0], sources)])
+    nodes = np.unique(np.concatenate([out_targets, sources]))
+    rp, perm = np.asarray(ocsr[0], np.int64), np.asarray(ocsr[2], np.int64)
+    ids = np.concatenate([perm[rp[t]:rp[t + 1]] for t in nodes])
+    return np.sort(ids)
+
+
+def _backward_sources(ocsr):
+    deg = ocsr[3]
+    rng = np.random.default_rng(41)
+    hubs = np.argsort(deg)[-2:]
+    low = np.argsort(deg)[:3]
+    return np.unique(np.concatenate([hubs, low, rng.choice(len(deg), 10, replace=False)])).astype(np.int64)
+
+
+def test_dcsbm_gat_backward_sampled_rows(dcsbm):
+    """GAT backward at full size (the launch the benchmark's next-row times):
+    grad_x of sampled nodes -- the two largest hubs, the lowest-degree nodes and a
+    random sample -- against the oracle's backward on the exact sub-graph those
+    rows depend on."""
+    wl, ocsr, csr, _ = dcsbm
+    n, h, c = wl.num_nodes, wl.heads, wl.channels
+    ei = dev(wl.edge_index)
+    csr_src = tfg.tfg_build_csr_by_source(ei, n)
+    tfg.check_status(csr_src.status)
+    del ei
+    x = dev(wl.x_bf16.view(np.int16)).view(torch.bfloat16)
+    a_s, a_d = dev(wl.a_src), dev(wl.a_dst)
+    out, _ = tfg.tfg_edge_softmax_aggregate(csr.rowptr, csr.col, x, h, c, a_s, a_d,
+                                            wl.negative_slope)
+    g = np.random.default_rng(43).standard_normal((n, h * c)).astype(np.float32)
+    gx, _, _ = tfg.tfg_edge_softmax_aggregate_backward(csr.rowptr, csr.col, csr_src.rowptr,
+                                                       csr_src.col, x, h, c, a_s, a_d,
+                                                       wl.negative_slope, out, dev(g))
+    sources = _backward_sources(ocsr)
+    got = gx[dev(sources)].cpu().numpy()
+    ids = _dependency_subgraph(wl, ocsr, sources)
+    sub = np.ascontiguousarray(wl.edge_index[:, ids])
+    rgx, _, _, (sx, _, _) = oracle.edge_softmax_backward(sub, n, wl.x_bf16, h, c, wl.a_src,
+                                                         wl.a_dst, wl.negative_slope, g)
+    lam = gat_logit_mag(oracle.widen(wl.x_bf16), sub[0], sub[1], h, c, wl.a_src, wl.a_dst)
+    lam_max = np.zeros((n, h))
+    np.maximum.at(lam_max, sub[1], lam)
+    tol = TOL_F32 + KAPPA_GAT * float(np.max(lam + lam_max[sub[1]]))
+    assert_scaled_close(got, rgx[sources], sx[sources], tol, "dcsbm gat backward grad_x")
+
+
+def test_dcsbm_dot_backward_sampled_rows(dcsbm):
+    """Dot-product attention backward at full size: grad_q, grad_k and grad_v
+    of the same sampled nodes against the oracle on their dependency
+    sub-graph (q, k, v bf16 [N, 8 x 16] as in the forward test)."""
+    wl, ocsr, csr, _ = dcsbm
+    n = wl.num_nodes
+    ei = dev(wl.edge_index)
+    csr_src = tfg.tfg_build_csr_by_source(ei, n)
+    tfg.check_status(csr_src.status)
+    del ei
+    rng = np.random.default_rng(1305)
+    bits = [gg.bf16_bits_rne(rng.standard_normal((n, 128), dtype=np.float32)) for _ in range(3)]
+    q, k, v = (dev(b.view(np.int16)).view(torch.bfloat16) for b in bits)
+    out, _ = tfg.tfg_dot_edge_softmax_aggregate(csr.rowptr, csr.col, q, k, v, 8, 16, scale=0.25)
+    g = np.random.default_rng(47).standard_normal((n, 128)).astype(np.float32)
+    grads = tfg.tfg_dot_edge_softmax_aggregate_backward(csr.rowptr, csr.col, csr_src.rowptr,
+                                                        csr_src.col, q, k, v, 8, 16, 0.25, out,
+                                                        dev(g))
+    sources = _backward_sources(ocsr)
+    ids = _dependency_subgraph(wl, ocsr, sources)
+    sub = np.ascontiguousarray(wl.edge_index[:, ids])
+    rq, rk, rv, (sq, sk, sv) = oracle.dot_softmax_backward(sub, n, *bits, 8, 16, 0.25, g)
+    lam = dot_logit_mag(oracle.widen(bits[0]), oracle.widen(bits[1]), sub[0], sub[1], 8, 16, 0.25)
+    lam_max = np.zeros((n, 8))
+    np.maximum.at(lam_max, sub[1], lam)
+    tol = TOL_F32 + kappa_dot(16) * float(np.max(lam + lam_max[sub[1]]))
+    for name, got, ref, sc in (("grad_q", grads[0], rq, sq), ("grad_k", grads[1], rk, sk),
+                               ("grad_v", grads[2], rv, sv)):
+        assert_scaled_close(got[dev(sources)].cpu().numpy(), ref[sources], sc[sources], tol,
+                            f"dcsbm dot backward {name}")
