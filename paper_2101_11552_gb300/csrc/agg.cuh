@@ -84,7 +84,8 @@ struct Agg {
     static constexpr int kUnroll = unroll_for<VEC, kIsMax>();
     // a step's slots j + u * G + g must stay inside one 32-edge chunk: full
     // chunks take no slot test, so a wider step would add edges twice
-    static_assert(G * kUnroll <= 32, "G * kUnroll must not exceed the 32-edge chunk");
+    static_assert(G * kUnroll <= 32 && 32 % (G * kUnroll) == 0,
+                  "steps of G * kUnroll slots must tile the 32-edge chunk");
 
     static __device__ __forceinline__ float identity() { return kIsMax ? -CUDART_INF_F : 0.f; }
 
@@ -384,7 +385,8 @@ struct MpAgg {
     static constexpr int kDepth = kSlots < mp_depth<VEC, A::kIsMax>() ? kSlots
                                                                       : mp_depth<VEC, A::kIsMax>();
     static constexpr int kF = LPR * VEC;
-    static_assert(G * kDepth <= 32, "a batch must stay inside one 32-edge chunk");
+    static_assert(G * kDepth <= 32 && kSlots % kDepth == 0 && kDepth % 2 == 0,
+                  "batches of kDepth slots (pairs) must tile a group's slots of the chunk");
 
     // Write the finished row t from the lane groups' reduced accumulator.
     static __device__ __forceinline__ void store_row(const AggArgs &a, int64_t t,

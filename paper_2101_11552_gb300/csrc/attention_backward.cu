@@ -304,8 +304,14 @@ struct FastBwArgs {
 };
 
 constexpr int64_t kFbMinWork = 2048;   // edges + rows per CTA, at least
-constexpr int kFbUnroll = 4;       // row gathers in flight per lane, target pass
-constexpr int kFbUnrollSrc = 4;    // row gathers in flight per lane, source pass
+#ifndef TFG_FB_UNROLL_TGT
+#define TFG_FB_UNROLL_TGT 4        // row gathers in flight per lane, target pass
+#endif
+#ifndef TFG_FB_UNROLL_SRC
+#define TFG_FB_UNROLL_SRC 4        // row gathers in flight per lane, source pass
+#endif
+constexpr int kFbUnroll = TFG_FB_UNROLL_TGT;
+constexpr int kFbUnrollSrc = TFG_FB_UNROLL_SRC;
 // Measured on the 114.6M-edge graph (bf16, 8 heads x 16): 3 / 3 CTAs per SM
 // 13.43 ms, 4 target / 3 source 13.20, 3 / 4 12.60, 4 / 4 12.37.
 #ifndef TFG_FB_TGT_BLOCKS
@@ -328,7 +334,8 @@ __device__ __forceinline__ void fast_bwd_target(const FastBwArgs &a, int64_t t, 
     constexpr int ES = 32 / H;      // edges per score step
     constexpr int R = H;            // score steps per 32-edge chunk
     static_assert(ES % G == 0, "score step must hold whole feature steps");
-    static_assert(G * kFbUnroll <= 32, "a feature step must stay inside the 32-edge chunk");
+    static_assert(G * kFbUnroll <= 32 && 32 % (G * kFbUnroll) == 0,
+                  "feature steps of G * kFbUnroll slots must tile the 32-edge chunk");
     const int se = lane / H, sh = lane % H;
     const int g = lane / LPR, sub = lane % LPR;
     const int f = H * a.channels;
@@ -447,7 +454,8 @@ __device__ __forceinline__ void fast_bwd_source(const FastBwArgs &a, int64_t s, 
     constexpr int ES = 32 / H;      // edges per score step
     constexpr int R = H;
     static_assert(ES % G == 0, "score step must hold whole feature steps");
-    static_assert(G * kFbUnrollSrc <= 32, "a feature step must stay inside the 32-edge chunk");
+    static_assert(G * kFbUnrollSrc <= 32 && 32 % (G * kFbUnrollSrc) == 0,
+                  "feature steps of G * kFbUnrollSrc slots must tile the 32-edge chunk");
     const int se = lane / H, sh = lane % H;
     const int g = lane / LPR, sub = lane % LPR;
     const int f = H * a.channels;

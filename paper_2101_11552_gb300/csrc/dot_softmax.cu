@@ -133,7 +133,8 @@ __device__ __forceinline__ void dot_fast_row(const DotArgs &a, int lh_arg, int64
     constexpr int kDotUnroll = dot_unroll<VEC>();
     // a step's slots j + u * G + g must stay inside one 32-edge chunk: full
     // chunks take no slot test, so a wider step would add edges twice
-    static_assert(G * kDotUnroll <= 32, "G * kDotUnroll must not exceed the 32-edge chunk");
+    static_assert(G * kDotUnroll <= 32 && 32 % (G * kDotUnroll) == 0,
+                  "steps of G * kDotUnroll slots must tile the 32-edge chunk");
     const int g = lane / LPR, sub = lane % LPR;
     const int64_t f = static_cast<int64_t>(a.heads) * a.channels;
     const XT *qp = static_cast<const XT *>(a.q);

@@ -228,7 +228,8 @@ __device__ __forceinline__ void fast_row(const int32_t *__restrict__ rowptr,
     static_assert(ES % G == 0, "score step must hold whole feature steps");
     // a step's slots e + u * G + g must stay inside one 32-edge chunk (full
     // chunks take no slot test, and p[k0 / ES] must stay inside p[R])
-    static_assert(G * kSmUnroll <= 32, "G * kSmUnroll must not exceed the 32-edge chunk");
+    static_assert(G * kSmUnroll <= 32 && 32 % (G * kSmUnroll) == 0,
+                  "steps of G * kSmUnroll slots must tile the 32-edge chunk");
     const int se = lane / H, sh = lane % H;
     const int g = lane / LPR, sub = lane % LPR;
     const int f = H * channels;
@@ -438,7 +439,8 @@ struct SmMp {
     static constexpr int R = 32 / ES;      // score steps per 32-edge chunk (= H)
     static constexpr int kF = LPR * VEC;
     static_assert(ES % G == 0, "score step must hold whole feature steps");
-    static_assert(G * kSmUnroll <= 32, "G * kSmUnroll must not exceed the 32-edge chunk");
+    static_assert(G * kSmUnroll <= 32 && 32 % (G * kSmUnroll) == 0,
+                  "steps of G * kSmUnroll slots must tile the 32-edge chunk");
 
     // One chunk of up to 32 edges of one row (ids in c, lane j holds edge j):
     // the logits of the chunk (score lanes), the running maximum, then the
