@@ -304,6 +304,9 @@ struct FastBwArgs {
 };
 
 constexpr int64_t kFbMinWork = 2048;   // edges + rows per CTA, at least
+#ifndef TFG_FB_STAGE
+#define TFG_FB_STAGE 1             // source pass: per-chunk weights staged in shared memory
+#endif
 #ifndef TFG_FB_UNROLL_TGT
 #define TFG_FB_UNROLL_TGT 4        // row gathers in flight per lane, target pass
 #endif
@@ -449,7 +452,8 @@ __device__ __forceinline__ void fast_bwd_target(const FastBwArgs &a, int64_t t, 
 // 14.65 ms in one launch, 14.59 in two, 15.06 in four -- the pass is bound by
 // latency, not by DRAM bytes.)
 template <typename XT, int LPR, int H>
-__device__ __forceinline__ void fast_bwd_source(const FastBwArgs &a, int64_t s, int lane) {
+__device__ __forceinline__ void fast_bwd_source(const FastBwArgs &a, int64_t s, int lane,
+                                                float4 *__restrict__ stage) {
     constexpr int G = 32 / LPR;     // edges per feature step
     constexpr int ES = 32 / H;      // edges per score step
     constexpr int R = H;
@@ -484,6 +488,26 @@ __device__ __forceinline__ void fast_bwd_source(const FastBwArgs &a, int64_t s, 
         for (int u = 0; u < kFbUnrollSrc; ++u)
             raw0[u] = gather(static_cast<uint32_t>(__shfl_sync(kFull, c, (u * G + g) & 31)));
         // alpha, af = alpha * slope(z) and ab = af * beta of (edge, head)
+#if TFG_FB_STAGE
+        // score lanes stage them per (edge, head) in the warp's shared-memory
+        // slots (lane-consecutive: conflict-free); feature lanes read their
+        // (edge, head) with one 16-byte load instead of three shuffles
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const int k = r * ES + se;
+            const int t = __shfl_sync(kFull, c, k);
+            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (k < cnt) {
+                const float4 st = __ldg(a.stats + static_cast<int64_t>(t) * H + sh);
+                const float z = ss + st.x;
+                v.x = exp2f(bw_leaky(z, a.slope) - st.y) * st.z;
+                v.y = v.x * (z > 0.f ? 1.f : a.slope);
+                v.z = v.y * st.w;
+            }
+            stage[k * H + sh] = v;
+        }
+        __syncwarp();
+#else
         float al[R], af[R], ab[R];
 #pragma unroll
         for (int r = 0; r < R; ++r) {
@@ -498,6 +522,7 @@ __device__ __forceinline__ void fast_bwd_source(const FastBwArgs &a, int64_t s, 
                 ab[r] = af[r] * st.w;
             }
         }
+#endif
         float part[4] = {0.f, 0.f, 0.f, 0.f}, partd = 0.f;
 #pragma unroll
         for (int e = 0; e < 32; e += G * kFbUnrollSrc) {
@@ -508,10 +533,17 @@ __device__ __forceinline__ void fast_bwd_source(const FastBwArgs &a, int64_t s, 
             for (int u = 0; u < kFbUnrollSrc; ++u) {
                 const int k0 = e + u * G;
                 const int k = k0 + g;
+#if TFG_FB_STAGE
+                const float4 w = stage[k * H + fh];
+                wa[u] = w.x;
+                wf[u] = w.y;
+                wb[u] = w.z;
+#else
                 const int from = ((k0 % ES) + g) * H + fh;
                 wa[u] = __shfl_sync(kFull, al[k0 / ES], from);
                 wf[u] = __shfl_sync(kFull, af[k0 / ES], from);
                 wb[u] = __shfl_sync(kFull, ab[k0 / ES], from);
+#endif
                 if (e == 0) raw[u] = raw0[u];
                 else raw[u] = gather(static_cast<uint32_t>(__shfl_sync(kFull, c, k & 31)));
             }
@@ -530,6 +562,9 @@ __device__ __forceinline__ void fast_bwd_source(const FastBwArgs &a, int64_t s, 
 #pragma unroll
         for (int q = 0; q < 4; ++q) px[q] += part[q];
         pdz += partd;
+#if TFG_FB_STAGE
+        __syncwarp();   // every lane has read the stage before the next chunk writes it
+#endif
     }
 #pragma unroll
     for (int o = LPR; o < 32; o <<= 1) {
@@ -559,7 +594,9 @@ __global__ void __launch_bounds__(kBwThreads, TFG_FB_TGT_BLOCKS) fast_bwd_target
 
 template <typename XT, int LPR, int H>
 __global__ void __launch_bounds__(kBwThreads, TFG_FB_SRC_BLOCKS) fast_bwd_sources(FastBwArgs a) {
-    for_each_row(a.rowptr_src, a.n, [&](int64_t s, int lane) { fast_bwd_source<XT, LPR, H>(a, s, lane); });
+    __shared__ float4 s_stage[TFG_FB_STAGE ? kBwWarps : 1][TFG_FB_STAGE ? 32 * H : 1];
+    float4 *stage = s_stage[TFG_FB_STAGE ? (threadIdx.x >> 5) : 0];
+    for_each_row(a.rowptr_src, a.n, [&](int64_t s, int lane) { fast_bwd_source<XT, LPR, H>(a, s, lane, stage); });
 }
 
 // ---------------------------------------------------------------------------
