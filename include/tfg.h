@@ -74,6 +74,16 @@ int tfg_version(void);
 /* Description of the last host-side failure on this thread ("" if none). */
 const char *tfg_last_error(void);
 
+/* 1 in the bounds-checked debug build (compiled with TFG_CHECK_BOUNDS=1),
+ * 0 in the default build.  The debug build checks, before every launch,
+ * that each device buffer a call touches lies inside its allocation and
+ * that caller-built index arrays are valid (rowptr[0] = 0, rowptr[N] = E,
+ * rowptr non-decreasing, col ids in [0, N), perm ids in [0, E)); a
+ * violation returns TFG_ERR_INDEX_RANGE (TFG_ERR_INVALID_ARG for a pointer
+ * that is not device memory) and launches nothing.  Each check reads the
+ * arrays once on the device and synchronises the stream: a debugging aid. */
+int tfg_check_bounds_enabled(void);
+
 /* ------------------------------------------------------------------------
  * Grouping by the reduce key: COO -> CSR by target.
  * Section 2.1.2 / Fig. 5b: a reducer gathers the elements that share a key

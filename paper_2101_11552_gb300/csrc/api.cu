@@ -67,6 +67,79 @@ int check_dtype(const char *fn, int dtype) {
             return fail(TFG_ERR_INVALID_ARG, "%s: %s must not be NULL", fn, name);    \
     } while (0)
 
+// ---- bounds-checked debug build (TFG_CHECK_BOUNDS=1) ----------------------
+// Before any launch, every device buffer is checked against the allocation
+// that holds it (the bytes the call will touch must lie inside it), and every
+// caller-built index array is read once on the device: rowptr[0] = 0,
+// rowptr[N] = E, rowptr non-decreasing, col ids in [0, N), perm ids in
+// [0, E).  A violation returns TFG_ERR_INDEX_RANGE with the reason and
+// launches nothing, so no kernel reads out of bounds.  Each check copies a
+// few values to the host and synchronises the stream: a debugging aid, not a
+// production mode.  The default build compiles none of it.
+#ifndef TFG_CHECK_BOUNDS
+#define TFG_CHECK_BOUNDS 0
+#endif
+
+#if TFG_CHECK_BOUNDS
+int debug_extent(const char *fn, const char *name, const void *p, size_t bytes) {
+    if (p == nullptr || bytes == 0) return TFG_OK;
+    uintptr_t base = 0;
+    size_t size = 0;
+    if (!tfg::allocation_range(p, &base, &size))
+        return fail(TFG_ERR_INVALID_ARG, "%s: %s is not device memory of the current context", fn,
+                    name);
+    const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+    if (a + bytes > base + size)
+        return fail(TFG_ERR_INDEX_RANGE,
+                    "%s: %s must hold %zu bytes, its allocation ends %zu bytes after it", fn, name,
+                    bytes, static_cast<size_t>(base + size - a));
+    return TFG_OK;
+}
+
+// rowptr [N + 1] (or NULL: col ids only, E = e_given), col [E] and perm [E]
+// each NULL when the call does not read it (a NULL col that the call reads
+// is refused when E > 0); e_given < 0 takes E from rowptr[N].  E is returned
+// in *e_out.
+int debug_csr(const char *fn, const char *which, const int32_t *rowptr, const int32_t *col,
+              const int32_t *perm, int64_t n, int64_t e_given, int64_t *e_out,
+              tfg_stream_t stream, bool col_read = true) {
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    int64_t e = e_given;
+    if (rowptr) {
+        TFG_TRY(debug_extent(fn, "rowptr", rowptr, sizeof(int32_t) * size_t(n + 1)));
+        int32_t first = 0, last = 0;
+        cudaError_t err = tfg::csr_ends(rowptr, n, &first, &last, s);
+        if (err != cudaSuccess) return cuda_result(err, fn);
+        if (first != 0 || last < 0 || (e_given >= 0 && last != e_given))
+            return fail(TFG_ERR_INDEX_RANGE, "%s: %s rowptr[0] = %d, rowptr[N] = %d (E = %lld)",
+                        fn, which, first, last, (long long)e_given);
+        e = last;
+    }
+    if (e_out) *e_out = e;
+    if (e > 0 && col_read && col == nullptr)
+        return fail(TFG_ERR_INVALID_ARG, "%s: %s is NULL but the graph has %lld edges", fn, which,
+                    (long long)e);
+    if (e > 0) {
+        TFG_TRY(debug_extent(fn, "col", col, sizeof(int32_t) * size_t(e)));
+        TFG_TRY(debug_extent(fn, "perm", perm, sizeof(int32_t) * size_t(e)));
+    }
+    int flags = 0;
+    cudaError_t err = tfg::validate_csr(rowptr, col, perm, n, e, &flags, s);
+    if (err != cudaSuccess) return cuda_result(err, fn);
+    if (flags & 1) return fail(TFG_ERR_INDEX_RANGE, "%s: %s rowptr decreases", fn, which);
+    if (flags & 2) return fail(TFG_ERR_INDEX_RANGE, "%s: a %s id lies outside [0, N)", fn, which);
+    if (flags & 4) return fail(TFG_ERR_INDEX_RANGE, "%s: a %s perm id lies outside [0, E)", fn, which);
+    return TFG_OK;
+}
+#define TFG_DEBUG(expr) TFG_TRY(expr)
+
+size_t elem_bytes(int dtype) { return dtype == TFG_BF16 ? 2 : 4; }
+#else
+#define TFG_DEBUG(expr) \
+    do {                \
+    } while (0)
+#endif
+
 int aggregate_common(const char *fn, int mode, const int32_t *rowptr, const int32_t *col,
                      const float *w, const float *dinv, const void *x, int dtype, int64_t n,
                      int64_t f, int add_self, float fill, float *out, tfg_stream_t stream) {
@@ -77,6 +150,16 @@ int aggregate_common(const char *fn, int mode, const int32_t *rowptr, const int3
     TFG_NEED(x, n > 0, fn, "x");
     TFG_NEED(out, n > 0, fn, "out");
     TFG_NEED(dinv, mode == 3 && n > 0, fn, "dinv");
+#if TFG_CHECK_BOUNDS
+    {
+        int64_t e = 0;
+        TFG_DEBUG(debug_csr(fn, "col", rowptr, col, nullptr, n, -1, &e, stream));
+        TFG_DEBUG(debug_extent(fn, "w_csr", w, sizeof(float) * size_t(e)));
+        TFG_DEBUG(debug_extent(fn, "dinv", dinv, sizeof(float) * size_t(n)));
+        TFG_DEBUG(debug_extent(fn, "x", x, elem_bytes(dtype) * size_t(n * f)));
+        TFG_DEBUG(debug_extent(fn, "out", out, sizeof(float) * size_t(n * f)));
+    }
+#endif
     return cuda_result(tfg::launch_aggregate(mode, rowptr, col, w, dinv, x, dtype, n, f, add_self,
                                              fill, out, reinterpret_cast<cudaStream_t>(stream)),
                        fn);
@@ -107,6 +190,17 @@ int propagate_common(const char *fn, const int32_t *rowptr, const int32_t *col, 
         if (reinterpret_cast<uintptr_t>(ws) % 16 != 0)
             return fail(TFG_ERR_INVALID_ARG, "%s: workspace must be 16-byte aligned", fn);
     }
+#if TFG_CHECK_BOUNDS
+    if (hops > 0) {
+        int64_t e = 0;
+        TFG_DEBUG(debug_csr(fn, "col", rowptr, col, nullptr, n, -1, &e, stream));
+        TFG_DEBUG(debug_extent(fn, "w_csr", w, sizeof(float) * size_t(e)));
+        TFG_DEBUG(debug_extent(fn, "dinv", dinv, sizeof(float) * size_t(n)));
+    }
+    TFG_DEBUG(debug_extent(fn, "x0", x0, elem_bytes(dtype) * size_t(n * f)));
+    TFG_DEBUG(debug_extent(fn, "out", out, sizeof(float) * size_t(n * f)));
+    TFG_DEBUG(debug_extent(fn, "workspace", ws, need));
+#endif
     return cuda_result(tfg::launch_propagate(rowptr, col, w, dinv, x0, dtype, n, f, hops, alpha,
                                              add_self, fill, out, ws,
                                              reinterpret_cast<cudaStream_t>(stream)),
@@ -141,6 +235,8 @@ extern "C" {
 
 int tfg_version(void) { return 200; }
 
+int tfg_check_bounds_enabled(void) { return TFG_CHECK_BOUNDS; }
+
 const char *tfg_last_error(void) { return g_err; }
 
 int tfg_build_csr_workspace_size(int64_t num_nodes, int64_t num_edges, size_t *bytes) {
@@ -171,6 +267,12 @@ int build_csr_common(const char *fn, bool by_source, const int64_t *edge_index, 
         if (reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
             return fail(TFG_ERR_INVALID_ARG, "%s: workspace must be 256-byte aligned", fn);
     }
+    TFG_DEBUG(debug_extent(fn, "edge_index", edge_index, sizeof(int64_t) * 2 * size_t(num_edges)));
+    TFG_DEBUG(debug_extent(fn, "rowptr", rowptr, sizeof(int32_t) * size_t(num_nodes + 1)));
+    TFG_DEBUG(debug_extent(fn, "col", col, sizeof(int32_t) * size_t(num_edges)));
+    TFG_DEBUG(debug_extent(fn, "perm", perm, sizeof(int32_t) * size_t(num_edges)));
+    TFG_DEBUG(debug_extent(fn, "in_degree", in_degree, sizeof(int32_t) * size_t(num_nodes)));
+    TFG_DEBUG(debug_extent(fn, "workspace", num_edges > 0 ? workspace : nullptr, need));
     return cuda_result(tfg::launch_build_csr(edge_index, num_edges, num_nodes, rowptr, col, perm,
                                              in_degree, workspace, status,
                                              reinterpret_cast<cudaStream_t>(stream), by_source),
@@ -205,6 +307,11 @@ int tfg_gcn_norm(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
     TFG_NEED(dinv, num_nodes > 0, fn, "dinv");
     TFG_NEED(col, w_csr != nullptr && num_edges > 0, fn, "col");
     TFG_NEED(perm, (w_csr != nullptr || edge_weight != nullptr) && num_edges > 0, fn, "perm");
+    TFG_DEBUG(debug_csr(fn, "col", rowptr, w_csr ? col : nullptr, w_csr || edge_weight ? perm : nullptr,
+                        num_nodes, num_edges, nullptr, stream, w_csr != nullptr));
+    TFG_DEBUG(debug_extent(fn, "edge_weight", edge_weight, sizeof(float) * size_t(num_edges)));
+    TFG_DEBUG(debug_extent(fn, "dinv", dinv, sizeof(float) * size_t(num_nodes)));
+    TFG_DEBUG(debug_extent(fn, "w_csr", w_csr, sizeof(float) * size_t(num_edges)));
     return cuda_result(tfg::launch_gcn_norm(rowptr, col, perm, edge_weight, num_nodes,
                                             add_self_loops, self_loop_fill, dinv, w_csr,
                                             reinterpret_cast<cudaStream_t>(stream)),
@@ -272,6 +379,14 @@ int tfg_aggregate_backward(int reduce, const int32_t *rowptr_src, const int32_t 
     if (need > 0 && (workspace == nullptr || workspace_bytes < need))
         return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
                     workspace ? workspace_bytes : size_t(0));
+    TFG_DEBUG(debug_csr(fn, "col_src", rowptr_src, col_src, weighted ? perm_src : nullptr, num_nodes,
+                        num_edges, nullptr, stream));
+    TFG_DEBUG(debug_extent(fn, "edge_weight", edge_weight, sizeof(float) * size_t(num_edges)));
+    TFG_DEBUG(debug_extent(fn, "in_degree", reduce == TFG_MEAN ? in_degree : nullptr,
+                           sizeof(int32_t) * size_t(num_nodes)));
+    TFG_DEBUG(debug_extent(fn, "grad_out", grad_out, sizeof(float) * size_t(num_nodes * num_features)));
+    TFG_DEBUG(debug_extent(fn, "grad_x", grad_x, sizeof(float) * size_t(num_nodes * num_features)));
+    TFG_DEBUG(debug_extent(fn, "workspace", need ? workspace : nullptr, need));
     return cuda_result(tfg::launch_aggregate_backward(reduce, rowptr_src, col_src, perm_src,
                                                       edge_weight, in_degree, grad_out, num_nodes,
                                                       num_edges, num_features, grad_x, workspace,
@@ -301,6 +416,16 @@ int tfg_aggregate_max_argmax(const int32_t *rowptr, const int32_t *col, const in
     TFG_NEED(x, num_nodes > 0, fn, "x");
     TFG_NEED(out, num_nodes > 0, fn, "out");
     TFG_NEED(argmax, num_nodes > 0, fn, "argmax");
+#if TFG_CHECK_BOUNDS
+    {
+        int64_t e = 0;
+        TFG_DEBUG(debug_csr(fn, "col", rowptr, col, perm, num_nodes, -1, &e, stream));
+        TFG_DEBUG(debug_extent(fn, "w_csr", w_csr, sizeof(float) * size_t(e)));
+        TFG_DEBUG(debug_extent(fn, "x", x, elem_bytes(x_dtype) * size_t(num_nodes * num_features)));
+        TFG_DEBUG(debug_extent(fn, "out", out, sizeof(float) * size_t(num_nodes * num_features)));
+        TFG_DEBUG(debug_extent(fn, "argmax", argmax, sizeof(int32_t) * size_t(num_nodes * num_features)));
+    }
+#endif
     return cuda_result(tfg::launch_max_argmax(rowptr, col, perm, w_csr, x, x_dtype, num_nodes,
                                               num_features, out, argmax,
                                               reinterpret_cast<cudaStream_t>(stream)),
@@ -320,6 +445,16 @@ int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src
     TFG_NEED(argmax, num_nodes > 0, fn, "argmax");
     TFG_NEED(grad_out, num_nodes > 0, fn, "grad_out");
     TFG_NEED(grad_x, num_nodes > 0, fn, "grad_x");
+#if TFG_CHECK_BOUNDS
+    {
+        int64_t e = 0;
+        TFG_DEBUG(debug_csr(fn, "col_src", rowptr_src, col_src, perm_src, num_nodes, -1, &e, stream));
+        TFG_DEBUG(debug_extent(fn, "edge_weight", edge_weight, sizeof(float) * size_t(e)));
+        TFG_DEBUG(debug_extent(fn, "argmax", argmax, sizeof(int32_t) * size_t(num_nodes * num_features)));
+        TFG_DEBUG(debug_extent(fn, "grad_out", grad_out, sizeof(float) * size_t(num_nodes * num_features)));
+        TFG_DEBUG(debug_extent(fn, "grad_x", grad_x, sizeof(float) * size_t(num_nodes * num_features)));
+    }
+#endif
     return cuda_result(tfg::launch_max_backward(rowptr_src, col_src, perm_src, argmax,
                                                 edge_weight, grad_out, num_nodes, num_features,
                                                 grad_x,
@@ -390,6 +525,13 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
     if (num_nodes > 0 && (workspace == nullptr || workspace_bytes < need))
         return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
                     workspace ? workspace_bytes : size_t(0));
+    TFG_DEBUG(debug_csr(fn, "col", rowptr, col, nullptr, num_nodes, num_edges, nullptr, stream));
+    TFG_DEBUG(debug_extent(fn, "x", x, elem_bytes(x_dtype) * size_t(num_nodes * heads * channels)));
+    TFG_DEBUG(debug_extent(fn, "out", out, sizeof(float) * size_t(num_nodes * heads * channels)));
+    TFG_DEBUG(debug_extent(fn, "alpha", alpha, sizeof(float) * size_t(num_edges * heads)));
+    TFG_DEBUG(debug_extent(fn, "a_src", a_src, sizeof(float) * size_t(heads * channels)));
+    TFG_DEBUG(debug_extent(fn, "a_dst", a_dst, sizeof(float) * size_t(heads * channels)));
+    TFG_DEBUG(debug_extent(fn, "workspace", num_nodes > 0 ? workspace : nullptr, need));
     return cuda_result(tfg::launch_edge_softmax(rowptr, num_edges > 0 ? col : nullptr, x, x_dtype,
                                                 num_nodes, num_edges, heads, channels, a_src, a_dst,
                                                 negative_slope, out, alpha, workspace,
@@ -443,6 +585,19 @@ int tfg_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t *co
     if (workspace == nullptr || workspace_bytes < need)
         return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
                     workspace ? workspace_bytes : size_t(0));
+#if TFG_CHECK_BOUNDS
+    {
+        const size_t nf = size_t(num_nodes) * size_t(heads) * size_t(channels);
+        TFG_DEBUG(debug_csr(fn, "col", rowptr, col, nullptr, num_nodes, num_edges, nullptr, stream));
+        TFG_DEBUG(debug_csr(fn, "col_src", rowptr_src, col_src, nullptr, num_nodes, num_edges,
+                            nullptr, stream));
+        TFG_DEBUG(debug_extent(fn, "x", x, elem_bytes(x_dtype) * nf));
+        TFG_DEBUG(debug_extent(fn, "out", out, sizeof(float) * nf));
+        TFG_DEBUG(debug_extent(fn, "grad_out", grad_out, sizeof(float) * nf));
+        TFG_DEBUG(debug_extent(fn, "grad_x", grad_x, sizeof(float) * nf));
+        TFG_DEBUG(debug_extent(fn, "workspace", workspace, need));
+    }
+#endif
     return cuda_result(tfg::launch_edge_softmax_backward(
                            rowptr, col, rowptr_src, col_src, x, x_dtype, num_nodes,
                            num_edges, heads, channels, a_src, a_dst, negative_slope, out, grad_out, grad_x,
@@ -498,6 +653,23 @@ int tfg_dot_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t
     if (workspace == nullptr || workspace_bytes < need)
         return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
                     workspace ? workspace_bytes : size_t(0));
+#if TFG_CHECK_BOUNDS
+    {
+        const size_t nf = size_t(num_nodes) * size_t(heads) * size_t(channels);
+        TFG_DEBUG(debug_csr(fn, "col", rowptr, col, nullptr, num_nodes, num_edges, nullptr, stream));
+        TFG_DEBUG(debug_csr(fn, "col_src", rowptr_src, col_src, nullptr, num_nodes, num_edges,
+                            nullptr, stream));
+        TFG_DEBUG(debug_extent(fn, "q", q, elem_bytes(x_dtype) * nf));
+        TFG_DEBUG(debug_extent(fn, "k", k, elem_bytes(x_dtype) * nf));
+        TFG_DEBUG(debug_extent(fn, "v", v, elem_bytes(x_dtype) * nf));
+        TFG_DEBUG(debug_extent(fn, "out", out, sizeof(float) * nf));
+        TFG_DEBUG(debug_extent(fn, "grad_out", grad_out, sizeof(float) * nf));
+        TFG_DEBUG(debug_extent(fn, "grad_q", grad_q, sizeof(float) * nf));
+        TFG_DEBUG(debug_extent(fn, "grad_k", grad_k, sizeof(float) * nf));
+        TFG_DEBUG(debug_extent(fn, "grad_v", grad_v, sizeof(float) * nf));
+        TFG_DEBUG(debug_extent(fn, "workspace", workspace, need));
+    }
+#endif
     return cuda_result(tfg::launch_dot_softmax_backward(
                            rowptr, col, rowptr_src, col_src, q, k, v, x_dtype, num_nodes,
                            num_edges, heads, channels, scale, out, grad_out, grad_q, grad_k,
@@ -526,6 +698,17 @@ int tfg_dot_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, co
     TFG_NEED(k, num_nodes > 0, fn, "k");
     TFG_NEED(v, num_nodes > 0, fn, "v");
     TFG_NEED(out, num_nodes > 0, fn, "out");
+#if TFG_CHECK_BOUNDS
+    {
+        const size_t nf = size_t(num_nodes) * size_t(heads) * size_t(channels);
+        TFG_DEBUG(debug_csr(fn, "col", rowptr, col, nullptr, num_nodes, num_edges, nullptr, stream));
+        TFG_DEBUG(debug_extent(fn, "q", q, elem_bytes(x_dtype) * nf));
+        TFG_DEBUG(debug_extent(fn, "k", k, elem_bytes(x_dtype) * nf));
+        TFG_DEBUG(debug_extent(fn, "v", v, elem_bytes(x_dtype) * nf));
+        TFG_DEBUG(debug_extent(fn, "out", out, sizeof(float) * nf));
+        TFG_DEBUG(debug_extent(fn, "alpha", alpha, sizeof(float) * size_t(num_edges * heads)));
+    }
+#endif
     return cuda_result(tfg::launch_dot_softmax(rowptr, num_edges > 0 ? col : nullptr, q, k, v,
                                                x_dtype, num_nodes, num_edges, heads, channels,
                                                scale, out, alpha,
@@ -557,6 +740,10 @@ int tfg_edge_softmax_aggregate_noalloc(const int32_t *rowptr, const int32_t *col
     TFG_NEED(a_src, true, fn, "a_src");
     TFG_NEED(a_dst, true, fn, "a_dst");
     if (num_nodes == 0) return ok();
+    TFG_DEBUG(debug_csr(fn, "col", rowptr, col, nullptr, num_nodes, num_edges, nullptr, stream));
+    TFG_DEBUG(debug_extent(fn, "x", x, elem_bytes(x_dtype) * size_t(num_nodes * heads * channels)));
+    TFG_DEBUG(debug_extent(fn, "out", out, sizeof(float) * size_t(num_nodes * heads * channels)));
+    TFG_DEBUG(debug_extent(fn, "alpha", alpha, sizeof(float) * size_t(num_edges * heads)));
     void *scratch = nullptr;
     size_t scratch_bytes = 0;
     cudaError_t err = tfg::noalloc_softmax_scratch(&scratch, &scratch_bytes);
@@ -585,6 +772,9 @@ int tfg_segment_pool_meanmax(const void *x, int x_dtype, const int64_t *batch,
     TFG_NEED(batch, num_nodes > 0, fn, "batch");
     TFG_NEED(out, num_graphs > 0, fn, "out");
     TFG_NEED(status, true, fn, "status");
+    TFG_DEBUG(debug_extent(fn, "x", x, elem_bytes(x_dtype) * size_t(num_nodes * num_features)));
+    TFG_DEBUG(debug_extent(fn, "batch", batch, sizeof(int64_t) * size_t(num_nodes)));
+    TFG_DEBUG(debug_extent(fn, "out", out, sizeof(float) * 2 * size_t(num_graphs * num_features)));
     return cuda_result(tfg::launch_segment_pool(x, x_dtype, batch, num_nodes, num_graphs,
                                                 num_features, 3 /* mean | max */, out, status,
                                                 reinterpret_cast<cudaStream_t>(stream)),
@@ -621,6 +811,13 @@ int tfg_batch_graphs(int64_t num_graphs, const int64_t *node_counts, const int64
     if (workspace == nullptr || workspace_bytes < need)
         return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
                     workspace ? workspace_bytes : size_t(0));
+    TFG_DEBUG(debug_extent(fn, "node_counts", node_counts, sizeof(int64_t) * size_t(num_graphs)));
+    TFG_DEBUG(debug_extent(fn, "edge_counts", edge_counts, sizeof(int64_t) * size_t(num_graphs)));
+    TFG_DEBUG(debug_extent(fn, "edge_index", edge_index, sizeof(int64_t) * 2 * size_t(total_edges)));
+    TFG_DEBUG(debug_extent(fn, "out_edge_index", out_edge_index,
+                           sizeof(int64_t) * 2 * size_t(total_edges)));
+    TFG_DEBUG(debug_extent(fn, "batch", batch, sizeof(int64_t) * size_t(total_nodes)));
+    TFG_DEBUG(debug_extent(fn, "node_offsets", node_offsets, sizeof(int64_t) * size_t(num_graphs + 1)));
     return cuda_result(tfg::launch_batch_graphs(num_graphs, node_counts, edge_counts, edge_index,
                                                 total_edges, total_nodes, out_edge_index, batch,
                                                 node_offsets, workspace, status,
@@ -645,6 +842,9 @@ int tfg_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n
     TFG_NEED(batch, num_nodes > 0, fn, "batch");
     TFG_NEED(out, num_graphs > 0, fn, "out");
     TFG_NEED(status, true, fn, "status");
+    TFG_DEBUG(debug_extent(fn, "x", x, elem_bytes(x_dtype) * size_t(num_nodes * num_features)));
+    TFG_DEBUG(debug_extent(fn, "batch", batch, sizeof(int64_t) * size_t(num_nodes)));
+    TFG_DEBUG(debug_extent(fn, "out", out, sizeof(float) * size_t(num_graphs * num_features)));
     return cuda_result(tfg::launch_segment_pool(x, x_dtype, batch, num_nodes, num_graphs,
                                                 num_features, reduce, out, status,
                                                 reinterpret_cast<cudaStream_t>(stream)),
@@ -663,6 +863,9 @@ int tfg_gather_xor(const int32_t *col, int64_t num_edges, const void *x, int64_t
     TFG_NEED(out, true, fn, "out");
     if (reinterpret_cast<uintptr_t>(x) % 16 != 0)
         return fail(TFG_ERR_INVALID_ARG, "%s: x must be 16-byte aligned", fn);
+    TFG_DEBUG(debug_csr(fn, "col", nullptr, col, nullptr, num_nodes, num_edges, nullptr, stream));
+    TFG_DEBUG(debug_extent(fn, "x", num_edges > 0 ? x : nullptr, size_t(num_nodes) * size_t(row_bytes)));
+    TFG_DEBUG(debug_extent(fn, "out", out, size_t(row_bytes)));
     return cuda_result(tfg::launch_gather_xor(col, num_edges, x, row_bytes, out,
                                               reinterpret_cast<cudaStream_t>(stream)),
                        fn);

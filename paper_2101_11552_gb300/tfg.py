@@ -48,55 +48,70 @@ def lib() -> ctypes.CDLL:
     global _lib
     with _lock:
         if _lib is None:
-            if not os.path.exists(LIB_PATH):
-                raise RuntimeError(
-                    f"{LIB_PATH} is missing: build it first (python -m paper_2101_11552_gb300.build "
-                    "or __graft_entry__.build()); there is no CPU fallback")
-            L = ctypes.CDLL(LIB_PATH)
-            P, I64, I, F, SZ = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float,
-                                ctypes.c_size_t)
-            sigs = {
-                "tfg_version": [],
-                "tfg_build_csr_workspace_size": [I64, I64, ctypes.POINTER(SZ)],
-                "tfg_build_csr": [P, I64, I64, P, P, P, P, P, SZ, P, P],
-                "tfg_build_csr_by_source": [P, I64, I64, P, P, P, P, P, SZ, P, P],
-                "tfg_aggregate_backward_workspace_size": [I, I64, ctypes.POINTER(SZ)],
-                "tfg_aggregate_backward": [I, P, P, P, P, P, P, I64, I64, I64, P, P, SZ, P],
-                "tfg_gcn_aggregate_backward": [P, P, P, P, I64, I64, I, F, P, P],
-                "tfg_aggregate_max_argmax": [P, P, P, P, P, I, I64, I64, P, P, P],
-                "tfg_aggregate_max_backward": [P, P, P, P, P, P, I64, I64, P, P],
-                "tfg_gcn_norm": [P, P, P, P, I64, I64, I, F, P, P, P],
-                "tfg_aggregate_sum": [P, P, P, P, I, I64, I64, P, P],
-                "tfg_aggregate_mean": [P, P, P, P, I, I64, I64, P, P],
-                "tfg_aggregate_max": [P, P, P, P, I, I64, I64, P, P],
-                "tfg_gcn_aggregate_sum": [P, P, P, P, P, I, I64, I64, I, F, P, P],
-                "tfg_propagate_workspace_size": [I64, I64, I64, ctypes.POINTER(SZ)],
-                "tfg_appnp_propagate": [P, P, P, P, P, I, I64, I64, I64, F, I, F, P, P, SZ, P],
-                "tfg_sgc_propagate": [P, P, P, P, P, I, I64, I64, I64, I, F, P, P, SZ, P],
-                "tfg_edge_softmax_workspace_size": [I64, I, ctypes.POINTER(SZ)],
-                "tfg_edge_softmax_aggregate": [P, P, P, I, I64, I64, I, I, P, P, F, P, P, P, SZ, P],
-                "tfg_dot_edge_softmax_aggregate": [P, P, P, P, P, I, I64, I64, I, I, F, P, P, P],
-                "tfg_edge_softmax_aggregate_noalloc": [P, P, P, I, I64, I64, I, I, P, P, F, P, P, P],
-                "tfg_segment_pool": [P, I, P, I64, I64, I64, I, P, P, P],
-                "tfg_segment_pool_meanmax": [P, I, P, I64, I64, I64, P, P, P],
-                "tfg_batch_graphs_workspace_size": [I64, ctypes.POINTER(SZ)],
-                "tfg_batch_graphs": [I64, P, P, P, I64, I64, P, P, P, P, SZ, P, P],
-                "tfg_gather_xor": [P, I64, P, I64, I64, P, P],
-                "tfg_edge_softmax_backward_workspace_size": [I64, I, I, ctypes.POINTER(SZ)],
-                "tfg_edge_softmax_aggregate_backward": [P, P, P, P, P, I, I64, I64, I, I, P, P, F,
-                                                        P, P, P, P, P, P, SZ, P],
-                "tfg_dot_edge_softmax_backward_workspace_size": [I64, I, I, ctypes.POINTER(SZ)],
-                "tfg_dot_edge_softmax_aggregate_backward": [P, P, P, P, P, P, P, I, I64, I64, I, I,
-                                                            F, P, P, P, P, P, P, SZ, P],
-            }
-            for name, args in sigs.items():
-                fn = getattr(L, name)
-                fn.argtypes = args
-                fn.restype = ctypes.c_int
-            L.tfg_last_error.argtypes = []
-            L.tfg_last_error.restype = ctypes.c_char_p
-            _lib = L
+            _lib = _load(LIB_PATH)
         return _lib
+
+
+def use_library(path: str) -> ctypes.CDLL:
+    """Switch every call of this module to another build of the library (for
+    example the bounds-checked debug build, ``build.build_library(defines=
+    ("TFG_CHECK_BOUNDS=1",), lib_path=...)``); returns the loaded library."""
+    global _lib
+    with _lock:
+        _lib = _load(path)
+        return _lib
+
+
+def _load(path: str) -> ctypes.CDLL:
+    if not os.path.exists(path):
+        raise RuntimeError(
+            f"{path} is missing: build it first (python -m paper_2101_11552_gb300.build "
+            "or __graft_entry__.build()); there is no CPU fallback")
+    L = ctypes.CDLL(path)
+    P, I64, I, F, SZ = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float,
+                        ctypes.c_size_t)
+    sigs = {
+        "tfg_version": [],
+        "tfg_check_bounds_enabled": [],
+        "tfg_build_csr_workspace_size": [I64, I64, ctypes.POINTER(SZ)],
+        "tfg_build_csr": [P, I64, I64, P, P, P, P, P, SZ, P, P],
+        "tfg_build_csr_by_source": [P, I64, I64, P, P, P, P, P, SZ, P, P],
+        "tfg_aggregate_backward_workspace_size": [I, I64, ctypes.POINTER(SZ)],
+        "tfg_aggregate_backward": [I, P, P, P, P, P, P, I64, I64, I64, P, P, SZ, P],
+        "tfg_gcn_aggregate_backward": [P, P, P, P, I64, I64, I, F, P, P],
+        "tfg_aggregate_max_argmax": [P, P, P, P, P, I, I64, I64, P, P, P],
+        "tfg_aggregate_max_backward": [P, P, P, P, P, P, I64, I64, P, P],
+        "tfg_gcn_norm": [P, P, P, P, I64, I64, I, F, P, P, P],
+        "tfg_aggregate_sum": [P, P, P, P, I, I64, I64, P, P],
+        "tfg_aggregate_mean": [P, P, P, P, I, I64, I64, P, P],
+        "tfg_aggregate_max": [P, P, P, P, I, I64, I64, P, P],
+        "tfg_gcn_aggregate_sum": [P, P, P, P, P, I, I64, I64, I, F, P, P],
+        "tfg_propagate_workspace_size": [I64, I64, I64, ctypes.POINTER(SZ)],
+        "tfg_appnp_propagate": [P, P, P, P, P, I, I64, I64, I64, F, I, F, P, P, SZ, P],
+        "tfg_sgc_propagate": [P, P, P, P, P, I, I64, I64, I64, I, F, P, P, SZ, P],
+        "tfg_edge_softmax_workspace_size": [I64, I, ctypes.POINTER(SZ)],
+        "tfg_edge_softmax_aggregate": [P, P, P, I, I64, I64, I, I, P, P, F, P, P, P, SZ, P],
+        "tfg_dot_edge_softmax_aggregate": [P, P, P, P, P, I, I64, I64, I, I, F, P, P, P],
+        "tfg_edge_softmax_aggregate_noalloc": [P, P, P, I, I64, I64, I, I, P, P, F, P, P, P],
+        "tfg_segment_pool": [P, I, P, I64, I64, I64, I, P, P, P],
+        "tfg_segment_pool_meanmax": [P, I, P, I64, I64, I64, P, P, P],
+        "tfg_batch_graphs_workspace_size": [I64, ctypes.POINTER(SZ)],
+        "tfg_batch_graphs": [I64, P, P, P, I64, I64, P, P, P, P, SZ, P, P],
+        "tfg_gather_xor": [P, I64, P, I64, I64, P, P],
+        "tfg_edge_softmax_backward_workspace_size": [I64, I, I, ctypes.POINTER(SZ)],
+        "tfg_edge_softmax_aggregate_backward": [P, P, P, P, P, I, I64, I64, I, I, P, P, F,
+                                                P, P, P, P, P, P, SZ, P],
+        "tfg_dot_edge_softmax_backward_workspace_size": [I64, I, I, ctypes.POINTER(SZ)],
+        "tfg_dot_edge_softmax_aggregate_backward": [P, P, P, P, P, P, P, I, I64, I64, I, I,
+                                                    F, P, P, P, P, P, P, SZ, P],
+    }
+    for name, args in sigs.items():
+        fn = getattr(L, name)
+        fn.argtypes = args
+        fn.restype = ctypes.c_int
+    L.tfg_last_error.argtypes = []
+    L.tfg_last_error.restype = ctypes.c_char_p
+    return L
 
 
 def tfg_version() -> int:
