@@ -6,6 +6,15 @@
 
 #include "common.cuh"
 
+// Helpers of the bounds-checked debug build (check_bounds.cu).
+namespace tfg {
+bool allocation_range(const void *p, uintptr_t *base, size_t *size);
+cudaError_t csr_ends(const int32_t *rowptr, int64_t n, int32_t *first, int32_t *last,
+                     cudaStream_t s);
+cudaError_t validate_csr(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
+                         int64_t n, int64_t e, int *flags, cudaStream_t s);
+}  // namespace tfg
+
 namespace {
 
 thread_local char g_err[512];

@@ -272,12 +272,6 @@ cudaError_t launch_dot_softmax_backward(const int32_t *rowptr, const int32_t *co
                                         int64_t n, int64_t e, int heads, int channels, float scale,
                                         const float *out, const float *grad_out, float *grad_q,
                                         float *grad_k, float *grad_v, void *ws, cudaStream_t s);
-// Bounds-checked debug build (check_bounds.cu)
-bool allocation_range(const void *p, uintptr_t *base, size_t *size);
-cudaError_t csr_ends(const int32_t *rowptr, int64_t n, int32_t *first, int32_t *last,
-                     cudaStream_t s);
-cudaError_t validate_csr(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
-                         int64_t n, int64_t e, int *flags, cudaStream_t s);
 cudaError_t launch_gather_xor(const int32_t *col, int64_t e, const void *x, int64_t row_bytes,
                               uint32_t *out, cudaStream_t s);
 cudaError_t launch_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n,
