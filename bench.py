@@ -331,12 +331,13 @@ def cold_l2_ms(fns: dict, stream, reps: int = 5) -> dict:
     return out
 
 
-def small_configs(L, stream, hbm_peak):
-    """The four smaller workloads, each call timed hot (mean of repeated calls,
-    inputs left in L2 by the previous call) and cold (after an L2 flush):
-    edge-features/s, algorithmic GB/s and its fraction of the measured HBM
-    peak (hot).  The 2,708-node and 19,717-node graphs fit in L2 and are
-    launch- or latency-bound; they are reported, not roofline targets."""
+def small_configs(L, stream, hbm_peak, only=None):
+    """The four smaller workloads (`only`: one of "c1".."c4", else all), each
+    call timed hot (mean of repeated calls, inputs left in L2 by the previous
+    call) and cold (after an L2 flush): edge-features/s, algorithmic GB/s and
+    its fraction of the measured HBM peak (hot).  The 2,708-node and
+    19,717-node graphs fit in L2 and are launch- or latency-bound; they are
+    reported, not roofline targets."""
     import torch
     from paper_2101_11552_gb300 import graphgen as gg
     from paper_2101_11552_gb300 import tfg
@@ -362,73 +363,77 @@ def small_configs(L, stream, hbm_peak):
         return csr
 
     out = {}
-    # GCN propagation on the 2,708-node graph (explicit self-loops), fp32 F = 64
-    wl = gg.make_er_2708()
-    n, e, f = wl.num_nodes, wl.num_edges, wl.num_features
-    csr = csr_of(wl)
-    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
-    x = torch.from_numpy(wl.x).to(dev)
-    y = torch.empty(n, f, dtype=torch.float32, device=dev)
-    out["er_2708_gcn"] = {"workload": "G(2708, 5278) + self-loops, F = 64 fp32, GCN sum",
-                          "nodes": n, "edges": e, "calls": {"gcn_aggregate": measure(
-        lambda: check(L.tfg_gcn_aggregate_sum(P(csr.rowptr), P(csr.col), P(dinv), None, P(x),
-                                              tfg.TFG_F32, n, f, 0, 1.0, P(y), sp)),
-        e * f, 4 * e + 4 * (n + 1) + 4 * n + 8 * n * f, 200)}}
-    # unweighted sum / mean / max on the 19,717-node power-law graph, fp32 F = 256
-    wl = gg.make_ba_19717()
-    n, e, f = wl.num_nodes, wl.num_edges, wl.num_features
-    csr = csr_of(wl)
-    x = torch.from_numpy(wl.x).to(dev)
-    y = torch.empty(n, f, dtype=torch.float32, device=dev)
-    calls = {}
-    for red, fn in (("sum", L.tfg_aggregate_sum), ("mean", L.tfg_aggregate_mean),
-                    ("max", L.tfg_aggregate_max)):
-        calls[red] = measure(
-            lambda fn=fn: check(fn(P(csr.rowptr), P(csr.col), None, P(x), tfg.TFG_F32, n, f,
-                                   P(y), sp)),
-            e * f, 4 * e + 4 * (n + 1) + 8 * n * f, 100)
-    out["ba_19717_sum_mean_max"] = {"workload": "BA(19717, m=2) + self-loops, F = 256 fp32",
-                                    "nodes": n, "edges": e, "calls": calls}
-    # GAT edge softmax on the 169,343-node oriented power-law graph, fp32 8 x 16
-    wl = gg.make_gat_169343()
-    n, e, f, heads, ch = wl.num_nodes, wl.num_edges, wl.num_features, wl.heads, wl.channels
-    csr = csr_of(wl)
-    x = torch.from_numpy(wl.x).to(dev)
-    y = torch.empty(n, f, dtype=torch.float32, device=dev)
-    a_s, a_d = torch.from_numpy(wl.a_src).to(dev), torch.from_numpy(wl.a_dst).to(dev)
-    ws = torch.empty(tfg.tfg_edge_softmax_workspace_size(n, heads), dtype=torch.uint8, device=dev)
-    out["gat_169343_edge_softmax"] = {
-        "workload": "BA(169343, m=7) subsampled to 1,166,243 edges, oriented; F = 8 x 16 fp32",
-        "nodes": n, "edges": e, "calls": {"edge_softmax": measure(
-            lambda: check(L.tfg_edge_softmax_aggregate(P(csr.rowptr), P(csr.col), P(x), tfg.TFG_F32,
-                                                       n, e, heads, ch, P(a_s), P(a_d), 0.2, P(y),
-                                                       None, P(ws), ws.numel(), sp)),
-            e * f, 4 * e + 4 * (n + 1) + 8 * n * f + 16 * n * heads, 50)}}
-    # 1,024 batched molecule-sized graphs: GCN, then sum / mean / max pooling
-    wl = gg.make_molecules_1024()
-    n, e, f, g = wl.num_nodes, wl.num_edges, wl.num_features, wl.num_graphs
-    csr = csr_of(wl)
-    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
-    x = torch.from_numpy(wl.x).to(dev)
-    hh = torch.empty(n, f, dtype=torch.float32, device=dev)
-    batch = torch.from_numpy(wl.batch).to(dev)
-    pooled = torch.empty(g, f, dtype=torch.float32, device=dev)
-    st = torch.zeros(1, dtype=torch.int32, device=dev)
-    calls = {"gcn_aggregate": measure(
-        lambda: check(L.tfg_gcn_aggregate_sum(P(csr.rowptr), P(csr.col), P(dinv), None, P(x),
-                                              tfg.TFG_F32, n, f, 0, 1.0, P(hh), sp)),
-        e * f, 4 * e + 4 * (n + 1) + 4 * n + 8 * n * f, 100)}
-    for red in ("sum", "mean", "max"):
-        calls[f"pool_{red}"] = measure(
-            lambda red=red: check(L.tfg_segment_pool(P(hh), tfg.TFG_F32, P(batch), n, g, f,
-                                                     tfg.REDUCERS[red], P(pooled), P(st), sp)),
-            n * f, 4 * n * f + 8 * n + 4 * g * f, 100)
-    torch.cuda.synchronize()
-    if int(st.item()) != 0:
-        raise RuntimeError("pooling status word set on the molecule batch")
-    out["molecules_1024_gcn_pool"] = {"workload": "1,024 graphs of 20-200 nodes (avg degree 4 + "
-                                      "self-loops), F = 128 fp32", "nodes": n, "edges": e,
-                                      "graphs": g, "calls": calls}
+    if only in (None, "c1"):
+        # GCN propagation on the 2,708-node graph (explicit self-loops), fp32 F = 64
+        wl = gg.make_er_2708()
+        n, e, f = wl.num_nodes, wl.num_edges, wl.num_features
+        csr = csr_of(wl)
+        dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
+        x = torch.from_numpy(wl.x).to(dev)
+        y = torch.empty(n, f, dtype=torch.float32, device=dev)
+        out["er_2708_gcn"] = {"workload": "G(2708, 5278) + self-loops, F = 64 fp32, GCN sum",
+                              "nodes": n, "edges": e, "calls": {"gcn_aggregate": measure(
+            lambda: check(L.tfg_gcn_aggregate_sum(P(csr.rowptr), P(csr.col), P(dinv), None, P(x),
+                                                  tfg.TFG_F32, n, f, 0, 1.0, P(y), sp)),
+            e * f, 4 * e + 4 * (n + 1) + 4 * n + 8 * n * f, 200)}}
+    if only in (None, "c2"):
+        # unweighted sum / mean / max on the 19,717-node power-law graph, fp32 F = 256
+        wl = gg.make_ba_19717()
+        n, e, f = wl.num_nodes, wl.num_edges, wl.num_features
+        csr = csr_of(wl)
+        x = torch.from_numpy(wl.x).to(dev)
+        y = torch.empty(n, f, dtype=torch.float32, device=dev)
+        calls = {}
+        for red, fn in (("sum", L.tfg_aggregate_sum), ("mean", L.tfg_aggregate_mean),
+                        ("max", L.tfg_aggregate_max)):
+            calls[red] = measure(
+                lambda fn=fn: check(fn(P(csr.rowptr), P(csr.col), None, P(x), tfg.TFG_F32, n, f,
+                                       P(y), sp)),
+                e * f, 4 * e + 4 * (n + 1) + 8 * n * f, 100)
+        out["ba_19717_sum_mean_max"] = {"workload": "BA(19717, m=2) + self-loops, F = 256 fp32",
+                                        "nodes": n, "edges": e, "calls": calls}
+    if only in (None, "c3"):
+        # GAT edge softmax on the 169,343-node oriented power-law graph, fp32 8 x 16
+        wl = gg.make_gat_169343()
+        n, e, f, heads, ch = wl.num_nodes, wl.num_edges, wl.num_features, wl.heads, wl.channels
+        csr = csr_of(wl)
+        x = torch.from_numpy(wl.x).to(dev)
+        y = torch.empty(n, f, dtype=torch.float32, device=dev)
+        a_s, a_d = torch.from_numpy(wl.a_src).to(dev), torch.from_numpy(wl.a_dst).to(dev)
+        ws = torch.empty(tfg.tfg_edge_softmax_workspace_size(n, heads), dtype=torch.uint8, device=dev)
+        out["gat_169343_edge_softmax"] = {
+            "workload": "BA(169343, m=7) subsampled to 1,166,243 edges, oriented; F = 8 x 16 fp32",
+            "nodes": n, "edges": e, "calls": {"edge_softmax": measure(
+                lambda: check(L.tfg_edge_softmax_aggregate(P(csr.rowptr), P(csr.col), P(x), tfg.TFG_F32,
+                                                           n, e, heads, ch, P(a_s), P(a_d), 0.2, P(y),
+                                                           None, P(ws), ws.numel(), sp)),
+                e * f, 4 * e + 4 * (n + 1) + 8 * n * f + 16 * n * heads, 50)}}
+    if only in (None, "c4"):
+        # 1,024 batched molecule-sized graphs: GCN, then sum / mean / max pooling
+        wl = gg.make_molecules_1024()
+        n, e, f, g = wl.num_nodes, wl.num_edges, wl.num_features, wl.num_graphs
+        csr = csr_of(wl)
+        dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, 0, 1.0, want_w_csr=False)
+        x = torch.from_numpy(wl.x).to(dev)
+        hh = torch.empty(n, f, dtype=torch.float32, device=dev)
+        batch = torch.from_numpy(wl.batch).to(dev)
+        pooled = torch.empty(g, f, dtype=torch.float32, device=dev)
+        st = torch.zeros(1, dtype=torch.int32, device=dev)
+        calls = {"gcn_aggregate": measure(
+            lambda: check(L.tfg_gcn_aggregate_sum(P(csr.rowptr), P(csr.col), P(dinv), None, P(x),
+                                                  tfg.TFG_F32, n, f, 0, 1.0, P(hh), sp)),
+            e * f, 4 * e + 4 * (n + 1) + 4 * n + 8 * n * f, 100)}
+        for red in ("sum", "mean", "max"):
+            calls[f"pool_{red}"] = measure(
+                lambda red=red: check(L.tfg_segment_pool(P(hh), tfg.TFG_F32, P(batch), n, g, f,
+                                                         tfg.REDUCERS[red], P(pooled), P(st), sp)),
+                n * f, 4 * n * f + 8 * n + 4 * g * f, 100)
+        torch.cuda.synchronize()
+        if int(st.item()) != 0:
+            raise RuntimeError("pooling status word set on the molecule batch")
+        out["molecules_1024_gcn_pool"] = {"workload": "1,024 graphs of 20-200 nodes (avg degree 4 + "
+                                          "self-loops), F = 128 fp32", "nodes": n, "edges": e,
+                                          "graphs": g, "calls": calls}
     return out
 
 
@@ -751,6 +756,10 @@ def parse():
                     help="skip the four smaller workloads")
     ap.add_argument("--configs-only", action="store_true",
                     help="measure only the four smaller workloads")
+    ap.add_argument("--config", choices=["c1", "c2", "c3", "c4", "c5"], default=None,
+                    help="one workload: c1 GCN on 2,708 nodes, c2 sum/mean/max on BA 19,717, "
+                         "c3 edge softmax on 169,343 nodes, c4 batched GCN + pooling, c5 the "
+                         "benchmark step on the 114.6M-edge graph (the default run)")
     ap.add_argument("--pairs", type=int, default=57_300_000, help=argparse.SUPPRESS)
     return ap.parse_args()
 
@@ -805,10 +814,12 @@ def main():
     tfg_build.build_library()
     L = tfg.lib()
 
-    if args.configs_only:   # the four smaller workloads alone (profiling their kernels)
+    one = args.config if args.config in ("c1", "c2", "c3", "c4") else None
+    if args.configs_only or one:   # the smaller workloads alone (profiling their kernels)
         peaks = os.path.join(ROOT, "MEASURED_PEAKS.json")
         hbm = float(json.load(open(peaks)).get("hbm_gbs", 6800.0)) if os.path.exists(peaks) else 6800.0
-        print(json.dumps({"configs": small_configs(L, torch.cuda.current_stream(), hbm)}), flush=True)
+        print(json.dumps({"configs": small_configs(L, torch.cuda.current_stream(), hbm, one)}),
+              flush=True)
         return
 
     wl = gg.make_dcsbm_232965(num_pairs=args.pairs)

@@ -6,6 +6,30 @@
 
 #include "common.cuh"
 
+// NVTX ranges (header-only NVTX 3; no-ops unless a profiler is attached):
+// every entry point opens a range named after itself around its host work
+// and launches, so ncu / nsys timelines show which call enqueued which
+// kernels.  TFG_NVTX=0 compiles them out.
+#ifndef TFG_NVTX
+#define TFG_NVTX 1
+#endif
+#if TFG_NVTX
+#include <nvtx3/nvToolsExt.h>
+namespace {
+struct NvtxRange {
+    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange &) = delete;
+    NvtxRange &operator=(const NvtxRange &) = delete;
+};
+}  // namespace
+#define TFG_RANGE(name) NvtxRange tfg_nvtx_range_(name)
+#else
+#define TFG_RANGE(name) \
+    do {                \
+    } while (0)
+#endif
+
 // Helpers of the bounds-checked debug build (check_bounds.cu).
 namespace tfg {
 bool allocation_range(const void *p, uintptr_t *base, size_t *size);
@@ -152,6 +176,7 @@ size_t elem_bytes(int dtype) { return dtype == TFG_BF16 ? 2 : 4; }
 int aggregate_common(const char *fn, int mode, const int32_t *rowptr, const int32_t *col,
                      const float *w, const float *dinv, const void *x, int dtype, int64_t n,
                      int64_t f, int add_self, float fill, float *out, tfg_stream_t stream) {
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, n, 0));
     TFG_TRY(check_features(fn, n, f));
     TFG_TRY(check_dtype(fn, dtype));
@@ -180,6 +205,7 @@ int propagate_common(const char *fn, const int32_t *rowptr, const int32_t *col, 
                      const float *w, const void *x0, int dtype, int64_t n, int64_t f, int64_t hops,
                      float alpha, int add_self, float fill, float *out, void *ws, size_t ws_bytes,
                      tfg_stream_t stream) {
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, n, 0));
     TFG_TRY(check_features(fn, n, f));
     TFG_TRY(check_dtype(fn, dtype));
@@ -250,6 +276,7 @@ const char *tfg_last_error(void) { return g_err; }
 
 int tfg_build_csr_workspace_size(int64_t num_nodes, int64_t num_edges, size_t *bytes) {
     const char *fn = "tfg_build_csr_workspace_size";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     TFG_NEED(bytes, true, fn, "bytes");
     *bytes = tfg::csr_workspace_bytes(num_nodes, num_edges);
@@ -261,6 +288,7 @@ int build_csr_common(const char *fn, bool by_source, const int64_t *edge_index, 
                      int64_t num_nodes, int32_t *rowptr, int32_t *col, int32_t *perm,
                      int32_t *in_degree, void *workspace, size_t workspace_bytes, int32_t *status,
                      tfg_stream_t stream) {
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     TFG_NEED(edge_index, num_edges > 0, fn, "edge_index");
     TFG_NEED(rowptr, true, fn, "rowptr");
@@ -311,6 +339,7 @@ int tfg_gcn_norm(const int32_t *rowptr, const int32_t *col, const int32_t *perm,
                  int add_self_loops, float self_loop_fill, float *dinv, float *w_csr,
                  tfg_stream_t stream) {
     const char *fn = "tfg_gcn_norm";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     TFG_NEED(rowptr, true, fn, "rowptr");
     TFG_NEED(dinv, num_nodes > 0, fn, "dinv");
@@ -358,6 +387,7 @@ int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float
 
 int tfg_aggregate_backward_workspace_size(int reduce, int64_t num_edges, size_t *bytes) {
     const char *fn = "tfg_aggregate_backward_workspace_size";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, 1, num_edges));
     if (reduce != TFG_SUM && reduce != TFG_MEAN)
         return fail(TFG_ERR_INVALID_ARG, "%s: reduce must be TFG_SUM or TFG_MEAN", fn);
@@ -372,6 +402,7 @@ int tfg_aggregate_backward(int reduce, const int32_t *rowptr_src, const int32_t 
                            int64_t num_edges, int64_t num_features, float *grad_x,
                            void *workspace, size_t workspace_bytes, tfg_stream_t stream) {
     const char *fn = "tfg_aggregate_backward";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     TFG_TRY(check_features(fn, num_nodes, num_features));
     if (reduce != TFG_SUM && reduce != TFG_MEAN)
@@ -417,6 +448,7 @@ int tfg_aggregate_max_argmax(const int32_t *rowptr, const int32_t *col, const in
                              int64_t num_features, float *out, int32_t *argmax,
                              tfg_stream_t stream) {
     const char *fn = "tfg_aggregate_max_argmax";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, 0));
     TFG_TRY(check_features(fn, num_nodes, num_features));
     TFG_TRY(check_dtype(fn, x_dtype));
@@ -447,6 +479,7 @@ int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src
                                int64_t num_nodes, int64_t num_features, float *grad_x,
                                tfg_stream_t stream) {
     const char *fn = "tfg_aggregate_max_backward";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, 0));
     TFG_TRY(check_features(fn, num_nodes, num_features));
     TFG_NEED(rowptr_src, true, fn, "rowptr_src");
@@ -474,6 +507,7 @@ int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src
 int tfg_propagate_workspace_size(int64_t num_nodes, int64_t num_features, int64_t num_hops,
                                  size_t *bytes) {
     const char *fn = "tfg_propagate_workspace_size";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, 0));
     TFG_TRY(check_features(fn, num_nodes, num_features));
     if (num_hops < 0 || num_hops > kMaxHops)
@@ -505,6 +539,7 @@ int tfg_sgc_propagate(const int32_t *rowptr, const int32_t *col, const float *di
 
 int tfg_edge_softmax_workspace_size(int64_t num_nodes, int heads, size_t *bytes) {
     const char *fn = "tfg_edge_softmax_workspace_size";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, 0));
     if (heads < 1) return fail(TFG_ERR_INVALID_ARG, "%s: heads must be >= 1", fn);
     TFG_NEED(bytes, true, fn, "bytes");
@@ -519,6 +554,7 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
                                float *out, float *alpha, void *workspace,
                                size_t workspace_bytes, tfg_stream_t stream) {
     const char *fn = "tfg_edge_softmax_aggregate";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     if (heads < 1 || channels < 1)
         return fail(TFG_ERR_INVALID_ARG, "%s: heads and channels must be >= 1", fn);
@@ -551,6 +587,7 @@ int tfg_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, const 
 int tfg_edge_softmax_backward_workspace_size(int64_t num_nodes, int heads, int channels,
                                              size_t *bytes) {
     const char *fn = "tfg_edge_softmax_backward_workspace_size";
+    TFG_RANGE(fn);
     TFG_NEED(bytes, true, fn, "bytes");
     TFG_TRY(check_counts(fn, num_nodes, 0));
     if (!tfg::attention_backward_layout_ok(heads, channels))
@@ -571,6 +608,7 @@ int tfg_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t *co
                                         float *grad_a_dst, void *workspace,
                                         size_t workspace_bytes, tfg_stream_t stream) {
     const char *fn = "tfg_edge_softmax_aggregate_backward";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     if (!tfg::attention_backward_layout_ok(heads, channels))
         return fail(TFG_ERR_INVALID_ARG,
@@ -617,6 +655,7 @@ int tfg_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t *co
 int tfg_dot_edge_softmax_backward_workspace_size(int64_t num_nodes, int heads, int channels,
                                                  size_t *bytes) {
     const char *fn = "tfg_dot_edge_softmax_backward_workspace_size";
+    TFG_RANGE(fn);
     TFG_NEED(bytes, true, fn, "bytes");
     TFG_TRY(check_counts(fn, num_nodes, 0));
     if (!tfg::attention_backward_layout_ok(heads, channels))
@@ -637,6 +676,7 @@ int tfg_dot_edge_softmax_aggregate_backward(const int32_t *rowptr, const int32_t
                                             void *workspace, size_t workspace_bytes,
                                             tfg_stream_t stream) {
     const char *fn = "tfg_dot_edge_softmax_aggregate_backward";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     if (!tfg::attention_backward_layout_ok(heads, channels))
         return fail(TFG_ERR_INVALID_ARG,
@@ -691,6 +731,7 @@ int tfg_dot_edge_softmax_aggregate(const int32_t *rowptr, const int32_t *col, co
                                    int64_t num_edges, int heads, int channels, float scale,
                                    float *out, float *alpha, tfg_stream_t stream) {
     const char *fn = "tfg_dot_edge_softmax_aggregate";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     if (heads < 1 || channels < 1)
         return fail(TFG_ERR_INVALID_ARG, "%s: heads and channels must be >= 1", fn);
@@ -731,6 +772,7 @@ int tfg_edge_softmax_aggregate_noalloc(const int32_t *rowptr, const int32_t *col
                                        const float *a_dst, float negative_slope, float *out,
                                        float *alpha, tfg_stream_t stream) {
     const char *fn = "tfg_edge_softmax_aggregate_noalloc";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     if (heads < 1 || channels < 1)
         return fail(TFG_ERR_INVALID_ARG, "%s: heads and channels must be >= 1", fn);
@@ -770,6 +812,7 @@ int tfg_segment_pool_meanmax(const void *x, int x_dtype, const int64_t *batch,
                              int64_t num_nodes, int64_t num_graphs, int64_t num_features,
                              float *out, int32_t *status, tfg_stream_t stream) {
     const char *fn = "tfg_segment_pool_meanmax";
+    TFG_RANGE(fn);
     if (num_nodes < 0 || num_graphs < 0)
         return fail(TFG_ERR_INVALID_ARG, "%s: negative size", fn);
     if (num_graphs >= kIndexLimit) return fail(TFG_ERR_TOO_LARGE, "%s: too many graphs", fn);
@@ -792,6 +835,7 @@ int tfg_segment_pool_meanmax(const void *x, int x_dtype, const int64_t *batch,
 
 int tfg_batch_graphs_workspace_size(int64_t num_graphs, size_t *bytes) {
     const char *fn = "tfg_batch_graphs_workspace_size";
+    TFG_RANGE(fn);
     if (num_graphs < 0) return fail(TFG_ERR_INVALID_ARG, "%s: negative size", fn);
     TFG_NEED(bytes, true, fn, "bytes");
     *bytes = tfg::batch_graphs_workspace_bytes(num_graphs);
@@ -804,6 +848,7 @@ int tfg_batch_graphs(int64_t num_graphs, const int64_t *node_counts, const int64
                      void *workspace, size_t workspace_bytes, int32_t *status,
                      tfg_stream_t stream) {
     const char *fn = "tfg_batch_graphs";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, total_nodes, total_edges));
     if (num_graphs < 0) return fail(TFG_ERR_INVALID_ARG, "%s: negative graph count", fn);
     if (num_graphs >= kIndexLimit) return fail(TFG_ERR_TOO_LARGE, "%s: too many graphs", fn);
@@ -838,6 +883,7 @@ int tfg_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n
                      int64_t num_graphs, int64_t num_features, int reduce, float *out,
                      int32_t *status, tfg_stream_t stream) {
     const char *fn = "tfg_segment_pool";
+    TFG_RANGE(fn);
     if (num_nodes < 0 || num_graphs < 0)
         return fail(TFG_ERR_INVALID_ARG, "%s: negative size", fn);
     if (num_graphs >= kIndexLimit) return fail(TFG_ERR_TOO_LARGE, "%s: too many graphs", fn);
@@ -863,6 +909,7 @@ int tfg_segment_pool(const void *x, int x_dtype, const int64_t *batch, int64_t n
 int tfg_gather_xor(const int32_t *col, int64_t num_edges, const void *x, int64_t num_nodes,
                    int64_t row_bytes, uint32_t *out, tfg_stream_t stream) {
     const char *fn = "tfg_gather_xor";
+    TFG_RANGE(fn);
     TFG_TRY(check_counts(fn, num_nodes, num_edges));
     if (row_bytes < 16 || row_bytes > 512 || (row_bytes & (row_bytes - 1)) != 0)
         return fail(TFG_ERR_INVALID_ARG, "%s: row_bytes must be a power of two in [16, 512] (%lld)",
