@@ -140,3 +140,28 @@ def test_feature_buffer_smaller_than_num_nodes_rows_is_refused(checked):
     finally:
         tfg.use_library(build.LIB_PATH)
     assert rc == tfg.TFG_ERR_INDEX_RANGE and "x must hold" in msg, (rc, msg)
+
+
+def test_backward_index_arrays_are_checked(checked):
+    """A bad id in the source-grouped CSR of a backward call, and a perm id
+    outside [0, E), are refused (the padded buffers keep even a launch in
+    bounds)."""
+    path, wl = checked
+    ei = dev(wl.edge_index)
+    csr = tfg.tfg_build_csr(ei, N)
+    src = tfg.tfg_build_csr_by_source(ei, N)
+    g = torch.randn(N, F, device="cuda")
+    dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, N, None, 1, 1.0, want_w_csr=False)
+    colp = torch.zeros(E + 64, dtype=torch.int32, device="cuda")
+    colp[:E] = src.col
+    colp[7] = N + 1                                    # a row the padding of gpad holds
+    gpad = torch.zeros(N + 64, F, device="cuda")
+    gpad[:N] = g
+    bad = src._replace(col=colp[:E])
+    _expect(path, lambda: tfg.tfg_gcn_aggregate_backward(bad, dinv, gpad[:N], 1, 1.0),
+            tfg.TFG_ERR_INDEX_RANGE, ["col", "outside [0, N)"])
+    permp = csr.perm.clone()
+    permp[11] = E + 2       # only ever copied into argmax, never used as an address
+    x = dev(wl.x)
+    _expect(path, lambda: tfg.tfg_aggregate_max_argmax(csr._replace(perm=permp), x),
+            tfg.TFG_ERR_INDEX_RANGE, ["perm id lies outside [0, E)"])
