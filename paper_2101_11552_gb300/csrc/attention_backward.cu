@@ -785,8 +785,17 @@ __global__ void __launch_bounds__(kBwThreads) dot_bwd_sources(DotBwArgs a) {
 //    grad_q[t] = scale * acc / den; stats[t, h] = (m, 1 / den, beta, 0).
 //  * source pass (CSR by source): per row s, alpha of each out-edge from
 //    stats[t]; grad_k[s] = scale * sum dl q[t], grad_v[s] = sum alpha grad_out[t].
-constexpr int kDbUnroll = 4;      // edges in flight per lane, target pass
-constexpr int kDbUnrollSrc = 2;   // edges in flight per lane, source pass
+// Measured on the 114.6M-edge graph (bf16, 8 x 16): 4 / 2 edges in flight
+// (target / source) at 2 CTAs per SM 21.60 ms, 4 / 4 20.95 ms (kept), 2 / 2
+// 23.32 ms, 2 / 1 at 3 CTAs 23.23 ms, 8 / 2 at 1 CTA 35.65 ms.
+#ifndef TFG_DB_UNROLL_TGT
+#define TFG_DB_UNROLL_TGT 4       // edges in flight per lane, target pass
+#endif
+#ifndef TFG_DB_UNROLL_SRC
+#define TFG_DB_UNROLL_SRC 4       // edges in flight per lane, source pass
+#endif
+constexpr int kDbUnroll = TFG_DB_UNROLL_TGT;
+constexpr int kDbUnrollSrc = TFG_DB_UNROLL_SRC;
 #ifndef TFG_DB_BLOCKS
 #define TFG_DB_BLOCKS 3           // resident CTAs per SM of the fast passes, fp32
 #endif
