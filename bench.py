@@ -864,14 +864,15 @@ def main():
     main_io = dict(edge=edge, xb=xb, batch=batch, a_src=a_src, a_dst=a_dst, h=h, att=att,
                    pool_mean=pool_mean, pool_max=pool_max)
 
-    def step(ev=None, io=None):
+    def step(ev=None, io=None, csr_fn=None):
         io = main_io if io is None else io
+        csr_fn = L.tfg_build_csr if csr_fn is None else csr_fn   # tfg_build_csr32: int32 edges
         edge, xb, batch, a_src, a_dst = (io[k] for k in ("edge", "xb", "batch", "a_src", "a_dst"))
         h, att, pool_mean, pool_max = (io[k] for k in ("h", "att", "pool_mean", "pool_max"))
         if ev is not None:
             ev[0].record(stream)
-        check(L.tfg_build_csr(P(edge), e, n, P(rowptr), P(col), P(perm), P(indeg), P(ws_csr),
-                              ws_csr.numel(), st0, sp))
+        check(csr_fn(P(edge), e, n, P(rowptr), P(col), P(perm), P(indeg), P(ws_csr),
+                     ws_csr.numel(), st0, sp))
         if ev is not None:
             ev[1].record(stream)
         check(L.tfg_gcn_norm(P(rowptr), P(col), P(perm), None, n, e, 1, 1.0, P(dinv), None, sp))
@@ -951,33 +952,33 @@ def main():
     host_in = dict(edge=hp_edge, xb=hp_xb, batch=hp_batch, a_src=hp_as, a_dst=hp_ad)
     host_out = dict(h=ho_h, att=ho_att, pool_mean=ho_pm, pool_max=ho_px)
 
-    def load(i):
+    def load(i, hin, ios):
         b = i % 2
         with torch.cuda.stream(s_in):
             if i >= 2:
                 s_in.wait_event(ev_computed[b])      # step i - 2 is done with these inputs
-            for k, t in host_in.items():
-                io_sets[b][k].copy_(t, non_blocking=True)
+            for k, t in hin.items():
+                ios[b][k].copy_(t, non_blocking=True)
             ev_loaded[b].record(s_in)
 
-    def e2e_run(k: int, start_ev=None, stop_ev=None):
+    def e2e_run(k: int, start_ev=None, stop_ev=None, hin=host_in, ios=io_sets, csr_fn=None):
         if start_ev is not None:
             start_ev.record(stream)
             s_in.wait_event(start_ev)
-        load(0)
+        load(0, hin, ios)
         for i in range(k):
             b = i % 2
             if i + 1 < k:
-                load(i + 1)
+                load(i + 1, hin, ios)
             stream.wait_event(ev_loaded[b])
             if i >= 2:
                 stream.wait_event(ev_drained[b])     # results of step i - 2 have left
-            step(io=io_sets[b])
+            step(io=ios[b], csr_fn=csr_fn)
             ev_computed[b].record(stream)
             with torch.cuda.stream(s_out):
                 s_out.wait_event(ev_computed[b])
                 for key, t in host_out.items():
-                    t.copy_(io_sets[b][key], non_blocking=True)
+                    t.copy_(ios[b][key], non_blocking=True)
                 ev_drained[b].record(s_out)
         stream.wait_event(ev_drained[(k - 1) % 2])
         if stop_ev is not None:
@@ -1006,6 +1007,43 @@ def main():
         c1.record(stream)
         torch.cuda.synchronize()
         link[name] = round(hp_edge.numel() * hp_edge.element_size() / (c0.elapsed_time(c1) * 1e-3) / 1e9, 1)
+
+    # The same step and the same pipeline with the edge list held as int32
+    # (tfg_build_csr32): informational, beside the int64 figures above.
+    ios32 = tuple(dict(d, edge=torch.empty(2, e, dtype=torch.int32, device=dev)) for d in io_sets)
+    ios32[0]["edge"].copy_(edge.to(torch.int32))
+    ev32 = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(20)]
+    for _ in range(3):
+        step(io=ios32[0], csr_fn=L.tfg_build_csr32)
+    torch.cuda.synchronize()
+    s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s0.record(stream)
+    for k32 in range(20):
+        step(ev32[k32], io=ios32[0], csr_fn=L.tfg_build_csr32)
+    s1.record(stream)
+    torch.cuda.synchronize()
+    if int(status[0].item()) != 0:
+        raise RuntimeError("int32 CSR build reported a bad id")
+    step32_ms = s0.elapsed_time(s1) / 20
+    csr32_ms = statistics.mean(ev[0].elapsed_time(ev[1]) for ev in ev32)
+    hp_edge32 = pin(h_edge.to(torch.int32))
+    host_in32 = dict(host_in, edge=hp_edge32)
+    e2e_run(2, hin=host_in32, ios=ios32, csr_fn=L.tfg_build_csr32)
+    torch.cuda.synchronize()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e2e_run(args.e2e_steps, f0, f1, hin=host_in32, ios=ios32, csr_fn=L.tfg_build_csr32)
+    torch.cuda.synchronize()
+    e2e32_t, e2e32_units = combine_ranks(f0.elapsed_time(f1) / 1e3,
+                                         units_per_step(n, e, f) * args.e2e_steps, world, pg)
+    h2d32 = sum(t.numel() * t.element_size() for t in host_in32.values())
+    int32_edges = {
+        "step_ms": round(step32_ms, 4), "build_csr32_ms": round(csr32_ms, 4),
+        "value": units_per_step(n, e, f) / (step32_ms * 1e-3),
+        "e2e": {"value": e2e32_units / e2e32_t, "unit": UNIT, "h2d_bytes_per_step": h2d32,
+                "d2h_bytes_per_step": d2h, "steps": args.e2e_steps},
+        "note": "the same step with edge_index held as int32 (tfg_build_csr32); not the "
+                "headline, which takes the int64 edge list"}
+    del ios32, hp_edge32, host_in32
 
     if rank != 0:
         if pg:
@@ -1058,6 +1096,7 @@ def main():
         "gpu_launches": launches_per_step(n, e) * args.steps,
         "e2e": {"value": e2e_units / e2e_t, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": args.e2e_steps, **link},
+        "int32_edges": int32_edges,
         "clocks": clocks.summary(),
     }
     line["kernels_cold_l2_ms"] = cold_l2_ms({

@@ -108,6 +108,13 @@ int tfg_build_csr(const int64_t *edge_index, int64_t num_edges, int64_t num_node
                   int32_t *rowptr, int32_t *col, int32_t *perm, int32_t *in_degree,
                   void *workspace, size_t workspace_bytes, int32_t *status,
                   tfg_stream_t stream);
+/* The same grouping from an int32 edge list (edge_index int32 [2, E], the
+ * same layout; ids are checked the same way).  Same outputs, workspace size
+ * and errors as tfg_build_csr; the first sort pass reads half the bytes. */
+int tfg_build_csr32(const int32_t *edge_index, int64_t num_edges, int64_t num_nodes,
+                    int32_t *rowptr, int32_t *col, int32_t *perm, int32_t *in_degree,
+                    void *workspace, size_t workspace_bytes, int32_t *status,
+                    tfg_stream_t stream);
 /* The same grouping by SOURCE (the CSR of the transposed graph, used by the
  * backward calls): rows are sources, col_src holds the targets, perm_src the
  * original edge ids (stable: original order within a row), out_degree the
@@ -116,6 +123,10 @@ int tfg_build_csr_by_source(const int64_t *edge_index, int64_t num_edges, int64_
                             int32_t *rowptr_src, int32_t *col_src, int32_t *perm_src,
                             int32_t *out_degree, void *workspace, size_t workspace_bytes,
                             int32_t *status, tfg_stream_t stream);
+int tfg_build_csr32_by_source(const int32_t *edge_index, int64_t num_edges, int64_t num_nodes,
+                              int32_t *rowptr_src, int32_t *col_src, int32_t *perm_src,
+                              int32_t *out_degree, void *workspace, size_t workspace_bytes,
+                              int32_t *status, tfg_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * GCN symmetric normalisation of A + I (the propagation rule of the GCN

@@ -30,8 +30,12 @@ struct NvtxRange {
     } while (0)
 #endif
 
-// Helpers of the bounds-checked debug build (check_bounds.cu).
+// Helpers of the bounds-checked debug build (check_bounds.cu), and the CSR
+// build over an int32 edge list (csr_build.cu).
 namespace tfg {
+cudaError_t launch_build_csr32(const int32_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
+                               int32_t *col, int32_t *perm, int32_t *in_degree, void *ws,
+                               int32_t *status, cudaStream_t s, bool by_source);
 bool allocation_range(const void *p, uintptr_t *base, size_t *size);
 cudaError_t csr_ends(const int32_t *rowptr, int64_t n, int32_t *first, int32_t *last,
                      cudaStream_t s);
@@ -284,7 +288,8 @@ int tfg_build_csr_workspace_size(int64_t num_nodes, int64_t num_edges, size_t *b
 }
 
 namespace {
-int build_csr_common(const char *fn, bool by_source, const int64_t *edge_index, int64_t num_edges,
+// edge_index: int64 [2, E], or int32 [2, E] when id32
+int build_csr_common(const char *fn, bool by_source, const void *edge_index, bool id32, int64_t num_edges,
                      int64_t num_nodes, int32_t *rowptr, int32_t *col, int32_t *perm,
                      int32_t *in_degree, void *workspace, size_t workspace_bytes, int32_t *status,
                      tfg_stream_t stream) {
@@ -304,16 +309,22 @@ int build_csr_common(const char *fn, bool by_source, const int64_t *edge_index, 
         if (reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
             return fail(TFG_ERR_INVALID_ARG, "%s: workspace must be 256-byte aligned", fn);
     }
-    TFG_DEBUG(debug_extent(fn, "edge_index", edge_index, sizeof(int64_t) * 2 * size_t(num_edges)));
+    TFG_DEBUG(debug_extent(fn, "edge_index", edge_index,
+                           (id32 ? sizeof(int32_t) : sizeof(int64_t)) * 2 * size_t(num_edges)));
     TFG_DEBUG(debug_extent(fn, "rowptr", rowptr, sizeof(int32_t) * size_t(num_nodes + 1)));
     TFG_DEBUG(debug_extent(fn, "col", col, sizeof(int32_t) * size_t(num_edges)));
     TFG_DEBUG(debug_extent(fn, "perm", perm, sizeof(int32_t) * size_t(num_edges)));
     TFG_DEBUG(debug_extent(fn, "in_degree", in_degree, sizeof(int32_t) * size_t(num_nodes)));
     TFG_DEBUG(debug_extent(fn, "workspace", num_edges > 0 ? workspace : nullptr, need));
-    return cuda_result(tfg::launch_build_csr(edge_index, num_edges, num_nodes, rowptr, col, perm,
-                                             in_degree, workspace, status,
-                                             reinterpret_cast<cudaStream_t>(stream), by_source),
-                       fn);
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    return cuda_result(
+        id32 ? tfg::launch_build_csr32(static_cast<const int32_t *>(edge_index), num_edges,
+                                       num_nodes, rowptr, col, perm, in_degree, workspace, status,
+                                       s, by_source)
+             : tfg::launch_build_csr(static_cast<const int64_t *>(edge_index), num_edges,
+                                     num_nodes, rowptr, col, perm, in_degree, workspace, status,
+                                     s, by_source),
+        fn);
 }
 }  // namespace
 
@@ -321,15 +332,33 @@ int tfg_build_csr(const int64_t *edge_index, int64_t num_edges, int64_t num_node
                   int32_t *rowptr, int32_t *col, int32_t *perm, int32_t *in_degree,
                   void *workspace, size_t workspace_bytes, int32_t *status,
                   tfg_stream_t stream) {
-    return build_csr_common("tfg_build_csr", false, edge_index, num_edges, num_nodes, rowptr, col,
-                            perm, in_degree, workspace, workspace_bytes, status, stream);
+    return build_csr_common("tfg_build_csr", false, edge_index, false, num_edges, num_nodes, rowptr,
+                            col, perm, in_degree, workspace, workspace_bytes, status, stream);
+}
+
+int tfg_build_csr32(const int32_t *edge_index, int64_t num_edges, int64_t num_nodes,
+                    int32_t *rowptr, int32_t *col, int32_t *perm, int32_t *in_degree,
+                    void *workspace, size_t workspace_bytes, int32_t *status,
+                    tfg_stream_t stream) {
+    return build_csr_common("tfg_build_csr32", false, edge_index, true, num_edges, num_nodes,
+                            rowptr, col, perm, in_degree, workspace, workspace_bytes, status,
+                            stream);
+}
+
+int tfg_build_csr32_by_source(const int32_t *edge_index, int64_t num_edges, int64_t num_nodes,
+                              int32_t *rowptr_src, int32_t *col_src, int32_t *perm_src,
+                              int32_t *out_degree, void *workspace, size_t workspace_bytes,
+                              int32_t *status, tfg_stream_t stream) {
+    return build_csr_common("tfg_build_csr32_by_source", true, edge_index, true, num_edges,
+                            num_nodes, rowptr_src, col_src, perm_src, out_degree, workspace,
+                            workspace_bytes, status, stream);
 }
 
 int tfg_build_csr_by_source(const int64_t *edge_index, int64_t num_edges, int64_t num_nodes,
                             int32_t *rowptr_src, int32_t *col_src, int32_t *perm_src,
                             int32_t *out_degree, void *workspace, size_t workspace_bytes,
                             int32_t *status, tfg_stream_t stream) {
-    return build_csr_common("tfg_build_csr_by_source", true, edge_index, num_edges, num_nodes,
+    return build_csr_common("tfg_build_csr_by_source", true, edge_index, false, num_edges, num_nodes,
                             rowptr_src, col_src, perm_src, out_degree, workspace, workspace_bytes,
                             status, stream);
 }

@@ -57,9 +57,11 @@ __device__ __forceinline__ uint32_t checked_id(int64_t v, int64_t n, int32_t *st
     return static_cast<uint32_t>(v);
 }
 
-template <bool FIRST>
+// IdT: the element type of the caller's edge_index (int64, or int32 for
+// tfg_build_csr32); only the first pass reads it.
+template <bool FIRST, typename IdT = int64_t>
 __global__ void __launch_bounds__(kUpThreads)
-radix_upsweep(const int64_t *__restrict__ dst64, const uint32_t *__restrict__ key32, int64_t e,
+radix_upsweep(const IdT *__restrict__ dst64, const uint32_t *__restrict__ key32, int64_t e,
               int64_t n, int shift, int width, int num_tiles, int32_t *__restrict__ cnt,
               int32_t *status) {
     extern __shared__ int32_t s_cnt[];
@@ -238,9 +240,9 @@ __device__ __forceinline__ unsigned same_digit_lanes(uint32_t dig, int bits) {
 
 // W > 0 fixes the digit width at compile time (the ballot loop unrolls and
 // the per-digit loops get constant bounds); W = 0 takes it from width_arg.
-template <bool FIRST, int W>
+template <bool FIRST, int W, typename IdT = int64_t>
 __global__ void __launch_bounds__(kDsThreads, 2)
-radix_downsweep(const int64_t *__restrict__ src64, const int64_t *__restrict__ dst64,
+radix_downsweep(const IdT *__restrict__ src64, const IdT *__restrict__ dst64,
                 const uint32_t *__restrict__ key_in, const int32_t *__restrict__ src_in,
                 const int32_t *__restrict__ eid_in, int64_t e, int64_t n, int shift,
                 int width_arg, int num_tiles, const int32_t *__restrict__ offs,
@@ -421,21 +423,24 @@ __global__ void degree_from_rowptr(const int32_t *__restrict__ rowptr, int64_t n
 #define TFG_DS_STATIC_WIDTH 1   // downsweeps with compile-time digit widths 6..10
 #endif
 
-using DownsweepFn = void (*)(const int64_t *, const int64_t *, const uint32_t *, const int32_t *,
+template <typename IdT>
+using DownsweepFn = void (*)(const IdT *, const IdT *, const uint32_t *, const int32_t *,
                              const int32_t *, int64_t, int64_t, int, int, int, const int32_t *,
                              uint32_t *, int32_t *, int32_t *, int32_t *);
 
 // Every multi-pass plan has digits of 6..10 bits (plan_for), so those widths
 // get their own code; single-pass sorts of small graphs take the generic one.
-template <bool FIRST>
-DownsweepFn downsweep_for(int width) {
+// Later passes read the library's own int32 arrays: they take IdT = int64_t
+// (their edge_index pointers are null) whatever the caller's id type.
+template <bool FIRST, typename IdT>
+DownsweepFn<IdT> downsweep_for(int width) {
     switch (TFG_DS_STATIC_WIDTH ? width : 0) {
-        case 6: return radix_downsweep<FIRST, 6>;
-        case 7: return radix_downsweep<FIRST, 7>;
-        case 8: return radix_downsweep<FIRST, 8>;
-        case 9: return radix_downsweep<FIRST, 9>;
-        case 10: return radix_downsweep<FIRST, 10>;
-        default: return radix_downsweep<FIRST, 0>;
+        case 6: return radix_downsweep<FIRST, 6, IdT>;
+        case 7: return radix_downsweep<FIRST, 7, IdT>;
+        case 8: return radix_downsweep<FIRST, 8, IdT>;
+        case 9: return radix_downsweep<FIRST, 9, IdT>;
+        case 10: return radix_downsweep<FIRST, 10, IdT>;
+        default: return radix_downsweep<FIRST, 0, IdT>;
     }
 }
 
@@ -453,9 +458,11 @@ size_t csr_workspace_bytes(int64_t n, int64_t e) {
     return a + b + h + sums;
 }
 
-cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
-                             int32_t *col, int32_t *perm, int32_t *in_degree, void *ws,
-                             int32_t *status, cudaStream_t s, bool by_source) {
+namespace {
+template <typename IdT>
+cudaError_t build_csr_impl(const IdT *edge_index, int64_t e, int64_t n, int32_t *rowptr,
+                           int32_t *col, int32_t *perm, int32_t *in_degree, void *ws,
+                           int32_t *status, cudaStream_t s, bool by_source) {
     cudaError_t err = cudaMemsetAsync(status, 0, sizeof(int32_t), s);
     if (err != cudaSuccess) return err;
     const uint32_t *sorted_keys = nullptr;
@@ -478,10 +485,10 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
         int32_t *sums = reinterpret_cast<int32_t *>(w);
 
         // the key row is row 1 (targets), or row 0 (sources) for the transposed CSR
-        const int64_t *src64 = by_source ? edge_index + e : edge_index;
-        const int64_t *dst64 = by_source ? edge_index : edge_index + e;
-        const DownsweepFn down_first = downsweep_for<true>(p.width);
-        const DownsweepFn down_later = downsweep_for<false>(p.width);
+        const IdT *src64 = by_source ? edge_index + e : edge_index;
+        const IdT *dst64 = by_source ? edge_index : edge_index + e;
+        const DownsweepFn<IdT> down_first = downsweep_for<true, IdT>(p.width);
+        const DownsweepFn<int64_t> down_later = downsweep_for<false, int64_t>(p.width);
         // the limit is set to the largest tile any width needs, so concurrent
         // builds of different sizes never lower it under one another's launch
         const int smem_max = static_cast<int>(downsweep_smem(1 << kMaxDigitBits));
@@ -496,10 +503,10 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
             Buf out = buf[pass & 1];
             if (last) { out.src = col; out.eid = perm; }
             if (first)
-                radix_upsweep<true><<<tiles, kUpThreads, radix * sizeof(int32_t), s>>>(
+                radix_upsweep<true, IdT><<<tiles, kUpThreads, radix * sizeof(int32_t), s>>>(
                     dst64, nullptr, e, n, shift, p.width, tiles, cnt, status);
             else
-                radix_upsweep<false><<<tiles, kUpThreads, radix * sizeof(int32_t), s>>>(
+                radix_upsweep<false, int64_t><<<tiles, kUpThreads, radix * sizeof(int32_t), s>>>(
                     nullptr, in.key, e, n, shift, p.width, tiles, cnt, status);
             err = exclusive_scan(cnt, int64_t(radix) * tiles, sums, s);
             if (err != cudaSuccess) return err;
@@ -520,6 +527,21 @@ cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, in
     rowptr_from_sorted<<<ceil_div(n + 1, 256), 256, 0, s>>>(sorted_keys, e, n, rowptr);
     if (n > 0) degree_from_rowptr<<<ceil_div(n, 256), 256, 0, s>>>(rowptr, n, in_degree);
     return cudaGetLastError();
+}
+}  // namespace
+
+cudaError_t launch_build_csr(const int64_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
+                             int32_t *col, int32_t *perm, int32_t *in_degree, void *ws,
+                             int32_t *status, cudaStream_t s, bool by_source) {
+    return build_csr_impl(edge_index, e, n, rowptr, col, perm, in_degree, ws, status, s,
+                          by_source);
+}
+
+cudaError_t launch_build_csr32(const int32_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
+                               int32_t *col, int32_t *perm, int32_t *in_degree, void *ws,
+                               int32_t *status, cudaStream_t s, bool by_source) {
+    return build_csr_impl(edge_index, e, n, rowptr, col, perm, in_degree, ws, status, s,
+                          by_source);
 }
 
 }  // namespace tfg

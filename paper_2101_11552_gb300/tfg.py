@@ -76,6 +76,8 @@ def _load(path: str) -> ctypes.CDLL:
         "tfg_build_csr_workspace_size": [I64, I64, ctypes.POINTER(SZ)],
         "tfg_build_csr": [P, I64, I64, P, P, P, P, P, SZ, P, P],
         "tfg_build_csr_by_source": [P, I64, I64, P, P, P, P, P, SZ, P, P],
+        "tfg_build_csr32": [P, I64, I64, P, P, P, P, P, SZ, P, P],
+        "tfg_build_csr32_by_source": [P, I64, I64, P, P, P, P, P, SZ, P, P],
         "tfg_aggregate_backward_workspace_size": [I, I64, ctypes.POINTER(SZ)],
         "tfg_aggregate_backward": [I, P, P, P, P, P, P, I64, I64, I64, P, P, SZ, P],
         "tfg_gcn_aggregate_backward": [P, P, P, P, I64, I64, I, F, P, P],
@@ -178,8 +180,10 @@ def tfg_build_csr_workspace_size(num_nodes: int, num_edges: int) -> int:
 
 def tfg_build_csr(edge_index: torch.Tensor, num_nodes: int,
                   workspace: Optional[torch.Tensor] = None) -> CSR:
-    """Group the edges of ``edge_index`` (int64 [2, E]) by target node."""
-    _need_cuda("edge_index", edge_index, torch.int64)
+    """Group the edges of ``edge_index`` (int64 or int32 [2, E]) by target node."""
+    _need_cuda("edge_index", edge_index, None)
+    if edge_index.dtype not in (torch.int64, torch.int32):
+        raise TypeError("edge_index must be int64 or int32")
     if edge_index.dim() != 2 or edge_index.shape[0] != 2:
         raise ValueError("edge_index must have shape [2, E]")
     dev = edge_index.device
@@ -192,9 +196,9 @@ def tfg_build_csr(edge_index: torch.Tensor, num_nodes: int,
     need = tfg_build_csr_workspace_size(num_nodes, e)
     if workspace is None:
         workspace = torch.empty(need, dtype=torch.uint8, device=dev)
-    _check(lib().tfg_build_csr(_ptr(edge_index), e, num_nodes, _ptr(rowptr), _ptr(col), _ptr(perm),
-                               _ptr(deg), _ptr(workspace), workspace.numel(), _ptr(status),
-                               _stream(dev)))
+    fn = lib().tfg_build_csr32 if edge_index.dtype == torch.int32 else lib().tfg_build_csr
+    _check(fn(_ptr(edge_index), e, num_nodes, _ptr(rowptr), _ptr(col), _ptr(perm), _ptr(deg),
+              _ptr(workspace), workspace.numel(), _ptr(status), _stream(dev)))
     return CSR(rowptr, col, perm, deg, status)
 
 
@@ -203,7 +207,9 @@ def tfg_build_csr_by_source(edge_index: torch.Tensor, num_nodes: int,
     """Group the edges by SOURCE (the transposed graph's CSR).  Returns the CSR
     tuple with rowptr over sources, col = targets, perm = original edge ids,
     in_degree = out-degrees."""
-    _need_cuda("edge_index", edge_index, torch.int64)
+    _need_cuda("edge_index", edge_index, None)
+    if edge_index.dtype not in (torch.int64, torch.int32):
+        raise TypeError("edge_index must be int64 or int32")
     if edge_index.dim() != 2 or edge_index.shape[0] != 2:
         raise ValueError("edge_index must have shape [2, E]")
     dev = edge_index.device
@@ -216,9 +222,10 @@ def tfg_build_csr_by_source(edge_index: torch.Tensor, num_nodes: int,
     need = tfg_build_csr_workspace_size(num_nodes, e)
     if workspace is None:
         workspace = torch.empty(need, dtype=torch.uint8, device=dev)
-    _check(lib().tfg_build_csr_by_source(_ptr(edge_index), e, num_nodes, _ptr(rowptr), _ptr(col),
-                                         _ptr(perm), _ptr(deg), _ptr(workspace), workspace.numel(),
-                                         _ptr(status), _stream(dev)))
+    fn = (lib().tfg_build_csr32_by_source if edge_index.dtype == torch.int32
+          else lib().tfg_build_csr_by_source)
+    _check(fn(_ptr(edge_index), e, num_nodes, _ptr(rowptr), _ptr(col), _ptr(perm), _ptr(deg),
+              _ptr(workspace), workspace.numel(), _ptr(status), _stream(dev)))
     return CSR(rowptr, col, perm, deg, status)
 
 

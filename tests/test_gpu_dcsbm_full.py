@@ -44,6 +44,10 @@ def test_dcsbm_csr_bit_exact(dcsbm):
     wl, ocsr, csr, _ = dcsbm
     for name, g, w in zip(("rowptr", "col", "perm", "in_degree"), csr[:4], ocsr):
         assert np.array_equal(g.cpu().numpy(), w), name
+    c32 = tfg.tfg_build_csr(dev(wl.edge_index.astype(np.int32)), wl.num_nodes)
+    tfg.check_status(c32.status)
+    for name, g, w in zip(("rowptr", "col", "perm", "in_degree"), c32[:4], csr[:4]):
+        assert torch.equal(g, w), f"int32 edge list: {name}"
 
 
 def test_dcsbm_gcn_bf16_sampled_rows(dcsbm):

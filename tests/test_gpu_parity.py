@@ -61,6 +61,26 @@ def test_csr_bit_exact(n, e, hub, iso, seed):
         assert np.array_equal(np_(g), w), name
 
 
+@pytest.mark.parametrize("by_source", [False, True])
+def test_csr_from_int32_edges_equals_int64(by_source):
+    """tfg_build_csr32 / _by_source: the same CSR from an int32 edge list, and
+    out-of-range int32 ids reported the same way."""
+    n = 50_000
+    wl = gg.random_edge_case_graph(n, 700_000, 1, 83, hub=4, isolated=50)
+    build = tfg.tfg_build_csr_by_source if by_source else tfg.tfg_build_csr
+    a = build(dev(wl.edge_index), n)
+    b = build(dev(wl.edge_index.astype(np.int32)), n)
+    tfg.check_status(b.status)
+    for name, u, v in zip(("rowptr", "col", "perm", "in_degree"), a[:4], b[:4]):
+        assert torch.equal(u, v), name
+    want = oracle.build_csr(np.ascontiguousarray(wl.edge_index[::-1]) if by_source else wl.edge_index, n)
+    for name, g, w in zip(("rowptr", "col", "perm", "in_degree"), b[:4], want):
+        assert np.array_equal(np_(g), w), name
+    bad = np.array([[0, 1, 2, 7], [1, 2, -1, 0]], dtype=np.int32)
+    got = build(dev(bad), 4)
+    assert int(got.status.item()) == tfg.TFG_ERR_INDEX_RANGE
+
+
 def test_csr_empty_graph():
     got = tfg.tfg_build_csr(torch.zeros(2, 0, dtype=torch.int64, device="cuda"), 0)
     tfg.check_status(got.status)
