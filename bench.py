@@ -864,9 +864,24 @@ def main():
     main_io = dict(edge=edge, xb=xb, batch=batch, a_src=a_src, a_dst=a_dst, h=h, att=att,
                    pool_mean=pool_mean, pool_max=pool_max)
 
-    def step(ev=None, io=None, csr_fn=None):
+    def cached_step(io):
+        xb, batch, a_src, a_dst = (io[k] for k in ("xb", "batch", "a_src", "a_dst"))
+        h, att, pool_mean, pool_max = (io[k] for k in ("h", "att", "pool_mean", "pool_max"))
+        check(L.tfg_gcn_aggregate_sum(P(rowptr), P(col), P(dinv), None, P(xb), tfg.TFG_BF16, n, f,
+                                      1, 1.0, P(h), sp))
+        check(L.tfg_edge_softmax_aggregate(P(rowptr), P(col), P(xb), tfg.TFG_BF16, n, e, heads, ch,
+                                           P(a_src), P(a_dst), 0.2, P(att), None, P(ws_sm),
+                                           ws_sm.numel(), sp))
+        check(L.tfg_segment_pool(P(h), tfg.TFG_F32, P(batch), n, g, f, tfg.REDUCERS["mean"],
+                                 P(pool_mean), st1, sp))
+        check(L.tfg_segment_pool(P(h), tfg.TFG_F32, P(batch), n, g, f, tfg.REDUCERS["max"],
+                                 P(pool_max), st1, sp))
+
+    def step(ev=None, io=None, csr_fn=None, cached=False):
         io = main_io if io is None else io
         csr_fn = L.tfg_build_csr if csr_fn is None else csr_fn   # tfg_build_csr32: int32 edges
+        if cached:   # graph-level cache: the CSR and dinv of an earlier step are reused
+            return cached_step(io)
         edge, xb, batch, a_src, a_dst = (io[k] for k in ("edge", "xb", "batch", "a_src", "a_dst"))
         h, att, pool_mean, pool_max = (io[k] for k in ("h", "att", "pool_mean", "pool_max"))
         if ev is not None:
@@ -961,7 +976,8 @@ def main():
                 ios[b][k].copy_(t, non_blocking=True)
             ev_loaded[b].record(s_in)
 
-    def e2e_run(k: int, start_ev=None, stop_ev=None, hin=host_in, ios=io_sets, csr_fn=None):
+    def e2e_run(k: int, start_ev=None, stop_ev=None, hin=host_in, ios=io_sets, csr_fn=None,
+                cached=False):
         if start_ev is not None:
             start_ev.record(stream)
             s_in.wait_event(start_ev)
@@ -973,7 +989,7 @@ def main():
             stream.wait_event(ev_loaded[b])
             if i >= 2:
                 stream.wait_event(ev_drained[b])     # results of step i - 2 have left
-            step(io=ios[b], csr_fn=csr_fn)
+            step(io=ios[b], csr_fn=csr_fn, cached=cached)
             ev_computed[b].record(stream)
             with torch.cuda.stream(s_out):
                 s_out.wait_event(ev_computed[b])
@@ -1045,6 +1061,39 @@ def main():
                 "headline, which takes the int64 edge list"}
     del ios32, hp_edge32, host_in32
 
+    # Graph-level cache (the paper's Sec. 3 cache of the normalised graph):
+    # the CSR and dinv built by the last step are reused, so a step is the
+    # GCN aggregation, the edge softmax and the two pools, and the pipeline
+    # copies only the features, batch vector and attention vectors per step.
+    # Informational, beside the headline step that rebuilds the graph.
+    step(io=io_sets[0])                      # a CSR and dinv of the current graph
+    for _ in range(3):
+        step(io=io_sets[0], cached=True)
+    torch.cuda.synchronize()
+    q0, q1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    q0.record(stream)
+    for _ in range(20):
+        step(io=io_sets[0], cached=True)
+    q1.record(stream)
+    torch.cuda.synchronize()
+    cached_ms = q0.elapsed_time(q1) / 20
+    host_in_c = {k: v for k, v in host_in.items() if k != "edge"}
+    e2e_run(2, hin=host_in_c, cached=True)
+    torch.cuda.synchronize()
+    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e2e_run(args.e2e_steps, g0, g1, hin=host_in_c, cached=True)
+    torch.cuda.synchronize()
+    ec_t, ec_units = combine_ranks(g0.elapsed_time(g1) / 1e3,
+                                   units_per_step(n, e, f) * args.e2e_steps, world, pg)
+    graph_cached = {
+        "step_ms": round(cached_ms, 4), "value": units_per_step(n, e, f) / (cached_ms * 1e-3),
+        "e2e": {"value": ec_units / ec_t, "unit": UNIT,
+                "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in host_in_c.values()),
+                "d2h_bytes_per_step": d2h, "steps": args.e2e_steps},
+        "note": "CSR and GCN normalisation built once and reused (graph-level cache); per step the "
+                "GCN aggregation, edge softmax and pools, copying features, batch vector and "
+                "attention vectors in and results out; not the headline, which rebuilds the graph"}
+
     if rank != 0:
         if pg:
             dist.destroy_process_group()
@@ -1097,6 +1146,7 @@ def main():
         "e2e": {"value": e2e_units / e2e_t, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": args.e2e_steps, **link},
         "int32_edges": int32_edges,
+        "graph_cached": graph_cached,
         "clocks": clocks.summary(),
     }
     line["kernels_cold_l2_ms"] = cold_l2_ms({
