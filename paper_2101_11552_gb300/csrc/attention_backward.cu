@@ -528,17 +528,14 @@ __device__ __forceinline__ void fast_bwd_source(const FastBwArgs &a, int64_t s, 
         for (int e = 0; e < 32; e += G * kFbUnrollSrc) {
             if (e >= cnt) break;   // warp-uniform
             float4 raw[kFbUnrollSrc];
+#if !TFG_FB_STAGE
             float wa[kFbUnrollSrc], wf[kFbUnrollSrc], wb[kFbUnrollSrc];
+#endif
 #pragma unroll
             for (int u = 0; u < kFbUnrollSrc; ++u) {
                 const int k0 = e + u * G;
                 const int k = k0 + g;
-#if TFG_FB_STAGE
-                const float4 w = stage[k * H + fh];
-                wa[u] = w.x;
-                wf[u] = w.y;
-                wb[u] = w.z;
-#else
+#if !TFG_FB_STAGE
                 const int from = ((k0 % ES) + g) * H + fh;
                 wa[u] = __shfl_sync(kFull, al[k0 / ES], from);
                 wf[u] = __shfl_sync(kFull, af[k0 / ES], from);
@@ -549,14 +546,22 @@ __device__ __forceinline__ void fast_bwd_source(const FastBwArgs &a, int64_t s, 
             }
 #pragma unroll
             for (int u = 0; u < kFbUnrollSrc; ++u) {
+#if TFG_FB_STAGE
+                // the staged weights are read when the row is used, so only
+                // the row slices are live while the gathers are in flight
+                const float4 w4 = stage[(e + u * G + g) * H + fh];
+                const float wa_u = w4.x, wf_u = w4.y, wb_u = w4.z;
+#else
+                const float wa_u = wa[u], wf_u = wf[u], wb_u = wb[u];
+#endif
                 const float gv[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
                 float d = 0.f;
 #pragma unroll
                 for (int q = 0; q < 4; ++q) d = fmaf(gv[q], xs[q], d);
                 d = group_sum(d, hl);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) part[q] = fmaf(wa[u], gv[q], part[q]);
-                partd += fmaf(wf[u], d, -wb[u]);
+                for (int q = 0; q < 4; ++q) part[q] = fmaf(wa_u, gv[q], part[q]);
+                partd += fmaf(wf_u, d, -wb_u);
             }
         }
 #pragma unroll
