@@ -60,6 +60,15 @@ def test_csr_at_max_nodes(huge_graph):
     _equal_in_chunks(csr.in_degree, deg, "in_degree")
 
 
+def test_csr_from_int32_edges_at_max_nodes(huge_graph):
+    """tfg_build_csr32 with ids up to 2^31 - 2: the same CSR as the int64 build."""
+    ei, csr = huge_graph
+    c32 = tfg.tfg_build_csr(dev(ei.astype(np.int32)), N_MAX)
+    tfg.check_status(c32.status)
+    assert torch.equal(c32.col, csr.col) and torch.equal(c32.perm, csr.perm)
+    assert torch.equal(c32.rowptr, csr.rowptr) and torch.equal(c32.in_degree, csr.in_degree)
+
+
 @pytest.mark.parametrize("reduce", ["sum", "mean", "max"])
 def test_aggregate_at_max_nodes(huge_graph, reduce):
     ei, csr = huge_graph
