@@ -72,9 +72,31 @@ struct AggArgs {
     const void *x0;     // APPNP mode: the teleport features x0 [N, F]
     float alpha;        // APPNP mode: teleport weight
     float beta;         // APPNP mode: 1 - alpha, rounded once on the host
+    int regime;         // kRegimeAny, or the degree regime the launched kernel serves
 };
 
+#ifndef TFG_MP_F32_DEGREE
+#define TFG_MP_F32_DEGREE 32   // mean in-degree splitting the fp32 sum regimes
+#endif
+constexpr int kRegimeAny = 0;      // the kernel runs whatever the degree
+constexpr int kRegimeShort = 1;    // runs only when E < TFG_MP_F32_DEGREE * N
+constexpr int kRegimeLong = 2;     // runs only when E >= TFG_MP_F32_DEGREE * N
+
+// True when a kernel launched for one degree regime finds the graph in the
+// other (the same answer in every thread: the caller returns before any
+// barrier).
+__device__ __forceinline__ bool other_regime(const int32_t *rowptr, int64_t n, int regime,
+                                             int64_t degree) {
+    if (regime == kRegimeAny) return false;
+    const bool short_rows = static_cast<int64_t>(__ldg(rowptr + n)) < degree * n;
+    return short_rows != (regime == kRegimeShort);
+}
+
 enum Kind { kSumLike = 0, kMax = 1, kGcn = 2, kAppnp = 3 };
+
+// The layouts whose launch splits by degree regime: fp32 sums in 16-byte slices.
+template <typename XT, int VEC, int KIND>
+constexpr bool kSplitsRegimes = sizeof(XT) == 4 && VEC == 4 && KIND != kMax;
 
 template <typename XT, int VEC, int LPR, int KIND, typename X0T = XT>
 struct Agg {
@@ -305,6 +327,9 @@ __global__ void __launch_bounds__(kAggThreads, VEC >= 8 ? TFG_AGG_MINB : 4) aggr
     __shared__ int s_next, s_nheavy;
     __shared__ int64_t s_heavy[kMaxHeavy];
     __shared__ float s_part[kAggWarps * LPR * VEC];
+    if constexpr (kSplitsRegimes<XT, VEC, KIND>) {
+        if (other_regime(a.rowptr, a.n, a.regime, TFG_MP_F32_DEGREE)) return;
+    }
     int64_t r0, r1;
     balanced_rows(a.rowptr, a.n, gridDim.x, blockIdx.x, r0, r1);
     const int64_t nrows = r1 - r0;
@@ -361,9 +386,18 @@ __global__ void __launch_bounds__(kAggThreads, VEC >= 8 ? TFG_AGG_MINB : 4) aggr
 // shared memory): GCN 1.82 ms at 4 CTAs per SM and 4 gathers in flight per
 // lane (3 CTAs and 8 in flight: 1.84 ms; 2 CTAs and 16: 2.06 ms; the
 // row-per-warp aggregate_kernel: 1.95 ms); max 2.84 ms (aggregate_kernel
-// 3.34 ms).  fp32 rows (512 bytes, one row per warp load) stay on
-// aggregate_kernel: 2.99 ms there against 3.10-3.50 ms here; bf16 rows as
-// 8-byte slices (4 features per lane, up to 16 in flight) measured 1.90-3.04 ms.
+// 3.34 ms).  bf16 rows as 8-byte slices (4 features per lane, up to 16 in
+// flight) measured 1.90-3.04 ms.
+// fp32 rows (16-byte slices of 4 features) depend on the degree.  On the
+// same graph in fp32 (mean in-degree 493) the GCN sum takes 2.99-3.04 ms in
+// aggregate_kernel against 3.15-3.31 ms here, at 2-4 CTAs per SM and 4-8 in
+// flight; max takes 3.35 ms here against 4.32 ms.  On graphs of mean
+// in-degree 4-8 (2,708 nodes F = 64; 169,343 nodes F = 128; 1,024 molecule
+// graphs F = 128) this kernel is 21-38% faster for sums and 26-42% for max.
+// So fp32 max always comes here, and an fp32 sum launches both kernels with
+// a degree regime: each reads E = rowptr[N] and returns at once unless the
+// mean in-degree E / N is on its side of TFG_MP_F32_DEGREE (the entry points
+// are not given E on the host, and reading it back would stall the stream).
 #ifndef TFG_MP_BLOCKS
 #define TFG_MP_BLOCKS 4    // resident CTAs per SM for sums (64 registers per thread)
 #endif
@@ -499,6 +533,9 @@ __global__ void __launch_bounds__(kAggThreads, mp_blocks<KIND == kMax>()) aggreg
     __shared__ float s_head[kAggWarps][kF];    // an owner's own part of a row begun by others
     __shared__ int32_t s_tail_row[kAggWarps], s_head_row[kAggWarps];
     __shared__ __align__(16) float2 s_stage[kAggWarps][32];   // a chunk's (id, weight) pairs
+    if constexpr (kSplitsRegimes<XT, VEC, KIND>) {
+        if (other_regime(a.rowptr, a.n, a.regime, TFG_MP_F32_DEGREE)) return;
+    }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int g = lane / LPR, sub = lane % LPR;
     const int64_t f0 = static_cast<int64_t>(sub) * VEC;
@@ -591,29 +628,49 @@ __global__ void __launch_bounds__(kAggThreads, mp_blocks<KIND == kMax>()) aggreg
     }
 }
 
-template <typename XT, int VEC, int KIND, typename X0T = XT>
-cudaError_t launch_lpr(const AggArgs &a, int lpr, cudaStream_t s) {
-    // E is not known on the host; the kernel reads rowptr[N] for the split.
-    // 16-byte bf16 slices in one feature tile: the merge-path kernel
-    if constexpr (sizeof(XT) == 2 && VEC == 8) {
-        if (TFG_AGG_MP && static_cast<int64_t>(lpr) * VEC >= a.f) {
-            const int grid = static_cast<int>(
-                min64(a.n, static_cast<int64_t>(sm_count()) * mp_blocks<KIND == kMax>()));
-            switch (lpr) {
-                case 32: aggregate_mp_kernel<XT, VEC, 32, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
-                case 16: aggregate_mp_kernel<XT, VEC, 16, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
-                default: aggregate_mp_kernel<XT, VEC, 8, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
-            }
-            return cudaGetLastError();
+template <typename XT, int VEC, int LPR, int KIND, typename X0T>
+cudaError_t launch_mp(const AggArgs &a, cudaStream_t s) {
+    const int grid = static_cast<int>(
+        min64(a.n, static_cast<int64_t>(sm_count()) * mp_blocks<KIND == kMax>()));
+    aggregate_mp_kernel<XT, VEC, LPR, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+template <typename XT, int VEC, int LPR, int KIND, typename X0T>
+cudaError_t launch_rows(const AggArgs &a, cudaStream_t s) {
+    aggregate_kernel<XT, VEC, LPR, KIND, X0T><<<balanced_grid(a.n, 0, 1), kAggThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+template <typename XT, int VEC, int LPR, int KIND, typename X0T>
+cudaError_t launch_agg(const AggArgs &a, cudaStream_t s) {
+    // E is not known on the host; the kernels read rowptr[N] for the split.
+    // Rows of one feature tile in 16-byte slices take the merge-path kernel:
+    // bf16 always, fp32 for max, and fp32 sums on graphs of short rows (the
+    // row-per-warp kernel is launched beside it for the long-row regime).
+    constexpr bool bf16 = sizeof(XT) == 2 && VEC == 8;
+    constexpr bool f32 = sizeof(XT) == 4 && VEC == 4;
+    if constexpr (bf16 || f32) {
+        if (TFG_AGG_MP && static_cast<int64_t>(LPR) * VEC >= a.f) {
+            if constexpr (!kSplitsRegimes<XT, VEC, KIND>) return launch_mp<XT, VEC, LPR, KIND, X0T>(a, s);
+            AggArgs shortr = a, longr = a;
+            shortr.regime = kRegimeShort;
+            longr.regime = kRegimeLong;
+            const cudaError_t err = launch_mp<XT, VEC, LPR, KIND, X0T>(shortr, s);
+            if (err != cudaSuccess) return err;
+            return launch_rows<XT, VEC, LPR, KIND, X0T>(longr, s);
         }
     }
-    const int grid = balanced_grid(a.n, 0, 1);
+    return launch_rows<XT, VEC, LPR, KIND, X0T>(a, s);
+}
+
+template <typename XT, int VEC, int KIND, typename X0T = XT>
+cudaError_t launch_lpr(const AggArgs &a, int lpr, cudaStream_t s) {
     switch (lpr) {
-        case 32: aggregate_kernel<XT, VEC, 32, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
-        case 16: aggregate_kernel<XT, VEC, 16, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
-        default: aggregate_kernel<XT, VEC, 8, KIND, X0T><<<grid, kAggThreads, 0, s>>>(a); break;
+        case 32: return launch_agg<XT, VEC, 32, KIND, X0T>(a, s);
+        case 16: return launch_agg<XT, VEC, 16, KIND, X0T>(a, s);
+        default: return launch_agg<XT, VEC, 8, KIND, X0T>(a, s);
     }
-    return cudaGetLastError();
 }
 
 inline int lanes_per_row(int64_t chunks) { return chunks >= 32 ? 32 : (chunks > 8 ? 16 : 8); }

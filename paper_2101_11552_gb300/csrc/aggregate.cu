@@ -21,7 +21,8 @@ cudaError_t launch_aggregate(int mode, const int32_t *rowptr, const int32_t *col
                              const float *dinv, const void *x, int x_dtype, int64_t n, int64_t f,
                              int add_self, float fill, float *out, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
-    AggArgs a{rowptr, col, w, dinv, x, out, n, f, mode == 1, add_self, fill, nullptr, 0.f, 1.f};
+    AggArgs a{rowptr, col, w, dinv, x, out, n, f, mode == 1, add_self, fill, nullptr, 0.f, 1.f,
+              kRegimeAny};
     const int kind = mode == 2 ? kMax : (mode == 3 ? kGcn : kSumLike);
     const bool aligned = (reinterpret_cast<uintptr_t>(x) % 16 == 0) &&
                          (reinterpret_cast<uintptr_t>(out) % 16 == 0);

@@ -81,7 +81,7 @@ cudaError_t launch_propagate(const int32_t *rowptr, const int32_t *col, const fl
     const void *h = x0;
     for (int64_t k = 0; k < hops; ++k) {
         float *dst = ((hops - 1 - k) % 2 == 0) ? out : spare;
-        AggArgs a{rowptr, col, w, dinv, h, dst, n, f, 0, add_self, fill, x0, alpha, beta};
+        AggArgs a{rowptr, col, w, dinv, h, dst, n, f, 0, add_self, fill, x0, alpha, beta, kRegimeAny};
         const cudaError_t err = x_dtype == TFG_BF16 ? launch_hop<uint16_t>(a, k == 0, s)
                                                     : launch_hop<float>(a, k == 0, s);
         if (err != cudaSuccess) return err;

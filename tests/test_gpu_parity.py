@@ -160,6 +160,33 @@ def test_aggregate(reduce, dtype, weighted, f):
             assert_scaled_close(got, ref, scale, TOL_F32, what)
 
 
+@pytest.mark.parametrize("f", [8, 64, 128])
+@pytest.mark.parametrize("n,e,hub", [(1000, 31999, -1), (1000, 32000, -1), (700, 35000, 2),
+                                     (64, 32 * 64, 0)])
+def test_fp32_sums_on_both_sides_of_the_degree_split(n, e, hub, f):
+    """fp32 sums in 16-byte slices run the merge-path kernel below a mean
+    in-degree of 32 and the row-per-warp kernel from 32 up (each kernel
+    reads E on the device); E = 32 N - 1 and E = 32 N sit on the two sides."""
+    wl = gg.random_edge_case_graph(n, e, f, 300 + e % 97 + f, hub=hub, isolated=3)
+    csr = gpu_csr(wl.edge_index, n)
+    x = features(wl, "f32")
+    for reduce, fn in (("sum", tfg.tfg_aggregate_sum), ("mean", tfg.tfg_aggregate_mean),
+                       ("max", tfg.tfg_aggregate_max)):
+        got = np_(fn(csr.rowptr, csr.col, x))
+        ref, scale = oracle.aggregate(wl.edge_index, n, wl.x, reduce)
+        what = f"{reduce} n={n} e={e} F={f}"
+        if reduce == "max":
+            assert_exact_f32(got, ref, what)
+        else:
+            assert_scaled_close(got, ref, scale, TOL_F32, what)
+    for add_self in (0, 1):
+        dinv, _ = tfg.tfg_gcn_norm(csr.rowptr, csr.col, csr.perm, n, None, add_self, 1.0,
+                                   want_w_csr=False)
+        got = np_(tfg.tfg_gcn_aggregate_sum(csr.rowptr, csr.col, dinv, x, None, add_self, 1.0))
+        ref, scale = oracle.gcn_aggregate(wl.edge_index, n, wl.x, None, add_self, 1.0)
+        assert_scaled_close(got, ref, scale, TOL_F32, f"gcn self={add_self} n={n} e={e} F={f}")
+
+
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("add_self", [0, 1])
 @pytest.mark.parametrize("f", [5, 64, 128])
