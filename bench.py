@@ -645,14 +645,23 @@ def next_rows(L, wl, bufs, stream, hbm_peak):
     ms_fwd = _event_ms(lambda: check(L.tfg_aggregate_max_argmax(
         P(bufs["rowptr"]), P(bufs["col"]), P(perm_fwd), None, P(bufs["xb"]), tfg.TFG_BF16, n, f,
         P(out_max), P(argmax), sp)), stream, 5)
+    ws_mark = torch.empty(max(tfg.tfg_aggregate_max_backward_workspace_size(n, e, f), 1),
+                          dtype=torch.uint8, device=dev)
     ms_bwd = _event_ms(lambda: check(L.tfg_aggregate_max_backward(
-        P(csr_src.rowptr), P(csr_src.col), P(csr_src.perm), P(argmax), None, P(bufs["h"]), n, f,
-        P(grad_x), sp)), stream, 5)
+        P(csr_src.rowptr), P(csr_src.col), P(csr_src.perm), P(argmax), None, P(bufs["h"]), n, e, f,
+        P(grad_x), P(ws_mark), ws_mark.numel(), sp)), stream, 5)
+    ms_bwd_all = _event_ms(lambda: check(L.tfg_aggregate_max_backward(
+        P(csr_src.rowptr), P(csr_src.col), P(csr_src.perm), P(argmax), None, P(bufs["h"]), n, e, f,
+        P(grad_x), None, 0, sp)), stream, 5)
+    marked = int((ws_mark[:e] != 0).sum().item()) if ws_mark.numel() > 1 else e
     rows["max_argmax_and_backward"] = {
         "forward_ms": round(ms_fwd, 4), "backward_ms": round(ms_bwd, 4),
+        "backward_without_marks_ms": round(ms_bwd_all, 4),
+        "edges_marked_frac": round(marked / max(e, 1), 4),
         "forward_edge_features_per_s": e * f / (ms_fwd * 1e-3),
         "backward_edge_features_per_s": e * f / (ms_bwd * 1e-3),
-        "note": "bf16 features, argmax int32 [N, F]; backward reads argmax and gradient rows per out-edge"}
+        "note": "bf16 features, argmax int32 [N, F]; the backward records per edge the features "
+                "it wins and reads argmax and gradient values for those alone"}
     # backward of the GAT edge softmax: grad_out = the softmax output of the
     # step (fp32), the forward's output taken from a fresh forward call
     heads, ch = wl.heads, wl.channels

@@ -224,7 +224,17 @@ int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float
  * tfg_aggregate_max_backward: grad_x[s, f] = sum over edges e = (s -> t)
  *   with argmax[t, f] == e of w_e grad_out[t, f], w_e = edge_weight[e] in
  *   ORIGINAL edge order (the weights of the forward, w_csr[k] =
- *   edge_weight[perm[k]]), or 1 when edge_weight is NULL.
+ *   edge_weight[perm[k]]), or 1 when edge_weight is NULL.  num_edges =
+ *   rowptr_src[num_nodes].  argmax values outside [0, num_edges) match no
+ *   edge.  tfg_aggregate_max_backward_workspace_size() gives the workspace
+ *   (16-byte aligned, overwritten) for win marks: on long rows (mean
+ *   in-degree num_edges / num_nodes >= 32), where an edge wins few
+ *   features, the call first marks, in a byte per edge, which eighths of
+ *   the features the edge is the argmax of, and then reads argmax and
+ *   gradient slices for those alone.  0 bytes: the marks would not pay and
+ *   no workspace is used.
+ *   Workspace NULL reads the argmax and gradient rows of every out-edge.
+ *   Both ways give the same bits.
  * grad_out, grad_x: fp32 [num_nodes, num_features]; grad_x is written.
  * Every sum runs in a fixed order: results are bitwise reproducible.
  * ---------------------------------------------------------------------- */
@@ -242,10 +252,13 @@ int tfg_aggregate_max_argmax(const int32_t *rowptr, const int32_t *col, const in
                              const float *w_csr, const void *x, int x_dtype, int64_t num_nodes,
                              int64_t num_features, float *out, int32_t *argmax,
                              tfg_stream_t stream);
+int tfg_aggregate_max_backward_workspace_size(int64_t num_nodes, int64_t num_edges,
+                                              int64_t num_features, size_t *bytes);
 int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src,
                                const int32_t *perm_src, const int32_t *argmax,
                                const float *edge_weight, const float *grad_out,
-                               int64_t num_nodes, int64_t num_features, float *grad_x,
+                               int64_t num_nodes, int64_t num_edges, int64_t num_features,
+                               float *grad_x, void *workspace, size_t workspace_bytes,
                                tfg_stream_t stream);
 
 /* ------------------------------------------------------------------------

@@ -30,9 +30,16 @@ struct NvtxRange {
     } while (0)
 #endif
 
-// Helpers of the bounds-checked debug build (check_bounds.cu), and the CSR
-// build over an int32 edge list (csr_build.cu).
+// Helpers of the bounds-checked debug build (check_bounds.cu), the CSR
+// build over an int32 edge list (csr_build.cu) and the max backward with
+// win marks (backward.cu).
 namespace tfg {
+size_t max_backward_workspace_bytes(int64_t n, int64_t e, int64_t f);
+cudaError_t launch_max_backward_marked(const int32_t *rowptr_src, const int32_t *col_src,
+                                       const int32_t *perm_src, const int32_t *argmax,
+                                       const float *edge_weight, const float *grad_out, int64_t n,
+                                       int64_t e, int64_t f, float *grad_x, void *ws,
+                                       cudaStream_t s);
 cudaError_t launch_build_csr32(const int32_t *edge_index, int64_t e, int64_t n, int32_t *rowptr,
                                int32_t *col, int32_t *perm, int32_t *in_degree, void *ws,
                                int32_t *status, cudaStream_t s, bool by_source);
@@ -502,35 +509,56 @@ int tfg_aggregate_max_argmax(const int32_t *rowptr, const int32_t *col, const in
                        fn);
 }
 
+int tfg_aggregate_max_backward_workspace_size(int64_t num_nodes, int64_t num_edges,
+                                              int64_t num_features, size_t *bytes) {
+    const char *fn = "tfg_aggregate_max_backward_workspace_size";
+    TFG_RANGE(fn);
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
+    TFG_TRY(check_features(fn, num_nodes, num_features));
+    TFG_NEED(bytes, true, fn, "bytes");
+    *bytes = tfg::max_backward_workspace_bytes(num_nodes, num_edges, num_features);
+    return ok();
+}
+
 int tfg_aggregate_max_backward(const int32_t *rowptr_src, const int32_t *col_src,
                                const int32_t *perm_src, const int32_t *argmax,
                                const float *edge_weight, const float *grad_out,
-                               int64_t num_nodes, int64_t num_features, float *grad_x,
+                               int64_t num_nodes, int64_t num_edges, int64_t num_features,
+                               float *grad_x, void *workspace, size_t workspace_bytes,
                                tfg_stream_t stream) {
     const char *fn = "tfg_aggregate_max_backward";
     TFG_RANGE(fn);
-    TFG_TRY(check_counts(fn, num_nodes, 0));
+    TFG_TRY(check_counts(fn, num_nodes, num_edges));
     TFG_TRY(check_features(fn, num_nodes, num_features));
     TFG_NEED(rowptr_src, true, fn, "rowptr_src");
-    TFG_NEED(perm_src, col_src != nullptr, fn, "perm_src");
+    TFG_NEED(col_src, num_edges > 0, fn, "col_src");
+    TFG_NEED(perm_src, num_edges > 0, fn, "perm_src");
     TFG_NEED(argmax, num_nodes > 0, fn, "argmax");
     TFG_NEED(grad_out, num_nodes > 0, fn, "grad_out");
     TFG_NEED(grad_x, num_nodes > 0, fn, "grad_x");
-#if TFG_CHECK_BOUNDS
-    {
-        int64_t e = 0;
-        TFG_DEBUG(debug_csr(fn, "col_src", rowptr_src, col_src, perm_src, num_nodes, -1, &e, stream));
-        TFG_DEBUG(debug_extent(fn, "edge_weight", edge_weight, sizeof(float) * size_t(e)));
-        TFG_DEBUG(debug_extent(fn, "argmax", argmax, sizeof(int32_t) * size_t(num_nodes * num_features)));
-        TFG_DEBUG(debug_extent(fn, "grad_out", grad_out, sizeof(float) * size_t(num_nodes * num_features)));
-        TFG_DEBUG(debug_extent(fn, "grad_x", grad_x, sizeof(float) * size_t(num_nodes * num_features)));
-    }
-#endif
-    return cuda_result(tfg::launch_max_backward(rowptr_src, col_src, perm_src, argmax,
-                                                edge_weight, grad_out, num_nodes, num_features,
-                                                grad_x,
-                                                reinterpret_cast<cudaStream_t>(stream)),
-                       fn);
+    const size_t need =
+        workspace ? tfg::max_backward_workspace_bytes(num_nodes, num_edges, num_features) : 0;
+    if (need > 0 && workspace_bytes < need)
+        return fail(TFG_ERR_WORKSPACE, "%s: workspace of %zu bytes needed, %zu given", fn, need,
+                    workspace_bytes);
+    if (need > 0 && reinterpret_cast<uintptr_t>(workspace) % 16 != 0)
+        return fail(TFG_ERR_INVALID_ARG, "%s: workspace must be 16-byte aligned", fn);
+    TFG_DEBUG(debug_csr(fn, "col_src", rowptr_src, col_src, perm_src, num_nodes, num_edges,
+                        nullptr, stream));
+    TFG_DEBUG(debug_extent(fn, "edge_weight", edge_weight, sizeof(float) * size_t(num_edges)));
+    TFG_DEBUG(debug_extent(fn, "argmax", argmax, sizeof(int32_t) * size_t(num_nodes * num_features)));
+    TFG_DEBUG(debug_extent(fn, "grad_out", grad_out, sizeof(float) * size_t(num_nodes * num_features)));
+    TFG_DEBUG(debug_extent(fn, "grad_x", grad_x, sizeof(float) * size_t(num_nodes * num_features)));
+    TFG_DEBUG(debug_extent(fn, "workspace", need ? workspace : nullptr, need));
+    const int32_t *col = num_edges > 0 ? col_src : nullptr;
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    return cuda_result(
+        need ? tfg::launch_max_backward_marked(rowptr_src, col, perm_src, argmax, edge_weight,
+                                               grad_out, num_nodes, num_edges, num_features, grad_x,
+                                               workspace, s)
+             : tfg::launch_max_backward(rowptr_src, col, perm_src, argmax, edge_weight, grad_out,
+                                        num_nodes, num_features, grad_x, s),
+        fn);
 }
 
 int tfg_propagate_workspace_size(int64_t num_nodes, int64_t num_features, int64_t num_hops,

@@ -73,6 +73,9 @@ struct MaxArgs {
     int64_t n, f;
     float *out;
     int32_t *argmax_out;        // forward only
+    const uint8_t *mark;        // backward: bit j of mark[e] when edge e wins some (t, f) of feature group j
+    int64_t e;                  // backward: edges (the extent of mark)
+    int group;                  // backward: features per group (a multiple of 4, at most 8 groups)
 };
 
 // Forward state of VEC features over an edge range, in CSR order (= original
@@ -104,7 +107,7 @@ __device__ __forceinline__ void max_combine(float &b, int32_t &p, float ob, int3
 
 template <typename XT, int VEC, int LPR>
 struct MaxFwd {
-    static constexpr int kVec = VEC, kLpr = LPR, kGroups = 32 / LPR;
+    static constexpr int kVec = VEC, kLpr = LPR, kGroups = 32 / LPR, kMinBlocks = 1;
     float best[VEC];
     int32_t pos[VEC];
 
@@ -192,13 +195,35 @@ struct MaxFwd {
 
 // Backward state: grad_x[s, f] = sum over the out-edges e = (s -> t) of s,
 // in CSR (= original) order, of w_e grad_out[t, f] where argmax[t, f] == e.
-// Per edge a lane requests its slice of the argmax row and of the gradient
-// row of t together, one round trip; this was measured faster than waiting
-// for the argmax row to skip gradient reads, and faster than more edges in
-// flight per warp, which cost registers and so resident warps.
-template <int VEC>
+#ifndef TFG_MXB_DEPTH
+#define TFG_MXB_DEPTH 4        // backward with win marks: marked out-edges in flight per warp
+#endif
+#ifndef TFG_MXB_DEPTH_ALL
+#define TFG_MXB_DEPTH_ALL 4    // backward over every out-edge: edges in flight per warp
+#endif
+#ifndef TFG_MXB_MINB
+#define TFG_MXB_MINB 4         // backward: resident CTAs per SM (64 registers per thread)
+#endif
+#ifndef TFG_MXB_GROUPS
+#define TFG_MXB_GROUPS 1       // 1: a marked edge's lanes read only the feature groups it wins
+#endif
+
+// Two ways to find the (edge, feature) pairs that contribute, with the same
+// sums in the same order:
+//  * every out-edge: a lane requests its slice of the argmax row and of the
+//    gradient row of t together (one round trip, D edges in flight) and
+//    adds where the argmax names the edge;
+//  * win marks (MASKED): the features are cut into at most 8 groups, and bit
+//    j of mark[e] is set when edge e is the argmax of some (t, f) with f in
+//    group j.  A chunk's edges with no bit set are skipped, and for the
+//    others only the lanes whose group bit is set read their slices.  On
+//    long rows few edges win anything and a winner wins few features, so
+//    most row reads disappear; the marks take a byte per edge and stay in
+//    L2.  A bit can come from another row's argmax naming the edge: the
+//    argmax check decides, as in the full walk.
+template <int VEC, bool MASKED>
 struct MaxBwd {
-    static constexpr int kVec = VEC, kLpr = 32;
+    static constexpr int kVec = VEC, kLpr = 32, kMinBlocks = TFG_MXB_MINB;
     float acc[VEC];
 
     __device__ void init() {
@@ -207,31 +232,61 @@ struct MaxBwd {
     }
 
     __device__ void scan(const MaxArgs &a, int64_t k0, int64_t k1, int64_t fl, bool, int lane) {
+        constexpr int D = MASKED ? TFG_MXB_DEPTH : TFG_MXB_DEPTH_ALL;
         const float *g = static_cast<const float *>(a.x);
         for (int64_t base = k0; base < k1; base += 32) {
             const int cnt = static_cast<int>(min64(32, k1 - base));
             const bool mine = lane < cnt;
             const int c = mine ? ld_stream(a.col + base + lane) : 0;
             const int32_t ec = mine ? __ldg(a.perm + base + lane) : 0;
-            const float wc = a.w ? (mine ? __ldg(a.w + ec) : 0.f) : 1.f;
-            for (int k = 0; k < cnt; ++k) {
-                const int64_t t = __shfl_sync(kFull, c, k);
-                const int32_t e = __shfl_sync(kFull, ec, k);
-                const float we = __shfl_sync(kFull, wc, k);
-                int32_t am[VEC];
-                float gv[VEC];
-                if constexpr (VEC == 4) {
-                    const int4 v = __ldg(reinterpret_cast<const int4 *>(a.argmax_in + t * a.f + fl));
-                    const float4 w4 = __ldg(reinterpret_cast<const float4 *>(g + t * a.f + fl));
-                    am[0] = v.x; am[1] = v.y; am[2] = v.z; am[3] = v.w;
-                    gv[0] = w4.x; gv[1] = w4.y; gv[2] = w4.z; gv[3] = w4.w;
-                } else {
-                    am[0] = __ldg(a.argmax_in + t * a.f + fl);
-                    gv[0] = __ldg(g + t * a.f + fl);
+            uint32_t mk = mine ? 0xffu : 0u;
+            if constexpr (MASKED)
+                mk = mine && static_cast<uint64_t>(ec) < static_cast<uint64_t>(a.e) ? __ldg(a.mark + ec)
+                                                                                   : 0u;
+            const bool win = mk != 0;
+            const float wc = a.w ? (win ? __ldg(a.w + ec) : 0.f) : 1.f;
+            const uint32_t my_bit =
+                MASKED && TFG_MXB_GROUPS ? 1u << static_cast<uint32_t>(fl / a.group) : 0xffu;
+            // the chunk's edges that may contribute, D at a time in chunk order
+            for (uint32_t m = __ballot_sync(kFull, win); m != 0;) {
+                int64_t t[D];
+                int32_t ed[D];
+                float we[D];
+                bool ok[D];
+#pragma unroll
+                for (int d = 0; d < D; ++d) {
+                    const bool any = m != 0;
+                    const int k = any ? __ffs(m) - 1 : 0;
+                    m &= m - 1;
+                    t[d] = __shfl_sync(kFull, c, k);
+                    ed[d] = __shfl_sync(kFull, ec, k);
+                    we[d] = __shfl_sync(kFull, wc, k);
+                    ok[d] = any && (__shfl_sync(kFull, mk, k) & my_bit) != 0;   // per lane
+                }
+                int32_t am[D][VEC];
+                float gv[D][VEC];
+                {
+#pragma unroll
+                    for (int d = 0; d < D; ++d) {
+                        if (!ok[d]) continue;
+                        if constexpr (VEC == 4) {
+                            const int4 v = __ldg(reinterpret_cast<const int4 *>(a.argmax_in + t[d] * a.f + fl));
+                            const float4 w4 = __ldg(reinterpret_cast<const float4 *>(g + t[d] * a.f + fl));
+                            am[d][0] = v.x; am[d][1] = v.y; am[d][2] = v.z; am[d][3] = v.w;
+                            gv[d][0] = w4.x; gv[d][1] = w4.y; gv[d][2] = w4.z; gv[d][3] = w4.w;
+                        } else {
+                            am[d][0] = __ldg(a.argmax_in + t[d] * a.f + fl);
+                            gv[d][0] = __ldg(g + t[d] * a.f + fl);
+                        }
+                    }
                 }
 #pragma unroll
-                for (int q = 0; q < VEC; ++q)
-                    if (am[q] == e) acc[q] = fmaf(we, gv[q], acc[q]);
+                for (int d = 0; d < D; ++d) {
+                    if (!ok[d]) continue;
+#pragma unroll
+                    for (int q = 0; q < VEC; ++q)
+                        if (am[d][q] == ed[d]) acc[q] = fmaf(we[d], gv[d][q], acc[q]);
+                }
             }
         }
     }
@@ -313,7 +368,7 @@ __device__ void max_cta_row(const MaxArgs &a, int64_t t, float *s_val, int32_t *
 }
 
 template <typename State>
-__global__ void __launch_bounds__(kMxThreads) max_rows_kernel(MaxArgs a) {
+__global__ void __launch_bounds__(kMxThreads, State::kMinBlocks) max_rows_kernel(MaxArgs a) {
     __shared__ int s_next, s_nheavy;
     __shared__ int64_t s_heavy[kMxMaxHeavy];
     __shared__ float s_val[kMxWarps * State::kLpr * State::kVec];
@@ -351,6 +406,33 @@ __global__ void __launch_bounds__(kMxThreads) max_rows_kernel(MaxArgs a) {
 
 bool aligned(const void *p, uintptr_t b) { return reinterpret_cast<uintptr_t>(p) % b == 0; }
 
+// Win marks of the max backward.  Every (t, f) has one winning edge (none
+// for a row without edges); a row of in-degree d has at most min(d, F)
+// distinct winners, so on long rows most out-edges win nothing and a
+// winner wins few features.  Two launches write the marks: zero them, then
+// for each e = argmax[t, f] set bit f / group of mark[e] (atomicOr on the
+// word holding the byte).  Ids outside [0, E) are ignored.
+__global__ void max_marks_zero(uint8_t *__restrict__ mark, int64_t bytes) {
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    const int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    const int64_t n16 = reinterpret_cast<uintptr_t>(mark) % 16 == 0 ? bytes / 16 : 0;
+    uint4 *m16 = reinterpret_cast<uint4 *>(mark);
+    for (int64_t i = i0; i < n16; i += stride) m16[i] = make_uint4(0, 0, 0, 0);
+    for (int64_t i = n16 * 16 + i0; i < bytes; i += stride) mark[i] = 0;
+}
+
+__global__ void max_marks_set(const int32_t *__restrict__ argmax, int64_t n, int64_t f, int64_t e,
+                              int group, uint8_t *__restrict__ mark) {
+    uint32_t *words = reinterpret_cast<uint32_t *>(mark);   // 4-byte aligned (checked by the caller)
+    // rows t over the grid, features over the threads of a block
+    for (int64_t t = blockIdx.x; t < n; t += gridDim.x)
+        for (int64_t c = threadIdx.x; c < f; c += blockDim.x) {
+            const int32_t k = __ldg(argmax + t * f + c);
+            if (static_cast<uint64_t>(k) >= static_cast<uint64_t>(e)) continue;
+            const uint32_t bit = 1u << static_cast<uint32_t>(c / group);
+            atomicOr(words + (k >> 2), bit << (8 * (k & 3)));
+        }
+}
 
 }  // namespace
 
@@ -402,18 +484,61 @@ cudaError_t launch_max_argmax(const int32_t *rowptr, const int32_t *col, const i
     return cudaGetLastError();
 }
 
+// The win marks pay on long rows, where an edge wins a feature with
+// probability about 1 / in-degree: on the 114.6M-edge graph (mean in-degree
+// 492, bf16) they cut the call 1.7-2x for F = 128-2048 and 1.4x at F =
+// 4096; on the 1.17M-edge graph (mean in-degree 6.9) they cost 2-60 % for
+// F = 8-128 (the marks' own launches and a dependent mark read per chunk
+// outweigh the short rows they skip).  So they are used when E >=
+// kMxbMarkDegree * N.
+#ifndef TFG_MXB_MARK_DEGREE
+#define TFG_MXB_MARK_DEGREE 32
+#endif
+constexpr int64_t kMxbMarkDegree = TFG_MXB_MARK_DEGREE;
+
+size_t max_backward_workspace_bytes(int64_t n, int64_t e, int64_t f) {
+    if (n <= 0 || e <= 0 || f <= 0 || e < kMxbMarkDegree * n) return 0;
+    return (static_cast<size_t>(e) + 255) & ~size_t(255);
+}
+
+// Features per mark bit: at most 8 groups, each a multiple of 4 features so
+// that a lane's 16-byte slice lies in one group.
+int mark_group(int64_t f) { return static_cast<int>(((f + 7) / 8 + 3) / 4 * 4); }
+
+cudaError_t launch_max_backward_marked(const int32_t *rowptr_src, const int32_t *col_src,
+                                       const int32_t *perm_src, const int32_t *argmax,
+                                       const float *edge_weight, const float *grad_out, int64_t n,
+                                       int64_t e, int64_t f, float *grad_x, void *ws,
+                                       cudaStream_t s) {
+    if (n <= 0) return cudaSuccess;
+    const bool marked = ws != nullptr && col_src != nullptr && max_backward_workspace_bytes(n, e, f) > 0;
+    uint8_t *mark = marked ? static_cast<uint8_t *>(ws) : nullptr;
+    const int group = mark_group(f);
+    if (marked) {
+        const int grid = sm_count() * 8;
+        max_marks_zero<<<grid, 256, 0, s>>>(mark, e);
+        max_marks_set<<<grid, f >= 256 ? 256 : 128, 0, s>>>(argmax, n, f, e, group, mark);
+    }
+    const MaxArgs a{rowptr_src, col_src, perm_src, edge_weight, grad_out, argmax, n, f, grad_x,
+                    nullptr, mark, e, group};
+    const int grid = balanced_grid(n, 0, 1);
+    const bool v4 = f % 4 == 0 && aligned(argmax, 16) && aligned(grad_out, 16) && aligned(grad_x, 16);
+    if (marked) {
+        if (v4) max_rows_kernel<MaxBwd<4, true>><<<grid, kMxThreads, 0, s>>>(a);
+        else max_rows_kernel<MaxBwd<1, true>><<<grid, kMxThreads, 0, s>>>(a);
+    } else {
+        if (v4) max_rows_kernel<MaxBwd<4, false>><<<grid, kMxThreads, 0, s>>>(a);
+        else max_rows_kernel<MaxBwd<1, false>><<<grid, kMxThreads, 0, s>>>(a);
+    }
+    return cudaGetLastError();
+}
+
 cudaError_t launch_max_backward(const int32_t *rowptr_src, const int32_t *col_src,
                                 const int32_t *perm_src, const int32_t *argmax,
                                 const float *edge_weight, const float *grad_out, int64_t n,
                                 int64_t f, float *grad_x, cudaStream_t s) {
-    if (n <= 0) return cudaSuccess;
-    const MaxArgs a{rowptr_src, col_src, perm_src, edge_weight, grad_out, argmax, n, f, grad_x,
-                    nullptr};
-    const int grid = balanced_grid(n, 0, 1);
-    const bool v4 = f % 4 == 0 && aligned(argmax, 16) && aligned(grad_out, 16) && aligned(grad_x, 16);
-    if (v4) max_rows_kernel<MaxBwd<4>><<<grid, kMxThreads, 0, s>>>(a);
-    else max_rows_kernel<MaxBwd<1>><<<grid, kMxThreads, 0, s>>>(a);
-    return cudaGetLastError();
+    return launch_max_backward_marked(rowptr_src, col_src, perm_src, argmax, edge_weight, grad_out,
+                                      n, 0, f, grad_x, nullptr, s);
 }
 
 }  // namespace tfg

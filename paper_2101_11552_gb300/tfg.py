@@ -82,7 +82,8 @@ def _load(path: str) -> ctypes.CDLL:
         "tfg_aggregate_backward": [I, P, P, P, P, P, P, I64, I64, I64, P, P, SZ, P],
         "tfg_gcn_aggregate_backward": [P, P, P, P, I64, I64, I, F, P, P],
         "tfg_aggregate_max_argmax": [P, P, P, P, P, I, I64, I64, P, P, P],
-        "tfg_aggregate_max_backward": [P, P, P, P, P, P, I64, I64, P, P],
+        "tfg_aggregate_max_backward_workspace_size": [I64, I64, I64, ctypes.POINTER(SZ)],
+        "tfg_aggregate_max_backward": [P, P, P, P, P, P, I64, I64, I64, P, P, SZ, P],
         "tfg_gcn_norm": [P, P, P, P, I64, I64, I, F, P, P, P],
         "tfg_aggregate_sum": [P, P, P, P, I, I64, I64, P, P],
         "tfg_aggregate_mean": [P, P, P, P, I, I64, I64, P, P],
@@ -277,17 +278,33 @@ def tfg_aggregate_max_argmax(csr: CSR, x, w_csr=None):
     return out, arg
 
 
-def tfg_aggregate_max_backward(csr_src: CSR, argmax, grad_out, edge_weight=None, out=None):
+def tfg_aggregate_max_backward_workspace_size(num_nodes: int, num_edges: int,
+                                              num_features: int) -> int:
+    nb = ctypes.c_size_t(0)
+    _check(lib().tfg_aggregate_max_backward_workspace_size(num_nodes, num_edges, num_features,
+                                                           ctypes.byref(nb)))
+    return nb.value
+
+
+def tfg_aggregate_max_backward(csr_src: CSR, argmax, grad_out, edge_weight=None, out=None,
+                               marks: bool = True):
     """grad_x of the max: w_e grad_out[t, f] to the source of the edge argmax[t, f]
-    (edge_weight in original edge order, or None)."""
+    (edge_weight in original edge order, or None).  marks=False runs without the
+    win-mark workspace (every out-edge's rows read; the same result)."""
     _need_cuda("grad_out", grad_out, torch.float32)
     dev = grad_out.device
     n, f = grad_out.shape
+    e = csr_src.col.numel()
+    ws = None
+    nb = tfg_aggregate_max_backward_workspace_size(n, e, f) if marks else 0
+    if nb > 0:
+        ws = torch.empty(nb, dtype=torch.uint8, device=dev)
     if out is None:
         out = torch.empty(n, f, dtype=torch.float32, device=dev)
     _check(lib().tfg_aggregate_max_backward(_ptr(csr_src.rowptr), _ptr(csr_src.col), _ptr(csr_src.perm),
-                                            _ptr(argmax), _ptr(edge_weight), _ptr(grad_out), n, f,
-                                            _ptr(out), _stream(dev)))
+                                            _ptr(argmax), _ptr(edge_weight), _ptr(grad_out), n, e, f,
+                                            _ptr(out), _ptr(ws), ws.numel() if ws is not None else 0,
+                                            _stream(dev)))
     return out
 
 

@@ -201,8 +201,19 @@ def test_backward_rejects(lib):
     assert am(FAKE, FAKE, FAKE, None, FAKE, 0, 10, 4, FAKE, None, None) == -1           # argmax
     assert am(FAKE, FAKE, FAKE, None, FAKE, 3, 10, 4, FAKE, FAKE, None) == -1           # dtype
     mb = lib.tfg_aggregate_max_backward
-    assert mb(FAKE, FAKE, None, FAKE, None, FAKE, 10, 4, FAKE, None) == -1              # perm_src
-    assert mb(FAKE, FAKE, FAKE, None, None, FAKE, 10, 4, FAKE, None) == -1              # argmax
+    assert mb(FAKE, FAKE, None, FAKE, None, FAKE, 10, 30, 4, FAKE, None, 0, None) == -1   # perm_src
+    assert mb(FAKE, FAKE, FAKE, None, None, FAKE, 10, 30, 4, FAKE, None, 0, None) == -1   # argmax
+    assert mb(FAKE, None, FAKE, FAKE, None, FAKE, 10, 30, 4, FAKE, None, 0, None) == -1   # col_src
+    assert mb(FAKE, FAKE, FAKE, FAKE, None, FAKE, 10, 320, 4, FAKE, FAKE, 256, None) == -3  # workspace
+    assert mb(FAKE, FAKE, FAKE, FAKE, None, FAKE, 10, 320, 4, FAKE, ctypes.c_void_p(0x1004), 1 << 20, None) == -1
+    nb = ctypes.c_size_t(0)
+    ws = lib.tfg_aggregate_max_backward_workspace_size
+    assert ws(10, 320, 4, ctypes.byref(nb)) == 0
+    assert nb.value == 512                           # a mark byte per edge, 256-byte rounded
+    assert ws(2, 300, 4000, ctypes.byref(nb)) == 0 and nb.value == 512
+    assert ws(10, 319, 4, ctypes.byref(nb)) == 0 and nb.value == 0     # E < 32 N: no marks
+    assert ws(10, 0, 4, ctypes.byref(nb)) == 0 and nb.value == 0
+    assert ws(10, -1, 4, ctypes.byref(nb)) == -1
     assert lib.tfg_build_csr_by_source(None, 10, 5, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20, FAKE, None) == -1
 
 

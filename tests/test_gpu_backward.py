@@ -97,6 +97,71 @@ def test_max_argmax_and_backward(dtype, weighted, f, reverse):
     refg, scale = oracle.max_backward(wl.edge_index, n, ref_arg, g,
                                       None if ew is None else ew.astype(np.float64))
     assert_scaled_close(got.cpu().numpy(), refg, scale, TOL_F32, "max backward")
+    # without the win marks every out-edge's rows are read: the same bits
+    plain = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g), None if ew is None else dev(ew),
+                                           marks=False)
+    assert torch.equal(got, plain)
+
+
+def test_max_backward_ignores_argmax_ids_outside_the_edges():
+    """argmax values outside [0, E) (and ids of edges into another row) match
+    no out-edge of the row, with and without the win marks."""
+    n, e, f = 400, 60000, 32
+    wl, csr, csr_src = _graphs(n, e, 41, f)
+    assert tfg.tfg_aggregate_max_backward_workspace_size(n, e, f) > 0
+    rng = np.random.default_rng(41)
+    _, arg = tfg.tfg_aggregate_max_argmax(csr, features(wl, "f32"))
+    bad = arg.cpu().numpy().copy()
+    pick = rng.random(bad.shape)
+    bad[pick < 0.05] = -7
+    bad[(pick >= 0.05) & (pick < 0.1)] = e + 3
+    bad[(pick >= 0.1) & (pick < 0.12)] = np.iinfo(np.int32).max
+    other = (pick >= 0.12) & (pick < 0.2)
+    bad[other] = rng.integers(0, e, size=int(other.sum()))    # mostly edges into other rows
+    g = rng.standard_normal((n, f)).astype(np.float32)
+    refg, scale = oracle.max_backward(wl.edge_index, n, bad, g, None)
+    for marks in (True, False):
+        got = tfg.tfg_aggregate_max_backward(csr_src, dev(bad), dev(g), marks=marks)
+        assert_scaled_close(got.cpu().numpy(), refg, scale, TOL_F32, f"max backward marks={marks}")
+
+
+@pytest.mark.parametrize("reverse", [False, True])
+@pytest.mark.parametrize("weighted", [False, True])
+@pytest.mark.parametrize("f", [4, 33, 36, 64])
+def test_max_backward_with_win_marks(f, weighted, reverse):
+    """Long rows (E >= 32 N): the call marks which eighths of the
+    features each edge wins and reads argmax and gradient slices for those
+    alone; the same bits as the walk over every out-edge.  Reversed, the hub (about half of the
+    edges) is a source row split over a CTA."""
+    n, e = 400, 60000
+    wl, csr, csr_src = _graphs(n, e, 90 + f, f, reverse)
+    assert tfg.tfg_aggregate_max_backward_workspace_size(n, e, f) > 0
+    rng = np.random.default_rng(f)
+    ew = rng.uniform(0.1, 3.0, size=e).astype(np.float32) if weighted else None
+    w_csr = None if ew is None else dev(ew[csr.perm.cpu().numpy()])
+    _, arg = tfg.tfg_aggregate_max_argmax(csr, features(wl, "bf16"), w_csr)
+    g = rng.standard_normal((n, f)).astype(np.float32)
+    got = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g), None if ew is None else dev(ew))
+    plain = tfg.tfg_aggregate_max_backward(csr_src, arg, dev(g), None if ew is None else dev(ew),
+                                           marks=False)
+    assert torch.equal(got, plain)
+    refg, scale = oracle.max_backward(wl.edge_index, n, arg.cpu().numpy(), g,
+                                      None if ew is None else ew.astype(np.float64))
+    assert_scaled_close(got.cpu().numpy(), refg, scale, TOL_F32, f"max backward with marks F={f}")
+
+
+def test_max_backward_workspace_is_checked():
+    n, e, f = 100, 4000, 4
+    wl, csr, csr_src = _graphs(n, e, 43, f)
+    _, arg = tfg.tfg_aggregate_max_argmax(csr, features(wl, "f32"))
+    g = dev(np.ones((n, f), np.float32))
+    out = torch.empty(n, f, device="cuda")
+    assert tfg.tfg_aggregate_max_backward_workspace_size(n, e, f) > 100
+    small = torch.empty(100, dtype=torch.uint8, device="cuda")
+    rc = tfg.lib().tfg_aggregate_max_backward(
+        tfg._ptr(csr_src.rowptr), tfg._ptr(csr_src.col), tfg._ptr(csr_src.perm), tfg._ptr(arg),
+        None, tfg._ptr(g), n, e, f, tfg._ptr(out), tfg._ptr(small), small.numel(), None)
+    assert rc == tfg.TFG_ERR_WORKSPACE
 
 
 def test_backward_is_deterministic_and_validates():
