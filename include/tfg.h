@@ -228,11 +228,11 @@ int tfg_gcn_aggregate_sum(const int32_t *rowptr, const int32_t *col, const float
  *   rowptr_src[num_nodes].  argmax values outside [0, num_edges) match no
  *   edge.  tfg_aggregate_max_backward_workspace_size() gives the workspace
  *   (16-byte aligned, overwritten) for win marks: on long rows (mean
- *   in-degree num_edges / num_nodes >= 32), where an edge wins few
- *   features, the call first marks, in a byte per edge, which eighths of
- *   the features the edge is the argmax of, and then reads argmax and
- *   gradient slices for those alone.  0 bytes: the marks would not pay and
- *   no workspace is used.
+ *   in-degree num_edges / num_nodes >= min(num_features, 128)), where most
+ *   edges win nothing, the call first marks, in a byte per edge, which
+ *   eighths of the features the edge is the argmax of, and then reads
+ *   argmax and gradient slices for those alone.  0 bytes: the marks would
+ *   not pay and no workspace is used.
  *   Workspace NULL reads the argmax and gradient rows of every out-edge.
  *   Both ways give the same bits.
  * grad_out, grad_x: fp32 [num_nodes, num_features]; grad_x is written.

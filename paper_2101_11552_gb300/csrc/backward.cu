@@ -107,7 +107,7 @@ __device__ __forceinline__ void max_combine(float &b, int32_t &p, float ob, int3
 
 template <typename XT, int VEC, int LPR>
 struct MaxFwd {
-    static constexpr int kVec = VEC, kLpr = LPR, kGroups = 32 / LPR, kMinBlocks = 1;
+    static constexpr int kVec = VEC, kLpr = LPR, kGroups = 32 / LPR;
     float best[VEC];
     int32_t pos[VEC];
 
@@ -223,7 +223,7 @@ struct MaxFwd {
 //    argmax check decides, as in the full walk.
 template <int VEC, bool MASKED>
 struct MaxBwd {
-    static constexpr int kVec = VEC, kLpr = 32, kMinBlocks = TFG_MXB_MINB;
+    static constexpr int kVec = VEC, kLpr = 32;
     float acc[VEC];
 
     __device__ void init() {
@@ -368,7 +368,7 @@ __device__ void max_cta_row(const MaxArgs &a, int64_t t, float *s_val, int32_t *
 }
 
 template <typename State>
-__global__ void __launch_bounds__(kMxThreads, State::kMinBlocks) max_rows_kernel(MaxArgs a) {
+__device__ __forceinline__ void max_rows(const MaxArgs &a) {
     __shared__ int s_next, s_nheavy;
     __shared__ int64_t s_heavy[kMxMaxHeavy];
     __shared__ float s_val[kMxWarps * State::kLpr * State::kVec];
@@ -402,6 +402,16 @@ __global__ void __launch_bounds__(kMxThreads, State::kMinBlocks) max_rows_kernel
     __syncthreads();
     const int nh = min(s_nheavy, kMxMaxHeavy);
     for (int h = 0; h < nh; ++h) max_cta_row<State>(a, s_heavy[h], s_val, s_pos);
+}
+
+// The forward keeps the compiler's register choice; the backward is held
+// to TFG_MXB_MINB resident CTAs per SM (64 registers per thread).
+template <typename State>
+__global__ void __launch_bounds__(kMxThreads) max_rows_kernel(MaxArgs a) { max_rows<State>(a); }
+
+template <typename State>
+__global__ void __launch_bounds__(kMxThreads, TFG_MXB_MINB) max_bwd_kernel(MaxArgs a) {
+    max_rows<State>(a);
 }
 
 bool aligned(const void *p, uintptr_t b) { return reinterpret_cast<uintptr_t>(p) % b == 0; }
@@ -484,20 +494,23 @@ cudaError_t launch_max_argmax(const int32_t *rowptr, const int32_t *col, const i
     return cudaGetLastError();
 }
 
-// The win marks pay on long rows, where an edge wins a feature with
-// probability about 1 / in-degree: on the 114.6M-edge graph (mean in-degree
-// 492, bf16) they cut the call 1.7-2x for F = 128-2048 and 1.4x at F =
-// 4096; on the 1.17M-edge graph (mean in-degree 6.9) they cost 2-60 % for
-// F = 8-128 (the marks' own launches and a dependent mark read per chunk
-// outweigh the short rows they skip).  So they are used when E >=
-// kMxbMarkDegree * N.
-#ifndef TFG_MXB_MARK_DEGREE
-#define TFG_MXB_MARK_DEGREE 32
+// The win marks pay when most edges win nothing in a row tile of kMxbSpan
+// features: an edge into a row of in-degree d wins a given feature with
+// probability about 1 / d, so it is visited in a tile with probability
+// about 1 - exp(-span / d), span = min(F, kMxbSpan).  They are used when
+// the mean in-degree E / N is at least span.  Measured: 114.6M edges, mean
+// in-degree 492, bf16: 1.7-2x faster for F = 128-2048, 1.4x at F = 4096;
+// 12.0M edges over the same nodes (mean in-degree 51.5, F = 128): 0.94 ms
+// for the marked walk + 0.15 ms for the marks against 0.91 ms unmarked
+// (ncu, serialised); 1.17M edges, mean in-degree 6.9: 2-60 % slower for F =
+// 8-128.
+#ifndef TFG_MXB_SPAN
+#define TFG_MXB_SPAN 128
 #endif
-constexpr int64_t kMxbMarkDegree = TFG_MXB_MARK_DEGREE;
+constexpr int64_t kMxbSpan = TFG_MXB_SPAN;
 
 size_t max_backward_workspace_bytes(int64_t n, int64_t e, int64_t f) {
-    if (n <= 0 || e <= 0 || f <= 0 || e < kMxbMarkDegree * n) return 0;
+    if (n <= 0 || e <= 0 || f <= 0 || e < n * (f < kMxbSpan ? f : kMxbSpan)) return 0;
     return (static_cast<size_t>(e) + 255) & ~size_t(255);
 }
 
@@ -524,11 +537,11 @@ cudaError_t launch_max_backward_marked(const int32_t *rowptr_src, const int32_t 
     const int grid = balanced_grid(n, 0, 1);
     const bool v4 = f % 4 == 0 && aligned(argmax, 16) && aligned(grad_out, 16) && aligned(grad_x, 16);
     if (marked) {
-        if (v4) max_rows_kernel<MaxBwd<4, true>><<<grid, kMxThreads, 0, s>>>(a);
-        else max_rows_kernel<MaxBwd<1, true>><<<grid, kMxThreads, 0, s>>>(a);
+        if (v4) max_bwd_kernel<MaxBwd<4, true>><<<grid, kMxThreads, 0, s>>>(a);
+        else max_bwd_kernel<MaxBwd<1, true>><<<grid, kMxThreads, 0, s>>>(a);
     } else {
-        if (v4) max_rows_kernel<MaxBwd<4, false>><<<grid, kMxThreads, 0, s>>>(a);
-        else max_rows_kernel<MaxBwd<1, false>><<<grid, kMxThreads, 0, s>>>(a);
+        if (v4) max_bwd_kernel<MaxBwd<4, false>><<<grid, kMxThreads, 0, s>>>(a);
+        else max_bwd_kernel<MaxBwd<1, false>><<<grid, kMxThreads, 0, s>>>(a);
     }
     return cudaGetLastError();
 }

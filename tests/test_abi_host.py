@@ -211,7 +211,9 @@ def test_backward_rejects(lib):
     assert ws(10, 320, 4, ctypes.byref(nb)) == 0
     assert nb.value == 512                           # a mark byte per edge, 256-byte rounded
     assert ws(2, 300, 4000, ctypes.byref(nb)) == 0 and nb.value == 512
-    assert ws(10, 319, 4, ctypes.byref(nb)) == 0 and nb.value == 0     # E < 32 N: no marks
+    assert ws(10, 39, 4, ctypes.byref(nb)) == 0 and nb.value == 0      # E < 4 N: no marks
+    assert ws(100, 12799, 200, ctypes.byref(nb)) == 0 and nb.value == 0  # E < 128 N: no marks
+    assert ws(100, 12800, 200, ctypes.byref(nb)) == 0 and nb.value == 12800
     assert ws(10, 0, 4, ctypes.byref(nb)) == 0 and nb.value == 0
     assert ws(10, -1, 4, ctypes.byref(nb)) == -1
     assert lib.tfg_build_csr_by_source(None, 10, 5, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20, FAKE, None) == -1

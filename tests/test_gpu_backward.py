@@ -129,7 +129,7 @@ def test_max_backward_ignores_argmax_ids_outside_the_edges():
 @pytest.mark.parametrize("weighted", [False, True])
 @pytest.mark.parametrize("f", [4, 33, 36, 64])
 def test_max_backward_with_win_marks(f, weighted, reverse):
-    """Long rows (E >= 32 N): the call marks which eighths of the
+    """Long rows (E >= min(F, 128) N): the call marks which eighths of the
     features each edge wins and reads argmax and gradient slices for those
     alone; the same bits as the walk over every out-edge.  Reversed, the hub (about half of the
     edges) is a source row split over a CTA."""
