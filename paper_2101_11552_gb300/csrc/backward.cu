@@ -231,22 +231,44 @@ struct MaxBwd {
         for (int q = 0; q < VEC; ++q) acc[q] = 0.f;
     }
 
+    // A chunk's loads: its target ids and edge ids, then (given the edge
+    // ids) its marks and weights.  Requesting the next chunk's ids and marks
+    // before this chunk's rows measured slower (more registers, spills).
+    struct Chunk {
+        int c;
+        int32_t ec;
+    };
+    static __device__ __forceinline__ Chunk ids(const MaxArgs &a, int64_t base, int64_t k1, int lane) {
+        Chunk r{0, 0};
+        if (base + lane < k1) {
+            r.c = ld_stream(a.col + base + lane);
+            r.ec = __ldg(a.perm + base + lane);
+        }
+        return r;
+    }
+    static __device__ __forceinline__ uint32_t mark_of(const MaxArgs &a, int64_t base, int64_t k1,
+                                                       int lane, int32_t ec) {
+        const bool mine = base + lane < k1;
+        if constexpr (MASKED)
+            return mine && static_cast<uint64_t>(ec) < static_cast<uint64_t>(a.e) ? __ldg(a.mark + ec) : 0u;
+        return mine ? 0xffu : 0u;
+    }
+    static __device__ __forceinline__ float weight_of(const MaxArgs &a, uint32_t mk, int32_t ec) {
+        return a.w ? (mk != 0 ? __ldg(a.w + ec) : 0.f) : 1.f;
+    }
+
     __device__ void scan(const MaxArgs &a, int64_t k0, int64_t k1, int64_t fl, bool, int lane) {
         constexpr int D = MASKED ? TFG_MXB_DEPTH : TFG_MXB_DEPTH_ALL;
         const float *g = static_cast<const float *>(a.x);
+        const uint32_t my_bit =
+            MASKED && TFG_MXB_GROUPS ? 1u << static_cast<uint32_t>(fl / a.group) : 0xffu;
         for (int64_t base = k0; base < k1; base += 32) {
-            const int cnt = static_cast<int>(min64(32, k1 - base));
-            const bool mine = lane < cnt;
-            const int c = mine ? ld_stream(a.col + base + lane) : 0;
-            const int32_t ec = mine ? __ldg(a.perm + base + lane) : 0;
-            uint32_t mk = mine ? 0xffu : 0u;
-            if constexpr (MASKED)
-                mk = mine && static_cast<uint64_t>(ec) < static_cast<uint64_t>(a.e) ? __ldg(a.mark + ec)
-                                                                                   : 0u;
+            const Chunk ch = ids(a, base, k1, lane);
+            const int c = ch.c;
+            const int32_t ec = ch.ec;
+            const uint32_t mk = mark_of(a, base, k1, lane, ec);
+            const float wc = weight_of(a, mk, ec);
             const bool win = mk != 0;
-            const float wc = a.w ? (win ? __ldg(a.w + ec) : 0.f) : 1.f;
-            const uint32_t my_bit =
-                MASKED && TFG_MXB_GROUPS ? 1u << static_cast<uint32_t>(fl / a.group) : 0xffu;
             // the chunk's edges that may contribute, D at a time in chunk order
             for (uint32_t m = __ballot_sync(kFull, win); m != 0;) {
                 int64_t t[D];
