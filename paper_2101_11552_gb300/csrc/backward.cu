@@ -287,19 +287,17 @@ struct MaxBwd {
                 }
                 int32_t am[D][VEC];
                 float gv[D][VEC];
-                {
 #pragma unroll
-                    for (int d = 0; d < D; ++d) {
-                        if (!ok[d]) continue;
-                        if constexpr (VEC == 4) {
-                            const int4 v = __ldg(reinterpret_cast<const int4 *>(a.argmax_in + t[d] * a.f + fl));
-                            const float4 w4 = __ldg(reinterpret_cast<const float4 *>(g + t[d] * a.f + fl));
-                            am[d][0] = v.x; am[d][1] = v.y; am[d][2] = v.z; am[d][3] = v.w;
-                            gv[d][0] = w4.x; gv[d][1] = w4.y; gv[d][2] = w4.z; gv[d][3] = w4.w;
-                        } else {
-                            am[d][0] = __ldg(a.argmax_in + t[d] * a.f + fl);
-                            gv[d][0] = __ldg(g + t[d] * a.f + fl);
-                        }
+                for (int d = 0; d < D; ++d) {
+                    if (!ok[d]) continue;
+                    if constexpr (VEC == 4) {
+                        const int4 v = __ldg(reinterpret_cast<const int4 *>(a.argmax_in + t[d] * a.f + fl));
+                        const float4 w4 = __ldg(reinterpret_cast<const float4 *>(g + t[d] * a.f + fl));
+                        am[d][0] = v.x; am[d][1] = v.y; am[d][2] = v.z; am[d][3] = v.w;
+                        gv[d][0] = w4.x; gv[d][1] = w4.y; gv[d][2] = w4.z; gv[d][3] = w4.w;
+                    } else {
+                        am[d][0] = __ldg(a.argmax_in + t[d] * a.f + fl);
+                        gv[d][0] = __ldg(g + t[d] * a.f + fl);
                     }
                 }
 #pragma unroll
