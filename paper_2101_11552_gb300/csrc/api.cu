@@ -279,7 +279,7 @@ int balanced_grid(int64_t n, int64_t e, int64_t min_work) {
 
 extern "C" {
 
-int tfg_version(void) { return 200; }
+int tfg_version(void) { return 300; }
 
 int tfg_check_bounds_enabled(void) { return TFG_CHECK_BOUNDS; }
 

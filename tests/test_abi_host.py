@@ -37,7 +37,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version(lib):
-    assert lib.tfg_version() == 200
+    assert lib.tfg_version() == 300
 
 
 def test_workspace_queries(lib):
